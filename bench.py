@@ -1,0 +1,405 @@
+#!/usr/bin/env python
+"""Throughput of the EOGP hot path on GB300.
+
+One step compresses one batch of B training examples through every module of
+the GPT-2-small-shaped stack (48 linears, T = 512 tokens, m = 4096 retained
+first-stage coordinates, k = 1024 PCA coordinates per module) into one-bit
+codes: Kronecker rotations, per-example contraction with the scale-and-gather
+epilogue, PCA projection, sign packing (Alg. 1 "Storing one training
+example"). Inputs are synthetic (Gaussian a and s, Haar eigenbases,
+power-law spectra with exponent 1.2), drawn on the device before timing; each
+step reads B x 151 MB of inputs, far more than L2, so no flush is needed.
+
+The JSON line's `value` is examples compressed per second per layer stack
+(whole job, all ranks). `scoring` reports the query x train scan (Q = 1024
+one-bit queries against N = 16384 stored codes). `e2e` repeats the
+compression through the same public API with the inputs in pinned host
+memory, host-to-device and device-to-host copies inside the timed region.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--batch B]
+    python bench.py --impl reference ...   # the CPU oracle on the host cores
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+WORKLOAD = "gpt2_small_bf16"
+METRIC = "training examples compressed/sec per layer stack"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# dram__bytes_read.sum + dram__bytes_write.sum per rotation launch from the committed
+# ncu capture (profiles/), or None when the kernel changed after the capture.
+ROTATE_TRAFFIC_BYTES = None
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return PEAKS_FALLBACK, "fallback"
+
+
+# --------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples every 200 ms while running."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.idx = None
+        try:
+            import torch
+            self.idx = "GPU-" + str(torch.cuda.get_device_properties(device_index).uuid)
+        except Exception:
+            vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+            self.idx = vis.split(",")[device_index] if vis else str(device_index)
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        rows = []
+        with open(self.path) as f:
+            for ln in f:
+                parts = [x.strip() for x in ln.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+# ----------------------------------------------------------- workload
+def build_stack(w, B, dev, seed):
+    """Per-module plans, retained eigenvector rows, PCA directions and inputs."""
+    import torch
+    from paper_2609_37842_gb300 import eogp as E
+    from paper_2609_37842_gb300 import synth
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    mods = []
+    plans = {}
+    for u, mod in enumerate(w.modules):
+        key = (mod.d_in, mod.d_out)
+        if key not in plans:
+            plans[key] = E.Plan.from_factors(synth.power_spectrum(mod.d_out, w.alpha),
+                                             synth.power_spectrum(mod.d_in, w.alpha), w.m,
+                                             w.damping_rel)
+        plan = plans[key]
+        inf = plan.info()
+        # The spectra are sorted, so C and R are index prefixes: the retained rows are the
+        # leading eigenvectors of fresh Haar bases.
+        R, C = plan.sets()
+        assert (C == range(inf.nC)).all() and (R == range(inf.nR)).all()
+        VA = synth.torch_eigvec_rows(mod.d_in, inf.nC, dev, g, torch.bfloat16)
+        VS = synth.torch_eigvec_rows(mod.d_out, inf.nR, dev, g, torch.bfloat16)
+        Pt = synth.torch_eigvec_rows(w.m, w.k, dev, g, torch.bfloat16)
+        a, s = synth.torch_layer_inputs(w, u, B, dev, g)
+        desc = E.layer_desc(plan, w.T, w.k, VA, VS, Pt)
+        mods.append(dict(desc=desc, a=a, s=s, d_in=mod.d_in, d_out=mod.d_out, nC=inf.nC,
+                         nR=inf.nR))
+    return mods
+
+
+def compress_step(mods, E, codes, scales, ws, words):
+    for u, md in enumerate(mods):
+        E.compress_layer(md["desc"], md["a"], md["s"], E.OUT_CODES,
+                         codes=codes[:, u * words:(u + 1) * words], scales=scales[:, u], ws=ws)
+
+
+def rotate_flops(mods, B, T):
+    return sum(2.0 * B * T * (md["d_in"] * md["nC"] + md["d_out"] * md["nR"]) for md in mods)
+
+
+# ------------------------------------------------------------ CPU oracle
+def cpu_sample(w, n_examples, seed=1):
+    """Time the oracle compressing `n_examples` examples through one module of each
+    distinct shape; returns (seconds per example per stack, cores, description)."""
+    import numpy as np
+    from oracle import eogp_oracle as O
+    from paper_2609_37842_gb300 import synth
+    shapes = {}
+    for u, mod in enumerate(w.modules):
+        shapes.setdefault((mod.d_in, mod.d_out), []).append(u)
+    rng = np.random.default_rng(seed)
+    total = 0.0
+    for (d_in, d_out), us in shapes.items():
+        u = us[0]
+        QA = synth.round_bf16(synth.haar_orthogonal(d_in, rng))
+        QS = synth.round_bf16(synth.haar_orthogonal(d_out, rng))
+        lamA, lamS = synth.power_spectrum(d_in, w.alpha), synth.power_spectrum(d_out, w.alpha)
+        P = synth.round_bf16(synth.haar_orthogonal(w.m, rng, w.k))
+        a, s = synth.layer_inputs(w, u, n_examples)
+        t0 = time.perf_counter()
+        Lam = O.kfac_eigenvalues(lamS, lamA)
+        lam = O.damping(Lam, w.damping_rel)
+        O.compress_layer(a, s, QA, QS, Lam, lam, w.m, P)
+        dt = (time.perf_counter() - t0) / n_examples
+        total += dt * len(us)
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    desc = (f"{n_examples} example(s) x one module of each of the {len(shapes)} distinct shapes, "
+            f"scaled by the shape counts to the {len(w.modules)}-module stack")
+    return total, cores, desc
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    from paper_2609_37842_gb300 import synth
+    w = synth.WORKLOADS[WORKLOAD]
+    for _ in range(args.warmup):
+        cpu_sample(w, 1)
+    ts = []
+    cores, desc = None, None
+    for _ in range(args.steps):
+        t, cores, desc = cpu_sample(w, 1)
+        ts.append(t)
+    sec = sum(ts)
+    value = args.steps / sec
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "examples/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000 * sec / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "batch": 1, "seq_len": w.T, "m": w.m, "k": w.k,
+                       "modules": len(w.modules)},
+            "cpu_baseline": {"value": value, "unit": "examples/s", "cores": cores,
+                             "kind": "oracle", "sample": desc},
+            "e2e": {"value": value, "unit": "examples/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+# ------------------------------------------------------------------ main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--batch", type=int, default=128)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-score", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_37842_gb300 import eogp as E
+    from paper_2609_37842_gb300 import synth
+
+    w = synth.WORKLOADS[WORKLOAD]
+    B, T, U = args.batch, w.T, len(w.modules)
+    words = (w.k + 31) // 32
+    peaks, peaks_src = load_peaks()
+
+    mods = build_stack(w, B, dev, seed=1000 + rank)
+    ws_bytes = max(E.compress_workspace_size(md["desc"], B, E.OUT_CODES) for md in mods)
+    ws = E.workspace(ws_bytes, dev)
+    codes = torch.empty((B, U * words), dtype=torch.int32, device=dev)
+    scales = torch.empty((B, U), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        compress_step(mods, E, codes, scales, ws, words)
+    E.sync_status()
+
+    # ---- timed region: K compression steps, kernel events on ----
+    for kk in E.KERNEL_KINDS:
+        E.profile_read(kk, reset=True)
+    E.profile_enable(True)
+    clocks = ClockSampler(local)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        compress_step(mods, E, codes, scales, ws, words)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    E.profile_enable(False)
+    E.sync_status()
+    ms = ev0.elapsed_time(ev1)
+    kern = {}
+    for kk, name in E.KERNEL_KINDS.items():
+        n, t = E.profile_read(kk, reset=True)
+        if n:
+            kern[name] = {"launches": n, "ms": t}
+    t_max = ms
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t_max = float(tt.item())
+    value = world * B * args.steps / (t_max / 1000.0)
+    launches = sum(v["launches"] for v in kern.values())
+    ktot = sum(v["ms"] for v in kern.values())
+    for v in kern.values():
+        v["share"] = v["ms"] / ktot if ktot else None
+
+    rot = kern.get("rotate", {"launches": 0, "ms": 0.0})
+    flops_per_launch = rotate_flops(mods, B, T) / (2 * U)
+    avg_ms = rot["ms"] / max(1, rot["launches"])
+    achieved = flops_per_launch / (avg_ms / 1000.0) / 1e12 if avg_ms > 0 else None
+    peak = peaks.get("bf16_tflops_sustained") or PEAKS_FALLBACK["bf16_tflops_sustained"]
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": (achieved / peak) if achieved else None,
+                "traffic": ROTATE_TRAFFIC_BYTES, "kernel": "k_tc_gemm (Kronecker rotation)",
+                "peak_source": f"{peaks_src} bf16_tflops_sustained",
+                "flops_per_launch": flops_per_launch}
+
+    # ---- scoring: Q = 1024 one-bit queries x N = 16384 stored codes ----
+    scoring = None
+    if not args.no_score:
+        N, Q = w.N, w.Q
+        g = torch.Generator(device=dev)
+        g.manual_seed(77 + rank)
+        tc = torch.randint(-2 ** 31, 2 ** 31 - 1, (N, U * words), generator=g, device=dev,
+                           dtype=torch.int32)
+        qc = torch.randint(-2 ** 31, 2 ** 31 - 1, (Q, U * words), generator=g, device=dev,
+                           dtype=torch.int32)
+        tsc = torch.exp(0.5 * torch.randn((N, U), generator=g, device=dev))
+        qsc = torch.exp(0.5 * torch.randn((Q, U), generator=g, device=dev))
+        out = torch.empty((Q, N), dtype=torch.float32, device=dev)
+        ks = [w.k] * U
+        E.score(tc, tsc, ks, E.SCORE_CODES, qc, qsc, out=out)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = 3
+        e0.record(stream)
+        for _ in range(reps):
+            E.score(tc, tsc, ks, E.SCORE_CODES, qc, qsc, out=out)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        E.sync_status()
+        sms = e0.elapsed_time(e1) / reps
+        words_total = N * Q * U * words
+        scoring = {"metric": "query x train scores/sec", "value": N * Q / (sms / 1000.0),
+                   "unit": "scores/s", "ms_per_call": sms, "N": N, "Q": Q, "bits": U * w.k,
+                   "mode": "CODES (xor-popcount)", "word_ops_per_s": words_total / (sms / 1000.0)}
+
+    # ---- end to end through the public API with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        host = []
+        for md in mods:
+            ha = torch.empty(md["a"].shape, dtype=md["a"].dtype, pin_memory=True)
+            hs = torch.empty(md["s"].shape, dtype=md["s"].dtype, pin_memory=True)
+            ha.copy_(md["a"])
+            hs.copy_(md["s"])
+            host.append((ha, hs))
+        hcodes = torch.empty(codes.shape, dtype=codes.dtype, pin_memory=True)
+        hscales = torch.empty(scales.shape, dtype=scales.dtype, pin_memory=True)
+        h2d = sum(ha.numel() * ha.element_size() + hs.numel() * hs.element_size() for ha, hs in host)
+        d2h = hcodes.numel() * 4 + hscales.numel() * 4
+
+        def e2e_step():
+            for md, (ha, hs) in zip(mods, host):
+                md["a"].copy_(ha, non_blocking=True)
+                md["s"].copy_(hs, non_blocking=True)
+            compress_step(mods, E, codes, scales, ws, words)
+            hcodes.copy_(codes, non_blocking=True)
+            hscales.copy_(scales, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        E.sync_status()
+        ems = e0.elapsed_time(e1)
+        if world > 1:
+            tt = torch.tensor([ems], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            ems = float(tt.item())
+        e2e = {"value": world * B * args.e2e_steps / (ems / 1000.0), "unit": "examples/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps}
+        del host
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        sec, cores, desc = cpu_sample(w, 1)
+        cpu = {"value": 1.0 / sec, "unit": "examples/s", "cores": cores, "kind": "oracle",
+               "sample": desc}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": t_max / args.steps, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+                "config": {"workload": WORKLOAD, "batch_per_gpu": B, "seq_len": T, "m": w.m,
+                           "k": w.k, "modules": U, "parallelism": f"replicas x{world}",
+                           "l2": "inputs > L2 (B x 151 MB per step)"},
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "scoring": scoring,
+                "gpu_launches": launches, "kernels": kern, "clocks": clk}
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,259 @@
+/*
+ * eogp.h -- C ABI of libeogp, a GB300 (sm_103a) implementation of the
+ * data-parallel hot path of EOGP, "Scaling Influence Functions in LLMs through
+ * Eigenbasis-Corrected One-Bit Gradient Projection" (arxiv 2609.37842):
+ * per-example gradient compression into one-bit codes and influence scoring
+ * of queries against the stored codes.
+ *
+ * Notation (the paper's). One linear module ("module u") has input
+ * activations a_t in R^{d_in} and output gradients s_t in R^{d_out} for tokens
+ * t = 1..T of an example. Its per-example gradient is G = sum_t s_t a_t^T
+ * (d_out x d_in, Sec. 2.2). Q_A, Q_S are the K-FAC eigenbases of the two
+ * Kronecker factors (Sec. 2.2, Eq. kfac_factorization) and Lambda[j][i] the
+ * (corrected) eigenvalue of the Kronecker coordinate (j, i), i.e. of the basis
+ * vector Q_A[:, i] (x) Q_S[:, j] (Eq. ekfac_eigendecompose).
+ *
+ * General conventions for every entry point:
+ *  - Array arguments named "device" are device pointers owned by the caller;
+ *    the library never frees or retains them after the call returns.
+ *  - Matrices are row-major with an explicit leading dimension in ELEMENTS
+ *    (ld >= row length). "bf16" means IEEE bfloat16 stored in uint16.
+ *  - Calls that take a stream are asynchronous on that stream (0 = the legacy
+ *    default stream) unless stated otherwise; the current CUDA device must be
+ *    the device that owns the pointers. They do not allocate: scratch memory
+ *    ("workspace") is sized with the matching *_workspace_size call and passed
+ *    in, 256-byte aligned.
+ *  - Every call returns an int status: EOGP_OK (0) or a negative EOGP_E*
+ *    code; eogp_last_error() then returns a thread-local message. Argument
+ *    errors are detected on the host before anything is launched.
+ *  - Kernels never trap. A bounded wait that expires (or another device-side
+ *    fault the kernels detect) sets a device status word; eogp_sync_status()
+ *    synchronizes a stream and returns / clears it (EOGP_ETIMEOUT, EOGP_EDEVICE).
+ *  - Unsupported shape/dtype combinations return EOGP_EUNSUPPORTED; there is
+ *    no CPU fallback.
+ */
+#ifndef EOGP_H
+#define EOGP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* cudaStream_t without including the CUDA headers. */
+typedef struct CUstream_st* eogp_stream_t;
+
+/* ---- status codes ------------------------------------------------------ */
+#define EOGP_OK            0
+#define EOGP_EINVAL       (-1) /* invalid argument (null pointer, size, stride, alignment) */
+#define EOGP_EUNSUPPORTED (-2) /* valid request that this build does not implement */
+#define EOGP_ECUDA        (-3) /* a CUDA runtime/driver call failed */
+#define EOGP_ETIMEOUT     (-4) /* a kernel's bounded wait expired (from eogp_sync_status) */
+#define EOGP_EWORKSPACE   (-5) /* workspace smaller than *_workspace_size reported */
+#define EOGP_EDEVICE      (-6) /* other device-side error recorded by a kernel */
+
+/* ---- element types ----------------------------------------------------- */
+#define EOGP_F32  0 /* float32 inputs; computed with fp32 CUDA-core kernels */
+#define EOGP_BF16 1 /* bfloat16 inputs; tcgen05 tensor-core kernels, fp32 accumulation */
+
+/* ---- eogp_compress_layer output modes ---------------------------------- */
+#define EOGP_OUT_FIRST_STAGE 0 /* z = (Lambda_m + lambda I)^{-1/2} Q_m^T g   [B x m] fp32 */
+#define EOGP_OUT_COORDS      1 /* x = P^T z                                  [B x k] fp32 */
+#define EOGP_OUT_CODES       2 /* sign bits of x (packed) + scale ||x||_1/k              */
+
+/* ---- eogp_score modes -------------------------------------------------- */
+#define EOGP_SCORE_CODES 0 /* sum_u s_iu s_qu <b_iu, b_qu>  (both sides one-bit)     */
+#define EOGP_SCORE_PAPER 1 /* sum_u s_iu <y_u, b_iu>        (query unquantized)      */
+#define EOGP_SCORE_FP    2 /* <y, x>                        (no quantization)        */
+
+/* Last error message of the calling thread ("" if none). Never NULL. */
+const char* eogp_last_error(void);
+
+/* Library version string. */
+const char* eogp_version(void);
+
+/* Synchronizes `stream`, then returns and clears the device status word of the
+ * current device: EOGP_OK, EOGP_ETIMEOUT (a bounded mbarrier/flag wait expired)
+ * or EOGP_EDEVICE (another kernel-detected error, e.g. a non-finite input to
+ * eogp_pack_sign). EOGP_ECUDA if the synchronization itself failed. */
+int eogp_sync_status(eogp_stream_t stream);
+
+/* ---- kernel timing ------------------------------------------------------
+ * While enabled (process-wide), every kernel the library launches is
+ * bracketed by two CUDA events recorded on the stream it is launched on.
+ * eogp_profile_read synchronizes on the recorded events and returns, for one
+ * kernel kind, the number of launches and their summed device time; reset = 1
+ * releases the records of that kind. Kinds: */
+#define EOGP_K_ROTATE   0 /* tcgen05 Kronecker rotation GEMM (A and S sides)    */
+#define EOGP_K_CONTRACT 1 /* tcgen05 per-example contraction + gather          */
+#define EOGP_K_PROJECT  2 /* tcgen05 second-stage projection (split K)         */
+#define EOGP_K_PACK     3 /* sign/scale packing (also the split-K finalise)    */
+#define EOGP_K_SCORE    4 /* scoring kernels                                   */
+#define EOGP_K_SIMT     5 /* fp32 CUDA-core kernels of the EOGP_F32 path       */
+#define EOGP_K_COUNT    6
+int eogp_profile_enable(int on);
+int eogp_profile_read(int kind, int* launches, double* total_ms, int reset);
+
+/* ========================================================================
+ * Retained-set plan (host; once per module)
+ *
+ * Selects the m Kronecker eigen-coordinates with the largest eigenvalues
+ * (Sec. 3.2: the top-m eigenvectors of Sigma_proxy, Eq. sigma_ekfac, are those
+ * of the m largest corrected eigenvalues; Alg. 1 "Select Q_{u,m}, Lambda_{u,m}")
+ * and the damping lambda = damping_rel * tr(Lambda)/d (App. C.2,
+ * Eq. app_module_damping; the paper uses damping_rel = 0.1).
+ * ======================================================================== */
+typedef struct eogp_plan eogp_plan;
+
+typedef struct {
+  int d_in, d_out, m;
+  int nR;        /* distinct rows j of the retained set (size of R)            */
+  int nC;        /* distinct columns i (size of C)                             */
+  int n_tiles;   /* active 128 x 128 tiles of the R x C block                  */
+  double lambda; /* damping actually used                                      */
+} eogp_plan_info;
+
+/* Build a plan. Eigenvalues are given EITHER as the two K-FAC factor spectra
+ * (lam_S [d_out], lam_A [d_in]; Lambda[j][i] = lam_S[j] * lam_A[i] formed in
+ * double) with Lambda == NULL, OR as the full corrected table Lambda
+ * [d_out x d_in] (row-major, double) with lam_S == lam_A == NULL. All are HOST
+ * arrays, read during the call only.
+ * Canonical retained order: eigenvalue descending, ties broken by the
+ * Kronecker column position i*d_out + j ascending. R and C are the distinct
+ * j / i of the retained set in ascending order.
+ * The plan owns small device tables (allocated here on the current device,
+ * freed by eogp_plan_destroy); it must be used on that device only.
+ * Errors: EOGP_EINVAL (null out, d_in/d_out < 1, m outside [1, d_in*d_out],
+ * damping_rel < 0, both or neither eigenvalue forms, non-finite or negative
+ * eigenvalues), EOGP_ECUDA. */
+int eogp_plan_layer(const double* lam_S, const double* lam_A, const double* Lambda,
+                    int d_in, int d_out, int m, double damping_rel, eogp_plan** out);
+
+void eogp_plan_destroy(eogp_plan* plan);
+
+int eogp_plan_get_info(const eogp_plan* plan, eogp_plan_info* info);
+
+/* Host copies of the canonical retained list: j[m], i[m] (int32) and the
+ * fp32 scale (Lambda[j][i] + lambda)^{-1/2} of Eq. first_stage. Any output
+ * pointer may be NULL. */
+int eogp_plan_get_retained(const eogp_plan* plan, int32_t* j, int32_t* i, float* scale);
+
+/* Host copies of R [nR] and C [nC] (either may be NULL). */
+int eogp_plan_get_sets(const eogp_plan* plan, int32_t* R, int32_t* C);
+
+/* Gather the retained eigenvectors as rows, the layout eogp_compress_layer
+ * reads: which = 0 copies V_full row C[r] (an eigenvector of A, i.e. column
+ * C[r] of Q_A) to row r of V_ret [nC x d_in]; which = 1 copies row R[r] of
+ * V_full (eigenvectors of S as rows, d_out x d_out) to V_ret [nR x d_out].
+ * dtype EOGP_F32 or EOGP_BF16; V_full with leading dimension ld_full; V_ret
+ * dense. Device pointers, asynchronous on `stream`. */
+int eogp_plan_gather_rows(const eogp_plan* plan, int which, int dtype, const void* V_full,
+                          int ld_full, void* V_ret, eogp_stream_t stream);
+
+/* ========================================================================
+ * Compression of one module (Alg. 1 "Storing one training example", applied
+ * to a batch of B examples; also the query projection y_u = T_u(L_u q_u)).
+ * ======================================================================== */
+typedef struct {
+  int d_in, d_out; /* module shape                                             */
+  int T;           /* tokens per example                                       */
+  int m;           /* retained first-stage coordinates (= plan m)              */
+  int k;           /* PCA output coordinates (sign bits) per example           */
+  int dtype;       /* EOGP_F32 or EOGP_BF16: type of a, s, VA, VS, Pt          */
+  const void* VA;  /* device [nC x d_in]: row r = eigenvector Q_A[:, C[r]]     */
+  const void* VS;  /* device [nR x d_out]: row r = eigenvector Q_S[:, R[r]]    */
+  const void* Pt;  /* device [k x m]: row c = PCA direction c (column c of P,
+                      App. B.2) over the canonical retained order; may be NULL
+                      for EOGP_OUT_FIRST_STAGE                                 */
+  const eogp_plan* plan;
+} eogp_layer_desc;
+
+/* Workspace bytes eogp_compress_layer needs for this descriptor, batch B and
+ * output mode. */
+int eogp_compress_workspace_size(const eogp_layer_desc* L, int B, int out_mode, size_t* bytes);
+
+/* For each example b < B (Sec. 3.2 Eq. first_stage and Eq. second_stage;
+ * Sec. 3.3 Eq. onebit):
+ *   G~_b = Q_S^T G_b Q_A evaluated on the retained rows/columns only, as
+ *          sum_t (V_S s_t)(V_A a_t)^T  (the Kronecker identity of Sec. 2.2),
+ *   z_b[r] = (Lambda[j_r][i_r] + lambda)^{-1/2} G~_b[j_r][i_r],
+ *   x_b = P^T z_b,
+ *   codes_b: bit (c % 32) of word c / 32 is 1 iff x_b[c] >= 0 (App. E.1 byte
+ *            order; pad bits 0), scales_b = ||x_b||_1 / k.
+ * Inputs: a [B x T x d_in], s [B x T x d_out] (dtype, dense, device).
+ * Outputs by out_mode:
+ *   FIRST_STAGE: out = z [B x ld_out], ld_out >= m;
+ *   COORDS:      out = x [B x ld_out], ld_out >= k;
+ *   CODES:       codes [B x ld_codes] uint32 (ld_codes >= ceil(k/32), so a
+ *                module's words can sit at an offset inside a wider store row)
+ *                and scales[b * ld_scales] fp32; `out` is ignored.
+ * BF16 requires d_in, d_out, m multiples of 8 (16-byte TMA strides) and
+ * 16-byte aligned a, s, VA, VS, Pt; F32 has no extra constraint.
+ * Errors: EOGP_EINVAL, EOGP_EUNSUPPORTED, EOGP_EWORKSPACE, EOGP_ECUDA. */
+int eogp_compress_layer(const eogp_layer_desc* L, const void* a, const void* s, int B,
+                        int out_mode, float* out, int ld_out, uint32_t* codes, int ld_codes,
+                        float* scales, int ld_scales, void* ws, size_t ws_bytes,
+                        eogp_stream_t stream);
+
+/* ========================================================================
+ * PCA fit (App. B.2 "PCA fitting"; Alg. 1 "fit P_u by uncentered PCA")
+ * ======================================================================== */
+int eogp_fit_pca_workspace_size(int n, int m, int k, size_t* bytes);
+
+/* Z [n x ldz] fp32 device (rows = first-stage coordinates of n fitting
+ * examples). Writes Pt [k x ld_pt] (row c = unit eigenvector c of Z^T Z / n,
+ * eigenvalue descending; sign fixed so that its largest-magnitude entry is
+ * positive, ties to the lowest index) as EOGP_F32 or EOGP_BF16 (pt_dtype), and
+ * eig [k] fp32 (the eigenvalues of Z^T Z / n). Uses the n x n Gram matrix when
+ * n < m, as the paper describes. Eigenpairs come from a cyclic Jacobi
+ * eigensolver on the device, in fp64. This call BLOCKS the host until the fit
+ * is done (it reads a convergence measure once per sweep).
+ * Errors: EOGP_EINVAL (k < 1 or k > min(n, m), ldz < m, ld_pt < m),
+ * EOGP_EWORKSPACE, EOGP_EUNSUPPORTED (min(n, m) > 12288), EOGP_ECUDA. */
+int eogp_fit_pca(const float* Z, int n, int m, int ldz, int k, void* Pt, int ld_pt, int pt_dtype,
+                 float* eig, void* ws, size_t ws_bytes, eogp_stream_t stream);
+
+/* ========================================================================
+ * One-bit encoding (Sec. 3.3 Eq. onebit; Alg. 1 "Store packed binary signs")
+ * ======================================================================== */
+/* x [B x ldx] fp32 device -> codes [B x ld_codes] uint32 (bit c % 32 of word
+ * c / 32 = [x_c >= 0], pad bits 0) and scales[b * ld_scales] = ||x_b||_1 / k
+ * (fixed-order reduction: bitwise reproducible). A NaN input sets
+ * EOGP_EDEVICE in the device status word. */
+int eogp_pack_sign(const float* x, int B, int k, int ldx, uint32_t* codes, int ld_codes,
+                   float* scales, int ld_scales, eogp_stream_t stream);
+
+/* ========================================================================
+ * Scoring (Sec. 3.3 Eq. onebit_influence; App. B.3 Eq. app_stored_influence;
+ * scan cost Eq. app_scan_complexity). Module contributions are summed.
+ * ======================================================================== */
+int eogp_score_workspace_size(int N, const int* k_per_module, int U, int mode, int Q,
+                              size_t* bytes);
+
+/* U modules with k_per_module[u] coordinates (HOST array). A stored row holds
+ * the modules' codes back to back, module u starting at word
+ * sum_{v<u} ceil(k_v/32); W = total words.
+ *   CODES: train = uint32 codes [N x ld_train] (ld_train >= W),
+ *          train_scales [N x ld_tscale], query = uint32 codes [Q x ld_query],
+ *          query_scales [Q x ld_qscale];
+ *          scores[q][i] = sum_u fl(fl(s_qu * s_iu) * (k_u - 2 popc(b_iu ^ b_qu))),
+ *          accumulated in fp32 in module order with no fused multiply-add
+ *          (bitwise reproducible).
+ *   PAPER: train = codes as above, train_scales as above, query = fp32
+ *          coordinates [Q x ld_query] (module u at column sum_{v<u} k_v),
+ *          query_scales ignored; scores[q][i] = sum_u s_iu <y_qu, b_iu>.
+ *   FP:    train = fp32 coordinates [N x ld_train], query = fp32 [Q x ld_query];
+ *          scores[q][i] = <y_q, x_i>; scales ignored.
+ * scores [Q x ld_scores] fp32 device, ld_scores >= N.
+ * Errors: EOGP_EINVAL, EOGP_EWORKSPACE, EOGP_ECUDA. */
+int eogp_score(const void* train, int ld_train, const float* train_scales, int ld_tscale, int N,
+               const int* k_per_module, int U, int mode, const void* query, int ld_query,
+               const float* query_scales, int ld_qscale, int Q, float* scores, int ld_scores,
+               void* ws, size_t ws_bytes, eogp_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* EOGP_H */

@@ -1,0 +1,726 @@
+// C ABI of libeogp (include/eogp.h): argument checking, the retained-set plan,
+// workspace layout and kernel dispatch. No entry point allocates device memory
+// except eogp_plan_layer (its small tables, freed by eogp_plan_destroy).
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <numeric>
+#include <vector>
+
+#include "eogp_dev.cuh"
+#include "eogp_internal.h"
+
+// Device status word (one per device that loads the library), see eogp_sync_status.
+__device__ unsigned int g_eogp_status;
+
+namespace eogp {
+
+static thread_local char g_err[1024];
+
+int set_error(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+void clear_error() { g_err[0] = '\0'; }
+
+unsigned* status_word() {
+  static unsigned* addr[128] = {nullptr};
+  static std::mutex mu;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 128) return nullptr;
+  std::lock_guard<std::mutex> lk(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_eogp_status) != cudaSuccess) return nullptr;
+    addr[dev] = static_cast<unsigned*>(p);
+  }
+  return addr[dev];
+}
+
+static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+int make_tmap(CUtensorMap* tm, CUtensorMapDataType dt, int rank, const void* base,
+              const uint64_t* dims, const uint64_t* strides_bytes, const uint32_t* box,
+              CUtensorMapSwizzle swz) {
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  if (!g_encode) return set_error(EOGP_ECUDA, "cuTensorMapEncodeTiled is unavailable");
+  cuuint64_t d[5];
+  cuuint64_t s[4];
+  cuuint32_t b[5], es[5];
+  for (int r = 0; r < rank; ++r) {
+    d[r] = dims[r];
+    b[r] = box[r];
+    es[r] = 1;
+    if (r + 1 < rank) s[r] = strides_bytes[r];
+  }
+  const CUresult res = g_encode(tm, dt, static_cast<cuuint32_t>(rank), const_cast<void*>(base), d,
+                                s, b, es, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                                CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (res != CUDA_SUCCESS) return set_error(EOGP_ECUDA, "cuTensorMapEncodeTiled failed (%d)", (int)res);
+  return EOGP_OK;
+}
+
+}  // namespace eogp
+
+using namespace eogp;
+
+#define CUDA_TRY(x)                                                                      \
+  do {                                                                                   \
+    cudaError_t e_ = (x);                                                                \
+    if (e_ != cudaSuccess)                                                               \
+      return set_error(EOGP_ECUDA, "%s failed: %s", #x, cudaGetErrorString(e_));         \
+  } while (0)
+
+static inline size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
+static inline int round_up(int x, int a) { return (x + a - 1) / a * a; }
+
+static int sm_count() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0, v = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && v > 0)
+      n = v;
+    else
+      return 148;
+  }
+  return n;
+}
+
+static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// ----------------------------------------------------------- kernel timing
+namespace {
+struct ProfRec {
+  cudaEvent_t a, b;
+};
+std::mutex g_prof_mu;
+bool g_prof_on = false;
+std::vector<ProfRec> g_prof[EOGP_K_COUNT];
+std::vector<cudaEvent_t> g_prof_free;
+
+cudaEvent_t prof_event() {
+  if (!g_prof_free.empty()) {
+    cudaEvent_t e = g_prof_free.back();
+    g_prof_free.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+// Brackets the launches made during its lifetime with events on `st`.
+struct ProfScope {
+  int kind;
+  cudaStream_t st;
+  cudaEvent_t a = nullptr;
+  ProfScope(int k, cudaStream_t s) : kind(k), st(s) {
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    if (!g_prof_on) return;
+    a = prof_event();
+    if (a) cudaEventRecord(a, st);
+  }
+  ~ProfScope() {
+    if (!a) return;
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    cudaEvent_t b = prof_event();
+    if (!b) return;
+    cudaEventRecord(b, st);
+    g_prof[kind].push_back(ProfRec{a, b});
+  }
+};
+}  // namespace
+
+extern "C" int eogp_profile_enable(int on) {
+  clear_error();
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  g_prof_on = on != 0;
+  return EOGP_OK;
+}
+
+extern "C" int eogp_profile_read(int kind, int* launches, double* total_ms, int reset) {
+  clear_error();
+  if (kind < 0 || kind >= EOGP_K_COUNT || !launches || !total_ms) return set_error(EOGP_EINVAL, "bad argument");
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  double tot = 0.0;
+  for (const ProfRec& r : g_prof[kind]) {
+    CUDA_TRY(cudaEventSynchronize(r.b));
+    float ms = 0.f;
+    CUDA_TRY(cudaEventElapsedTime(&ms, r.a, r.b));
+    tot += ms;
+  }
+  *launches = static_cast<int>(g_prof[kind].size());
+  *total_ms = tot;
+  if (reset) {
+    for (const ProfRec& r : g_prof[kind]) {
+      g_prof_free.push_back(r.a);
+      g_prof_free.push_back(r.b);
+    }
+    g_prof[kind].clear();
+  }
+  return EOGP_OK;
+}
+
+extern "C" const char* eogp_last_error(void) { return g_err; }
+
+extern "C" const char* eogp_version(void) { return "eogp-gb300 0.1 (sm_103a)"; }
+
+extern "C" int eogp_sync_status(eogp_stream_t stream) {
+  clear_error();
+  CUDA_TRY(cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)));
+  unsigned* w = status_word();
+  if (!w) return set_error(EOGP_ECUDA, "device status word unavailable");
+  unsigned v = 0;
+  CUDA_TRY(cudaMemcpy(&v, w, sizeof(v), cudaMemcpyDeviceToHost));
+  if (v) CUDA_TRY(cudaMemset(w, 0, sizeof(unsigned)));
+  if (v & EOGP_ST_TIMEOUT) return set_error(EOGP_ETIMEOUT, "a kernel's bounded wait expired");
+  if (v) return set_error(EOGP_EDEVICE, "device-side error flag 0x%x", v);
+  return EOGP_OK;
+}
+
+// =================================================================== plan
+
+static void plan_free_device(eogp_plan* p) {
+  int32_t** ip[] = {&p->d_tile_rc, &p->d_tile_start, &p->d_ent_r, &p->d_ent_off,
+                    &p->d_posR,    &p->d_posC,       &p->d_R,     &p->d_C};
+  for (auto q : ip) {
+    if (*q) cudaFree(*q);
+    *q = nullptr;
+  }
+  float** fp[] = {&p->d_ent_scale, &p->d_scale};
+  for (auto q : fp) {
+    if (*q) cudaFree(*q);
+    *q = nullptr;
+  }
+}
+
+template <typename T>
+static int upload(T** dst, const std::vector<T>& src) {
+  const size_t bytes = std::max<size_t>(1, src.size()) * sizeof(T);
+  CUDA_TRY(cudaMalloc(reinterpret_cast<void**>(dst), bytes));
+  if (!src.empty()) CUDA_TRY(cudaMemcpy(*dst, src.data(), src.size() * sizeof(T), cudaMemcpyHostToDevice));
+  return EOGP_OK;
+}
+
+extern "C" int eogp_plan_layer(const double* lam_S, const double* lam_A, const double* Lambda,
+                               int d_in, int d_out, int m, double damping_rel, eogp_plan** out) {
+  clear_error();
+  if (!out) return set_error(EOGP_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (d_in < 1 || d_out < 1) return set_error(EOGP_EINVAL, "d_in and d_out must be >= 1");
+  const long long d = static_cast<long long>(d_in) * d_out;
+  if (d > 0xFFFFFFFFLL) return set_error(EOGP_EUNSUPPORTED, "d_in * d_out must be < 2^32");
+  if (m < 1 || m > d) return set_error(EOGP_EINVAL, "m must be in [1, d_in*d_out]");
+  if (!(damping_rel >= 0.0) || !std::isfinite(damping_rel))
+    return set_error(EOGP_EINVAL, "damping_rel must be finite and >= 0");
+  const bool product = (lam_S != nullptr) || (lam_A != nullptr);
+  if (product && Lambda) return set_error(EOGP_EINVAL, "give either (lam_S, lam_A) or Lambda");
+  if (product && (!lam_S || !lam_A)) return set_error(EOGP_EINVAL, "both lam_S and lam_A are required");
+  if (!product && !Lambda) return set_error(EOGP_EINVAL, "no eigenvalues given");
+  // A plan made where no CUDA device is visible keeps only its host tables
+  // (device = -1); eogp_compress_layer rejects it.
+  int dev = -1, ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev == 0) {
+    cudaGetLastError();
+    dev = -1;
+  } else {
+    CUDA_TRY(cudaGetDevice(&dev));
+  }
+
+  // Eigenvalue of Kronecker position p = i*d_out + j (basis vector Q_A[:,i] (x) Q_S[:,j]).
+  auto val = [&](uint32_t p) -> double {
+    const uint32_t i = p / static_cast<uint32_t>(d_out), j = p % static_cast<uint32_t>(d_out);
+    return product ? lam_S[j] * lam_A[i] : Lambda[static_cast<size_t>(j) * d_in + i];
+  };
+  // Validate and form the damping lambda = rel * tr(Lambda) / d (Eq. app_module_damping).
+  double tr = 0.0;
+  if (product) {
+    for (int j = 0; j < d_out; ++j)
+      if (!std::isfinite(lam_S[j]) || lam_S[j] < 0) return set_error(EOGP_EINVAL, "lam_S must be finite, >= 0");
+    for (int i = 0; i < d_in; ++i)
+      if (!std::isfinite(lam_A[i]) || lam_A[i] < 0) return set_error(EOGP_EINVAL, "lam_A must be finite, >= 0");
+  }
+  for (long long p = 0; p < d; ++p) {
+    const double v = val(static_cast<uint32_t>(p));
+    if (!std::isfinite(v) || v < 0) return set_error(EOGP_EINVAL, "eigenvalues must be finite and >= 0");
+    tr += v;
+  }
+  auto* P = new eogp_plan();
+  P->d_in = d_in;
+  P->d_out = d_out;
+  P->m = m;
+  P->device = dev;
+  P->lambda = damping_rel * tr / static_cast<double>(d);
+
+  // Top-m selection: value descending, Kronecker position ascending on ties.
+  std::vector<uint32_t> pos(static_cast<size_t>(d));
+  std::iota(pos.begin(), pos.end(), 0u);
+  auto before = [&](uint32_t a, uint32_t b) {
+    const double va = val(a), vb = val(b);
+    if (va != vb) return va > vb;
+    return a < b;
+  };
+  if (m < d) std::nth_element(pos.begin(), pos.begin() + m, pos.end(), before);
+  std::sort(pos.begin(), pos.begin() + m, before);
+  pos.resize(m);
+
+  P->j.resize(m);
+  P->i.resize(m);
+  P->scale.resize(m);
+  std::vector<int32_t> rowmap(d_out, -1), colmap(d_in, -1);
+  for (int r = 0; r < m; ++r) {
+    P->i[r] = static_cast<int32_t>(pos[r] / d_out);
+    P->j[r] = static_cast<int32_t>(pos[r] % d_out);
+    P->scale[r] = static_cast<float>(1.0 / std::sqrt(val(pos[r]) + P->lambda));
+    rowmap[P->j[r]] = 1;
+    colmap[P->i[r]] = 1;
+  }
+  for (int j = 0; j < d_out; ++j)
+    if (rowmap[j] >= 0) {
+      rowmap[j] = static_cast<int32_t>(P->R.size());
+      P->R.push_back(j);
+    }
+  for (int i = 0; i < d_in; ++i)
+    if (colmap[i] >= 0) {
+      colmap[i] = static_cast<int32_t>(P->C.size());
+      P->C.push_back(i);
+    }
+  P->posR.resize(m);
+  P->posC.resize(m);
+  for (int r = 0; r < m; ++r) {
+    P->posR[r] = rowmap[P->j[r]];
+    P->posC[r] = colmap[P->i[r]];
+  }
+  // Active 128 x 128 tiles; entries grouped per tile, canonical order inside.
+  std::vector<int> order(m);
+  std::iota(order.begin(), order.end(), 0);
+  auto tkey = [&](int r) { return (static_cast<int64_t>(P->posR[r] / 128) << 32) | (P->posC[r] / 128); };
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return tkey(a) < tkey(b); });
+  int64_t last = -1;
+  for (int e = 0; e < m; ++e) {
+    const int r = order[e];
+    const int64_t k = tkey(r);
+    if (k != last) {
+      P->tile_rc.push_back(static_cast<int32_t>(((P->posR[r] / 128) << 16) | (P->posC[r] / 128)));
+      P->tile_start.push_back(e);
+      last = k;
+    }
+    P->ent_r.push_back(r);
+    P->ent_off.push_back(((P->posR[r] % 128) << 8) | (P->posC[r] % 128));
+    P->ent_scale.push_back(P->scale[r]);
+  }
+  P->tile_start.push_back(m);
+  if (P->nR() / 128 >= 32768 || P->nC() / 128 >= 65536) {
+    delete P;
+    return set_error(EOGP_EUNSUPPORTED, "retained block too large");
+  }
+
+  int rc = EOGP_OK;
+  if (dev >= 0 && ((rc = upload(&P->d_tile_rc, P->tile_rc)) || (rc = upload(&P->d_tile_start, P->tile_start)) ||
+      (rc = upload(&P->d_ent_r, P->ent_r)) || (rc = upload(&P->d_ent_off, P->ent_off)) ||
+      (rc = upload(&P->d_ent_scale, P->ent_scale)) || (rc = upload(&P->d_posR, P->posR)) ||
+      (rc = upload(&P->d_posC, P->posC)) || (rc = upload(&P->d_scale, P->scale)) ||
+      (rc = upload(&P->d_R, P->R)) || (rc = upload(&P->d_C, P->C)))) {
+    plan_free_device(P);
+    delete P;
+    return rc;
+  }
+  *out = P;
+  return EOGP_OK;
+}
+
+extern "C" void eogp_plan_destroy(eogp_plan* plan) {
+  if (!plan) return;
+  if (plan->device >= 0) {
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (plan->device != cur) cudaSetDevice(plan->device);
+    plan_free_device(plan);
+    if (cur >= 0 && plan->device != cur) cudaSetDevice(cur);
+  }
+  delete plan;
+}
+
+extern "C" int eogp_plan_get_info(const eogp_plan* plan, eogp_plan_info* info) {
+  clear_error();
+  if (!plan || !info) return set_error(EOGP_EINVAL, "NULL argument");
+  info->d_in = plan->d_in;
+  info->d_out = plan->d_out;
+  info->m = plan->m;
+  info->nR = plan->nR();
+  info->nC = plan->nC();
+  info->n_tiles = plan->n_tiles();
+  info->lambda = plan->lambda;
+  return EOGP_OK;
+}
+
+extern "C" int eogp_plan_get_retained(const eogp_plan* plan, int32_t* j, int32_t* i, float* scale) {
+  clear_error();
+  if (!plan) return set_error(EOGP_EINVAL, "NULL plan");
+  if (j) std::memcpy(j, plan->j.data(), plan->j.size() * sizeof(int32_t));
+  if (i) std::memcpy(i, plan->i.data(), plan->i.size() * sizeof(int32_t));
+  if (scale) std::memcpy(scale, plan->scale.data(), plan->scale.size() * sizeof(float));
+  return EOGP_OK;
+}
+
+extern "C" int eogp_plan_get_sets(const eogp_plan* plan, int32_t* R, int32_t* C) {
+  clear_error();
+  if (!plan) return set_error(EOGP_EINVAL, "NULL plan");
+  if (R) std::memcpy(R, plan->R.data(), plan->R.size() * sizeof(int32_t));
+  if (C) std::memcpy(C, plan->C.data(), plan->C.size() * sizeof(int32_t));
+  return EOGP_OK;
+}
+
+static int check_device(const eogp_plan* plan) {
+  if (plan->device < 0) return set_error(EOGP_EINVAL, "plan was built without a CUDA device");
+  int dev = 0;
+  CUDA_TRY(cudaGetDevice(&dev));
+  if (dev != plan->device) return set_error(EOGP_EINVAL, "plan belongs to device %d, current is %d", plan->device, dev);
+  return EOGP_OK;
+}
+
+extern "C" int eogp_plan_gather_rows(const eogp_plan* plan, int which, int dtype, const void* V_full,
+                                     int ld_full, void* V_ret, eogp_stream_t stream) {
+  clear_error();
+  if (!plan || !V_full || !V_ret) return set_error(EOGP_EINVAL, "NULL argument");
+  if (which != 0 && which != 1) return set_error(EOGP_EINVAL, "which must be 0 (A) or 1 (S)");
+  if (dtype != EOGP_F32 && dtype != EOGP_BF16) return set_error(EOGP_EINVAL, "bad dtype");
+  const int d = which == 0 ? plan->d_in : plan->d_out;
+  if (ld_full < d) return set_error(EOGP_EINVAL, "ld_full < row length");
+  if (int rc = check_device(plan)) return rc;
+  const int n = which == 0 ? plan->nC() : plan->nR();
+  const int32_t* idx = which == 0 ? plan->d_C : plan->d_R;
+  CUDA_TRY(launch_gather_rows(V_full, ld_full, dtype == EOGP_F32 ? 4 : 2, idx, n, d, V_ret,
+                              reinterpret_cast<cudaStream_t>(stream)));
+  return EOGP_OK;
+}
+
+// ============================================================ compression
+
+namespace {
+
+struct Layout {
+  // bf16 path
+  int ldA = 0, ldS = 0, ldzb = 0, ldp = 0, splits = 1;
+  size_t at_hi = 0, at_lo = 0, st_hi = 0, st_lo = 0, zhi = 0, zlo = 0, part = 0;
+  // f32 path
+  size_t at = 0, st = 0, z = 0, x = 0;
+  size_t total = 0;
+};
+
+TcGemmCfg rot_cfg() { return TcGemmCfg{128, 4}; }
+TcGemmCfg proj_cfg() { return TcGemmCfg{128, 4}; }
+constexpr int kContractStages = 3;
+
+int proj_splits(int B, int k, int m) {
+  const int tiles = ((B + 127) / 128) * ((k + proj_cfg().BN - 1) / proj_cfg().BN);
+  const int nkb = (m + 63) / 64;
+  int want = (2 * sm_count() + tiles - 1) / tiles;
+  want = std::min(want, std::max(1, nkb / 4));
+  return tc_gemm_splits_used(m, std::max(1, want));
+}
+
+int make_layout(const eogp_layer_desc* L, int B, int mode, Layout* o) {
+  const eogp_plan* P = L->plan;
+  const size_t M = static_cast<size_t>(B) * L->T;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off += al256(bytes);
+    return at;
+  };
+  if (L->dtype == EOGP_BF16) {
+    o->ldA = round_up(std::max(1, P->nC()), 128);
+    o->ldS = round_up(std::max(1, P->nR()), 128);
+    o->at_hi = take(M * o->ldA * 2);
+    o->at_lo = take(M * o->ldA * 2);
+    o->st_hi = take(M * o->ldS * 2);
+    o->st_lo = take(M * o->ldS * 2);
+    if (mode != EOGP_OUT_FIRST_STAGE) {
+      o->ldzb = round_up(L->m, 64);
+      o->zhi = take(static_cast<size_t>(B) * o->ldzb * 2);
+      o->zlo = take(static_cast<size_t>(B) * o->ldzb * 2);
+      o->ldp = round_up(L->k, 16);
+      o->splits = proj_splits(B, L->k, L->m);
+      o->part = take(static_cast<size_t>(o->splits) * B * o->ldp * 4);
+    }
+  } else {
+    o->at = take(M * P->nC() * 4);
+    o->st = take(M * P->nR() * 4);
+    if (mode != EOGP_OUT_FIRST_STAGE) o->z = take(static_cast<size_t>(B) * L->m * 4);
+    if (mode == EOGP_OUT_CODES) o->x = take(static_cast<size_t>(B) * L->k * 4);
+  }
+  o->total = std::max<size_t>(off, 256);
+  return EOGP_OK;
+}
+
+int check_desc(const eogp_layer_desc* L, int B, int mode) {
+  if (!L) return set_error(EOGP_EINVAL, "descriptor is NULL");
+  if (!L->plan) return set_error(EOGP_EINVAL, "descriptor has no plan");
+  const eogp_plan* P = L->plan;
+  if (L->d_in != P->d_in || L->d_out != P->d_out || L->m != P->m)
+    return set_error(EOGP_EINVAL, "descriptor shape (%d, %d, m=%d) differs from the plan (%d, %d, m=%d)",
+                     L->d_in, L->d_out, L->m, P->d_in, P->d_out, P->m);
+  if (L->T < 1) return set_error(EOGP_EINVAL, "T must be >= 1");
+  if (B < 0) return set_error(EOGP_EINVAL, "B must be >= 0");
+  if (mode < EOGP_OUT_FIRST_STAGE || mode > EOGP_OUT_CODES) return set_error(EOGP_EINVAL, "bad out_mode");
+  if (L->dtype != EOGP_F32 && L->dtype != EOGP_BF16) return set_error(EOGP_EINVAL, "bad dtype");
+  if (mode != EOGP_OUT_FIRST_STAGE) {
+    if (L->k < 1 || L->k > L->m) return set_error(EOGP_EINVAL, "k must be in [1, m]");
+    if (!L->Pt) return set_error(EOGP_EINVAL, "Pt is NULL");
+  }
+  if (!L->VA || !L->VS) return set_error(EOGP_EINVAL, "VA / VS is NULL");
+  if (L->dtype == EOGP_BF16) {
+    if (L->d_in % 8 || L->d_out % 8 || L->m % 8)
+      return set_error(EOGP_EUNSUPPORTED, "bf16 path needs d_in, d_out, m multiples of 8");
+    if (!aligned16(L->VA) || !aligned16(L->VS) || (L->Pt && !aligned16(L->Pt)))
+      return set_error(EOGP_EINVAL, "bf16 operands must be 16-byte aligned");
+    if (static_cast<long long>(B) * L->T > 0x7FFFFFFFLL) return set_error(EOGP_EUNSUPPORTED, "B*T too large");
+  }
+  return EOGP_OK;
+}
+
+}  // namespace
+
+extern "C" int eogp_compress_workspace_size(const eogp_layer_desc* L, int B, int out_mode, size_t* bytes) {
+  clear_error();
+  if (!bytes) return set_error(EOGP_EINVAL, "bytes is NULL");
+  if (int rc = check_desc(L, B, out_mode)) return rc;
+  Layout lo;
+  make_layout(L, B, out_mode, &lo);
+  *bytes = lo.total;
+  return EOGP_OK;
+}
+
+extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, const void* s, int B,
+                                   int out_mode, float* out, int ld_out, uint32_t* codes,
+                                   int ld_codes, float* scales, int ld_scales, void* ws,
+                                   size_t ws_bytes, eogp_stream_t stream) {
+  clear_error();
+  if (int rc = check_desc(L, B, out_mode)) return rc;
+  if (B == 0) return EOGP_OK;
+  if (!a || !s) return set_error(EOGP_EINVAL, "a / s is NULL");
+  if (out_mode == EOGP_OUT_CODES) {
+    if (!codes || !scales) return set_error(EOGP_EINVAL, "codes / scales is NULL");
+    if (ld_codes < (L->k + 31) / 32 || ld_scales < 1) return set_error(EOGP_EINVAL, "ld_codes / ld_scales too small");
+  } else {
+    if (!out) return set_error(EOGP_EINVAL, "out is NULL");
+    const int need = out_mode == EOGP_OUT_FIRST_STAGE ? L->m : L->k;
+    if (ld_out < need) return set_error(EOGP_EINVAL, "ld_out too small");
+  }
+  if (int rc = check_device(L->plan)) return rc;
+  Layout lo;
+  make_layout(L, B, out_mode, &lo);
+  if (!ws || ws_bytes < lo.total)
+    return set_error(EOGP_EWORKSPACE, "workspace of %zu bytes needed, %zu given", lo.total, ws_bytes);
+  if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
+  const eogp_plan* P = L->plan;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  unsigned* status = status_word();
+  if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
+  char* w = static_cast<char*>(ws);
+  const int M = B * L->T;
+
+  if (L->dtype == EOGP_BF16) {
+    if (!aligned16(a) || !aligned16(s)) return set_error(EOGP_EINVAL, "a / s must be 16-byte aligned");
+    void* at_hi = w + lo.at_hi;
+    void* at_lo = w + lo.at_lo;
+    void* st_hi = w + lo.st_hi;
+    void* st_lo = w + lo.st_lo;
+    // Kronecker rotations restricted to the retained columns C / rows R (Sec. 2.2).
+    {
+      ProfScope ps(EOGP_K_ROTATE, st);
+      CUDA_TRY(launch_tc_gemm(M, lo.ldA, L->d_in, a, nullptr, L->d_in, L->VA, L->d_in, P->nC(), 1,
+                              0, at_hi, at_lo, lo.ldA, 0, rot_cfg(), status, st));
+    }
+    {
+      ProfScope ps(EOGP_K_ROTATE, st);
+      CUDA_TRY(launch_tc_gemm(M, lo.ldS, L->d_out, s, nullptr, L->d_out, L->VS, L->d_out, P->nR(),
+                              1, 0, st_hi, st_lo, lo.ldS, 0, rot_cfg(), status, st));
+    }
+    // Per-example contraction over tokens + scale/gather into z (Eq. first_stage).
+    const bool fs = out_mode == EOGP_OUT_FIRST_STAGE;
+    {
+      ProfScope ps(EOGP_K_CONTRACT, st);
+      CUDA_TRY(launch_tc_contract(st_hi, st_lo, lo.ldS, at_hi, at_lo, lo.ldA, B, L->T, P,
+                                  fs ? out : nullptr, ld_out, fs ? nullptr : w + lo.zhi,
+                                  fs ? nullptr : w + lo.zlo, lo.ldzb, kContractStages, status, st));
+    }
+    if (fs) return EOGP_OK;
+    // x = P^T z (Eq. second_stage), split over K; then sum + sign/pack (Eq. onebit).
+    float* part = reinterpret_cast<float*>(w + lo.part);
+    const size_t slab = static_cast<size_t>(B) * lo.ldp;
+    {
+      ProfScope ps(EOGP_K_PROJECT, st);
+      CUDA_TRY(launch_tc_gemm(B, L->k, L->m, w + lo.zhi, w + lo.zlo, lo.ldzb, L->Pt, L->m, L->k,
+                              lo.splits, 1, part, nullptr, lo.ldp, slab, proj_cfg(), status, st));
+    }
+    ProfScope ps(EOGP_K_PACK, st);
+    if (out_mode == EOGP_OUT_COORDS)
+      CUDA_TRY(launch_pack(part, lo.splits, slab, lo.ldp, B, L->k, out, ld_out, nullptr, 0, nullptr,
+                           0, status, st));
+    else
+      CUDA_TRY(launch_pack(part, lo.splits, slab, lo.ldp, B, L->k, nullptr, 0, codes, ld_codes,
+                           scales, ld_scales, status, st));
+    return EOGP_OK;
+  }
+
+  // fp32 CUDA-core path.
+  ProfScope ps(EOGP_K_SIMT, st);
+  const float* af = static_cast<const float*>(a);
+  const float* sf = static_cast<const float*>(s);
+  float* at = reinterpret_cast<float*>(w + lo.at);
+  float* stt = reinterpret_cast<float*>(w + lo.st);
+  const int nC = P->nC(), nR = P->nR();
+  CUDA_TRY(launch_simt_gemm(M, nC, L->d_in, 1.f, af, L->d_in, 1, static_cast<const float*>(L->VA),
+                            L->d_in, 1, at, nC, st));
+  CUDA_TRY(launch_simt_gemm(M, nR, L->d_out, 1.f, sf, L->d_out, 1, static_cast<const float*>(L->VS),
+                            L->d_out, 1, stt, nR, st));
+  float* z = out_mode == EOGP_OUT_FIRST_STAGE ? out : reinterpret_cast<float*>(w + lo.z);
+  const int ldz = out_mode == EOGP_OUT_FIRST_STAGE ? ld_out : L->m;
+  CUDA_TRY(launch_contract_f32(at, nC, stt, nR, B, L->T, L->m, P->d_posR, P->d_posC, P->d_scale, z,
+                               ldz, st));
+  if (out_mode == EOGP_OUT_FIRST_STAGE) return EOGP_OK;
+  float* x = out_mode == EOGP_OUT_COORDS ? out : reinterpret_cast<float*>(w + lo.x);
+  const int ldx = out_mode == EOGP_OUT_COORDS ? ld_out : L->k;
+  CUDA_TRY(launch_simt_gemm(B, L->k, L->m, 1.f, z, ldz, 1, static_cast<const float*>(L->Pt), L->m, 1,
+                            x, ldx, st));
+  if (out_mode == EOGP_OUT_CODES)
+    CUDA_TRY(launch_pack(x, 1, 0, ldx, B, L->k, nullptr, 0, codes, ld_codes, scales, ld_scales,
+                         status, st));
+  return EOGP_OK;
+}
+
+// ================================================================ fit PCA
+
+extern "C" int eogp_fit_pca_workspace_size(int n, int m, int k, size_t* bytes) {
+  clear_error();
+  if (!bytes) return set_error(EOGP_EINVAL, "bytes is NULL");
+  if (n < 1 || m < 1 || k < 1 || k > std::min(n, m)) return set_error(EOGP_EINVAL, "need 1 <= k <= min(n, m)");
+  if (std::min(n, m) > 12288) return set_error(EOGP_EUNSUPPORTED, "min(n, m) > 12288");
+  *bytes = fit_pca_ws_bytes(n, m, k);
+  return EOGP_OK;
+}
+
+extern "C" int eogp_fit_pca(const float* Z, int n, int m, int ldz, int k, void* Pt, int ld_pt,
+                            int pt_dtype, float* eig, void* ws, size_t ws_bytes, eogp_stream_t stream) {
+  clear_error();
+  size_t need = 0;
+  if (int rc = eogp_fit_pca_workspace_size(n, m, k, &need)) return rc;
+  if (!Z || !Pt || !eig) return set_error(EOGP_EINVAL, "NULL argument");
+  if (ldz < m || ld_pt < m) return set_error(EOGP_EINVAL, "ldz / ld_pt must be >= m");
+  if (pt_dtype != EOGP_F32 && pt_dtype != EOGP_BF16) return set_error(EOGP_EINVAL, "bad pt_dtype");
+  if (!ws || ws_bytes < need) return set_error(EOGP_EWORKSPACE, "workspace of %zu bytes needed", need);
+  if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
+  const int nn = std::min(n, m);
+  char* w = static_cast<char*>(ws);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    char* p = w + off;
+    off += al256(bytes);
+    return p;
+  };
+  PcaWs pw;
+  pw.A = reinterpret_cast<double*>(take(static_cast<size_t>(nn) * nn * 8));
+  pw.Vt = reinterpret_cast<double*>(take(static_cast<size_t>(nn) * nn * 8));
+  pw.cs = reinterpret_cast<double*>(take((static_cast<size_t>(nn) / 2 + 1) * 2 * 8));
+  pw.mu = reinterpret_cast<double*>(take(static_cast<size_t>(nn) * 8));
+  pw.sel = reinterpret_cast<int*>(take(static_cast<size_t>(k) * 4));
+  pw.red = reinterpret_cast<double*>(take(4 * 8));
+  pw.Pr = n < m ? reinterpret_cast<double*>(take(static_cast<size_t>(k) * m * 8)) : nullptr;
+  return fit_pca_device(Z, n, m, ldz, k, Pt, ld_pt, pt_dtype, eig, pw, status_word(),
+                        reinterpret_cast<cudaStream_t>(stream));
+}
+
+// ============================================================== pack, score
+
+extern "C" int eogp_pack_sign(const float* x, int B, int k, int ldx, uint32_t* codes, int ld_codes,
+                              float* scales, int ld_scales, eogp_stream_t stream) {
+  clear_error();
+  if (B < 0 || k < 1) return set_error(EOGP_EINVAL, "need B >= 0, k >= 1");
+  if (B == 0) return EOGP_OK;
+  if (!x || !codes || !scales) return set_error(EOGP_EINVAL, "NULL argument");
+  if (ldx < k || ld_codes < (k + 31) / 32 || ld_scales < 1) return set_error(EOGP_EINVAL, "leading dimension too small");
+  unsigned* status = status_word();
+  if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
+  ProfScope ps(EOGP_K_PACK, reinterpret_cast<cudaStream_t>(stream));
+  CUDA_TRY(launch_pack(x, 1, 0, ldx, B, k, nullptr, 0, codes, ld_codes, scales, ld_scales, status,
+                       reinterpret_cast<cudaStream_t>(stream)));
+  return EOGP_OK;
+}
+
+extern "C" int eogp_score_workspace_size(int N, const int* k_per_module, int U, int mode, int Q,
+                                         size_t* bytes) {
+  clear_error();
+  if (!bytes) return set_error(EOGP_EINVAL, "bytes is NULL");
+  (void)N;
+  (void)k_per_module;
+  (void)U;
+  (void)mode;
+  (void)Q;
+  *bytes = 0;
+  return EOGP_OK;
+}
+
+extern "C" int eogp_score(const void* train, int ld_train, const float* train_scales, int ld_tscale,
+                          int N, const int* k_per_module, int U, int mode, const void* query,
+                          int ld_query, const float* query_scales, int ld_qscale, int Q,
+                          float* scores, int ld_scores, void* ws, size_t ws_bytes,
+                          eogp_stream_t stream) {
+  clear_error();
+  (void)ws;
+  (void)ws_bytes;
+  if (N < 0 || Q < 0) return set_error(EOGP_EINVAL, "N, Q must be >= 0");
+  if (!k_per_module || U < 1 || U > 1024) return set_error(EOGP_EINVAL, "need 1 <= U <= 1024 modules");
+  long long W = 0, D = 0;
+  for (int u = 0; u < U; ++u) {
+    if (k_per_module[u] < 1) return set_error(EOGP_EINVAL, "k_per_module must be >= 1");
+    W += (k_per_module[u] + 31) / 32;
+    D += k_per_module[u];
+  }
+  if (N == 0 || Q == 0) return EOGP_OK;
+  if (!train || !query || !scores) return set_error(EOGP_EINVAL, "NULL argument");
+  if (ld_scores < N) return set_error(EOGP_EINVAL, "ld_scores < N");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  ProfScope ps(EOGP_K_SCORE, st);
+  if (mode == EOGP_SCORE_CODES) {
+    if (!train_scales || !query_scales) return set_error(EOGP_EINVAL, "scales are NULL");
+    if (ld_train < W || ld_query < W || ld_tscale < U || ld_qscale < U)
+      return set_error(EOGP_EINVAL, "leading dimension too small");
+    CUDA_TRY(launch_score_codes(static_cast<const uint32_t*>(train), ld_train, train_scales, ld_tscale,
+                                N, k_per_module, U, static_cast<const uint32_t*>(query), ld_query,
+                                query_scales, ld_qscale, Q, scores, ld_scores, st));
+  } else if (mode == EOGP_SCORE_PAPER) {
+    if (!train_scales) return set_error(EOGP_EINVAL, "train_scales is NULL");
+    if (ld_train < W || ld_query < D || ld_tscale < U) return set_error(EOGP_EINVAL, "leading dimension too small");
+    CUDA_TRY(launch_score_paper(static_cast<const uint32_t*>(train), ld_train, train_scales, ld_tscale,
+                                N, k_per_module, U, static_cast<const float*>(query), ld_query, Q,
+                                scores, ld_scores, st));
+  } else if (mode == EOGP_SCORE_FP) {
+    if (ld_train < D || ld_query < D) return set_error(EOGP_EINVAL, "leading dimension too small");
+    CUDA_TRY(launch_simt_gemm(Q, N, static_cast<int>(D), 1.f, static_cast<const float*>(query), ld_query,
+                              1, static_cast<const float*>(train), ld_train, 1, scores, ld_scores, st));
+  } else {
+    return set_error(EOGP_EINVAL, "bad score mode");
+  }
+  return EOGP_OK;
+}

@@ -1,0 +1,124 @@
+// Host-side internals shared by the library's translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include <vector>
+
+#include "../../include/eogp.h"
+
+namespace eogp {
+
+// Records a thread-local error message and returns `code`.
+int set_error(int code, const char* fmt, ...);
+// Clears the thread-local message.
+void clear_error();
+
+// Address of the device status word on the current device (nullptr on failure).
+unsigned* status_word();
+
+// Encodes a tiled TMA descriptor (driver entry point resolved once).
+// dims/strides: innermost first; strides in bytes for dims 1..rank-1.
+int make_tmap(CUtensorMap* tm, CUtensorMapDataType dt, int rank, const void* base,
+              const uint64_t* dims, const uint64_t* strides_bytes, const uint32_t* box,
+              CUtensorMapSwizzle swz);
+
+}  // namespace eogp
+
+// Retained-set plan.
+struct eogp_plan {
+  int d_in = 0, d_out = 0, m = 0;
+  double lambda = 0.0;
+  int device = -1;
+  std::vector<int32_t> j, i;        // canonical order
+  std::vector<float> scale;         // (Lambda + lambda)^{-1/2}, fp32
+  std::vector<int32_t> R, C;        // distinct rows / columns, ascending
+  std::vector<int32_t> posR, posC;  // per retained r: index of j_r in R, of i_r in C
+  // Active 128x128 tiles of the R x C block, CSR over entries.
+  std::vector<int32_t> tile_rc;     // (rt << 16) | ct
+  std::vector<int32_t> tile_start;  // n_tiles + 1
+  std::vector<int32_t> ent_r;       // retained index r
+  std::vector<int32_t> ent_off;     // (ro << 8) | co inside the tile
+  std::vector<float> ent_scale;
+  // Device copies (owned).
+  int32_t* d_tile_rc = nullptr;
+  int32_t* d_tile_start = nullptr;
+  int32_t* d_ent_r = nullptr;
+  int32_t* d_ent_off = nullptr;
+  float* d_ent_scale = nullptr;
+  int32_t* d_posR = nullptr;
+  int32_t* d_posC = nullptr;
+  float* d_scale = nullptr;
+  int32_t* d_R = nullptr;
+  int32_t* d_C = nullptr;
+  int nR() const { return static_cast<int>(R.size()); }
+  int nC() const { return static_cast<int>(C.size()); }
+  int n_tiles() const { return static_cast<int>(tile_rc.size()); }
+};
+
+// ---------------------------------------------------------------- launchers
+// All return cudaError_t of the launch.
+
+// k_pack.cu: x (sum of `splits` partial slabs, slab stride `slab`) -> optional x
+// copy, sign codes and scales. One warp per row.
+cudaError_t launch_pack(const float* part, int splits, size_t slab, int ldp, int B, int k,
+                        float* x_out, int ldx, uint32_t* codes, int ld_codes, float* scales,
+                        int ld_scales, unsigned* status, cudaStream_t st);
+
+// k_score.cu
+cudaError_t launch_score_codes(const uint32_t* train, int ldt, const float* ts, int ldts, int N,
+                               const int* ks, int U, const uint32_t* query, int ldq,
+                               const float* qs, int ldqs, int Q, float* out, int ldo,
+                               cudaStream_t st);
+cudaError_t launch_score_paper(const uint32_t* train, int ldt, const float* ts, int ldts, int N,
+                               const int* ks, int U, const float* y, int ldy, int Q, float* out,
+                               int ldo, cudaStream_t st);
+
+// k_simt.cu: C[i][j] = alpha * sum_k A(i,k) B(j,k), A(i,k) = A[i*sai + k*sak], etc.
+cudaError_t launch_simt_gemm(int M, int N, int K, float alpha, const float* A, long long sai,
+                             long long sak, const float* Bm, long long sbj, long long sbk,
+                             float* C, long long ldc, cudaStream_t st);
+// z[b*ldz + r] = scale[r] * sum_t St[(b*T+t)*ldS + posR[r]] * At[(b*T+t)*ldA + posC[r]]
+cudaError_t launch_contract_f32(const float* At, int ldA, const float* St, int ldS, int B, int T,
+                                int m, const int32_t* posR, const int32_t* posC,
+                                const float* scale, float* z, int ldz, cudaStream_t st);
+cudaError_t launch_gather_rows(const void* src, int ld_src, int elem_bytes, const int32_t* idx,
+                               int n_rows, int row_len, void* dst, cudaStream_t st);
+
+// k_tc.cu: tcgen05 kernels (bf16).
+struct TcGemmCfg {
+  int BN;      // N tile, multiple of 16, <= 256
+  int stages;  // smem pipeline depth
+};
+// D[M x N] = sum_a X_a[M x K] * W[N x K]^T (X_a, W bf16 K-major; W has Wrows
+// real rows, rows beyond read as zero). epi 0: out0 = bf16 hi, out1 = bf16 lo
+// of D, row stride ldo, columns < ldo written; epi 1: out0 = fp32 partial slab
+// per K split (slab elements apart), columns < N written.
+cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, int ldx,
+                           const void* W, int ldw, int Wrows, int splits, int epi, void* out0,
+                           void* out1, int ldo, size_t slab, TcGemmCfg cfg, unsigned* status,
+                           cudaStream_t st);
+// Number of K splits launch_tc_gemm actually uses for a requested count.
+int tc_gemm_splits_used(int K, int splits);
+// Per-example tile-sparse contraction over tokens with the scale-and-gather epilogue.
+cudaError_t launch_tc_contract(const void* St_hi, const void* St_lo, int ldS, const void* At_hi,
+                               const void* At_lo, int ldA, int B, int T, const eogp_plan* plan,
+                               float* z, int ldz, void* zhi, void* zlo, int ldzb, int stages,
+                               unsigned* status, cudaStream_t st);
+
+// k_pca.cu
+struct PcaWs {
+  double* A;     // [n' x n'] symmetric matrix, diagonalised in place
+  double* Vt;    // [n' x n'] eigenvectors as rows
+  double* cs;    // [n'/2+1][2] rotation (c, s)
+  double* mu;    // [n']
+  int* sel;      // [k]
+  double* red;   // [4] reduction scratch
+  double* Pr;    // [k x m] raw directions (Gram route)
+};
+int fit_pca_device(const float* Z, int n, int m, int ldz, int k, void* Pt, int ld_pt, int pt_dtype,
+                   float* eig, PcaWs ws, unsigned* status, cudaStream_t st);
+size_t fit_pca_ws_bytes(int n, int m, int k);

@@ -1,0 +1,104 @@
+// One-bit encoding (Sec. 3.3, Eq. onebit): per row x in R^k, sign bits packed
+// LSB-first into 32-bit words (bit c % 32 of word c / 32 is [x_c >= 0]; the
+// per-module byte packing of App. E.1 read as little-endian words) and the
+// scale ||x||_1 / k. The same kernel finalises the split-K projection: x is
+// the fixed-order sum of `splits` partial slabs.
+//
+// One warp per row. Full 128-column chunks use float4 loads: each lane holds 4
+// columns, forms a 4-bit nibble, and 8 lanes OR their nibbles into one word.
+// The remainder uses one column per lane and a warp ballot. The |x| sum is
+// accumulated per lane in column order, then reduced by a fixed butterfly, so
+// the scale is bitwise reproducible run to run. HBM-bound: it reads 4k bytes
+// per row (times `splits`) and writes k/8 + 4.
+#include "eogp_dev.cuh"
+#include "eogp_internal.h"
+
+namespace {
+
+__device__ __forceinline__ float4 ld_stream4(const float* p) {
+  return __ldcs(reinterpret_cast<const float4*>(p));
+}
+
+__global__ void __launch_bounds__(256) k_pack(const float* __restrict__ part, int splits,
+                                               size_t slab, int ldp, int B, int k,
+                                               float* __restrict__ x_out, int ldx,
+                                               uint32_t* __restrict__ codes, int ld_codes,
+                                               float* __restrict__ scales, int ld_scales,
+                                               unsigned* status) {
+  const int row = static_cast<int>((blockIdx.x * static_cast<unsigned>(blockDim.x) + threadIdx.x) >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= B) return;
+  const float* src = part + static_cast<size_t>(row) * ldp;
+  float* xo = x_out ? x_out + static_cast<size_t>(row) * ldx : nullptr;
+  uint32_t* co = codes ? codes + static_cast<size_t>(row) * ld_codes : nullptr;
+  float acc = 0.f;
+  bool bad = false;
+
+  const bool vec = ((ldp & 3) == 0) && ((reinterpret_cast<uintptr_t>(part) & 15) == 0) &&
+                   ((slab & 3) == 0) &&
+                   (x_out == nullptr ||
+                    (((ldx & 3) == 0) && ((reinterpret_cast<uintptr_t>(x_out) & 15) == 0)));
+  int c0 = 0;
+  if (vec) {
+    const int nfull = k >> 7;
+#pragma unroll 4
+    for (int it = 0; it < nfull; ++it) {
+      const int c = (it << 7) + (lane << 2);
+      float4 v = ld_stream4(src + c);
+      for (int s = 1; s < splits; ++s) {
+        const float4 w = ld_stream4(src + static_cast<size_t>(s) * slab + c);
+        v.x += w.x;
+        v.y += w.y;
+        v.z += w.z;
+        v.w += w.w;
+      }
+      if (xo) *reinterpret_cast<float4*>(xo + c) = v;
+      bad |= isnan(v.x) | isnan(v.y) | isnan(v.z) | isnan(v.w);
+      acc += fabsf(v.x);
+      acc += fabsf(v.y);
+      acc += fabsf(v.z);
+      acc += fabsf(v.w);
+      uint32_t nib = (v.x >= 0.f ? 1u : 0u) | (v.y >= 0.f ? 2u : 0u) | (v.z >= 0.f ? 4u : 0u) |
+                     (v.w >= 0.f ? 8u : 0u);
+      uint32_t word = nib << (4 * (lane & 7));
+      word |= __shfl_xor_sync(0xffffffffu, word, 1);
+      word |= __shfl_xor_sync(0xffffffffu, word, 2);
+      word |= __shfl_xor_sync(0xffffffffu, word, 4);
+      if (co && (lane & 7) == 0) co[(it << 2) + (lane >> 3)] = word;
+    }
+    c0 = nfull << 7;
+  }
+  for (int base = c0; base < k; base += 32) {
+    const int c = base + lane;
+    const bool in = c < k;
+    float v = 0.f;
+    if (in) {
+      v = src[c];
+      for (int s = 1; s < splits; ++s) v += src[static_cast<size_t>(s) * slab + c];
+      if (xo) xo[c] = v;
+      bad |= isnan(v);
+      acc += fabsf(v);
+    }
+    const uint32_t word = __ballot_sync(0xffffffffu, in && v >= 0.f);
+    if (co && lane == 0) co[base >> 5] = word;
+  }
+  // Fixed-order butterfly; lane 0's value is the row total.
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+  if (__any_sync(0xffffffffu, bad) && lane == 0) eogp::flag_status(status, EOGP_ST_DEVICE);
+  if (scales && lane == 0) scales[static_cast<size_t>(row) * ld_scales] = acc / static_cast<float>(k);
+}
+
+}  // namespace
+
+cudaError_t launch_pack(const float* part, int splits, size_t slab, int ldp, int B, int k,
+                        float* x_out, int ldx, uint32_t* codes, int ld_codes, float* scales,
+                        int ld_scales, unsigned* status, cudaStream_t st) {
+  if (B <= 0) return cudaSuccess;
+  const int threads = 256;
+  const long long blocks = (static_cast<long long>(B) * 32 + threads - 1) / threads;
+  k_pack<<<static_cast<unsigned>(blocks), threads, 0, st>>>(part, splits, slab, ldp, B, k, x_out,
+                                                           ldx, codes, ld_codes, scales,
+                                                           ld_scales, status);
+  return cudaGetLastError();
+}

@@ -1,0 +1,436 @@
+// tcgen05 tensor-core kernels (bf16 in, fp32 accumulate in TMEM), fed by TMA.
+//
+// k_tc_gemm -- D[M x N] = sum_a X_a[M x K] W[N x K]^T, both operands K-major.
+//   Used twice per module for the Kronecker rotations of Sec. 2.2
+//   (A~ = A V_A[C]^T over the retained columns, S~ = S V_S[R]^T over the
+//   retained rows; M = B*T tokens) and once for the second-stage projection
+//   x = P^T z (Eq. second_stage; M = B examples, N = k, K = m) where z enters as
+//   a bf16 hi + lo pair (two A operands into the same accumulator).
+//   Epilogue 0 writes D as a bf16 hi/lo pair (hi = rn(D), lo = rn(D - hi)), so
+//   the next contraction sees D to ~16 significant bits; epilogue 1 writes an
+//   fp32 partial slab per K split.
+//
+// k_tc_contract -- for example b and one active 128 x 128 tile (R block rt,
+//   C block ct) of the retained block: G~_b[tile] = sum_t S~_b[t, rows]^T
+//   A~_b[t, cols] with K = tokens, both operands MN-major (token rows).
+//   hi*hi + hi*lo + lo*hi: three MMAs per K step. The epilogue stages the fp32
+//   tile in shared memory and gathers the retained entries of the tile,
+//   scaled by (Lambda + lambda)^{-1/2} (Eq. first_stage), into z.
+//
+// Warp roles (192 threads): warp 0 issues TMA, warp 1 owns TMEM and issues
+// MMAs (one lane), warps 2-5 run the epilogue (warp w reads TMEM lanes
+// 32*(w%4)..+31). Every mbarrier wait is bounded (eogp_dev.cuh); after a
+// timeout every role falls through to the common exit, which frees TMEM.
+#include <mutex>
+
+#include "eogp_dev.cuh"
+#include "eogp_internal.h"
+
+using namespace eogp;
+
+namespace {
+
+constexpr int kThreads = 192;
+constexpr uint32_t kABytes = 128u * 64u * 2u;  // 128 rows x 64 bf16 (one 128-byte swizzle row each)
+
+struct GemmArgs {
+  int M, N, K, BN, stages, nA, kbps, epi, ldo;
+  void* out0;
+  void* out1;
+  size_t slab;
+  unsigned* status;
+};
+
+__device__ __forceinline__ uint32_t pack_bf16x2(__nv_bfloat16 a, __nv_bfloat16 b) {
+  return static_cast<uint32_t>(__bfloat16_as_ushort(a)) |
+         (static_cast<uint32_t>(__bfloat16_as_ushort(b)) << 16);
+}
+
+__device__ __forceinline__ uint32_t tmem_cols_for(int n) {
+  return n <= 32 ? 32u : n <= 64 ? 64u : n <= 128 ? 128u : 256u;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_tc_gemm(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__ CUtensorMap tmX1,
+              const __grid_constant__ CUtensorMap tmW, const GemmArgs g) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t b_bytes = static_cast<uint32_t>(g.BN) * 128u;
+  const uint32_t stage_bytes = static_cast<uint32_t>(g.nA) * kABytes + b_bytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(g.stages) * stage_bytes);
+  uint64_t* empty = full + g.stages;
+  uint64_t* done = empty + g.stages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  const uint32_t tmem_cols = tmem_cols_for(g.BN);
+
+  const int n0 = blockIdx.x * g.BN, m0 = blockIdx.y * 128;
+  const int nkb_total = (g.K + 63) / 64;
+  const int kb0 = blockIdx.z * g.kbps;
+  const int nkb = max(0, min(g.kbps, nkb_total - kb0));
+
+  if (threadIdx.x == 0) {
+    tma_prefetch_desc(&tmX0);
+    if (g.nA > 1) tma_prefetch_desc(&tmX1);
+    tma_prefetch_desc(&tmW);
+    for (int s = 0; s < g.stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(done, 1);
+    fence_barrier_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, tmem_cols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int i = 0; i < nkb; ++i) {
+        const int s = i % g.stages;
+        const uint32_t ph = static_cast<uint32_t>(i / g.stages) & 1u;
+        if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) break;
+        uint8_t* st = smem + static_cast<size_t>(s) * stage_bytes;
+        mbar_arrive_expect_tx(&full[s], stage_bytes);
+        const int kx = (kb0 + i) * 64;
+        tma_load_2d(st, &tmX0, kx, m0, &full[s]);
+        if (g.nA > 1) tma_load_2d(st + kABytes, &tmX1, kx, m0, &full[s]);
+        tma_load_2d(st + g.nA * kABytes, &tmW, kx, n0, &full[s]);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(128, g.BN, 0, 0);
+      for (int i = 0; i < nkb; ++i) {
+        const int s = i % g.stages;
+        const uint32_t ph = static_cast<uint32_t>(i / g.stages) & 1u;
+        if (!mbar_wait(&full[s], ph, g.status)) break;
+        tc_fence_after();
+        const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
+        const uint32_t sb = sa + g.nA * kABytes;
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          const uint64_t bd = sdesc_sw128(sb + kk * 32, 16, 1024);
+          for (int a = 0; a < g.nA; ++a) {
+            const uint64_t ad = sdesc_sw128(sa + a * kABytes + kk * 32, 16, 1024);
+            tc_mma_f16(tmem, ad, bd, idesc, (i | kk | a) != 0 ? 1u : 0u);
+          }
+        }
+        tc_commit(&empty[s]);
+      }
+      tc_commit(done);
+    }
+    __syncwarp();
+  } else {
+    const int q = warp & 3;
+    uint32_t ok = 1;
+    if (lane == 0) ok = mbar_wait(done, 0, g.status) ? 1u : 0u;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    __syncwarp();
+    tc_fence_after();
+    if (ok && nkb > 0) {
+      const int row = m0 + q * 32 + lane;
+      const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16);
+      if (g.epi == 0) {
+        __nv_bfloat16* hi = static_cast<__nv_bfloat16*>(g.out0);
+        __nv_bfloat16* lo = static_cast<__nv_bfloat16*>(g.out1);
+        for (int c = 0; c < g.BN; c += 16) {
+          float v[16];
+          tmem_ld16(tbase + c, v);
+          const int col = n0 + c;
+          if (row < g.M && col < g.ldo) {
+            uint32_t h[8], l[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * e]);
+              const __nv_bfloat16 h1 = __float2bfloat16_rn(v[2 * e + 1]);
+              const __nv_bfloat16 l0 = __float2bfloat16_rn(v[2 * e] - __bfloat162float(h0));
+              const __nv_bfloat16 l1 = __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1));
+              h[e] = pack_bf16x2(h0, h1);
+              l[e] = pack_bf16x2(l0, l1);
+            }
+            const size_t off = static_cast<size_t>(row) * g.ldo + col;
+            uint4* ph = reinterpret_cast<uint4*>(hi + off);
+            uint4* pl = reinterpret_cast<uint4*>(lo + off);
+            ph[0] = make_uint4(h[0], h[1], h[2], h[3]);
+            ph[1] = make_uint4(h[4], h[5], h[6], h[7]);
+            pl[0] = make_uint4(l[0], l[1], l[2], l[3]);
+            pl[1] = make_uint4(l[4], l[5], l[6], l[7]);
+          }
+        }
+      } else {
+        float* out = static_cast<float*>(g.out0) + static_cast<size_t>(blockIdx.z) * g.slab;
+        for (int c = 0; c < g.BN; c += 16) {
+          float v[16];
+          tmem_ld16(tbase + c, v);
+          const int col = n0 + c;
+          if (row < g.M && col < g.N) {
+            float* o = out + static_cast<size_t>(row) * g.ldo + col;
+            if (col + 16 <= g.N) {
+#pragma unroll
+              for (int e = 0; e < 4; ++e)
+                reinterpret_cast<float4*>(o)[e] =
+                    make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+            } else {
+              for (int e = 0; e < 16; ++e)
+                if (col + e < g.N) o[e] = v[e];
+            }
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, tmem_cols);
+}
+
+struct ContractArgs {
+  int T, stages;
+  const int32_t* tile_rc;
+  const int32_t* tile_start;
+  const int32_t* ent_r;
+  const int32_t* ent_off;
+  const float* ent_scale;
+  float* z;
+  int ldz;
+  __nv_bfloat16* zhi;
+  __nv_bfloat16* zlo;
+  int ldzb;
+  unsigned* status;
+};
+
+constexpr uint32_t kOpBytes = 16384u;          // one 128-wide operand tile, 64 tokens
+constexpr uint32_t kCStage = 4u * kOpBytes;    // S hi, S lo, A hi, A lo
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_tc_contract(const __grid_constant__ CUtensorMap tmShi, const __grid_constant__ CUtensorMap tmSlo,
+                  const __grid_constant__ CUtensorMap tmAhi, const __grid_constant__ CUtensorMap tmAlo,
+                  const ContractArgs g) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(g.stages) * kCStage);
+  uint64_t* empty = full + g.stages;
+  uint64_t* done = empty + g.stages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+
+  const int tile = blockIdx.x, b = blockIdx.y;
+  const int rc = g.tile_rc[tile];
+  const int r0 = (rc >> 16) * 128, c0 = (rc & 0xFFFF) * 128;
+  const int nkb = (g.T + 63) / 64;
+
+  if (threadIdx.x == 0) {
+    tma_prefetch_desc(&tmShi);
+    tma_prefetch_desc(&tmSlo);
+    tma_prefetch_desc(&tmAhi);
+    tma_prefetch_desc(&tmAlo);
+    for (int s = 0; s < g.stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(done, 1);
+    fence_barrier_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, 128);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int i = 0; i < nkb; ++i) {
+        const int s = i % g.stages;
+        const uint32_t ph = static_cast<uint32_t>(i / g.stages) & 1u;
+        if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) break;
+        uint8_t* st = smem + static_cast<size_t>(s) * kCStage;
+        mbar_arrive_expect_tx(&full[s], kCStage);
+        const int t0 = i * 64;
+        tma_load_3d(st + 0 * kOpBytes, &tmShi, r0, t0, b, &full[s]);
+        tma_load_3d(st + 0 * kOpBytes + 8192, &tmShi, r0 + 64, t0, b, &full[s]);
+        tma_load_3d(st + 1 * kOpBytes, &tmSlo, r0, t0, b, &full[s]);
+        tma_load_3d(st + 1 * kOpBytes + 8192, &tmSlo, r0 + 64, t0, b, &full[s]);
+        tma_load_3d(st + 2 * kOpBytes, &tmAhi, c0, t0, b, &full[s]);
+        tma_load_3d(st + 2 * kOpBytes + 8192, &tmAhi, c0 + 64, t0, b, &full[s]);
+        tma_load_3d(st + 3 * kOpBytes, &tmAlo, c0, t0, b, &full[s]);
+        tma_load_3d(st + 3 * kOpBytes + 8192, &tmAlo, c0 + 64, t0, b, &full[s]);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(128, 128, 1, 1);
+      for (int i = 0; i < nkb; ++i) {
+        const int s = i % g.stages;
+        const uint32_t ph = static_cast<uint32_t>(i / g.stages) & 1u;
+        if (!mbar_wait(&full[s], ph, g.status)) break;
+        tc_fence_after();
+        const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * kCStage);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          const uint32_t o = kk * 2048u;  // 16 token rows of 128 bytes
+          const uint64_t sh = sdesc_sw128(sa + 0 * kOpBytes + o, 8192, 1024);
+          const uint64_t sl = sdesc_sw128(sa + 1 * kOpBytes + o, 8192, 1024);
+          const uint64_t ah = sdesc_sw128(sa + 2 * kOpBytes + o, 8192, 1024);
+          const uint64_t al = sdesc_sw128(sa + 3 * kOpBytes + o, 8192, 1024);
+          tc_mma_f16(tmem, sh, ah, idesc, (i | kk) != 0 ? 1u : 0u);
+          tc_mma_f16(tmem, sh, al, idesc, 1u);
+          tc_mma_f16(tmem, sl, ah, idesc, 1u);
+        }
+        tc_commit(&empty[s]);
+      }
+      tc_commit(done);
+    }
+    __syncwarp();
+  } else {
+    const int q = warp & 3;
+    uint32_t ok = 1;
+    if (lane == 0) ok = mbar_wait(done, 0, g.status) ? 1u : 0u;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    __syncwarp();
+    tc_fence_after();
+    float* tilebuf = reinterpret_cast<float*>(smem);  // [128][129], reuses the drained stages
+    if (ok) {
+      const int row = q * 32 + lane;
+      const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16);
+      for (int c = 0; c < 128; c += 16) {
+        float v[16];
+        tmem_ld16(tbase + c, v);
+#pragma unroll
+        for (int e = 0; e < 16; ++e) tilebuf[row * 129 + c + e] = v[e];
+      }
+    }
+    named_bar_sync(1, 128);
+    if (ok) {
+      const int etid = threadIdx.x - 64;
+      const int e0 = g.tile_start[tile], e1 = g.tile_start[tile + 1];
+      for (int e = e0 + etid; e < e1; e += 128) {
+        const int r = g.ent_r[e];
+        const int off = g.ent_off[e];
+        const float val = g.ent_scale[e] * tilebuf[(off >> 8) * 129 + (off & 255)];
+        if (g.z) g.z[static_cast<size_t>(b) * g.ldz + r] = val;
+        if (g.zhi) {
+          const __nv_bfloat16 h = __float2bfloat16_rn(val);
+          g.zhi[static_cast<size_t>(b) * g.ldzb + r] = h;
+          g.zlo[static_cast<size_t>(b) * g.ldzb + r] = __float2bfloat16_rn(val - __bfloat162float(h));
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, 128);
+}
+
+size_t gemm_smem_bytes(int BN, int stages, int nA) {
+  return 1024 + static_cast<size_t>(stages) * (nA * kABytes + BN * 128u) + (2 * stages + 1) * 8 + 16;
+}
+
+size_t contract_smem_bytes(int stages) {
+  return 1024 + static_cast<size_t>(stages) * kCStage + (2 * stages + 1) * 8 + 16;
+}
+
+}  // namespace
+
+static int tmap_bf16_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t rows,
+                        uint64_t row_stride_elems, uint32_t box_inner, uint32_t box_rows) {
+  const uint64_t dims[2] = {inner, rows};
+  const uint64_t strides[1] = {row_stride_elems * 2};
+  const uint32_t box[2] = {box_inner, box_rows};
+  return make_tmap(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box,
+                   CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+static int tmap_bf16_3d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t T, uint64_t B,
+                        uint64_t ld) {
+  const uint64_t dims[3] = {inner, T, B};
+  const uint64_t strides[2] = {ld * 2, ld * 2 * T};
+  const uint32_t box[3] = {64, 64, 1};
+  return make_tmap(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box,
+                   CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, int ldx,
+                                const void* W, int ldw, int Wrows, int splits, int epi,
+                                void* out0, void* out1, int ldo, size_t slab, TcGemmCfg cfg,
+                                unsigned* status, cudaStream_t st) {
+  if (M <= 0 || N <= 0) return cudaSuccess;
+  const int nA = X1 ? 2 : 1;
+  CUtensorMap tX0, tX1, tW;
+  if (tmap_bf16_2d(&tX0, X0, static_cast<uint64_t>(K), static_cast<uint64_t>(M), ldx, 64, 128))
+    return cudaErrorInvalidValue;
+  if (nA > 1) {
+    if (tmap_bf16_2d(&tX1, X1, K, M, ldx, 64, 128)) return cudaErrorInvalidValue;
+  } else {
+    tX1 = tX0;
+  }
+  if (tmap_bf16_2d(&tW, W, K, Wrows, ldw, 64, cfg.BN)) return cudaErrorInvalidValue;
+  const int nkb = (K + 63) / 64;
+  splits = max(1, min(splits, nkb));
+  const int kbps = (nkb + splits - 1) / splits;
+  splits = (nkb + kbps - 1) / kbps;
+  GemmArgs g;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.BN = cfg.BN;
+  g.stages = cfg.stages;
+  g.nA = nA;
+  g.kbps = kbps;
+  g.epi = epi;
+  g.ldo = ldo;
+  g.out0 = out0;
+  g.out1 = out1;
+  g.slab = slab;
+  g.status = status;
+  const size_t smem = gemm_smem_bytes(cfg.BN, cfg.stages, nA);
+  cudaError_t e = cudaFuncSetAttribute(k_tc_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  dim3 grid((N + cfg.BN - 1) / cfg.BN, (M + 127) / 128, splits);
+  k_tc_gemm<<<grid, kThreads, smem, st>>>(tX0, tX1, tW, g);
+  return cudaGetLastError();
+}
+
+int tc_gemm_splits_used(int K, int splits) {
+  const int nkb = (K + 63) / 64;
+  splits = max(1, min(splits, nkb));
+  const int kbps = (nkb + splits - 1) / splits;
+  return (nkb + kbps - 1) / kbps;
+}
+
+cudaError_t launch_tc_contract(const void* St_hi, const void* St_lo, int ldS, const void* At_hi,
+                               const void* At_lo, int ldA, int B, int T, const eogp_plan* plan,
+                               float* z, int ldz, void* zhi, void* zlo, int ldzb, int stages,
+                               unsigned* status, cudaStream_t st) {
+  if (B <= 0 || plan->n_tiles() == 0) return cudaSuccess;
+  CUtensorMap tSh, tSl, tAh, tAl;
+  if (tmap_bf16_3d(&tSh, St_hi, ldS, T, B, ldS) || tmap_bf16_3d(&tSl, St_lo, ldS, T, B, ldS) ||
+      tmap_bf16_3d(&tAh, At_hi, ldA, T, B, ldA) || tmap_bf16_3d(&tAl, At_lo, ldA, T, B, ldA))
+    return cudaErrorInvalidValue;
+  ContractArgs g;
+  g.T = T;
+  g.stages = stages;
+  g.tile_rc = plan->d_tile_rc;
+  g.tile_start = plan->d_tile_start;
+  g.ent_r = plan->d_ent_r;
+  g.ent_off = plan->d_ent_off;
+  g.ent_scale = plan->d_ent_scale;
+  g.z = z;
+  g.ldz = ldz;
+  g.zhi = static_cast<__nv_bfloat16*>(zhi);
+  g.zlo = static_cast<__nv_bfloat16*>(zlo);
+  g.ldzb = ldzb;
+  g.status = status;
+  const size_t smem = contract_smem_bytes(stages);
+  cudaError_t e = cudaFuncSetAttribute(k_tc_contract, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  dim3 grid(plan->n_tiles(), B);
+  k_tc_contract<<<grid, kThreads, smem, st>>>(tSh, tSl, tAh, tAl, g);
+  return cudaGetLastError();
+}

@@ -1,0 +1,338 @@
+"""Python binding of libeogp (include/eogp.h): argument marshalling only.
+
+Every computation runs in the library's CUDA kernels; PyTorch supplies device
+memory and streams. Functions keep the C names without the ``eogp_`` prefix.
+If libeogp.so has not been built, the first call raises: there is no
+fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, c_double, c_float, c_int, c_int32, c_size_t, c_uint32, c_void_p
+from typing import Optional, Sequence, Tuple
+
+import numpy as np
+
+from . import build as _build
+
+OK, EINVAL, EUNSUPPORTED, ECUDA, ETIMEOUT, EWORKSPACE, EDEVICE = 0, -1, -2, -3, -4, -5, -6
+F32, BF16 = 0, 1
+OUT_FIRST_STAGE, OUT_COORDS, OUT_CODES = 0, 1, 2
+SCORE_CODES, SCORE_PAPER, SCORE_FP = 0, 1, 2
+K_ROTATE, K_CONTRACT, K_PROJECT, K_PACK, K_SCORE, K_SIMT = range(6)
+KERNEL_KINDS = {K_ROTATE: "rotate", K_CONTRACT: "contract", K_PROJECT: "project", K_PACK: "pack",
+                K_SCORE: "score", K_SIMT: "simt_f32"}
+
+_ERRNAMES = {EINVAL: "EINVAL", EUNSUPPORTED: "EUNSUPPORTED", ECUDA: "ECUDA",
+             ETIMEOUT: "ETIMEOUT", EWORKSPACE: "EWORKSPACE", EDEVICE: "EDEVICE"}
+
+
+class EOGPError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"{_ERRNAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+class PlanInfo(ctypes.Structure):
+    _fields_ = [("d_in", c_int), ("d_out", c_int), ("m", c_int), ("nR", c_int), ("nC", c_int),
+                ("n_tiles", c_int), ("lam", c_double)]
+
+
+class LayerDesc(ctypes.Structure):
+    _fields_ = [("d_in", c_int), ("d_out", c_int), ("T", c_int), ("m", c_int), ("k", c_int),
+                ("dtype", c_int), ("VA", c_void_p), ("VS", c_void_p), ("Pt", c_void_p),
+                ("plan", c_void_p)]
+
+
+EXPORTS = {
+    # name: (restype, argtypes)
+    "eogp_last_error": (ctypes.c_char_p, []),
+    "eogp_version": (ctypes.c_char_p, []),
+    "eogp_sync_status": (c_int, [c_void_p]),
+    "eogp_profile_enable": (c_int, [c_int]),
+    "eogp_profile_read": (c_int, [c_int, POINTER(c_int), POINTER(c_double), c_int]),
+    "eogp_plan_layer": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_double,
+                                POINTER(c_void_p)]),
+    "eogp_plan_destroy": (None, [c_void_p]),
+    "eogp_plan_get_info": (c_int, [c_void_p, POINTER(PlanInfo)]),
+    "eogp_plan_get_retained": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p]),
+    "eogp_plan_get_sets": (c_int, [c_void_p, c_void_p, c_void_p]),
+    "eogp_plan_gather_rows": (c_int, [c_void_p, c_int, c_int, c_void_p, c_int, c_void_p, c_void_p]),
+    "eogp_compress_workspace_size": (c_int, [POINTER(LayerDesc), c_int, c_int, POINTER(c_size_t)]),
+    "eogp_compress_layer": (c_int, [POINTER(LayerDesc), c_void_p, c_void_p, c_int, c_int, c_void_p,
+                                    c_int, c_void_p, c_int, c_void_p, c_int, c_void_p, c_size_t,
+                                    c_void_p]),
+    "eogp_fit_pca_workspace_size": (c_int, [c_int, c_int, c_int, POINTER(c_size_t)]),
+    "eogp_fit_pca": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int,
+                             c_void_p, c_void_p, c_size_t, c_void_p]),
+    "eogp_pack_sign": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_int, c_void_p, c_int,
+                               c_void_p]),
+    "eogp_score_workspace_size": (c_int, [c_int, c_void_p, c_int, c_int, c_int, POINTER(c_size_t)]),
+    "eogp_score": (c_int, [c_void_p, c_int, c_void_p, c_int, c_int, c_void_p, c_int, c_int,
+                           c_void_p, c_int, c_void_p, c_int, c_int, c_void_p, c_int, c_void_p,
+                           c_size_t, c_void_p]),
+}
+
+_LIB = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load libeogp.so (built in-tree by build.py). Raises if it is missing."""
+    global _LIB
+    if _LIB is None:
+        path = _build.LIB
+        if not os.path.exists(path):
+            raise RuntimeError(f"libeogp.so is not built ({path}); run "
+                               "`python -m paper_2609_37842_gb300.build` first")
+        L = ctypes.CDLL(path)
+        for name, (res, args) in EXPORTS.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _LIB = L
+    return _LIB
+
+
+def _check(rc: int):
+    if rc != OK:
+        raise EOGPError(rc, lib().eogp_last_error().decode(errors="replace"))
+
+
+def _ptr(t) -> Optional[int]:
+    if t is None:
+        return None
+    return t.data_ptr()
+
+
+def _rows(t, name: str):
+    """Require a row-major matrix view (unit inner stride); returns t."""
+    if t is not None and t.dim() >= 1 and t.numel() > 0 and t.stride(-1) != 1:
+        raise ValueError(f"{name} must have unit stride along its last dimension")
+    return t
+
+
+def _dense(t, name: str):
+    if t is not None and t.numel() > 0 and not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t
+
+
+def _stream(stream) -> Optional[int]:
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def version() -> str:
+    return lib().eogp_version().decode()
+
+
+def sync_status(stream=None) -> None:
+    _check(lib().eogp_sync_status(_stream(stream)))
+
+
+def profile_enable(on: bool) -> None:
+    _check(lib().eogp_profile_enable(1 if on else 0))
+
+
+def profile_read(kind: int, reset: bool = True) -> Tuple[int, float]:
+    """(launches, total device ms) of one kernel kind since the last reset."""
+    n = c_int()
+    ms = c_double()
+    _check(lib().eogp_profile_read(int(kind), ctypes.byref(n), ctypes.byref(ms), 1 if reset else 0))
+    return n.value, ms.value
+
+
+def _dtype_code(t) -> int:
+    import torch
+    if t.dtype == torch.bfloat16:
+        return BF16
+    if t.dtype == torch.float32:
+        return F32
+    raise ValueError(f"unsupported dtype {t.dtype}")
+
+
+# ------------------------------------------------------------------- plan
+class Plan:
+    """Retained-set plan of one module (wraps eogp_plan*)."""
+
+    def __init__(self, handle: int):
+        self._h = c_void_p(handle)
+
+    @classmethod
+    def from_factors(cls, lam_S, lam_A, m: int, damping_rel: float) -> "Plan":
+        lam_S = np.ascontiguousarray(lam_S, np.float64)
+        lam_A = np.ascontiguousarray(lam_A, np.float64)
+        h = c_void_p()
+        _check(lib().eogp_plan_layer(lam_S.ctypes.data, lam_A.ctypes.data, None, len(lam_A),
+                                     len(lam_S), int(m), float(damping_rel), ctypes.byref(h)))
+        return cls(h.value)
+
+    @classmethod
+    def from_table(cls, Lambda, m: int, damping_rel: float) -> "Plan":
+        Lam = np.ascontiguousarray(Lambda, np.float64)
+        d_out, d_in = Lam.shape
+        h = c_void_p()
+        _check(lib().eogp_plan_layer(None, None, Lam.ctypes.data, d_in, d_out, int(m),
+                                     float(damping_rel), ctypes.byref(h)))
+        return cls(h.value)
+
+    @property
+    def handle(self) -> int:
+        return self._h.value
+
+    def info(self) -> PlanInfo:
+        inf = PlanInfo()
+        _check(lib().eogp_plan_get_info(self._h, ctypes.byref(inf)))
+        return inf
+
+    def retained(self) -> Tuple[np.ndarray, np.ndarray, np.ndarray]:
+        m = self.info().m
+        j = np.empty(m, np.int32)
+        i = np.empty(m, np.int32)
+        sc = np.empty(m, np.float32)
+        _check(lib().eogp_plan_get_retained(self._h, j.ctypes.data, i.ctypes.data, sc.ctypes.data))
+        return j, i, sc
+
+    def sets(self) -> Tuple[np.ndarray, np.ndarray]:
+        inf = self.info()
+        R = np.empty(inf.nR, np.int32)
+        C = np.empty(inf.nC, np.int32)
+        _check(lib().eogp_plan_get_sets(self._h, R.ctypes.data, C.ctypes.data))
+        return R, C
+
+    def gather_rows(self, which: int, V_full, out=None, stream=None):
+        """Retained eigenvector rows: which=0 -> V_A[C] [nC, d_in], 1 -> V_S[R] [nR, d_out]."""
+        import torch
+        inf = self.info()
+        n = inf.nC if which == 0 else inf.nR
+        d = inf.d_in if which == 0 else inf.d_out
+        if out is None:
+            out = torch.empty((n, d), dtype=V_full.dtype, device=V_full.device)
+        _check(lib().eogp_plan_gather_rows(self._h, which, _dtype_code(V_full), _ptr(V_full),
+                                           V_full.stride(0), _ptr(out), _stream(stream)))
+        return out
+
+    def __del__(self):
+        if getattr(self, "_h", None) is not None and self._h.value and _LIB is not None:
+            _LIB.eogp_plan_destroy(self._h)
+            self._h = c_void_p()
+
+
+# ------------------------------------------------------------- compression
+def layer_desc(plan: Plan, T: int, k: int, VA, VS, Pt=None) -> LayerDesc:
+    """Descriptor of one module. It keeps references to the plan and tensors so
+    their device memory outlives the descriptor."""
+    inf = plan.info()
+    _dense(VA, "VA")
+    _dense(VS, "VS")
+    _dense(Pt, "Pt")
+    d = LayerDesc(inf.d_in, inf.d_out, int(T), inf.m, int(k), _dtype_code(VA), _ptr(VA),
+                  _ptr(VS), _ptr(Pt), plan.handle)
+    d._refs = (plan, VA, VS, Pt)
+    return d
+
+
+def compress_workspace_size(desc: LayerDesc, B: int, out_mode: int) -> int:
+    n = c_size_t()
+    _check(lib().eogp_compress_workspace_size(ctypes.byref(desc), int(B), int(out_mode),
+                                              ctypes.byref(n)))
+    return n.value
+
+
+def workspace(nbytes: int, device):
+    import torch
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+def compress_layer(desc: LayerDesc, a, s, out_mode: int, out=None, codes=None, scales=None,
+                   ws=None, stream=None):
+    """eogp_compress_layer on a [B, T, d_in], s [B, T, d_out]. Returns `out` (z or x) for
+    FIRST_STAGE / COORDS, (codes, scales) for CODES. Output tensors may be given
+    (strided rows: codes/scales of one module inside a wider store row)."""
+    import torch
+    _dense(a, "a")
+    _dense(s, "s")
+    _rows(out, "out")
+    _rows(codes, "codes")
+    B = a.shape[0]
+    dev = a.device
+    if ws is None:
+        ws = workspace(compress_workspace_size(desc, B, out_mode), dev)
+    if out_mode == OUT_CODES:
+        if codes is None:
+            codes = torch.empty((B, (desc.k + 31) // 32), dtype=torch.int32, device=dev)
+        if scales is None:
+            scales = torch.empty((B,), dtype=torch.float32, device=dev)
+        ld_sc = scales.stride(0)
+        _check(lib().eogp_compress_layer(ctypes.byref(desc), _ptr(a), _ptr(s), B, out_mode, None, 0,
+                                         _ptr(codes), codes.stride(0), _ptr(scales), ld_sc,
+                                         _ptr(ws), ws.numel(), _stream(stream)))
+        return codes, scales
+    width = desc.m if out_mode == OUT_FIRST_STAGE else desc.k
+    if out is None:
+        out = torch.empty((B, width), dtype=torch.float32, device=dev)
+    _check(lib().eogp_compress_layer(ctypes.byref(desc), _ptr(a), _ptr(s), B, out_mode, _ptr(out),
+                                     out.stride(0), None, 0, None, 0, _ptr(ws), ws.numel(),
+                                     _stream(stream)))
+    return out
+
+
+# ------------------------------------------------------------------ fit PCA
+def fit_pca_workspace_size(n: int, m: int, k: int) -> int:
+    v = c_size_t()
+    _check(lib().eogp_fit_pca_workspace_size(int(n), int(m), int(k), ctypes.byref(v)))
+    return v.value
+
+
+def fit_pca(Z, k: int, pt_dtype: int = F32, ws=None, stream=None):
+    """Top-k PCA directions of Z [n, m] (fp32, device): returns (Pt [k, m], eig [k])."""
+    import torch
+    _rows(Z, "Z")
+    n, m = Z.shape
+    if ws is None:
+        ws = workspace(fit_pca_workspace_size(n, m, k), Z.device)
+    Pt = torch.empty((k, m), dtype=torch.bfloat16 if pt_dtype == BF16 else torch.float32,
+                     device=Z.device)
+    eig = torch.empty((k,), dtype=torch.float32, device=Z.device)
+    _check(lib().eogp_fit_pca(_ptr(Z), n, m, Z.stride(0), int(k), _ptr(Pt), Pt.stride(0), pt_dtype,
+                              _ptr(eig), _ptr(ws), ws.numel(), _stream(stream)))
+    return Pt, eig
+
+
+# --------------------------------------------------------------- pack, score
+def pack_sign(x, codes=None, scales=None, stream=None):
+    """Sign bits and ||x||_1/k of each row of x [B, k] (fp32, device)."""
+    import torch
+    _rows(x, "x")
+    _rows(codes, "codes")
+    B, k = x.shape
+    if codes is None:
+        codes = torch.empty((B, (k + 31) // 32), dtype=torch.int32, device=x.device)
+    if scales is None:
+        scales = torch.empty((B,), dtype=torch.float32, device=x.device)
+    _check(lib().eogp_pack_sign(_ptr(x), B, k, x.stride(0), _ptr(codes), codes.stride(0),
+                                _ptr(scales), scales.stride(0), _stream(stream)))
+    return codes, scales
+
+
+def score(train, train_scales, ks: Sequence[int], mode: int, query, query_scales=None, out=None,
+          stream=None):
+    """eogp_score: returns scores [Q, N] fp32."""
+    import torch
+    for t, nm in ((train, "train"), (query, "query"), (train_scales, "train_scales"),
+                  (query_scales, "query_scales")):
+        _rows(t, nm)
+    N = train.shape[0]
+    Q = query.shape[0]
+    karr = (c_int * len(ks))(*[int(k) for k in ks])
+    if out is None:
+        out = torch.empty((Q, N), dtype=torch.float32, device=train.device)
+    ts_ld = train_scales.stride(0) if train_scales is not None else 0
+    qs_ld = query_scales.stride(0) if query_scales is not None else 0
+    _check(lib().eogp_score(_ptr(train), train.stride(0), _ptr(train_scales), ts_ld, N, karr,
+                            len(ks), int(mode), _ptr(query), query.stride(0), _ptr(query_scales),
+                            qs_ld, Q, _ptr(out), out.stride(0), None, 0, _stream(stream)))
+    return out

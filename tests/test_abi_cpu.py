@@ -1,0 +1,130 @@
+"""CPU checks of the C ABI: the library loads, exports every function that
+include/eogp.h declares, rejects bad arguments on the host, and its host-side
+retained-set plan matches the oracle's selection exactly."""
+import os
+import re
+import subprocess
+
+import numpy as np
+import pytest
+
+from oracle import eogp_oracle as O
+from paper_2609_37842_gb300 import build as B
+from paper_2609_37842_gb300 import eogp as E
+from paper_2609_37842_gb300 import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    B.build()
+    E.lib()
+
+
+def declared_functions():
+    names = set()
+    inc = os.path.join(ROOT, "include")
+    for f in os.listdir(inc):
+        if f.endswith(".h"):
+            txt = open(os.path.join(inc, f)).read()
+            txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+            names |= set(re.findall(r"\b(eogp_\w+)\s*\(", txt))
+    return sorted(names)
+
+
+def test_every_declared_symbol_is_exported():
+    names = declared_functions()
+    assert len(names) >= 14
+    out = subprocess.run(["nm", "-D", "--defined-only", B.LIB], capture_output=True, text=True).stdout
+    exported = set(re.findall(r"\bT (eogp_\w+)", out))
+    missing = [n for n in names if n not in exported]
+    assert not missing, missing
+    for n in names:
+        assert n in E.EXPORTS, f"binding lacks {n}"
+    # nothing but the ABI leaks out of the library
+    assert all(n.startswith("eogp_") for n in exported)
+
+
+def test_version_and_error_string():
+    assert "sm_103a" in E.version()
+    assert isinstance(E.lib().eogp_last_error(), bytes)
+
+
+@pytest.mark.parametrize("d_in,d_out,m,alpha,rel", [
+    (64, 64, 512, 1.5, 1e-3),      # the tiny fp32 workload: 6 ties at the boundary
+    (8, 8, 7, 1.5, 0.1),           # cut inside a tie group
+    (8, 8, 64, 1.0, 0.1),          # keep everything
+    (768, 2304, 4096, 1.2, 0.1),   # GPT-2 c_attn
+    (3072, 768, 4096, 1.2, 0.1),   # GPT-2 mlp c_proj
+    (33, 17, 100, 0.7, 0.1),       # ragged sizes
+])
+def test_plan_matches_oracle_selection(d_in, d_out, m, alpha, rel):
+    lamA = synth.power_spectrum(d_in, alpha)
+    lamS = synth.power_spectrum(d_out, alpha)
+    plan = E.Plan.from_factors(lamS, lamA, m, rel)
+    j, i, sc = plan.retained()
+    Lam = O.kfac_eigenvalues(lamS, lamA)
+    jo, io = O.select_retained(Lam, m)
+    np.testing.assert_array_equal(j, jo)
+    np.testing.assert_array_equal(i, io)
+    lam = O.damping(Lam, rel)
+    inf = plan.info()
+    assert inf.lam == pytest.approx(lam, rel=1e-12)
+    want = (1.0 / np.sqrt(Lam[jo, io] + lam)).astype(np.float32)
+    np.testing.assert_allclose(sc, want, rtol=2e-7, atol=0)
+    R, C = plan.sets()
+    np.testing.assert_array_equal(R, np.unique(jo))
+    np.testing.assert_array_equal(C, np.unique(io))
+    assert inf.nR == len(R) and inf.nC == len(C)
+
+
+def test_plan_full_table_form():
+    rng = np.random.default_rng(3)
+    Lam = rng.uniform(0, 1, (20, 12))
+    Lam[3, 4] = Lam[5, 6] = Lam[0, 0] = 0.99999   # ties in the table
+    plan = E.Plan.from_table(Lam, 37, 0.1)
+    j, i, _ = plan.retained()
+    jo, io = O.select_retained(Lam, 37)
+    np.testing.assert_array_equal(j, jo)
+    np.testing.assert_array_equal(i, io)
+
+
+@pytest.mark.parametrize("kwargs,code", [
+    (dict(m=0), E.EINVAL), (dict(m=10_000), E.EINVAL), (dict(rel=-1.0), E.EINVAL),
+    (dict(bad_lam=True), E.EINVAL)])
+def test_plan_rejects_bad_arguments(kwargs, code):
+    lam = np.arange(1, 9, dtype=np.float64) ** -1.0
+    if kwargs.get("bad_lam"):
+        lam = lam.copy()
+        lam[2] = np.nan
+    with pytest.raises(E.EOGPError) as ei:
+        E.Plan.from_factors(lam, lam, kwargs.get("m", 10), kwargs.get("rel", 0.1))
+    assert ei.value.code == code
+
+
+def test_host_only_plan_is_rejected_by_compress():
+    lam = np.arange(1, 9, dtype=np.float64) ** -1.0
+    plan = E.Plan.from_factors(lam, lam, 10, 0.1)
+    desc = E.LayerDesc(8, 8, 4, 10, 4, E.F32, 16, 16, 16, plan.handle)
+    import ctypes
+    n = ctypes.c_size_t()
+    assert E.lib().eogp_compress_workspace_size(ctypes.byref(desc), 2, E.OUT_CODES, ctypes.byref(n)) == 0
+    rc = E.lib().eogp_compress_layer(ctypes.byref(desc), 16, 16, 2, E.OUT_CODES, None, 0, 16, 1, 16,
+                                     1, 256, n.value, None)
+    assert rc == E.EINVAL
+
+
+def test_host_argument_checks():
+    L = E.lib()
+    import ctypes
+    n = ctypes.c_size_t()
+    assert L.eogp_fit_pca_workspace_size(10, 20, 0, ctypes.byref(n)) == E.EINVAL
+    assert L.eogp_fit_pca_workspace_size(10, 20, 11, ctypes.byref(n)) == E.EINVAL
+    assert L.eogp_fit_pca_workspace_size(10, 20, 5, ctypes.byref(n)) == E.OK and n.value > 0
+    assert L.eogp_pack_sign(None, -1, 8, 8, None, 1, None, 1, None) == E.EINVAL
+    assert L.eogp_pack_sign(None, 4, 0, 8, None, 1, None, 1, None) == E.EINVAL
+    assert L.eogp_pack_sign(None, 0, 8, 8, None, 1, None, 1, None) == E.OK   # empty batch
+    ks = (ctypes.c_int * 2)(32, 0)
+    assert L.eogp_score(16, 2, 16, 2, 4, ks, 2, 0, 16, 2, 16, 2, 4, 16, 4, None, 0, None) == E.EINVAL
+    assert L.eogp_compress_workspace_size(None, 1, 0, ctypes.byref(n)) == E.EINVAL
