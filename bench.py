@@ -114,23 +114,29 @@ def build_stack(w, B, dev, seed):
     from paper_2609_37842_gb300 import synth
     g = torch.Generator(device=dev)
     g.manual_seed(seed)
+    gh = torch.Generator()
+    gh.manual_seed(seed)
     mods = []
     plans = {}
+    bases = {}
+    Pt = synth.torch_eigvec_rows(w.m, w.k, dev, gh, torch.bfloat16)
     for u, mod in enumerate(w.modules):
         key = (mod.d_in, mod.d_out)
         if key not in plans:
             plans[key] = E.Plan.from_factors(synth.power_spectrum(mod.d_out, w.alpha),
                                              synth.power_spectrum(mod.d_in, w.alpha), w.m,
                                              w.damping_rel)
+            inf = plans[key].info()
+            # The spectra are sorted, so C and R are index prefixes: the retained rows are
+            # the leading eigenvectors of Haar bases (shared by modules of one shape; the
+            # work per module does not depend on their values).
+            R, C = plans[key].sets()
+            assert (C == range(inf.nC)).all() and (R == range(inf.nR)).all()
+            bases[key] = (synth.torch_eigvec_rows(mod.d_in, inf.nC, dev, gh, torch.bfloat16),
+                          synth.torch_eigvec_rows(mod.d_out, inf.nR, dev, gh, torch.bfloat16))
         plan = plans[key]
         inf = plan.info()
-        # The spectra are sorted, so C and R are index prefixes: the retained rows are the
-        # leading eigenvectors of fresh Haar bases.
-        R, C = plan.sets()
-        assert (C == range(inf.nC)).all() and (R == range(inf.nR)).all()
-        VA = synth.torch_eigvec_rows(mod.d_in, inf.nC, dev, g, torch.bfloat16)
-        VS = synth.torch_eigvec_rows(mod.d_out, inf.nR, dev, g, torch.bfloat16)
-        Pt = synth.torch_eigvec_rows(w.m, w.k, dev, g, torch.bfloat16)
+        VA, VS = bases[key]
         a, s = synth.torch_layer_inputs(w, u, B, dev, g)
         desc = E.layer_desc(plan, w.T, w.k, VA, VS, Pt)
         mods.append(dict(desc=desc, a=a, s=s, d_in=mod.d_in, d_out=mod.d_out, nC=inf.nC,
@@ -220,6 +226,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-score", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--modules", type=int, default=0,
+                    help="use only the first N modules of the stack (small profiling cases)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -242,6 +250,9 @@ def main():
     from paper_2609_37842_gb300 import synth
 
     w = synth.WORKLOADS[WORKLOAD]
+    if args.modules:
+        import dataclasses
+        w = dataclasses.replace(w, modules=w.modules[:args.modules])
     B, T, U = args.batch, w.T, len(w.modules)
     words = (w.k + 31) // 32
     peaks, peaks_src = load_peaks()
@@ -303,7 +314,7 @@ def main():
     peak = peaks.get("bf16_tflops_sustained") or PEAKS_FALLBACK["bf16_tflops_sustained"]
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": (achieved / peak) if achieved else None,
-                "traffic": ROTATE_TRAFFIC_BYTES, "kernel": "k_tc_gemm (Kronecker rotation)",
+                "traffic": ROTATE_TRAFFIC_BYTES, "kernel": "k_tc_rotate (Kronecker rotation)",
                 "peak_source": f"{peaks_src} bf16_tflops_sustained",
                 "flops_per_launch": flops_per_launch}
 
@@ -390,7 +401,8 @@ def main():
                 "steps": args.steps, "warmup": args.warmup,
                 "ms_per_step": t_max / args.steps, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-                "config": {"workload": WORKLOAD, "batch_per_gpu": B, "seq_len": T, "m": w.m,
+                "config": {"workload": WORKLOAD if not args.modules else
+                           f"{WORKLOAD} (first {U} modules)", "batch_per_gpu": B, "seq_len": T, "m": w.m,
                            "k": w.k, "modules": U, "parallelism": f"replicas x{world}",
                            "l2": "inputs > L2 (B x 151 MB per step)"},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "scoring": scoring,

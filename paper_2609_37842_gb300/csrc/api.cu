@@ -427,7 +427,6 @@ struct Layout {
   size_t total = 0;
 };
 
-TcGemmCfg rot_cfg() { return TcGemmCfg{128, 4}; }
 TcGemmCfg proj_cfg() { return TcGemmCfg{128, 4}; }
 constexpr int kContractStages = 3;
 
@@ -549,13 +548,13 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
     // Kronecker rotations restricted to the retained columns C / rows R (Sec. 2.2).
     {
       ProfScope ps(EOGP_K_ROTATE, st);
-      CUDA_TRY(launch_tc_gemm(M, lo.ldA, L->d_in, a, nullptr, L->d_in, L->VA, L->d_in, P->nC(), 1,
-                              0, at_hi, at_lo, lo.ldA, 0, rot_cfg(), status, st));
+      CUDA_TRY(launch_tc_rotate(M, L->d_in, a, L->d_in, L->VA, L->d_in, P->nC(), at_hi, at_lo,
+                                lo.ldA, sm_count(), status, st));
     }
     {
       ProfScope ps(EOGP_K_ROTATE, st);
-      CUDA_TRY(launch_tc_gemm(M, lo.ldS, L->d_out, s, nullptr, L->d_out, L->VS, L->d_out, P->nR(),
-                              1, 0, st_hi, st_lo, lo.ldS, 0, rot_cfg(), status, st));
+      CUDA_TRY(launch_tc_rotate(M, L->d_out, s, L->d_out, L->VS, L->d_out, P->nR(), st_hi, st_lo,
+                                lo.ldS, sm_count(), status, st));
     }
     // Per-example contraction over tokens + scale/gather into z (Eq. first_stage).
     const bool fs = out_mode == EOGP_OUT_FIRST_STAGE;

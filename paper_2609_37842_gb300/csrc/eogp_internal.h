@@ -101,6 +101,10 @@ cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, 
                            const void* W, int ldw, int Wrows, int splits, int epi, void* out0,
                            void* out1, int ldo, size_t slab, TcGemmCfg cfg, unsigned* status,
                            cudaStream_t st);
+// Persistent rotation GEMM: hi/lo = split(X[M x K] W[Wrows x K]^T), columns < ldo.
+cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W, int ldw, int Wrows,
+                             void* hi, void* lo, int ldo, int num_sms, unsigned* status,
+                             cudaStream_t st);
 // Number of K splits launch_tc_gemm actually uses for a requested count.
 int tc_gemm_splits_used(int K, int splits);
 // Per-example tile-sparse contraction over tokens with the scale-and-gather epilogue.

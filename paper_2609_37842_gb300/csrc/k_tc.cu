@@ -21,6 +21,8 @@
 // MMAs (one lane), warps 2-5 run the epilogue (warp w reads TMEM lanes
 // 32*(w%4)..+31). Every mbarrier wait is bounded (eogp_dev.cuh); after a
 // timeout every role falls through to the common exit, which frees TMEM.
+#include <algorithm>
+#include <cstdlib>
 #include <mutex>
 
 #include "eogp_dev.cuh"
@@ -334,6 +336,170 @@ size_t contract_smem_bytes(int stages) {
   return 1024 + static_cast<size_t>(stages) * kCStage + (2 * stages + 1) * 8 + 16;
 }
 
+
+// ------------------------------------------------------------------------
+// k_tc_rotate -- persistent rotation GEMM: D = X W^T written as bf16 hi/lo.
+// One CTA per SM walks a static tile schedule (tile t -> M block t / nN,
+// N block t % nN, so the nN CTAs sharing an activation block run together and
+// the block is read from HBM once). Two TMEM accumulators alternate between
+// tiles: the MMA warp fills one while the epilogue warps drain the other.
+// Epilogue: 32-column TMEM loads, hi/lo split, 32-byte stores (a full sector
+// per thread).
+struct RotArgs {
+  int M, K, BN, stages, nN, n_tiles, ldo;
+  __nv_bfloat16* hi;
+  __nv_bfloat16* lo;
+  unsigned* status;
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_tc_rotate(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
+                const RotArgs g) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t stage_bytes = kABytes + static_cast<uint32_t>(g.BN) * 128u;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(g.stages) * stage_bytes);
+  uint64_t* empty = full + g.stages;
+  uint64_t* tfull = empty + g.stages;  // accumulator ready, per TMEM buffer
+  uint64_t* tempty = tfull + 2;        // accumulator drained, per TMEM buffer
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  const uint32_t tcols = g.BN <= 64 ? 128u : g.BN <= 128 ? 256u : 512u;
+  const uint32_t bstride = tcols / 2;
+  const int nkb = (g.K + 63) / 64;
+
+  if (threadIdx.x == 0) {
+    tma_prefetch_desc(&tmX);
+    tma_prefetch_desc(&tmW);
+    for (int s = 0; s < g.stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 4);  // one arrive per epilogue warp
+    }
+    fence_barrier_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, tcols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < g.n_tiles && ok; t += gridDim.x) {
+        const int m0 = (t / g.nN) * 128, n0 = (t % g.nN) * g.BN;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = static_cast<int>(it % g.stages);
+          const uint32_t ph = (it / g.stages) & 1u;
+          if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) {
+            ok = false;
+            break;
+          }
+          uint8_t* st = smem + static_cast<size_t>(s) * stage_bytes;
+          mbar_arrive_expect_tx(&full[s], stage_bytes);
+          tma_load_2d(st, &tmX, kb * 64, m0, &full[s]);
+          tma_load_2d(st + kABytes, &tmW, kb * 64, n0, &full[s]);
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(128, g.BN, 0, 0);
+      uint32_t it = 0;
+      int i = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < g.n_tiles && ok; t += gridDim.x, ++i) {
+        const int buf = i & 1;
+        const uint32_t aph = static_cast<uint32_t>(i >> 1) & 1u;
+        if (!mbar_wait(&tempty[buf], aph ^ 1u, g.status)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + buf * bstride;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = static_cast<int>(it % g.stages);
+          const uint32_t ph = (it / g.stages) & 1u;
+          if (!mbar_wait(&full[s], ph, g.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
+          const uint32_t sb = sa + kABytes;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            tc_mma_f16(d, sdesc_sw128(sa + kk * 32, 16, 1024), sdesc_sw128(sb + kk * 32, 16, 1024),
+                       idesc, (kb | kk) != 0 ? 1u : 0u);
+          }
+          tc_commit(&empty[s]);
+        }
+        tc_commit(&tfull[buf]);
+      }
+    }
+    __syncwarp();
+  } else {
+    const int q = warp & 3;
+    int i = 0;
+    for (int t = blockIdx.x; t < g.n_tiles; t += gridDim.x, ++i) {
+      const int buf = i & 1;
+      const uint32_t aph = static_cast<uint32_t>(i >> 1) & 1u;
+      uint32_t ok = 1;
+      if (lane == 0) ok = mbar_wait(&tfull[buf], aph, g.status) ? 1u : 0u;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      __syncwarp();
+      tc_fence_after();
+      if (!ok) break;
+      const int m0 = (t / g.nN) * 128, n0 = (t % g.nN) * g.BN;
+      const int row = m0 + q * 32 + lane;
+      const uint32_t tb = tmem + buf * bstride + (static_cast<uint32_t>(q * 32) << 16);
+      for (int c = 0; c < g.BN; c += 32) {
+        float v[32];
+        tmem_ld32(tb + c, v);
+        const int col = n0 + c;
+        if (row < g.M && col < g.ldo) {
+          uint32_t h[16], l[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * e]);
+            const __nv_bfloat16 h1 = __float2bfloat16_rn(v[2 * e + 1]);
+            h[e] = pack_bf16x2(h0, h1);
+            l[e] = pack_bf16x2(__float2bfloat16_rn(v[2 * e] - __bfloat162float(h0)),
+                               __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1)));
+          }
+          const size_t off = static_cast<size_t>(row) * g.ldo + col;
+          uint32_t w[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w[e] = h[e];
+          st_global_v8(g.hi + off, w);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w[e] = h[8 + e];
+          st_global_v8(g.hi + off + 16, w);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w[e] = l[e];
+          st_global_v8(g.lo + off, w);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w[e] = l[8 + e];
+          st_global_v8(g.lo + off + 16, w);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[buf]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, tcols);
+}
+
+size_t rotate_smem_bytes(int BN, int stages) {
+  return 1024 + static_cast<size_t>(stages) * (kABytes + BN * 128u) + (2 * stages + 4) * 8 + 16;
+}
+
 }  // namespace
 
 static int tmap_bf16_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t rows,
@@ -393,6 +559,57 @@ cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, 
   if (e != cudaSuccess) return e;
   dim3 grid((N + cfg.BN - 1) / cfg.BN, (M + 127) / 128, splits);
   k_tc_gemm<<<grid, kThreads, smem, st>>>(tX0, tX1, tW, g);
+  return cudaGetLastError();
+}
+
+
+int rotate_bn(int ldo) {
+  static int forced = -1;
+  if (forced < 0) {
+    const char* e = getenv("EOGP_ROT_BN");
+    forced = e ? atoi(e) : 0;
+  }
+  if (forced > 0 && forced % 32 == 0 && forced <= 256) return forced;
+  const int n0 = (ldo + 255) / 256;
+  int best = 0, best_cost = 1 << 30;
+  for (int nN = n0; nN <= n0 + 1; ++nN) {
+    const int bn = ((ldo + nN - 1) / nN + 31) / 32 * 32;
+    const int cost = nN * bn + 32 * nN;
+    if (cost < best_cost) {
+      best_cost = cost;
+      best = bn;
+    }
+  }
+  return best;
+}
+
+cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W, int ldw, int Wrows,
+                             void* hi, void* lo, int ldo, int num_sms, unsigned* status,
+                             cudaStream_t st) {
+  if (M <= 0) return cudaSuccess;
+  const int BN = rotate_bn(ldo);
+  const int stages = BN > 128 ? 4 : 5;
+  CUtensorMap tX, tW;
+  if (tmap_bf16_2d(&tX, X, static_cast<uint64_t>(K), static_cast<uint64_t>(M), ldx, 64, 128) ||
+      tmap_bf16_2d(&tW, W, K, Wrows, ldw, 64, BN))
+    return cudaErrorInvalidValue;
+  RotArgs g;
+  g.M = M;
+  g.K = K;
+  g.BN = BN;
+  g.stages = stages;
+  g.nN = (ldo + BN - 1) / BN;
+  g.n_tiles = ((M + 127) / 128) * g.nN;
+  g.ldo = ldo;
+  g.hi = static_cast<__nv_bfloat16*>(hi);
+  g.lo = static_cast<__nv_bfloat16*>(lo);
+  g.status = status;
+  const size_t smem = rotate_smem_bytes(BN, stages);
+  cudaError_t e = cudaFuncSetAttribute(k_tc_rotate, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  const int grid = std::min(g.n_tiles, std::max(1, num_sms));
+  k_tc_rotate<<<grid, kThreads, smem, st>>>(tX, tW, g);
   return cudaGetLastError();
 }
 

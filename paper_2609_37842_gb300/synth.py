@@ -264,12 +264,13 @@ def torch_layer_inputs(w: Workload, module_index: int, n: int, device, generator
 
 
 def torch_eigvec_rows(d: int, n_rows: int, device, generator, dtype):
-    """n_rows orthonormal rows of length d (leading rows of a Haar orthogonal matrix),
-    drawn on the device with a thin QR."""
+    """n_rows orthonormal rows of length d (leading rows of a Haar orthogonal matrix):
+    thin QR of a Gaussian d x n_rows matrix on the host, then moved to `device`.
+    `generator` is a CPU torch.Generator."""
     import torch
-    g = torch.randn((d, n_rows), device=device, generator=generator, dtype=torch.float32)
+    g = torch.randn((d, n_rows), generator=generator, dtype=torch.float32)
     q, r = torch.linalg.qr(g)
     sgn = torch.sign(torch.diagonal(r))
     sgn[sgn == 0] = 1.0
     q = q * sgn[None, :]
-    return q.t().contiguous().to(dtype)
+    return q.t().contiguous().to(device=device, dtype=dtype)
