@@ -197,6 +197,25 @@ int eogp_compress_layer(const eogp_layer_desc* L, const void* a, const void* s, 
                         float* scales, int ld_scales, void* ws, size_t ws_bytes,
                         eogp_stream_t stream);
 
+/* Same computation and outputs as eogp_compress_layer, for callers that cannot
+ * allocate device memory (a plugin whose host framework owns every device
+ * allocation, a service confined to a memory budget fixed at start-up, a C
+ * program with no allocator of its own). The paper has no counterpart: this is
+ * a library convenience. Its scratch is a built-in device array of
+ * EOGP_STATIC_WORKSPACE_BYTES that every GPU loading the library keeps until
+ * the process exits; the call itself allocates nothing.
+ *  - Requests whose eogp_compress_workspace_size exceeds the array return
+ *    EOGP_EUNSUPPORTED with a message; use a smaller B or eogp_compress_layer.
+ *  - All calls on a device share the one array and it keeps the last call's
+ *    contents. Calls whose kernels overlap on the GPU (e.g. on two streams
+ *    without ordering between them) race on it and corrupt each other's results.
+ *  - The first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress); make that first call before any stream capture. */
+#define EOGP_STATIC_WORKSPACE_BYTES (32u << 20)
+int eogp_compress_layer_static(const eogp_layer_desc* L, const void* a, const void* s, int B,
+                               int out_mode, float* out, int ld_out, uint32_t* codes, int ld_codes,
+                               float* scales, int ld_scales, eogp_stream_t stream);
+
 /* ========================================================================
  * PCA fit (App. B.2 "PCA fitting"; Alg. 1 "fit P_u by uncentered PCA")
  * ======================================================================== */

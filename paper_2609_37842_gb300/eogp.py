@@ -63,6 +63,9 @@ EXPORTS = {
     "eogp_compress_layer": (c_int, [POINTER(LayerDesc), c_void_p, c_void_p, c_int, c_int, c_void_p,
                                     c_int, c_void_p, c_int, c_void_p, c_int, c_void_p, c_size_t,
                                     c_void_p]),
+    "eogp_compress_layer_static": (c_int, [POINTER(LayerDesc), c_void_p, c_void_p, c_int, c_int,
+                                           c_void_p, c_int, c_void_p, c_int, c_void_p, c_int,
+                                           c_void_p]),
     "eogp_fit_pca_workspace_size": (c_int, [c_int, c_int, c_int, POINTER(c_size_t)]),
     "eogp_fit_pca": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int,
                              c_void_p, c_void_p, c_size_t, c_void_p]),
