@@ -200,8 +200,9 @@ extern "C" int eogp_sync_status(eogp_stream_t stream) {
 // =================================================================== plan
 
 static void plan_free_device(eogp_plan* p) {
-  int32_t** ip[] = {&p->d_tile_rc, &p->d_tile_start, &p->d_ent_r, &p->d_ent_off,
-                    &p->d_posR,    &p->d_posC,       &p->d_R,     &p->d_C};
+  int32_t** ip[] = {&p->d_tile_rc, &p->d_tile_start, &p->d_grp_start, &p->d_ent, &p->d_ent_r,
+                    &p->d_ent_off, &p->d_posR,       &p->d_posC,      &p->d_R,
+                    &p->d_C};
   for (auto q : ip) {
     if (*q) cudaFree(*q);
     *q = nullptr;
@@ -310,11 +311,18 @@ extern "C" int eogp_plan_layer(const double* lam_S, const double* lam_A, const d
     P->posR[r] = rowmap[P->j[r]];
     P->posC[r] = colmap[P->i[r]];
   }
-  // Active 128 x 128 tiles; entries grouped per tile, canonical order inside.
+  // Active 128 x 128 tiles; inside a tile, entries grouped by the 32-column
+  // chunk co / 32 that the contraction epilogue stages at a time, canonical
+  // order inside a group.
   std::vector<int> order(m);
   std::iota(order.begin(), order.end(), 0);
   auto tkey = [&](int r) { return (static_cast<int64_t>(P->posR[r] / 128) << 32) | (P->posC[r] / 128); };
-  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return tkey(a) < tkey(b); });
+  auto gkey = [&](int r) { return (P->posC[r] % 128) / 32; };
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) {
+    const int64_t ta = tkey(a), tb = tkey(b);
+    if (ta != tb) return ta < tb;
+    return gkey(a) < gkey(b);
+  });
   int64_t last = -1;
   for (int e = 0; e < m; ++e) {
     const int r = order[e];
@@ -329,6 +337,25 @@ extern "C" int eogp_plan_layer(const double* lam_S, const double* lam_A, const d
     P->ent_scale.push_back(P->scale[r]);
   }
   P->tile_start.push_back(m);
+  // Group boundaries: for tile t, group g = co / 32.
+  P->grp_start.assign(static_cast<size_t>(P->n_tiles()) * 4 + 1, 0);
+  for (int t = 0; t < P->n_tiles(); ++t) {
+    int e = P->tile_start[t];
+    for (int grp = 0; grp < 4; ++grp) {
+      P->grp_start[t * 4 + grp] = e;
+      while (e < P->tile_start[t + 1] && (P->ent_off[e] & 255) / 32 == grp) ++e;
+    }
+  }
+  P->grp_start[static_cast<size_t>(P->n_tiles()) * 4] = m;
+  P->ent.resize(static_cast<size_t>(m) * 4);
+  for (int e = 0; e < m; ++e) {
+    int32_t sbits;
+    std::memcpy(&sbits, &P->ent_scale[e], 4);
+    P->ent[4 * e + 0] = P->ent_r[e];
+    P->ent[4 * e + 1] = P->ent_off[e];
+    P->ent[4 * e + 2] = sbits;
+    P->ent[4 * e + 3] = 0;
+  }
   if (P->nR() / 128 >= 32768 || P->nC() / 128 >= 65536) {
     delete P;
     return set_error(EOGP_EUNSUPPORTED, "retained block too large");
@@ -336,6 +363,7 @@ extern "C" int eogp_plan_layer(const double* lam_S, const double* lam_A, const d
 
   int rc = EOGP_OK;
   if (dev >= 0 && ((rc = upload(&P->d_tile_rc, P->tile_rc)) || (rc = upload(&P->d_tile_start, P->tile_start)) ||
+      (rc = upload(&P->d_grp_start, P->grp_start)) || (rc = upload(&P->d_ent, P->ent)) ||
       (rc = upload(&P->d_ent_r, P->ent_r)) || (rc = upload(&P->d_ent_off, P->ent_off)) ||
       (rc = upload(&P->d_ent_scale, P->ent_scale)) || (rc = upload(&P->d_posR, P->posR)) ||
       (rc = upload(&P->d_posC, P->posC)) || (rc = upload(&P->d_scale, P->scale)) ||
@@ -549,12 +577,12 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
     {
       ProfScope ps(EOGP_K_ROTATE, st);
       CUDA_TRY(launch_tc_rotate(M, L->d_in, a, L->d_in, L->VA, L->d_in, P->nC(), at_hi, at_lo,
-                                lo.ldA, sm_count(), status, st));
+                                lo.ldA, L->T, sm_count(), status, st));
     }
     {
       ProfScope ps(EOGP_K_ROTATE, st);
       CUDA_TRY(launch_tc_rotate(M, L->d_out, s, L->d_out, L->VS, L->d_out, P->nR(), st_hi, st_lo,
-                                lo.ldS, sm_count(), status, st));
+                                lo.ldS, L->T, sm_count(), status, st));
     }
     // Per-example contraction over tokens + scale/gather into z (Eq. first_stage).
     const bool fs = out_mode == EOGP_OUT_FIRST_STAGE;
@@ -562,7 +590,8 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
       ProfScope ps(EOGP_K_CONTRACT, st);
       CUDA_TRY(launch_tc_contract(st_hi, st_lo, lo.ldS, at_hi, at_lo, lo.ldA, B, L->T, P,
                                   fs ? out : nullptr, ld_out, fs ? nullptr : w + lo.zhi,
-                                  fs ? nullptr : w + lo.zlo, lo.ldzb, kContractStages, status, st));
+                                  fs ? nullptr : w + lo.zlo, lo.ldzb, kContractStages, sm_count(),
+                                  status, st));
     }
     if (fs) return EOGP_OK;
     // x = P^T z (Eq. second_stage), split over K; then sum + sign/pack (Eq. onebit).

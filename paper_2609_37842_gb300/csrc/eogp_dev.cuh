@@ -215,4 +215,18 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+// AND of `pred` over the 128 threads of the four epilogue warps (named barrier 2).
+__device__ __forceinline__ uint32_t __syncthreads_and_named(uint32_t pred) {
+  uint32_t out;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, 2, 128, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}\n"
+      : "=r"(out)
+      : "r"(pred)
+      : "memory");
+  return out;
+}
+
 }  // namespace eogp

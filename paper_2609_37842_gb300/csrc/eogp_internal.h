@@ -40,12 +40,16 @@ struct eogp_plan {
   // Active 128x128 tiles of the R x C block, CSR over entries.
   std::vector<int32_t> tile_rc;     // (rt << 16) | ct
   std::vector<int32_t> tile_start;  // n_tiles + 1
+  std::vector<int32_t> grp_start;   // n_tiles * 4 + 1: (tile, co / 32) groups
+  std::vector<int32_t> ent;         // 4 ints per entry: r, (ro << 8) | co, scale bits, 0
   std::vector<int32_t> ent_r;       // retained index r
   std::vector<int32_t> ent_off;     // (ro << 8) | co inside the tile
   std::vector<float> ent_scale;
   // Device copies (owned).
   int32_t* d_tile_rc = nullptr;
   int32_t* d_tile_start = nullptr;
+  int32_t* d_grp_start = nullptr;
+  int32_t* d_ent = nullptr;
   int32_t* d_ent_r = nullptr;
   int32_t* d_ent_off = nullptr;
   float* d_ent_scale = nullptr;
@@ -101,9 +105,11 @@ cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, 
                            const void* W, int ldw, int Wrows, int splits, int epi, void* out0,
                            void* out1, int ldo, size_t slab, TcGemmCfg cfg, unsigned* status,
                            cudaStream_t st);
-// Persistent rotation GEMM: hi/lo = split(X[M x K] W[Wrows x K]^T), columns < ldo.
+// Persistent rotation GEMM: hi/lo = split(X[M x K] W[Wrows x K]^T), columns < ldo
+// (a multiple of 128), rows M = B * T, written in the blocked layout
+// [B][ldo / 128][T][128] that launch_tc_contract reads.
 cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W, int ldw, int Wrows,
-                             void* hi, void* lo, int ldo, int num_sms, unsigned* status,
+                             void* hi, void* lo, int ldo, int T, int num_sms, unsigned* status,
                              cudaStream_t st);
 // Number of K splits launch_tc_gemm actually uses for a requested count.
 int tc_gemm_splits_used(int K, int splits);
@@ -111,7 +117,7 @@ int tc_gemm_splits_used(int K, int splits);
 cudaError_t launch_tc_contract(const void* St_hi, const void* St_lo, int ldS, const void* At_hi,
                                const void* At_lo, int ldA, int B, int T, const eogp_plan* plan,
                                float* z, int ldz, void* zhi, void* zlo, int ldzb, int stages,
-                               unsigned* status, cudaStream_t st);
+                               int num_sms, unsigned* status, cudaStream_t st);
 
 // k_pca.cu
 struct PcaWs {

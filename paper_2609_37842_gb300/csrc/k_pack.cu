@@ -4,12 +4,10 @@
 // scale ||x||_1 / k. The same kernel finalises the split-K projection: x is
 // the fixed-order sum of `splits` partial slabs.
 //
-// One warp per row. Full 128-column chunks use float4 loads: each lane holds 4
-// columns, forms a 4-bit nibble, and 8 lanes OR their nibbles into one word.
-// The remainder uses one column per lane and a warp ballot. The |x| sum is
-// accumulated per lane in column order, then reduced by a fixed butterfly, so
-// the scale is bitwise reproducible run to run. HBM-bound: it reads 4k bytes
-// per row (times `splits`) and writes k/8 + 4.
+// Full 128-column chunks use float4 loads: each lane holds 4 columns, forms a
+// 4-bit nibble, and 8 lanes OR their nibbles into one word. The remainder uses
+// one column per lane and a warp ballot. HBM-bound: it reads 4k bytes per row
+// (times `splits`) and writes k/8 + 4.
 #include "eogp_dev.cuh"
 #include "eogp_internal.h"
 
@@ -19,15 +17,18 @@ __device__ __forceinline__ float4 ld_stream4(const float* p) {
   return __ldcs(reinterpret_cast<const float4*>(p));
 }
 
+// One block (8 warps) per row. 128-column chunks go to warps round-robin; each
+// warp sums |x| over its chunks in column order, then the 8 warp totals are
+// added in warp order, so the scale is bitwise reproducible.
 __global__ void __launch_bounds__(256) k_pack(const float* __restrict__ part, int splits,
                                                size_t slab, int ldp, int B, int k,
                                                float* __restrict__ x_out, int ldx,
                                                uint32_t* __restrict__ codes, int ld_codes,
                                                float* __restrict__ scales, int ld_scales,
                                                unsigned* status) {
-  const int row = static_cast<int>((blockIdx.x * static_cast<unsigned>(blockDim.x) + threadIdx.x) >> 5);
-  const int lane = threadIdx.x & 31;
-  if (row >= B) return;
+  __shared__ float wsum[8];
+  const int row = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float* src = part + static_cast<size_t>(row) * ldp;
   float* xo = x_out ? x_out + static_cast<size_t>(row) * ldx : nullptr;
   uint32_t* co = codes ? codes + static_cast<size_t>(row) * ld_codes : nullptr;
@@ -38,37 +39,34 @@ __global__ void __launch_bounds__(256) k_pack(const float* __restrict__ part, in
                    ((slab & 3) == 0) &&
                    (x_out == nullptr ||
                     (((ldx & 3) == 0) && ((reinterpret_cast<uintptr_t>(x_out) & 15) == 0)));
-  int c0 = 0;
-  if (vec) {
-    const int nfull = k >> 7;
-#pragma unroll 4
-    for (int it = 0; it < nfull; ++it) {
-      const int c = (it << 7) + (lane << 2);
-      float4 v = ld_stream4(src + c);
-      for (int s = 1; s < splits; ++s) {
-        const float4 w = ld_stream4(src + static_cast<size_t>(s) * slab + c);
-        v.x += w.x;
-        v.y += w.y;
-        v.z += w.z;
-        v.w += w.w;
-      }
-      if (xo) *reinterpret_cast<float4*>(xo + c) = v;
-      bad |= isnan(v.x) | isnan(v.y) | isnan(v.z) | isnan(v.w);
-      acc += fabsf(v.x);
-      acc += fabsf(v.y);
-      acc += fabsf(v.z);
-      acc += fabsf(v.w);
-      uint32_t nib = (v.x >= 0.f ? 1u : 0u) | (v.y >= 0.f ? 2u : 0u) | (v.z >= 0.f ? 4u : 0u) |
-                     (v.w >= 0.f ? 8u : 0u);
-      uint32_t word = nib << (4 * (lane & 7));
-      word |= __shfl_xor_sync(0xffffffffu, word, 1);
-      word |= __shfl_xor_sync(0xffffffffu, word, 2);
-      word |= __shfl_xor_sync(0xffffffffu, word, 4);
-      if (co && (lane & 7) == 0) co[(it << 2) + (lane >> 3)] = word;
+  const int nfull = vec ? (k >> 7) : 0;
+  for (int it = warp; it < nfull; it += 8) {
+    const int c = (it << 7) + (lane << 2);
+    float4 v = ld_stream4(src + c);
+    for (int s = 1; s < splits; ++s) {
+      const float4 w = ld_stream4(src + static_cast<size_t>(s) * slab + c);
+      v.x += w.x;
+      v.y += w.y;
+      v.z += w.z;
+      v.w += w.w;
     }
-    c0 = nfull << 7;
+    if (xo) *reinterpret_cast<float4*>(xo + c) = v;
+    bad |= isnan(v.x) | isnan(v.y) | isnan(v.z) | isnan(v.w);
+    acc += fabsf(v.x);
+    acc += fabsf(v.y);
+    acc += fabsf(v.z);
+    acc += fabsf(v.w);
+    const uint32_t nib = (v.x >= 0.f ? 1u : 0u) | (v.y >= 0.f ? 2u : 0u) |
+                         (v.z >= 0.f ? 4u : 0u) | (v.w >= 0.f ? 8u : 0u);
+    uint32_t word = nib << (4 * (lane & 7));
+    word |= __shfl_xor_sync(0xffffffffu, word, 1);
+    word |= __shfl_xor_sync(0xffffffffu, word, 2);
+    word |= __shfl_xor_sync(0xffffffffu, word, 4);
+    if (co && (lane & 7) == 0) co[(it << 2) + (lane >> 3)] = word;
   }
-  for (int base = c0; base < k; base += 32) {
+  // Remainder (or everything, when unaligned): 32-column words, one column per lane.
+  const int c0 = nfull << 7;
+  for (int base = c0 + 32 * warp; base < k; base += 256) {
     const int c = base + lane;
     const bool in = c < k;
     float v = 0.f;
@@ -82,11 +80,16 @@ __global__ void __launch_bounds__(256) k_pack(const float* __restrict__ part, in
     const uint32_t word = __ballot_sync(0xffffffffu, in && v >= 0.f);
     if (co && lane == 0) co[base >> 5] = word;
   }
-  // Fixed-order butterfly; lane 0's value is the row total.
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+  if (lane == 0) wsum[warp] = acc;
   if (__any_sync(0xffffffffu, bad) && lane == 0) eogp::flag_status(status, EOGP_ST_DEVICE);
-  if (scales && lane == 0) scales[static_cast<size_t>(row) * ld_scales] = acc / static_cast<float>(k);
+  __syncthreads();
+  if (threadIdx.x == 0 && scales) {
+    float t = 0.f;
+    for (int w = 0; w < 8; ++w) t += wsum[w];
+    scales[static_cast<size_t>(row) * ld_scales] = t / static_cast<float>(k);
+  }
 }
 
 }  // namespace
@@ -95,9 +98,7 @@ cudaError_t launch_pack(const float* part, int splits, size_t slab, int ldp, int
                         float* x_out, int ldx, uint32_t* codes, int ld_codes, float* scales,
                         int ld_scales, unsigned* status, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
-  const int threads = 256;
-  const long long blocks = (static_cast<long long>(B) * 32 + threads - 1) / threads;
-  k_pack<<<static_cast<unsigned>(blocks), threads, 0, st>>>(part, splits, slab, ldp, B, k, x_out,
+  k_pack<<<static_cast<unsigned>(B), 256, 0, st>>>(part, splits, slab, ldp, B, k, x_out,
                                                            ldx, codes, ld_codes, scales,
                                                            ld_scales, status);
   return cudaGetLastError();

@@ -191,12 +191,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 struct ContractArgs {
-  int T, stages;
+  int T, stages, n_tiles, n_items, nblkS, nblkA;
   const int32_t* tile_rc;
-  const int32_t* tile_start;
-  const int32_t* ent_r;
-  const int32_t* ent_off;
-  const float* ent_scale;
+  const int32_t* grp_start;  // [n_tiles * 4 + 1]: entries per (tile, 32-column chunk)
+  const int4* ent;           // {r, (ro << 8) | co, bits of the fp32 scale, 0}
   float* z;
   int ldz;
   __nv_bfloat16* zhi;
@@ -207,7 +205,12 @@ struct ContractArgs {
 
 constexpr uint32_t kOpBytes = 16384u;          // one 128-wide operand tile, 64 tokens
 constexpr uint32_t kCStage = 4u * kOpBytes;    // S hi, S lo, A hi, A lo
+constexpr uint32_t kCStageBuf = 128u * 33u * 4u;  // 128 x 32 (+1 pad) epilogue staging
 
+// Persistent: one CTA per SM walks items (example b, active tile) with
+// b = item / n_tiles, so the tiles of one example run together and share
+// operands through L2. Two TMEM accumulators let the gather epilogue of one
+// item overlap the loads and MMAs of the next.
 __global__ void __launch_bounds__(kThreads, 1)
     k_tc_contract(const __grid_constant__ CUtensorMap tmShi, const __grid_constant__ CUtensorMap tmSlo,
                   const __grid_constant__ CUtensorMap tmAhi, const __grid_constant__ CUtensorMap tmAlo,
@@ -215,14 +218,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(g.stages) * kCStage);
+  float* stage_buf = reinterpret_cast<float*>(smem + static_cast<size_t>(g.stages) * kCStage);
+  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(stage_buf) + kCStageBuf);
   uint64_t* empty = full + g.stages;
-  uint64_t* done = empty + g.stages;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
-
-  const int tile = blockIdx.x, b = blockIdx.y;
-  const int rc = g.tile_rc[tile];
-  const int r0 = (rc >> 16) * 128, c0 = (rc & 0xFFFF) * 128;
+  uint64_t* tfull = empty + g.stages;
+  uint64_t* tempty = tfull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
   const int nkb = (g.T + 63) / 64;
 
   if (threadIdx.x == 0) {
@@ -234,10 +235,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(done, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 4);
+    }
     fence_barrier_init();
   }
-  if (warp == 1) tmem_alloc(tmem_slot, 128);
+  if (warp == 1) tmem_alloc(tmem_slot, 256);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -245,87 +249,127 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      for (int i = 0; i < nkb; ++i) {
-        const int s = i % g.stages;
-        const uint32_t ph = static_cast<uint32_t>(i / g.stages) & 1u;
-        if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) break;
-        uint8_t* st = smem + static_cast<size_t>(s) * kCStage;
-        mbar_arrive_expect_tx(&full[s], kCStage);
-        const int t0 = i * 64;
-        tma_load_3d(st + 0 * kOpBytes, &tmShi, r0, t0, b, &full[s]);
-        tma_load_3d(st + 0 * kOpBytes + 8192, &tmShi, r0 + 64, t0, b, &full[s]);
-        tma_load_3d(st + 1 * kOpBytes, &tmSlo, r0, t0, b, &full[s]);
-        tma_load_3d(st + 1 * kOpBytes + 8192, &tmSlo, r0 + 64, t0, b, &full[s]);
-        tma_load_3d(st + 2 * kOpBytes, &tmAhi, c0, t0, b, &full[s]);
-        tma_load_3d(st + 2 * kOpBytes + 8192, &tmAhi, c0 + 64, t0, b, &full[s]);
-        tma_load_3d(st + 3 * kOpBytes, &tmAlo, c0, t0, b, &full[s]);
-        tma_load_3d(st + 3 * kOpBytes + 8192, &tmAlo, c0 + 64, t0, b, &full[s]);
+      uint32_t it = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < g.n_items && ok; item += gridDim.x) {
+        const int b = item / g.n_tiles, tile = item % g.n_tiles;
+        const int rc = g.tile_rc[tile];
+        const int zs = b * g.nblkS + (rc >> 16), za = b * g.nblkA + (rc & 0xFFFF);
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = static_cast<int>(it % g.stages);
+          const uint32_t ph = (it / g.stages) & 1u;
+          if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) {
+            ok = false;
+            break;
+          }
+          uint8_t* st = smem + static_cast<size_t>(s) * kCStage;
+          mbar_arrive_expect_tx(&full[s], kCStage);
+          const int t0 = kb * 64;
+          tma_load_3d(st + 0 * kOpBytes, &tmShi, 0, t0, zs, &full[s]);
+          tma_load_3d(st + 0 * kOpBytes + 8192, &tmShi, 64, t0, zs, &full[s]);
+          tma_load_3d(st + 1 * kOpBytes, &tmSlo, 0, t0, zs, &full[s]);
+          tma_load_3d(st + 1 * kOpBytes + 8192, &tmSlo, 64, t0, zs, &full[s]);
+          tma_load_3d(st + 2 * kOpBytes, &tmAhi, 0, t0, za, &full[s]);
+          tma_load_3d(st + 2 * kOpBytes + 8192, &tmAhi, 64, t0, za, &full[s]);
+          tma_load_3d(st + 3 * kOpBytes, &tmAlo, 0, t0, za, &full[s]);
+          tma_load_3d(st + 3 * kOpBytes + 8192, &tmAlo, 64, t0, za, &full[s]);
+        }
       }
     }
     __syncwarp();
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16_f32(128, 128, 1, 1);
-      for (int i = 0; i < nkb; ++i) {
-        const int s = i % g.stages;
-        const uint32_t ph = static_cast<uint32_t>(i / g.stages) & 1u;
-        if (!mbar_wait(&full[s], ph, g.status)) break;
+      uint32_t it = 0;
+      int i = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < g.n_items && ok; item += gridDim.x, ++i) {
+        const int buf = i & 1;
+        const uint32_t aph = static_cast<uint32_t>(i >> 1) & 1u;
+        if (!mbar_wait(&tempty[buf], aph ^ 1u, g.status)) break;
         tc_fence_after();
-        const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * kCStage);
+        const uint32_t d = tmem + buf * 128u;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = static_cast<int>(it % g.stages);
+          const uint32_t ph = (it / g.stages) & 1u;
+          if (!mbar_wait(&full[s], ph, g.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * kCStage);
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-          const uint32_t o = kk * 2048u;  // 16 token rows of 128 bytes
-          const uint64_t sh = sdesc_sw128(sa + 0 * kOpBytes + o, 8192, 1024);
-          const uint64_t sl = sdesc_sw128(sa + 1 * kOpBytes + o, 8192, 1024);
-          const uint64_t ah = sdesc_sw128(sa + 2 * kOpBytes + o, 8192, 1024);
-          const uint64_t al = sdesc_sw128(sa + 3 * kOpBytes + o, 8192, 1024);
-          tc_mma_f16(tmem, sh, ah, idesc, (i | kk) != 0 ? 1u : 0u);
-          tc_mma_f16(tmem, sh, al, idesc, 1u);
-          tc_mma_f16(tmem, sl, ah, idesc, 1u);
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint32_t o = kk * 2048u;  // 16 token rows of 128 bytes
+            const uint64_t sh = sdesc_sw128(sa + 0 * kOpBytes + o, 8192, 1024);
+            const uint64_t sl = sdesc_sw128(sa + 1 * kOpBytes + o, 8192, 1024);
+            const uint64_t ah = sdesc_sw128(sa + 2 * kOpBytes + o, 8192, 1024);
+            const uint64_t al = sdesc_sw128(sa + 3 * kOpBytes + o, 8192, 1024);
+            tc_mma_f16(d, sh, ah, idesc, (kb | kk) != 0 ? 1u : 0u);
+            tc_mma_f16(d, sh, al, idesc, 1u);
+            tc_mma_f16(d, sl, ah, idesc, 1u);
+          }
+          tc_commit(&empty[s]);
         }
-        tc_commit(&empty[s]);
+        tc_commit(&tfull[buf]);
       }
-      tc_commit(done);
     }
     __syncwarp();
   } else {
     const int q = warp & 3;
-    uint32_t ok = 1;
-    if (lane == 0) ok = mbar_wait(done, 0, g.status) ? 1u : 0u;
-    ok = __shfl_sync(0xffffffffu, ok, 0);
-    __syncwarp();
-    tc_fence_after();
-    float* tilebuf = reinterpret_cast<float*>(smem);  // [128][129], reuses the drained stages
-    if (ok) {
-      const int row = q * 32 + lane;
-      const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16);
-      for (int c = 0; c < 128; c += 16) {
-        float v[16];
-        tmem_ld16(tbase + c, v);
+    const int etid = threadIdx.x - 64;  // 0..127 over the four epilogue warps
+    int i = 0;
+    for (int item = blockIdx.x; item < g.n_items; item += gridDim.x, ++i) {
+      const int buf = i & 1;
+      const uint32_t aph = static_cast<uint32_t>(i >> 1) & 1u;
+      uint32_t ok = 1;
+      if (lane == 0) ok = mbar_wait(&tfull[buf], aph, g.status) ? 1u : 0u;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      __syncwarp();
+      tc_fence_after();
+      // All four warps must agree before the shared staging is used.
+      ok = __syncthreads_and_named(ok);
+      if (!ok) break;
+      const int b = item / g.n_tiles, tile = item % g.n_tiles;
+      const uint32_t tb = tmem + buf * 128u + (static_cast<uint32_t>(q * 32) << 16);
+      const size_t zrow = static_cast<size_t>(b);
+      for (int j = 0; j < 4; ++j) {
+        float v[32];
+        tmem_ld32(tb + 32 * j, v);
 #pragma unroll
-        for (int e = 0; e < 16; ++e) tilebuf[row * 129 + c + e] = v[e];
-      }
-    }
-    named_bar_sync(1, 128);
-    if (ok) {
-      const int etid = threadIdx.x - 64;
-      const int e0 = g.tile_start[tile], e1 = g.tile_start[tile + 1];
-      for (int e = e0 + etid; e < e1; e += 128) {
-        const int r = g.ent_r[e];
-        const int off = g.ent_off[e];
-        const float val = g.ent_scale[e] * tilebuf[(off >> 8) * 129 + (off & 255)];
-        if (g.z) g.z[static_cast<size_t>(b) * g.ldz + r] = val;
-        if (g.zhi) {
-          const __nv_bfloat16 h = __float2bfloat16_rn(val);
-          g.zhi[static_cast<size_t>(b) * g.ldzb + r] = h;
-          g.zlo[static_cast<size_t>(b) * g.ldzb + r] = __float2bfloat16_rn(val - __bfloat162float(h));
+        for (int c = 0; c < 32; ++c) stage_buf[(q * 32 + lane) * 33 + c] = v[c];
+        named_bar_sync(1, 128);
+        const int e0 = g.grp_start[tile * 4 + j], e1 = g.grp_start[tile * 4 + j + 1];
+        for (int e = e0 + etid; e < e1; e += 4 * 128) {
+          int4 en[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int eu = e + u * 128;
+            en[u] = eu < e1 ? __ldg(&g.ent[eu]) : make_int4(-1, 0, 0, 0);
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            if (en[u].x < 0) continue;
+            const int r = en[u].x, off = en[u].y;
+            const float val = __int_as_float(en[u].z) * stage_buf[(off >> 8) * 33 + (off & 31)];
+            if (g.z) g.z[zrow * g.ldz + r] = val;
+            if (g.zhi) {
+              const __nv_bfloat16 h = __float2bfloat16_rn(val);
+              g.zhi[zrow * g.ldzb + r] = h;
+              g.zlo[zrow * g.ldzb + r] = __float2bfloat16_rn(val - __bfloat162float(h));
+            }
+          }
         }
+        named_bar_sync(1, 128);
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[buf]);
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) tmem_dealloc(tmem, 128);
+  if (warp == 1) tmem_dealloc(tmem, 256);
 }
 
 size_t gemm_smem_bytes(int BN, int stages, int nA) {
@@ -333,7 +377,7 @@ size_t gemm_smem_bytes(int BN, int stages, int nA) {
 }
 
 size_t contract_smem_bytes(int stages) {
-  return 1024 + static_cast<size_t>(stages) * kCStage + (2 * stages + 1) * 8 + 16;
+  return 1024 + static_cast<size_t>(stages) * kCStage + kCStageBuf + (2 * stages + 4) * 8 + 16;
 }
 
 
@@ -344,9 +388,11 @@ size_t contract_smem_bytes(int stages) {
 // the block is read from HBM once). Two TMEM accumulators alternate between
 // tiles: the MMA warp fills one while the epilogue warps drain the other.
 // Epilogue: 32-column TMEM loads, hi/lo split, 32-byte stores (a full sector
-// per thread).
+// per thread). The output is blocked for the contraction that reads it:
+// element (row = b*T + t, col) sits at ((b * (ldo/128) + col/128) * T + t) * 128
+// + col % 128, so one 128-column block of one example is T*256 contiguous bytes.
 struct RotArgs {
-  int M, K, BN, stages, nN, n_tiles, ldo;
+  int M, K, BN, stages, nN, n_tiles, ldo, T;
   __nv_bfloat16* hi;
   __nv_bfloat16* lo;
   unsigned* status;
@@ -470,7 +516,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             l[e] = pack_bf16x2(__float2bfloat16_rn(v[2 * e] - __bfloat162float(h0)),
                                __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1)));
           }
-          const size_t off = static_cast<size_t>(row) * g.ldo + col;
+          const int bex = row / g.T, tok = row - bex * g.T;
+          const size_t off =
+              ((static_cast<size_t>(bex) * (g.ldo >> 7) + (col >> 7)) * g.T + tok) * 128 + (col & 127);
           uint32_t w[8];
 #pragma unroll
           for (int e = 0; e < 8; ++e) w[e] = h[e];
@@ -511,10 +559,10 @@ static int tmap_bf16_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint6
                    CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
-static int tmap_bf16_3d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t T, uint64_t B,
-                        uint64_t ld) {
-  const uint64_t dims[3] = {inner, T, B};
-  const uint64_t strides[2] = {ld * 2, ld * 2 * T};
+// Blocked intermediate [B * nblk][T][128] (bf16): box of 64 columns x 64 tokens.
+static int tmap_bf16_blocked(CUtensorMap* tm, const void* base, uint64_t T, uint64_t nbatch) {
+  const uint64_t dims[3] = {128, T, nbatch};
+  const uint64_t strides[2] = {128 * 2, 128 * 2 * T};
   const uint32_t box[3] = {64, 64, 1};
   return make_tmap(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box,
                    CU_TENSOR_MAP_SWIZZLE_128B);
@@ -562,7 +610,6 @@ cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, 
   return cudaGetLastError();
 }
 
-
 int rotate_bn(int ldo) {
   static int forced = -1;
   if (forced < 0) {
@@ -584,7 +631,7 @@ int rotate_bn(int ldo) {
 }
 
 cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W, int ldw, int Wrows,
-                             void* hi, void* lo, int ldo, int num_sms, unsigned* status,
+                             void* hi, void* lo, int ldo, int T, int num_sms, unsigned* status,
                              cudaStream_t st) {
   if (M <= 0) return cudaSuccess;
   const int BN = rotate_bn(ldo);
@@ -601,6 +648,7 @@ cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W
   g.nN = (ldo + BN - 1) / BN;
   g.n_tiles = ((M + 127) / 128) * g.nN;
   g.ldo = ldo;
+  g.T = T;
   g.hi = static_cast<__nv_bfloat16*>(hi);
   g.lo = static_cast<__nv_bfloat16*>(lo);
   g.status = status;
@@ -623,20 +671,23 @@ int tc_gemm_splits_used(int K, int splits) {
 cudaError_t launch_tc_contract(const void* St_hi, const void* St_lo, int ldS, const void* At_hi,
                                const void* At_lo, int ldA, int B, int T, const eogp_plan* plan,
                                float* z, int ldz, void* zhi, void* zlo, int ldzb, int stages,
-                               unsigned* status, cudaStream_t st) {
+                               int num_sms, unsigned* status, cudaStream_t st) {
   if (B <= 0 || plan->n_tiles() == 0) return cudaSuccess;
   CUtensorMap tSh, tSl, tAh, tAl;
-  if (tmap_bf16_3d(&tSh, St_hi, ldS, T, B, ldS) || tmap_bf16_3d(&tSl, St_lo, ldS, T, B, ldS) ||
-      tmap_bf16_3d(&tAh, At_hi, ldA, T, B, ldA) || tmap_bf16_3d(&tAl, At_lo, ldA, T, B, ldA))
+  const uint64_t nS = static_cast<uint64_t>(B) * (ldS / 128), nA = static_cast<uint64_t>(B) * (ldA / 128);
+  if (tmap_bf16_blocked(&tSh, St_hi, T, nS) || tmap_bf16_blocked(&tSl, St_lo, T, nS) ||
+      tmap_bf16_blocked(&tAh, At_hi, T, nA) || tmap_bf16_blocked(&tAl, At_lo, T, nA))
     return cudaErrorInvalidValue;
   ContractArgs g;
   g.T = T;
+  g.nblkS = ldS / 128;
+  g.nblkA = ldA / 128;
   g.stages = stages;
+  g.n_tiles = plan->n_tiles();
+  g.n_items = g.n_tiles * B;
   g.tile_rc = plan->d_tile_rc;
-  g.tile_start = plan->d_tile_start;
-  g.ent_r = plan->d_ent_r;
-  g.ent_off = plan->d_ent_off;
-  g.ent_scale = plan->d_ent_scale;
+  g.grp_start = plan->d_grp_start;
+  g.ent = reinterpret_cast<const int4*>(plan->d_ent);
   g.z = z;
   g.ldz = ldz;
   g.zhi = static_cast<__nv_bfloat16*>(zhi);
@@ -647,7 +698,7 @@ cudaError_t launch_tc_contract(const void* St_hi, const void* St_lo, int ldS, co
   cudaError_t e = cudaFuncSetAttribute(k_tc_contract, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  dim3 grid(plan->n_tiles(), B);
+  const int grid = std::min(g.n_items, std::max(1, num_sms));
   k_tc_contract<<<grid, kThreads, smem, st>>>(tSh, tSl, tAh, tAl, g);
   return cudaGetLastError();
 }
