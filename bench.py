@@ -226,6 +226,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-score", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--copy-streams", type=int, default=2)
+    ap.add_argument("--no-scan", action="store_true")
     ap.add_argument("--modules", type=int, default=0,
                     help="use only the first N modules of the stack (small profiling cases)")
     args = ap.parse_args()
@@ -349,6 +351,10 @@ def main():
                    "mode": "CODES (xor-popcount)", "word_ops_per_s": words_total / (sms / 1000.0)}
 
     # ---- end to end through the public API with host buffers ----
+    # Per module: host -> device copy of (a, s) on a copy stream, then the
+    # compression on the compute stream once that copy has landed; module u+1's
+    # copy overlaps module u's compute. Step k+1 overwrites module u's device
+    # buffers only after step k's compute of u (event wait on the copy stream).
     e2e = None
     if not args.no_e2e:
         host = []
@@ -362,33 +368,105 @@ def main():
         hscales = torch.empty(scales.shape, dtype=scales.dtype, pin_memory=True)
         h2d = sum(ha.numel() * ha.element_size() + hs.numel() * hs.element_size() for ha, hs in host)
         d2h = hcodes.numel() * 4 + hscales.numel() * 4
+        cstreams = [torch.cuda.Stream() for _ in range(max(1, args.copy_streams))]
+        landed = [torch.cuda.Event() for _ in mods]
+        consumed = [None] * len(mods)
 
         def e2e_step():
-            for md, (ha, hs) in zip(mods, host):
-                md["a"].copy_(ha, non_blocking=True)
-                md["s"].copy_(hs, non_blocking=True)
-            compress_step(mods, E, codes, scales, ws, words)
+            for u, (md, (ha, hs)) in enumerate(zip(mods, host)):
+                cs = cstreams[u % len(cstreams)]
+                if consumed[u] is not None:
+                    cs.wait_event(consumed[u])
+                with torch.cuda.stream(cs):
+                    md["a"].copy_(ha, non_blocking=True)
+                    md["s"].copy_(hs, non_blocking=True)
+                    landed[u].record(cs)
+            for u, md in enumerate(mods):
+                stream.wait_event(landed[u])
+                E.compress_layer(md["desc"], md["a"], md["s"], E.OUT_CODES,
+                                 codes=codes[:, u * words:(u + 1) * words], scales=scales[:, u],
+                                 ws=ws, stream=stream)
+                ev = torch.cuda.Event()
+                ev.record(stream)
+                consumed[u] = ev
             hcodes.copy_(codes, non_blocking=True)
             hscales.copy_(scales, non_blocking=True)
 
         e2e_step()
         torch.cuda.synchronize()
         barrier()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
+        t0 = time.perf_counter()
         for _ in range(args.e2e_steps):
             e2e_step()
-        e1.record(stream)
         torch.cuda.synchronize()
+        ems = (time.perf_counter() - t0) * 1000.0
         E.sync_status()
-        ems = e0.elapsed_time(e1)
         if world > 1:
             tt = torch.tensor([ems], device=dev)
             dist.all_reduce(tt, op=dist.ReduceOp.MAX)
             ems = float(tt.item())
         e2e = {"value": world * B * args.e2e_steps / (ems / 1000.0), "unit": "examples/s",
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps}
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
+               "h2d_GBps": h2d * args.e2e_steps / (ems / 1000.0) / 1e9,
+               "copy_streams": len(cstreams)}
         del host
+
+    # ---- standalone sign-pack and the scoring sweep (HBM-bound kernels) ----
+    hbm = peaks.get("hbm_gbs") or PEAKS_FALLBACK["hbm_gbs"]
+    pack = None
+    scan = None
+    if rank == 0 and not args.no_scan:
+        del mods
+        torch.cuda.empty_cache()
+        g = torch.Generator(device=dev)
+        g.manual_seed(99)
+        xs = torch.randn((262144, 1024), generator=g, device=dev)
+        pc = torch.empty((262144, 32), dtype=torch.int32, device=dev)
+        psc = torch.empty((262144,), dtype=torch.float32, device=dev)
+        E.pack_sign(xs, pc, psc)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(5):
+            E.pack_sign(xs, pc, psc)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        E.sync_status()
+        pms = e0.elapsed_time(e1) / 5
+        pbytes = xs.numel() * 4 + pc.numel() * 4 + psc.numel() * 4
+        pack = {"rows": 262144, "k": 1024, "ms": pms, "GBps": pbytes / (pms / 1000.0) / 1e9,
+                "frac_of_hbm": pbytes / (pms / 1000.0) / 1e9 / hbm}
+        del xs, pc, psc
+        sc = synth.SCAN
+        N, ksc = sc["N"], sc["k"]
+        Wsc = ksc // 32
+        tr = torch.randint(-2 ** 31, 2 ** 31 - 1, (N, Wsc), generator=g, device=dev, dtype=torch.int32)
+        tsc = torch.exp(sc["scale_sigma"] * torch.randn((N, 1), generator=g, device=dev))
+        qmax = 1024
+        out = torch.empty((qmax, N), dtype=torch.float32, device=dev)
+        scan = {"N": N, "bits": ksc, "mode": "CODES", "per_Q": {}}
+        for Q in sc["Qs"]:
+            qc = torch.randint(-2 ** 31, 2 ** 31 - 1, (Q, Wsc), generator=g, device=dev,
+                               dtype=torch.int32)
+            qs = torch.exp(sc["scale_sigma"] * torch.randn((Q, 1), generator=g, device=dev))
+            chunks = [(q0, min(Q, q0 + qmax)) for q0 in range(0, Q, qmax)]
+            for q0, q1 in chunks[:1]:
+                E.score(tr, tsc, [ksc], E.SCORE_CODES, qc[q0:q1], qs[q0:q1], out=out[:q1 - q0])
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for q0, q1 in chunks:
+                E.score(tr, tsc, [ksc], E.SCORE_CODES, qc[q0:q1], qs[q0:q1], out=out[:q1 - q0])
+            e1.record(stream)
+            torch.cuda.synchronize()
+            E.sync_status()
+            qms = e0.elapsed_time(e1)
+            byts = len(chunks) * (N * Wsc * 4 + N * 4) + Q * N * 4
+            scan["per_Q"][str(Q)] = {"ms": qms, "scores_per_s": N * Q / (qms / 1000.0),
+                                     "GBps": byts / (qms / 1000.0) / 1e9,
+                                     "frac_of_hbm": byts / (qms / 1000.0) / 1e9 / hbm,
+                                     "word_ops_per_s": N * Q * Wsc / (qms / 1000.0)}
+        del tr, out
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -406,6 +484,7 @@ def main():
                            "k": w.k, "modules": U, "parallelism": f"replicas x{world}",
                            "l2": "inputs > L2 (B x 151 MB per step)"},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "scoring": scoring,
+                "pack_sign": pack, "scan": scan,
                 "gpu_launches": launches, "kernels": kern, "clocks": clk}
         print(json.dumps(line))
     if world > 1:

@@ -701,11 +701,9 @@ extern "C" int eogp_score_workspace_size(int N, const int* k_per_module, int U, 
   clear_error();
   if (!bytes) return set_error(EOGP_EINVAL, "bytes is NULL");
   (void)N;
-  (void)k_per_module;
-  (void)U;
-  (void)mode;
-  (void)Q;
   *bytes = 0;
+  if (mode == EOGP_SCORE_CODES && k_per_module && U >= 1 && score_tc_supported(k_per_module, U, Q))
+    *bytes = score_tc_ws_bytes(k_per_module, U, Q);
   return EOGP_OK;
 }
 
@@ -715,8 +713,6 @@ extern "C" int eogp_score(const void* train, int ld_train, const float* train_sc
                           float* scores, int ld_scores, void* ws, size_t ws_bytes,
                           eogp_stream_t stream) {
   clear_error();
-  (void)ws;
-  (void)ws_bytes;
   if (N < 0 || Q < 0) return set_error(EOGP_EINVAL, "N, Q must be >= 0");
   if (!k_per_module || U < 1 || U > 1024) return set_error(EOGP_EINVAL, "need 1 <= U <= 1024 modules");
   long long W = 0, D = 0;
@@ -734,9 +730,24 @@ extern "C" int eogp_score(const void* train, int ld_train, const float* train_sc
     if (!train_scales || !query_scales) return set_error(EOGP_EINVAL, "scales are NULL");
     if (ld_train < W || ld_query < W || ld_tscale < U || ld_qscale < U)
       return set_error(EOGP_EINVAL, "leading dimension too small");
-    CUDA_TRY(launch_score_codes(static_cast<const uint32_t*>(train), ld_train, train_scales, ld_tscale,
-                                N, k_per_module, U, static_cast<const uint32_t*>(query), ld_query,
-                                query_scales, ld_qscale, Q, scores, ld_scores, st));
+    // Tensor-core path when the caller provided the workspace eogp_score_workspace_size
+    // asks for (Q >= 64, every k_u a multiple of 128, 16-byte aligned code rows);
+    // otherwise the popcount kernels. Both give bitwise identical scores.
+    const bool tc = score_tc_supported(k_per_module, U, Q) && ws &&
+                    ws_bytes >= score_tc_ws_bytes(k_per_module, U, Q) && (ld_train % 4) == 0 &&
+                    aligned16(train) && (reinterpret_cast<uintptr_t>(ws) & 255) == 0;
+    if (tc) {
+      unsigned* status = status_word();
+      if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
+      CUDA_TRY(launch_score_tc(static_cast<const uint32_t*>(train), ld_train, train_scales, ld_tscale,
+                               N, k_per_module, U, static_cast<const uint32_t*>(query), ld_query,
+                               query_scales, ld_qscale, Q, scores, ld_scores, ws, sm_count(), status,
+                               st));
+    } else {
+      CUDA_TRY(launch_score_codes(static_cast<const uint32_t*>(train), ld_train, train_scales,
+                                  ld_tscale, N, k_per_module, U, static_cast<const uint32_t*>(query),
+                                  ld_query, query_scales, ld_qscale, Q, scores, ld_scores, st));
+    }
   } else if (mode == EOGP_SCORE_PAPER) {
     if (!train_scales) return set_error(EOGP_EINVAL, "train_scales is NULL");
     if (ld_train < W || ld_query < D || ld_tscale < U) return set_error(EOGP_EINVAL, "leading dimension too small");

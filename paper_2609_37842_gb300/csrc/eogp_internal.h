@@ -81,6 +81,14 @@ cudaError_t launch_score_paper(const uint32_t* train, int ldt, const float* ts, 
                                const int* ks, int U, const float* y, int ldy, int Q, float* out,
                                int ldo, cudaStream_t st);
 
+// k_score_tc.cu: CODES scoring on the tensor cores (e4m3 +-1 operands).
+bool score_tc_supported(const int* ks, int U, int Q);
+size_t score_tc_ws_bytes(const int* ks, int U, int Q);
+cudaError_t launch_score_tc(const uint32_t* train, int ldt, const float* ts, int ldts, int N,
+                            const int* ks, int U, const uint32_t* query, int ldq, const float* qs,
+                            int ldqs, int Q, float* out, int ldo, void* ws, int num_sms,
+                            unsigned* status, cudaStream_t st);
+
 // k_simt.cu: C[i][j] = alpha * sum_k A(i,k) B(j,k), A(i,k) = A[i*sai + k*sak], etc.
 cudaError_t launch_simt_gemm(int M, int N, int K, float alpha, const float* A, long long sai,
                              long long sak, const float* Bm, long long sbj, long long sbk,

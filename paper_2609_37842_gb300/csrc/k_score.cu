@@ -29,11 +29,34 @@ struct ModInfo {
   int coff[kMaxU + 1];
 };
 
+// Chunk c of the stored rows' words: module u, words [wc, wc + nw) of it.
+struct Chunk {
+  int u, wc, nw;
+};
+
+__device__ __forceinline__ bool next_chunk(const ModInfo& mi, Chunk& c) {
+  const int wu = mi.off[c.u + 1] - mi.off[c.u];
+  if (c.wc + 32 < wu) {
+    c.wc += 32;
+  } else {
+    ++c.u;
+    c.wc = 0;
+    if (c.u >= mi.U) return false;
+  }
+  c.nw = min(32, mi.off[c.u + 1] - mi.off[c.u] - c.wc);
+  return true;
+}
+
+// Stored rows are staged 256 rows x 32 words at a time in shared memory; the
+// next chunk's words are loaded into registers (128-bit loads) while the
+// current chunk is counted, so loads stay in flight during the popcounts.
+// vec requires every module's word count, ldt and the base to be multiples of
+// 4 words / 16 bytes.
 template <int QT>
 __global__ void __launch_bounds__(256) k_score_codes_smallq(
     const uint32_t* __restrict__ train, int ldt, const float* __restrict__ ts, int ldts, int N,
     const __grid_constant__ ModInfo mi, const uint32_t* __restrict__ query, int ldq,
-    const float* __restrict__ qs, int ldqs, int Q, float* __restrict__ out, int ldo) {
+    const float* __restrict__ qs, int ldqs, int Q, float* __restrict__ out, int ldo, int vec) {
   __shared__ uint32_t Ts[256][33];
   __shared__ uint32_t Qw[QT][32];
   const int tid = threadIdx.x;
@@ -41,50 +64,82 @@ __global__ void __launch_bounds__(256) k_score_codes_smallq(
   const int q0 = blockIdx.y * QT;
   const int i = i0 + tid;
   float acc[QT];
+  int cnt[QT];
 #pragma unroll
-  for (int a = 0; a < QT; ++a) acc[a] = 0.f;
-
-  for (int u = 0; u < mi.U; ++u) {
-    const int w0 = mi.off[u], wu = mi.off[u + 1] - w0;
-    int cnt[QT];
+  for (int a = 0; a < QT; ++a) {
+    acc[a] = 0.f;
+    cnt[a] = 0;
+  }
+  // vector loader: iteration r covers rows r*32 + tid/8, words (tid%8)*4 .. +3
+  const int lrow = tid >> 3, lword = (tid & 7) * 4;
+  uint4 pre[8];
+  auto issue = [&](const Chunk& c) {
+    const int base = mi.off[c.u] + c.wc;
 #pragma unroll
-    for (int a = 0; a < QT; ++a) cnt[a] = 0;
-    for (int wc = 0; wc < wu; wc += 32) {
-      const int nw = min(32, wu - wc);
-      // 256 rows x 32 words, one 128-byte row segment per warp instruction.
+    for (int r = 0; r < 8; ++r) {
+      const int row = i0 + r * 32 + lrow;
+      pre[r] = make_uint4(0, 0, 0, 0);
+      if (row < N && lword < c.nw)
+        pre[r] = __ldcs(reinterpret_cast<const uint4*>(train + static_cast<size_t>(row) * ldt + base + lword));
+    }
+  };
+  Chunk cur{0, 0, min(32, mi.off[1] - mi.off[0])};
+  if (vec) issue(cur);
+  for (;;) {
+    if (vec) {
+#pragma unroll
+      for (int r = 0; r < 8; ++r) {
+        uint32_t* d = &Ts[r * 32 + lrow][lword];
+        d[0] = pre[r].x;
+        d[1] = pre[r].y;
+        d[2] = pre[r].z;
+        d[3] = pre[r].w;
+      }
+    } else {
+      const int base = mi.off[cur.u] + cur.wc;
 #pragma unroll 8
       for (int r = 0; r < 32; ++r) {
         const int e = tid + 256 * r;
         const int row = e >> 5, w = e & 31;
         uint32_t v = 0;
-        if (i0 + row < N && w < nw) v = __ldcs(train + static_cast<size_t>(i0 + row) * ldt + w0 + wc + w);
+        if (i0 + row < N && w < cur.nw) v = __ldcs(train + static_cast<size_t>(i0 + row) * ldt + base + w);
         Ts[row][w] = v;
       }
-      if (tid < QT * 32) {
-        const int a = tid >> 5, w = tid & 31;
-        uint32_t v = 0;
-        if (q0 + a < Q && w < nw) v = query[static_cast<size_t>(q0 + a) * ldq + w0 + wc + w];
-        Qw[a][w] = v;
-      }
-      __syncthreads();
-      for (int w = 0; w < nw; ++w) {
-        const uint32_t t = Ts[tid][w];
-#pragma unroll
-        for (int a = 0; a < QT; ++a) cnt[a] += __popc(t ^ Qw[a][w]);
-      }
-      __syncthreads();
     }
-    if (i < N) {
-      const float si = ts[static_cast<size_t>(i) * ldts + u];
+    if (tid < QT * 32) {
+      const int a = tid >> 5, w = tid & 31;
+      uint32_t v = 0;
+      if (q0 + a < Q && w < cur.nw) v = query[static_cast<size_t>(q0 + a) * ldq + mi.off[cur.u] + cur.wc + w];
+      Qw[a][w] = v;
+    }
+    __syncthreads();
+    Chunk nxt = cur;
+    const bool more = next_chunk(mi, nxt);
+    if (more && vec) issue(nxt);
+    for (int w = 0; w < cur.nw; ++w) {
+      const uint32_t t = Ts[tid][w];
 #pragma unroll
-      for (int a = 0; a < QT; ++a) {
-        if (q0 + a < Q) {
-          const float sq = qs[static_cast<size_t>(q0 + a) * ldqs + u];
-          const float d = static_cast<float>(mi.k[u] - 2 * cnt[a]);
-          acc[a] = __fadd_rn(acc[a], __fmul_rn(__fmul_rn(sq, si), d));
+      for (int a = 0; a < QT; ++a) cnt[a] += __popc(t ^ Qw[a][w]);
+    }
+    const bool module_done = !more || nxt.u != cur.u;
+    if (module_done) {
+      if (i < N) {
+        const float si = ts[static_cast<size_t>(i) * ldts + cur.u];
+#pragma unroll
+        for (int a = 0; a < QT; ++a) {
+          if (q0 + a < Q) {
+            const float sq = qs[static_cast<size_t>(q0 + a) * ldqs + cur.u];
+            const float d = static_cast<float>(mi.k[cur.u] - 2 * cnt[a]);
+            acc[a] = __fadd_rn(acc[a], __fmul_rn(__fmul_rn(sq, si), d));
+          }
         }
       }
+#pragma unroll
+      for (int a = 0; a < QT; ++a) cnt[a] = 0;
     }
+    __syncthreads();
+    if (!more) break;
+    cur = nxt;
   }
   if (i < N) {
 #pragma unroll
@@ -271,11 +326,13 @@ cudaError_t launch_score_codes(const uint32_t* train, int ldt, const float* ts, 
   if (Q <= 8) {
     const int qt = Q <= 1 ? 1 : Q <= 2 ? 2 : Q <= 4 ? 4 : 8;
     dim3 grid((N + 255) / 256, (Q + qt - 1) / qt);
+    int vec = ((ldt & 3) == 0) && ((reinterpret_cast<uintptr_t>(train) & 15) == 0);
+    for (int u = 0; u < U; ++u) vec &= (((ks[u] + 31) / 32) % 4) == 0;
     switch (qt) {
-      case 1: k_score_codes_smallq<1><<<grid, 256, 0, st>>>(train, ldt, ts, ldts, N, local, query, ldq, qs, ldqs, Q, out, ldo); break;
-      case 2: k_score_codes_smallq<2><<<grid, 256, 0, st>>>(train, ldt, ts, ldts, N, local, query, ldq, qs, ldqs, Q, out, ldo); break;
-      case 4: k_score_codes_smallq<4><<<grid, 256, 0, st>>>(train, ldt, ts, ldts, N, local, query, ldq, qs, ldqs, Q, out, ldo); break;
-      default: k_score_codes_smallq<8><<<grid, 256, 0, st>>>(train, ldt, ts, ldts, N, local, query, ldq, qs, ldqs, Q, out, ldo); break;
+      case 1: k_score_codes_smallq<1><<<grid, 256, 0, st>>>(train, ldt, ts, ldts, N, local, query, ldq, qs, ldqs, Q, out, ldo, vec); break;
+      case 2: k_score_codes_smallq<2><<<grid, 256, 0, st>>>(train, ldt, ts, ldts, N, local, query, ldq, qs, ldqs, Q, out, ldo, vec); break;
+      case 4: k_score_codes_smallq<4><<<grid, 256, 0, st>>>(train, ldt, ts, ldts, N, local, query, ldq, qs, ldqs, Q, out, ldo, vec); break;
+      default: k_score_codes_smallq<8><<<grid, 256, 0, st>>>(train, ldt, ts, ldts, N, local, query, ldq, qs, ldqs, Q, out, ldo, vec); break;
     }
   } else {
     dim3 grid((N + 63) / 64, (Q + 63) / 64);

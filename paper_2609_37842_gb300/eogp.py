@@ -322,8 +322,10 @@ def pack_sign(x, codes=None, scales=None, stream=None):
 
 
 def score(train, train_scales, ks: Sequence[int], mode: int, query, query_scales=None, out=None,
-          stream=None):
-    """eogp_score: returns scores [Q, N] fp32."""
+          stream=None, ws=None):
+    """eogp_score: returns scores [Q, N] fp32. A workspace of the size
+    eogp_score_workspace_size asks for is allocated unless `ws` is given (pass an
+    empty tensor to force the popcount kernels)."""
     import torch
     for t, nm in ((train, "train"), (query, "query"), (train_scales, "train_scales"),
                   (query_scales, "query_scales")):
@@ -335,7 +337,12 @@ def score(train, train_scales, ks: Sequence[int], mode: int, query, query_scales
         out = torch.empty((Q, N), dtype=torch.float32, device=train.device)
     ts_ld = train_scales.stride(0) if train_scales is not None else 0
     qs_ld = query_scales.stride(0) if query_scales is not None else 0
+    if ws is None:
+        need = c_size_t()
+        _check(lib().eogp_score_workspace_size(N, karr, len(ks), int(mode), Q, ctypes.byref(need)))
+        ws = workspace(need.value, train.device) if need.value else None
     _check(lib().eogp_score(_ptr(train), train.stride(0), _ptr(train_scales), ts_ld, N, karr,
                             len(ks), int(mode), _ptr(query), query.stride(0), _ptr(query_scales),
-                            qs_ld, Q, _ptr(out), out.stride(0), None, 0, _stream(stream)))
+                            qs_ld, Q, _ptr(out), out.stride(0), _ptr(ws),
+                            ws.numel() if ws is not None else 0, _stream(stream)))
     return out

@@ -61,7 +61,7 @@ def check_bits(x_or, codes, k):
 # ---------------------------------------------------------------- pack_sign
 
 @pytest.mark.parametrize("B,k", [(1, 1), (7, 31), (5, 32), (300, 100), (64, 128), (33, 1000),
-                                 (16, 1024), (3, 16384 + 96)])
+                                 (16, 1024), (3, 16384 + 96), (5000, 1024), (4100, 100)])
 def test_pack_sign(B, k):
     rng = np.random.default_rng(B * 1000 + k)
     x = rng.standard_normal((B, k)).astype(np.float32)
@@ -102,8 +102,11 @@ def rand_store(rng, n, ks):
 
 
 @pytest.mark.parametrize("N,Q,ks", [(1, 1, [32]), (300, 1, [40, 64, 7]), (257, 3, [1024]),
+                                    (1000, 1, [128, 1024]), (513, 5, [256, 2048]),
                                     (1000, 8, [128, 5, 300]), (130, 9, [64, 64]),
-                                    (513, 70, [40, 1024, 7, 33]), (64, 64, [16384])])
+                                    (513, 70, [40, 1024, 7, 33]), (64, 64, [16384]),
+                                    (1000, 64, [128, 1024]), (300, 100, [256]),
+                                    (129, 200, [1024, 128, 2048]), (777, 257, [512] * 5)])
 def test_score_codes_bit_exact(N, Q, ks):
     rng = np.random.default_rng(N * 7 + Q)
     tc, qc = rand_store(rng, N, ks), rand_store(rng, Q, ks)
@@ -119,6 +122,12 @@ def test_score_codes_bit_exact(N, Q, ks):
     want64 = O.score_codes(tc, ts, ks, qc, qs)
     bound = 1e-6 * sum(np.abs(qs[:, u, None] * ts[None, :, u]) * k for u, k in enumerate(ks))
     assert np.all(np.abs(got - want64) <= bound)
+    # the tensor-core and popcount kernels agree bit for bit (an empty workspace
+    # selects the popcount kernels)
+    pop = E.score(dt(tc), dt(ts), ks, E.SCORE_CODES, dt(qc), dt(qs),
+                  ws=torch.empty(0, dtype=torch.uint8, device=DEV))
+    E.sync_status()
+    np.testing.assert_array_equal(pop.cpu().numpy(), got)
 
 
 @pytest.mark.parametrize("N,Q,ks", [(100, 3, [40, 64, 7]), (257, 70, [1024, 33])])
