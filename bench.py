@@ -1,7 +1,7 @@
 #!/usr/bin/env python
 """Throughput of the EOGP hot path on GB300.
 
-One step compresses one batch of B training examples through every module of
+One step compresses one batch of B = 256 training examples through every module of
 the GPT-2-small-shaped stack (48 linears, T = 512 tokens, m = 4096 retained
 first-stage coordinates, k = 1024 PCA coordinates per module) into one-bit
 codes: Kronecker rotations, per-example contraction with the scale-and-gather
@@ -220,13 +220,15 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--batch", type=int, default=128)
+    ap.add_argument("--batch", type=int, default=256)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-score", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--copy-streams", type=int, default=2)
+    ap.add_argument("--e2e-batch", type=int, default=128,
+                    help="examples per e2e step (pinned host staging is sized by it)")
     ap.add_argument("--no-scan", action="store_true")
     ap.add_argument("--modules", type=int, default=0,
                     help="use only the first N modules of the stack (small profiling cases)")
@@ -357,15 +359,17 @@ def main():
     # buffers only after step k's compute of u (event wait on the copy stream).
     e2e = None
     if not args.no_e2e:
+        Be = min(B, args.e2e_batch)
         host = []
         for md in mods:
-            ha = torch.empty(md["a"].shape, dtype=md["a"].dtype, pin_memory=True)
-            hs = torch.empty(md["s"].shape, dtype=md["s"].dtype, pin_memory=True)
-            ha.copy_(md["a"])
-            hs.copy_(md["s"])
+            ha = torch.empty(md["a"][:Be].shape, dtype=md["a"].dtype, pin_memory=True)
+            hs = torch.empty(md["s"][:Be].shape, dtype=md["s"].dtype, pin_memory=True)
+            ha.copy_(md["a"][:Be])
+            hs.copy_(md["s"][:Be])
             host.append((ha, hs))
-        hcodes = torch.empty(codes.shape, dtype=codes.dtype, pin_memory=True)
-        hscales = torch.empty(scales.shape, dtype=scales.dtype, pin_memory=True)
+        ecodes, escales = codes[:Be], scales[:Be]
+        hcodes = torch.empty(ecodes.shape, dtype=codes.dtype, pin_memory=True)
+        hscales = torch.empty(escales.shape, dtype=scales.dtype, pin_memory=True)
         h2d = sum(ha.numel() * ha.element_size() + hs.numel() * hs.element_size() for ha, hs in host)
         d2h = hcodes.numel() * 4 + hscales.numel() * 4
         cstreams = [torch.cuda.Stream() for _ in range(max(1, args.copy_streams))]
@@ -378,19 +382,19 @@ def main():
                 if consumed[u] is not None:
                     cs.wait_event(consumed[u])
                 with torch.cuda.stream(cs):
-                    md["a"].copy_(ha, non_blocking=True)
-                    md["s"].copy_(hs, non_blocking=True)
+                    md["a"][:Be].copy_(ha, non_blocking=True)
+                    md["s"][:Be].copy_(hs, non_blocking=True)
                     landed[u].record(cs)
             for u, md in enumerate(mods):
                 stream.wait_event(landed[u])
-                E.compress_layer(md["desc"], md["a"], md["s"], E.OUT_CODES,
-                                 codes=codes[:, u * words:(u + 1) * words], scales=scales[:, u],
+                E.compress_layer(md["desc"], md["a"][:Be], md["s"][:Be], E.OUT_CODES,
+                                 codes=ecodes[:, u * words:(u + 1) * words], scales=escales[:, u],
                                  ws=ws, stream=stream)
                 ev = torch.cuda.Event()
                 ev.record(stream)
                 consumed[u] = ev
-            hcodes.copy_(codes, non_blocking=True)
-            hscales.copy_(scales, non_blocking=True)
+            hcodes.copy_(ecodes, non_blocking=True)
+            hscales.copy_(escales, non_blocking=True)
 
         e2e_step()
         torch.cuda.synchronize()
@@ -405,7 +409,8 @@ def main():
             tt = torch.tensor([ems], device=dev)
             dist.all_reduce(tt, op=dist.ReduceOp.MAX)
             ems = float(tt.item())
-        e2e = {"value": world * B * args.e2e_steps / (ems / 1000.0), "unit": "examples/s",
+        e2e = {"value": world * Be * args.e2e_steps / (ems / 1000.0), "unit": "examples/s",
+               "batch": Be,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
                "h2d_GBps": h2d * args.e2e_steps / (ems / 1000.0) / 1e9,
                "copy_streams": len(cstreams)}

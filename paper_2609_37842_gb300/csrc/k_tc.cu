@@ -364,7 +364,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[buf]);
+      if (lane == 0) mbar_arrive_relaxed(&tempty[buf]);
     }
   }
   tc_fence_before();
@@ -536,7 +536,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[buf]);
+      if (lane == 0) mbar_arrive_relaxed(&tempty[buf]);
     }
   }
   tc_fence_before();
@@ -546,6 +546,173 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 size_t rotate_smem_bytes(int BN, int stages) {
   return 1024 + static_cast<size_t>(stages) * (kABytes + BN * 128u) + (2 * stages + 4) * 8 + 16;
+}
+
+
+// ------------------------------------------------------------------------
+// k_tc_rotate2 -- the rotation GEMM on CTA pairs (tcgen05 cta_group::2,
+// M = 256). Each CTA of a pair loads its own 128 activation rows and its own
+// half of the BN eigenvector rows (no multicast), so per-SM shared-memory
+// traffic per MMA flop drops by a third against one CTA per tile; the leader
+// CTA (rank 0) issues the M = 256 MMAs, whose accumulator rows are split over
+// the two CTAs' TMEM. Pipeline completion (TMA bytes) and accumulator release
+// are counted on the leader's barriers; MMA completion is multicast to both
+// CTAs. Epilogue as in k_tc_rotate (blocked hi/lo output).
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    k_tc_rotate2(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
+                 const RotArgs g) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const int half = g.BN / 2;  // W rows held by this CTA
+  const uint32_t stage_bytes = kABytes + static_cast<uint32_t>(half) * 128u;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(g.stages) * stage_bytes);
+  uint64_t* empty = full + g.stages;
+  uint64_t* tfull = empty + g.stages;
+  uint64_t* tempty = tfull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  const uint32_t tcols = g.BN <= 64 ? 128u : g.BN <= 128 ? 256u : 512u;
+  const uint32_t bstride = tcols / 2;
+  const int nkb = (g.K + 63) / 64;
+  const int cl = blockIdx.x >> 1, ncl = gridDim.x >> 1;
+
+  if (threadIdx.x == 0) {
+    tma_prefetch_desc(&tmX);
+    tma_prefetch_desc(&tmW);
+    for (int s = 0; s < g.stages; ++s) {
+      mbar_init(&full[s], 2);   // one expect_tx arrive from each CTA (leader's copy is used)
+      mbar_init(&empty[s], 1);  // MMA completion, multicast to both CTAs
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);   // multicast to both CTAs
+      mbar_init(&tempty[b], 8);  // 4 epilogue warps x 2 CTAs (leader's copy is used)
+    }
+    fence_barrier_init();
+  }
+  if (warp == 1) tmem_alloc_pair(tmem_slot, tcols);
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // barriers of both CTAs initialised before any remote arrive
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int t = cl; t < g.n_tiles && ok; t += ncl) {
+        const int m0 = (t / g.nN) * 256 + static_cast<int>(rank) * 128;
+        const int n0 = (t % g.nN) * g.BN + static_cast<int>(rank) * half;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = static_cast<int>(it % g.stages);
+          const uint32_t ph = (it / g.stages) & 1u;
+          if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) {
+            ok = false;
+            break;
+          }
+          const uint32_t st = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
+          const uint32_t fl = mapa_shared(smem_u32(&full[s]), 0);
+          mbar_arrive_expect_tx_cluster(fl, stage_bytes);
+          tma_load_2d_pair(st, &tmX, kb * 64, m0, fl);
+          tma_load_2d_pair(st + kABytes, &tmW, kb * 64, n0, fl);
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      const uint32_t idesc = idesc_bf16_f32(256, g.BN, 0, 0);
+      uint32_t it = 0;
+      int i = 0;
+      bool ok = true;
+      for (int t = cl; t < g.n_tiles && ok; t += ncl, ++i) {
+        const int buf = i & 1;
+        const uint32_t aph = static_cast<uint32_t>(i >> 1) & 1u;
+        if (!mbar_wait(&tempty[buf], aph ^ 1u, g.status)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + buf * bstride;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = static_cast<int>(it % g.stages);
+          const uint32_t ph = (it / g.stages) & 1u;
+          if (!mbar_wait(&full[s], ph, g.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
+          const uint32_t sb = sa + kABytes;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_f16_pair(d, sdesc_sw128(sa + kk * 32, 16, 1024), sdesc_sw128(sb + kk * 32, 16, 1024),
+                            idesc, (kb | kk) != 0 ? 1u : 0u);
+          tc_commit_pair_mc(&empty[s], 0x3);
+        }
+        tc_commit_pair_mc(&tfull[buf], 0x3);
+      }
+    }
+    __syncwarp();
+  } else {
+    const int q = warp & 3;
+    int i = 0;
+    for (int t = cl; t < g.n_tiles; t += ncl, ++i) {
+      const int buf = i & 1;
+      const uint32_t aph = static_cast<uint32_t>(i >> 1) & 1u;
+      uint32_t ok = 1;
+      if (lane == 0) ok = mbar_wait(&tfull[buf], aph, g.status) ? 1u : 0u;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      __syncwarp();
+      tc_fence_after();
+      if (!ok) break;
+      const int m0 = (t / g.nN) * 256 + static_cast<int>(rank) * 128, n0 = (t % g.nN) * g.BN;
+      const int row = m0 + q * 32 + lane;
+      const uint32_t tb = tmem + buf * bstride + (static_cast<uint32_t>(q * 32) << 16);
+      for (int c = 0; c < g.BN; c += 32) {
+        float v[32];
+        tmem_ld32(tb + c, v);
+        const int col = n0 + c;
+        if (row < g.M && col < g.ldo) {
+          uint32_t h[16], l[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * e]);
+            const __nv_bfloat16 h1 = __float2bfloat16_rn(v[2 * e + 1]);
+            h[e] = pack_bf16x2(h0, h1);
+            l[e] = pack_bf16x2(__float2bfloat16_rn(v[2 * e] - __bfloat162float(h0)),
+                               __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1)));
+          }
+          const int bex = row / g.T, tok = row - bex * g.T;
+          const size_t off =
+              ((static_cast<size_t>(bex) * (g.ldo >> 7) + (col >> 7)) * g.T + tok) * 128 + (col & 127);
+          uint32_t w[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w[e] = h[e];
+          st_global_v8(g.hi + off, w);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w[e] = h[8 + e];
+          st_global_v8(g.hi + off + 16, w);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w[e] = l[e];
+          st_global_v8(g.lo + off, w);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w[e] = l[8 + e];
+          st_global_v8(g.lo + off + 16, w);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_relaxed_cluster(mapa_shared(smem_u32(&tempty[buf]), 0));
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // neither CTA leaves while its peer may still signal it
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc_pair(tmem, tcols);
+}
+
+size_t rotate2_smem_bytes(int BN, int stages) {
+  return 1024 + static_cast<size_t>(stages) * (kABytes + (BN / 2) * 128u) + (2 * stages + 4) * 8 + 16;
 }
 
 }  // namespace
@@ -610,6 +777,19 @@ cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, 
   return cudaGetLastError();
 }
 
+// CTA pairs measured faster for short reductions (K <= 1536: the hi/lo
+// epilogue dominates and halving the per-SM operand stream helps) and slower
+// for long ones; EOGP_ROT_PAIRS = 0 / 1 forces one choice.
+static bool rotate_pairs(int K) {
+  static int v = -2;
+  if (v == -2) {
+    const char* e = getenv("EOGP_ROT_PAIRS");
+    v = e ? atoi(e) : -1;
+  }
+  if (v >= 0) return v != 0;
+  return K <= 1536;
+}
+
 int rotate_bn(int ldo) {
   static int forced = -1;
   if (forced < 0) {
@@ -635,7 +815,16 @@ cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W
                              cudaStream_t st) {
   if (M <= 0) return cudaSuccess;
   const int BN = rotate_bn(ldo);
-  const int stages = BN > 128 ? 4 : 5;
+  // As many pipeline stages as fit in 227 KB of shared memory (at most 8);
+  // EOGP_ROT_STAGES overrides for tuning sweeps.
+  static int forced_stages = -1;
+  if (forced_stages < 0) {
+    const char* e = getenv("EOGP_ROT_STAGES");
+    forced_stages = e ? atoi(e) : 0;
+  }
+  int stages = 2;
+  while (stages < 8 && rotate_smem_bytes(BN, stages + 1) <= 232448) ++stages;
+  if (forced_stages >= 2 && rotate_smem_bytes(BN, forced_stages) <= 232448) stages = forced_stages;
   CUtensorMap tX, tW;
   if (tmap_bf16_2d(&tX, X, static_cast<uint64_t>(K), static_cast<uint64_t>(M), ldx, 64, 128) ||
       tmap_bf16_2d(&tW, W, K, Wrows, ldw, 64, BN))
@@ -652,6 +841,23 @@ cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W
   g.hi = static_cast<__nv_bfloat16*>(hi);
   g.lo = static_cast<__nv_bfloat16*>(lo);
   g.status = status;
+  if (rotate_pairs(K) && BN % 32 == 0) {
+    // CTA pairs: tiles of 256 rows, W split in halves of BN / 2 rows.
+    CUtensorMap tWh;
+    if (tmap_bf16_2d(&tWh, W, K, Wrows, ldw, 64, BN / 2)) return cudaErrorInvalidValue;
+    int st2 = 2;
+    while (st2 < 8 && rotate2_smem_bytes(BN, st2 + 1) <= 232448) ++st2;
+    if (forced_stages >= 2 && rotate2_smem_bytes(BN, forced_stages) <= 232448) st2 = forced_stages;
+    g.stages = st2;
+    g.n_tiles = ((M + 255) / 256) * g.nN;
+    const size_t smem = rotate2_smem_bytes(BN, st2);
+    cudaError_t e = cudaFuncSetAttribute(k_tc_rotate2, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    const int clusters = std::min(g.n_tiles, std::max(1, num_sms / 2));
+    k_tc_rotate2<<<2 * clusters, kThreads, smem, st>>>(tX, tWh, g);
+    return cudaGetLastError();
+  }
   const size_t smem = rotate_smem_bytes(BN, stages);
   cudaError_t e = cudaFuncSetAttribute(k_tc_rotate, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));

@@ -84,7 +84,7 @@ def lib() -> ctypes.CDLL:
     """Load libeogp.so (built in-tree by build.py). Raises if it is missing."""
     global _LIB
     if _LIB is None:
-        path = _build.LIB
+        path = os.environ.get("EOGP_LIB") or _build.LIB   # EOGP_LIB: an alternative build
         if not os.path.exists(path):
             raise RuntimeError(f"libeogp.so is not built ({path}); run "
                                "`python -m paper_2609_37842_gb300.build` first")
