@@ -31,6 +31,8 @@ import sys
 import tempfile
 import time
 
+import numpy as np
+
 ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
@@ -40,7 +42,7 @@ METRIC = "training examples compressed/sec per layer stack"
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # dram__bytes_read.sum + dram__bytes_write.sum per rotation launch from the committed
 # ncu capture (profiles/), or None when the kernel changed after the capture.
-ROTATE_TRAFFIC_BYTES = 322.9e6  # mean over one transformer block (8 launches) at B = 128
+ROTATE_TRAFFIC_BYTES = 692.1e6  # mean over one transformer block (8 launches) at B = 256
 
 
 def load_peaks():
@@ -214,6 +216,189 @@ def run_reference(args):
     return 0
 
 
+
+
+# ------------------------------------------------ other workloads (throughput)
+def _config_stack(name, B, dev, gh, g):
+    """Plans, retained eigenvector rows and inputs for one layer's module types of a
+    workload; the per-layer inputs are reused by every layer (the work per layer is
+    identical, and each module's inputs still exceed L2)."""
+    import torch
+    from paper_2609_37842_gb300 import eogp as E
+    from paper_2609_37842_gb300 import synth
+    w = synth.WORKLOADS[name]
+    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    per_layer = {}
+    for u, mod in enumerate(w.modules):
+        key = (mod.d_in, mod.d_out, mod.gelu_input, u % 7 if name.startswith("olmo") else u % 4)
+        if key in per_layer:
+            continue
+        if w.spectrum == "channel":
+            spec = synth.layer_spec(w, u, 1, 1)
+            lamA, lamS = spec.lam_A, spec.lam_S
+        else:
+            lamA = synth.power_spectrum(mod.d_in, w.alpha)
+            lamS = synth.power_spectrum(mod.d_out, w.alpha)
+        plan = E.Plan.from_factors(lamS, lamA, w.m, w.damping_rel)
+        inf = plan.info()
+        R, C = plan.sets()
+        if w.spectrum == "channel":
+            # permutation eigenbasis: row r of V_A[C] is the unit vector at the channel
+            # holding the C[r]-th largest variance
+            pa = np.argsort(-spec.chan_A ** 2, kind="stable")
+            ps = np.argsort(-spec.chan_S ** 2, kind="stable")
+            VA = torch.zeros((inf.nC, mod.d_in), dtype=dt, device=dev)
+            VA[torch.arange(inf.nC), torch.from_numpy(pa[C]).long()] = 1
+            VS = torch.zeros((inf.nR, mod.d_out), dtype=dt, device=dev)
+            VS[torch.arange(inf.nR), torch.from_numpy(ps[R]).long()] = 1
+            sa = torch.from_numpy(spec.chan_A).float().to(dev)
+            ss = torch.from_numpy(spec.chan_S).float().to(dev)
+        else:
+            VA = synth.torch_eigvec_rows(mod.d_in, inf.nC, dev, gh, dt)
+            VS = synth.torch_eigvec_rows(mod.d_out, inf.nR, dev, gh, dt)
+            sa = ss = None
+        a, s = synth.torch_layer_inputs(w, u, B, dev, g)
+        if sa is not None:
+            a = (a.float() * sa).to(dt)
+            s = (s.float() * ss).to(dt)
+        per_layer[key] = dict(plan=plan, VA=VA, VS=VS, a=a, s=s, d_in=mod.d_in, d_out=mod.d_out,
+                              nC=inf.nC, nR=inf.nR)
+    keys = []
+    for u, mod in enumerate(w.modules):
+        keys.append((mod.d_in, mod.d_out, mod.gelu_input, u % 7 if name.startswith("olmo") else u % 4))
+    return w, per_layer, keys
+
+
+def bench_config(name, B, steps, warmup, dev, stream_bases=False):
+    """Examples/s per layer stack for one workload; with stream_bases the retained
+    eigenvector rows of every layer live in pinned host memory and are copied to
+    the device one layer ahead of its compute on a side stream."""
+    import torch
+    from paper_2609_37842_gb300 import eogp as E
+    from paper_2609_37842_gb300 import synth
+    g = torch.Generator(device=dev)
+    g.manual_seed(7)
+    gh = torch.Generator()
+    gh.manual_seed(7)
+    w, per_layer, keys = _config_stack(name, B, dev, gh, g)
+    Pt = synth.torch_eigvec_rows(w.m, w.k, dev, gh,
+                                 torch.bfloat16 if w.dtype == "bf16" else torch.float32)
+    words = (w.k + 31) // 32
+    U = len(w.modules)
+    codes = torch.empty((B, U * words), dtype=torch.int32, device=dev)
+    scales = torch.empty((B, U), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    nmod_layer = len(set(keys))
+    layers = U // nmod_layer if name.startswith("olmo") else 1
+    descs = {}
+    for key, L in per_layer.items():
+        descs[key] = E.layer_desc(L["plan"], w.T, w.k, L["VA"], L["VS"], Pt)
+    ws = E.workspace(max(E.compress_workspace_size(d, B, E.OUT_CODES) for d in descs.values()), dev)
+    host_bases = dev_bases = None
+    if stream_bases:
+        # one pinned host copy per module type (every layer copies it again) and two
+        # device slots, so layer l+1's rows land while layer l computes
+        host_one = {k: (L["VA"].cpu().pin_memory(), L["VS"].cpu().pin_memory())
+                    for k, L in per_layer.items()}
+        host_bases = [host_one] * layers
+        dev_bases = [{k: (torch.empty_like(L["VA"]), torch.empty_like(L["VS"]))
+                      for k, L in per_layer.items()} for _ in range(2)]
+        slot_descs = [{k: E.layer_desc(per_layer[k]["plan"], w.T, w.k, dev_bases[sl][k][0],
+                                       dev_bases[sl][k][1], Pt) for k in per_layer} for sl in range(2)]
+        cstream = torch.cuda.Stream()
+        landed = [torch.cuda.Event() for _ in range(2)]
+        freed = [None, None]
+
+    def step():
+        if not stream_bases:
+            for u, key in enumerate(keys):
+                L = per_layer[key]
+                E.compress_layer(descs[key], L["a"], L["s"], E.OUT_CODES,
+                                 codes=codes[:, u * words:(u + 1) * words], scales=scales[:, u], ws=ws)
+            return
+
+        def issue_copy(layer):
+            sl = layer % 2
+            if freed[sl] is not None:
+                cstream.wait_event(freed[sl])
+            with torch.cuda.stream(cstream):
+                for k in per_layer:
+                    dev_bases[sl][k][0].copy_(host_bases[layer][k][0], non_blocking=True)
+                    dev_bases[sl][k][1].copy_(host_bases[layer][k][1], non_blocking=True)
+                landed[sl].record(cstream)
+        issue_copy(0)
+        for layer in range(layers):
+            sl = layer % 2
+            if layer + 1 < layers:
+                issue_copy(layer + 1)
+            stream.wait_event(landed[sl])
+            for j in range(nmod_layer):
+                u = layer * nmod_layer + j
+                key = keys[u]
+                L = per_layer[key]
+                E.compress_layer(slot_descs[sl][key], L["a"], L["s"], E.OUT_CODES,
+                                 codes=codes[:, u * words:(u + 1) * words], scales=scales[:, u], ws=ws)
+            ev = torch.cuda.Event()
+            ev.record(stream)
+            freed[sl] = ev
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize()
+    E.sync_status()
+    for kk in E.KERNEL_KINDS:
+        E.profile_read(kk, reset=True)
+    E.profile_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    E.profile_enable(False)
+    E.sync_status()
+    ms = e0.elapsed_time(e1)
+    n, rms = E.profile_read(E.K_ROTATE, reset=True)
+    for kk in E.KERNEL_KINDS:
+        E.profile_read(kk, reset=True)
+    rot_flops = sum(2.0 * B * w.T * (per_layer[k]["d_in"] * per_layer[k]["nC"] +
+                                     per_layer[k]["d_out"] * per_layer[k]["nR"]) for k in keys)
+    in_bytes = sum(2.0 * B * w.T * (per_layer[k]["d_in"] + per_layer[k]["d_out"]) for k in keys)
+    sec = ms / 1000.0
+    out = {"examples_per_s": B * steps / sec, "ms_per_step": ms / steps, "batch": B,
+           "modules": U, "T": w.T, "m": w.m, "k": w.k,
+           "rotate_TFLOPs": rot_flops * steps / (rms / 1000.0) / 1e12 if rms else None,
+           "stack_TFLOPs": rot_flops * steps / sec / 1e12,
+           "input_GBps": in_bytes * steps / sec / 1e9,
+           "alg_GFLOP_per_example": rot_flops / B / 1e9,
+           "input_MB_per_example": in_bytes / B / 1e6}
+    if stream_bases:
+        out["eigenbases"] = "host-pinned, one layer ahead on a side stream"
+        out["h2d_bytes_per_step"] = layers * sum(2 * (L["VA"].numel() + L["VS"].numel())
+                                                 for L in per_layer.values())
+    if layers > 1:
+        out["inputs"] = f"one buffer per module type, shared by the {layers} layers"
+    del per_layer, descs, ws
+    torch.cuda.empty_cache()
+    return out
+
+
+def bench_fit(dev, n=10000, m=4096, k=1024):
+    import torch
+    from paper_2609_37842_gb300 import eogp as E
+    g = torch.Generator(device=dev)
+    g.manual_seed(11)
+    col = torch.arange(1, m + 1, device=dev, dtype=torch.float32) ** -0.7
+    Z = torch.randn((n, m), generator=g, device=dev) * col
+    E.fit_pca(Z[:512, :256], 32)   # warm-up (module load)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    Pt, eig = E.fit_pca(Z, k)
+    torch.cuda.synchronize()
+    E.sync_status()
+    return {"n": n, "m": m, "k": k, "seconds": time.perf_counter() - t0,
+            "route": "covariance (m x m) Jacobi, fp64"}
+
 # ------------------------------------------------------------------ main
 def main():
     ap = argparse.ArgumentParser()
@@ -230,6 +415,8 @@ def main():
     ap.add_argument("--e2e-batch", type=int, default=128,
                     help="examples per e2e step (pinned host staging is sized by it)")
     ap.add_argument("--no-scan", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the OLMo / 32B / tiny-fp32 throughput and the PCA-fit timing")
     ap.add_argument("--modules", type=int, default=0,
                     help="use only the first N modules of the stack (small profiling cases)")
     args = ap.parse_args()
@@ -318,7 +505,9 @@ def main():
     peak = peaks.get("bf16_tflops_sustained") or PEAKS_FALLBACK["bf16_tflops_sustained"]
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": (achieved / peak) if achieved else None,
-                "traffic": ROTATE_TRAFFIC_BYTES, "kernel": "k_tc_rotate (Kronecker rotation)",
+                # captured on the full stack's block structure at B = 256 only
+                "traffic": ROTATE_TRAFFIC_BYTES if (B == 256 and U % 4 == 0) else None,
+                "kernel": "k_tc_rotate / k_tc_rotate2 (Kronecker rotations)",
                 "peak_source": f"{peaks_src} bf16_tflops_sustained",
                 "flops_per_launch": flops_per_launch}
 
@@ -473,6 +662,18 @@ def main():
                                      "word_ops_per_s": N * Q * Wsc / (qms / 1000.0)}
         del tr, out
 
+    configs = None
+    fit = None
+    if rank == 0 and not args.no_configs:
+        torch.cuda.empty_cache()
+        configs = {
+            "tiny_f32": bench_config("tiny_f32", 4096, 5, 3, dev),
+            "olmo2_1b_bf16": bench_config("olmo2_1b_bf16", 8, 3, 3, dev),
+            "olmo2_7b_bf16": bench_config("olmo2_7b_bf16", 8, 3, 3, dev, stream_bases=True),
+            "olmo2_32b_gate_bf16": bench_config("olmo2_32b_gate_bf16", 32, 5, 3, dev),
+        }
+        fit = bench_fit(dev)
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         sec, cores, desc = cpu_sample(w, 1)
@@ -489,7 +690,7 @@ def main():
                            "k": w.k, "modules": U, "parallelism": f"replicas x{world}",
                            "l2": "inputs > L2 (B x 151 MB per step)"},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "scoring": scoring,
-                "pack_sign": pack, "scan": scan,
+                "pack_sign": pack, "scan": scan, "other_workloads": configs, "fit_pca": fit,
                 "gpu_launches": launches, "kernels": kern, "clocks": clk}
         print(json.dumps(line))
     if world > 1:
