@@ -358,9 +358,14 @@ def bench_config(name, B, steps, warmup, dev, stream_bases=False):
     E.profile_enable(False)
     E.sync_status()
     ms = e0.elapsed_time(e1)
-    n, rms = E.profile_read(E.K_ROTATE, reset=True)
-    for kk in E.KERNEL_KINDS:
-        E.profile_read(kk, reset=True)
+    kern = {}
+    for kk, nm in E.KERNEL_KINDS.items():
+        n, kms = E.profile_read(kk, reset=True)
+        if n:
+            kern[nm] = {"launches": n, "ms": kms}
+    rms = kern.get("rotate", {}).get("ms", 0.0)
+    peaks, _ = load_peaks()
+    hbm_peak = peaks.get("hbm_gbs") or PEAKS_FALLBACK["hbm_gbs"]
     rot_flops = sum(2.0 * B * w.T * (per_layer[k]["d_in"] * per_layer[k]["nC"] +
                                      per_layer[k]["d_out"] * per_layer[k]["nR"]) for k in keys)
     in_bytes = sum(2.0 * B * w.T * (per_layer[k]["d_in"] + per_layer[k]["d_out"]) for k in keys)
@@ -371,7 +376,9 @@ def bench_config(name, B, steps, warmup, dev, stream_bases=False):
            "stack_TFLOPs": rot_flops * steps / sec / 1e12,
            "input_GBps": in_bytes * steps / sec / 1e9,
            "alg_GFLOP_per_example": rot_flops / B / 1e9,
-           "input_MB_per_example": in_bytes / B / 1e6}
+           "input_MB_per_example": in_bytes / B / 1e6,
+           "input_frac_of_hbm": in_bytes * steps / sec / 1e9 / hbm_peak,
+           "kernels": kern}
     if stream_bases:
         out["eigenbases"] = "host-pinned, one layer ahead on a side stream"
         out["h2d_bytes_per_step"] = layers * sum(2 * (L["VA"].numel() + L["VS"].numel())
@@ -668,9 +675,9 @@ def main():
         torch.cuda.empty_cache()
         configs = {
             "tiny_f32": bench_config("tiny_f32", 4096, 5, 3, dev),
-            "olmo2_1b_bf16": bench_config("olmo2_1b_bf16", 8, 3, 3, dev),
-            "olmo2_7b_bf16": bench_config("olmo2_7b_bf16", 8, 3, 3, dev, stream_bases=True),
-            "olmo2_32b_gate_bf16": bench_config("olmo2_32b_gate_bf16", 32, 5, 3, dev),
+            "olmo2_1b_bf16": bench_config("olmo2_1b_bf16", 128, 3, 3, dev),
+            "olmo2_7b_bf16": bench_config("olmo2_7b_bf16", 32, 3, 3, dev, stream_bases=True),
+            "olmo2_32b_gate_bf16": bench_config("olmo2_32b_gate_bf16", 64, 5, 3, dev),
         }
         fit = bench_fit(dev)
 
