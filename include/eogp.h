@@ -263,14 +263,50 @@ int eogp_score_workspace_size(int N, const int* k_per_module, int U, int mode, i
  *   PAPER: train = codes as above, train_scales as above, query = fp32
  *          coordinates [Q x ld_query] (module u at column sum_{v<u} k_v),
  *          query_scales ignored; scores[q][i] = sum_u s_iu <y_qu, b_iu>.
+ *          With every k_u a multiple of 64 and the workspace
+ *          eogp_score_workspace_size reports (4 Q sum_u k_u bytes), this runs on
+ *          the tensor cores with y split into bf16 hi + lo (about 2^-17 relative)
+ *          and fp32 sums: |error| <= 1e-5 sum_u s_iu ||y_qu||_1 for k_u <= 16384.
  *   FP:    train = fp32 coordinates [N x ld_train], query = fp32 [Q x ld_query];
  *          scores[q][i] = <y_q, x_i>; scales ignored.
  * scores [Q x ld_scores] fp32 device, ld_scores >= N.
+ * ws: 256-byte aligned device workspace of at least eogp_score_workspace_size
+ * bytes (0 bytes for the CUDA-core kernels); CODES and PAPER use the tensor
+ * cores when it is given, the shape allows (CODES: Q >= 64, k_u % 128 == 0;
+ * PAPER: k_u % 64 == 0) and the code rows are aligned (CODES: ld_train % 4 == 0
+ * and a 16-byte aligned base; PAPER: ld_train % 2 == 0, 8-byte base).
  * Errors: EOGP_EINVAL, EOGP_EWORKSPACE, EOGP_ECUDA. */
 int eogp_score(const void* train, int ld_train, const float* train_scales, int ld_tscale, int N,
                const int* k_per_module, int U, int mode, const void* query, int ld_query,
                const float* query_scales, int ld_qscale, int Q, float* scores, int ld_scores,
                void* ws, size_t ws_bytes, eogp_stream_t stream);
+
+/* ---- ranking (App. C: stored examples ranked per query by score, descending;
+ * NDCG@20 reads the first 20) ------------------------------------------- */
+#define EOGP_TOPK_MAX 256
+
+int eogp_score_topk_workspace_size(int N, const int* k_per_module, int U, int mode, int Q,
+                                   int topk, size_t* bytes);
+
+/* Per query, the `topk` best stored rows under the eogp_score definition of
+ * `mode`, without materialising the Q x N scores when the tensor-core kernels
+ * apply and topk <= 64 (the ranking then runs in their epilogue; the Q x N
+ * matrix is never written). Otherwise the scores go to the workspace and a
+ * ranking kernel follows. Arguments as eogp_score, plus:
+ *   top_scores [Q x ld_top_scores] fp32 device and top_index [Q x ld_top_index]
+ *   int32 device (stored row numbers), ld >= topk: row q lists its best rows by
+ *   score descending, equal scores by lower row number; NaN scores never rank;
+ *   places beyond N hold (-inf, -1). CODES scores are bitwise those of
+ *   eogp_score, so the lists are exact.
+ * ws: 256-byte aligned, at least eogp_score_topk_workspace_size bytes.
+ * Errors: EOGP_EINVAL (topk outside [1, EOGP_TOPK_MAX], bad sizes),
+ *   EOGP_EWORKSPACE, EOGP_EUNSUPPORTED (tensor-core shape with code rows not
+ *   aligned as eogp_score's tensor-core path needs), EOGP_ECUDA. */
+int eogp_score_topk(const void* train, int ld_train, const float* train_scales, int ld_tscale,
+                    int N, const int* k_per_module, int U, int mode, const void* query,
+                    int ld_query, const float* query_scales, int ld_qscale, int Q, int topk,
+                    float* top_scores, int ld_top_scores, int* top_index, int ld_top_index,
+                    void* ws, size_t ws_bytes, eogp_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -299,6 +299,25 @@ def score_fp(x_train: np.ndarray, y: np.ndarray) -> np.ndarray:
     return np.asarray(y, np.float64) @ np.asarray(x_train, np.float64).T
 
 
+def top_k(scores: np.ndarray, K: int) -> Tuple[np.ndarray, np.ndarray]:
+    """Per query (row of scores [Q, N]) the K highest-scoring stored examples,
+    best first (App. C: stored examples ranked by score, descending; NDCG@20
+    reads the first 20). Equal scores rank the lower stored index first; NaN
+    scores never rank; places past the ranked examples hold (-inf, -1).
+    Returns (values [Q, K] float64, indices [Q, K] int64)."""
+    scores = np.asarray(scores, np.float64)
+    Q = scores.shape[0]
+    vals = np.full((Q, K), -np.inf)
+    idx = np.full((Q, K), -1, np.int64)
+    for q in range(Q):
+        row = scores[q]
+        cand = np.flatnonzero(~np.isnan(row))
+        order = cand[np.lexsort((cand, -row[cand]))][:K]   # key 1: score desc; key 2: index asc
+        vals[q, :len(order)] = row[order]
+        idx[q, :len(order)] = order
+    return vals, idx
+
+
 # --------------------------------------------------------------------------
 # Storage accounting
 # --------------------------------------------------------------------------

@@ -696,14 +696,78 @@ extern "C" int eogp_pack_sign(const float* x, int B, int k, int ldx, uint32_t* c
   return EOGP_OK;
 }
 
+static bool score_args_ok(int N, const int* ks, int U, long long* W, long long* D) {
+  *W = *D = 0;
+  if (N < 0 || !ks || U < 1 || U > 1024) return false;
+  for (int u = 0; u < U; ++u) {
+    if (ks[u] < 1) return false;
+    *W += (ks[u] + 31) / 32;
+    *D += ks[u];
+  }
+  return true;
+}
+
+// Row alignment the tensor-core scoring kernels load stored code rows with.
+static bool tc_rows_aligned(int mode, const void* train, int ld_train) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(train);
+  return mode == EOGP_SCORE_CODES ? ((ld_train % 4) == 0 && (a & 15) == 0)
+                                  : ((ld_train % 2) == 0 && (a & 7) == 0);
+}
+
 extern "C" int eogp_score_workspace_size(int N, const int* k_per_module, int U, int mode, int Q,
                                          size_t* bytes) {
   clear_error();
   if (!bytes) return set_error(EOGP_EINVAL, "bytes is NULL");
   (void)N;
   *bytes = 0;
-  if (mode == EOGP_SCORE_CODES && k_per_module && U >= 1 && score_tc_supported(k_per_module, U, Q))
-    *bytes = score_tc_ws_bytes(k_per_module, U, Q);
+  if ((mode == EOGP_SCORE_CODES || mode == EOGP_SCORE_PAPER) && k_per_module && U >= 1 &&
+      U <= 1024 && score_tc_supported(mode, k_per_module, U, Q))
+    *bytes = score_tc_ws_bytes(mode, k_per_module, U, Q);
+  return EOGP_OK;
+}
+
+// Dense scoring into `scores`; the tensor-core kernels when the shape, the
+// pointers and the workspace allow, otherwise the CUDA-core kernels.
+static int score_dense(const void* train, int ld_train, const float* train_scales, int ld_tscale,
+                       int N, const int* k_per_module, int U, int mode, const void* query,
+                       int ld_query, const float* query_scales, int ld_qscale, int Q,
+                       float* scores, int ld_scores, void* ws, size_t ws_bytes, long long W,
+                       long long D, cudaStream_t st) {
+  if (mode == EOGP_SCORE_CODES || mode == EOGP_SCORE_PAPER) {
+    if (!train_scales) return set_error(EOGP_EINVAL, "train_scales is NULL");
+    if (mode == EOGP_SCORE_CODES && !query_scales) return set_error(EOGP_EINVAL, "query_scales is NULL");
+    if (ld_train < W || ld_tscale < U ||
+        (mode == EOGP_SCORE_CODES ? (ld_query < W || ld_qscale < U) : ld_query < D))
+      return set_error(EOGP_EINVAL, "leading dimension too small");
+    // Tensor-core path when the caller provided the workspace eogp_score_workspace_size
+    // asks for and the stored rows are aligned for vector loads; CODES scores are
+    // bitwise identical either way.
+    const bool tc = score_tc_supported(mode, k_per_module, U, Q) && ws &&
+                    ws_bytes >= score_tc_ws_bytes(mode, k_per_module, U, Q) &&
+                    tc_rows_aligned(mode, train, ld_train) &&
+                    (reinterpret_cast<uintptr_t>(ws) & 255) == 0;
+    if (tc) {
+      unsigned* status = status_word();
+      if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
+      CUDA_TRY(launch_score_tc(mode, static_cast<const uint32_t*>(train), ld_train, train_scales,
+                               ld_tscale, N, k_per_module, U, query, ld_query, query_scales,
+                               ld_qscale, Q, scores, ld_scores, nullptr, ws, sm_count(), status, st));
+    } else if (mode == EOGP_SCORE_CODES) {
+      CUDA_TRY(launch_score_codes(static_cast<const uint32_t*>(train), ld_train, train_scales,
+                                  ld_tscale, N, k_per_module, U, static_cast<const uint32_t*>(query),
+                                  ld_query, query_scales, ld_qscale, Q, scores, ld_scores, st));
+    } else {
+      CUDA_TRY(launch_score_paper(static_cast<const uint32_t*>(train), ld_train, train_scales, ld_tscale,
+                                  N, k_per_module, U, static_cast<const float*>(query), ld_query, Q,
+                                  scores, ld_scores, st));
+    }
+  } else if (mode == EOGP_SCORE_FP) {
+    if (ld_train < D || ld_query < D) return set_error(EOGP_EINVAL, "leading dimension too small");
+    CUDA_TRY(launch_simt_gemm(Q, N, static_cast<int>(D), 1.f, static_cast<const float*>(query), ld_query,
+                              1, static_cast<const float*>(train), ld_train, 1, scores, ld_scores, st));
+  } else {
+    return set_error(EOGP_EINVAL, "bad score mode");
+  }
   return EOGP_OK;
 }
 
@@ -714,52 +778,113 @@ extern "C" int eogp_score(const void* train, int ld_train, const float* train_sc
                           eogp_stream_t stream) {
   clear_error();
   if (N < 0 || Q < 0) return set_error(EOGP_EINVAL, "N, Q must be >= 0");
-  if (!k_per_module || U < 1 || U > 1024) return set_error(EOGP_EINVAL, "need 1 <= U <= 1024 modules");
-  long long W = 0, D = 0;
-  for (int u = 0; u < U; ++u) {
-    if (k_per_module[u] < 1) return set_error(EOGP_EINVAL, "k_per_module must be >= 1");
-    W += (k_per_module[u] + 31) / 32;
-    D += k_per_module[u];
-  }
+  long long W, D;
+  if (!score_args_ok(N, k_per_module, U, &W, &D))
+    return set_error(EOGP_EINVAL, "need 1 <= U <= 1024 modules with k_per_module >= 1");
+  if (mode != EOGP_SCORE_CODES && mode != EOGP_SCORE_PAPER && mode != EOGP_SCORE_FP)
+    return set_error(EOGP_EINVAL, "bad score mode");
   if (N == 0 || Q == 0) return EOGP_OK;
   if (!train || !query || !scores) return set_error(EOGP_EINVAL, "NULL argument");
   if (ld_scores < N) return set_error(EOGP_EINVAL, "ld_scores < N");
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   ProfScope ps(EOGP_K_SCORE, st);
-  if (mode == EOGP_SCORE_CODES) {
-    if (!train_scales || !query_scales) return set_error(EOGP_EINVAL, "scales are NULL");
-    if (ld_train < W || ld_query < W || ld_tscale < U || ld_qscale < U)
-      return set_error(EOGP_EINVAL, "leading dimension too small");
-    // Tensor-core path when the caller provided the workspace eogp_score_workspace_size
-    // asks for (Q >= 64, every k_u a multiple of 128, 16-byte aligned code rows);
-    // otherwise the popcount kernels. Both give bitwise identical scores.
-    const bool tc = score_tc_supported(k_per_module, U, Q) && ws &&
-                    ws_bytes >= score_tc_ws_bytes(k_per_module, U, Q) && (ld_train % 4) == 0 &&
-                    aligned16(train) && (reinterpret_cast<uintptr_t>(ws) & 255) == 0;
-    if (tc) {
-      unsigned* status = status_word();
-      if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
-      CUDA_TRY(launch_score_tc(static_cast<const uint32_t*>(train), ld_train, train_scales, ld_tscale,
-                               N, k_per_module, U, static_cast<const uint32_t*>(query), ld_query,
-                               query_scales, ld_qscale, Q, scores, ld_scores, ws, sm_count(), status,
-                               st));
-    } else {
-      CUDA_TRY(launch_score_codes(static_cast<const uint32_t*>(train), ld_train, train_scales,
-                                  ld_tscale, N, k_per_module, U, static_cast<const uint32_t*>(query),
-                                  ld_query, query_scales, ld_qscale, Q, scores, ld_scores, st));
-    }
-  } else if (mode == EOGP_SCORE_PAPER) {
-    if (!train_scales) return set_error(EOGP_EINVAL, "train_scales is NULL");
-    if (ld_train < W || ld_query < D || ld_tscale < U) return set_error(EOGP_EINVAL, "leading dimension too small");
-    CUDA_TRY(launch_score_paper(static_cast<const uint32_t*>(train), ld_train, train_scales, ld_tscale,
-                                N, k_per_module, U, static_cast<const float*>(query), ld_query, Q,
-                                scores, ld_scores, st));
-  } else if (mode == EOGP_SCORE_FP) {
-    if (ld_train < D || ld_query < D) return set_error(EOGP_EINVAL, "leading dimension too small");
-    CUDA_TRY(launch_simt_gemm(Q, N, static_cast<int>(D), 1.f, static_cast<const float*>(query), ld_query,
-                              1, static_cast<const float*>(train), ld_train, 1, scores, ld_scores, st));
+  return score_dense(train, ld_train, train_scales, ld_tscale, N, k_per_module, U, mode, query,
+                     ld_query, query_scales, ld_qscale, Q, scores, ld_scores, ws, ws_bytes, W, D, st);
+}
+
+// ---------------------------------------------------------------- top-K
+// Workspace plan of eogp_score_topk: fused (tensor-core scoring with the ranking in
+// its epilogue) or dense (scores into the workspace, then a ranking kernel).
+struct TopkPlan {
+  bool fused;
+  int slots;
+  size_t q_bytes, dense_bytes, list_bytes, total;
+};
+
+static TopkPlan topk_plan(int N, const int* ks, int U, int mode, int Q, int K) {
+  TopkPlan p{};
+  const bool tc_ok = (mode == EOGP_SCORE_CODES || mode == EOGP_SCORE_PAPER) &&
+                     score_tc_supported(mode, ks, U, Q);
+  p.fused = tc_ok && score_tc_topk_fits(mode, Q, K);
+  p.q_bytes = tc_ok ? score_tc_ws_bytes(mode, ks, U, Q) : 0;
+  if (p.fused) {
+    p.slots = score_tc_grid(N, Q, sm_count());
+    p.dense_bytes = 0;
   } else {
-    return set_error(EOGP_EINVAL, "bad score mode");
+    p.slots = topk_dense_slots(N);
+    p.dense_bytes = al256(static_cast<size_t>(Q) * ((static_cast<size_t>(N) + 3) & ~size_t(3)) * 4);
   }
+  p.list_bytes = al256(static_cast<size_t>(p.slots) * Q * K * 4);
+  p.total = al256(p.q_bytes) + p.dense_bytes + 2 * p.list_bytes;
+  return p;
+}
+
+extern "C" int eogp_score_topk_workspace_size(int N, const int* k_per_module, int U, int mode, int Q,
+                                              int topk, size_t* bytes) {
+  clear_error();
+  if (!bytes) return set_error(EOGP_EINVAL, "bytes is NULL");
+  long long W, D;
+  if (!score_args_ok(N, k_per_module, U, &W, &D) || Q < 0)
+    return set_error(EOGP_EINVAL, "need N, Q >= 0 and 1 <= U <= 1024 modules with k_per_module >= 1");
+  if (topk < 1 || topk > EOGP_TOPK_MAX) return set_error(EOGP_EINVAL, "topk must be in [1, %d]", EOGP_TOPK_MAX);
+  *bytes = Q == 0 ? 0 : topk_plan(N, k_per_module, U, mode, Q, topk).total;
+  return EOGP_OK;
+}
+
+extern "C" int eogp_score_topk(const void* train, int ld_train, const float* train_scales,
+                               int ld_tscale, int N, const int* k_per_module, int U, int mode,
+                               const void* query, int ld_query, const float* query_scales,
+                               int ld_qscale, int Q, int topk, float* top_scores, int ld_top_scores,
+                               int* top_index, int ld_top_index, void* ws, size_t ws_bytes,
+                               eogp_stream_t stream) {
+  clear_error();
+  if (N < 0 || Q < 0) return set_error(EOGP_EINVAL, "N, Q must be >= 0");
+  long long W, D;
+  if (!score_args_ok(N, k_per_module, U, &W, &D))
+    return set_error(EOGP_EINVAL, "need 1 <= U <= 1024 modules with k_per_module >= 1");
+  if (mode != EOGP_SCORE_CODES && mode != EOGP_SCORE_PAPER && mode != EOGP_SCORE_FP)
+    return set_error(EOGP_EINVAL, "bad score mode");
+  if (topk < 1 || topk > EOGP_TOPK_MAX) return set_error(EOGP_EINVAL, "topk must be in [1, %d]", EOGP_TOPK_MAX);
+  if (Q == 0) return EOGP_OK;
+  if (!top_scores || !top_index) return set_error(EOGP_EINVAL, "NULL output");
+  if (ld_top_scores < topk || ld_top_index < topk) return set_error(EOGP_EINVAL, "output leading dimension < topk");
+  if (N > 0 && (!train || !query)) return set_error(EOGP_EINVAL, "NULL argument");
+  const TopkPlan p = topk_plan(N, k_per_module, U, mode, Q, topk);
+  if (!ws || ws_bytes < p.total) return set_error(EOGP_EWORKSPACE, "workspace too small: need %zu bytes", p.total);
+  if ((reinterpret_cast<uintptr_t>(ws) & 255) != 0) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  void* qws = w;
+  float* dense = reinterpret_cast<float*>(w + al256(p.q_bytes));
+  float* lst = reinterpret_cast<float*>(w + al256(p.q_bytes) + p.dense_bytes);
+  int* lsi = reinterpret_cast<int*>(w + al256(p.q_bytes) + p.dense_bytes + p.list_bytes);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  ProfScope ps(EOGP_K_SCORE, st);
+  if (p.fused && N > 0) {
+    if (!train_scales || (mode == EOGP_SCORE_CODES && !query_scales))
+      return set_error(EOGP_EINVAL, "scales are NULL");
+    if (ld_train < W || ld_tscale < U ||
+        (mode == EOGP_SCORE_CODES ? (ld_query < W || ld_qscale < U) : ld_query < D))
+      return set_error(EOGP_EINVAL, "leading dimension too small");
+    if (!tc_rows_aligned(mode, train, ld_train))
+      return set_error(EOGP_EUNSUPPORTED, mode == EOGP_SCORE_CODES
+                                              ? "fused top-K needs 16-byte aligned code rows (ld_train % 4 == 0)"
+                                              : "fused top-K needs 8-byte aligned code rows (ld_train % 2 == 0)");
+    unsigned* status = status_word();
+    if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
+    TcTopK tk{topk, lst, lsi, top_scores, ld_top_scores, top_index, ld_top_index};
+    CUDA_TRY(launch_score_tc(mode, static_cast<const uint32_t*>(train), ld_train, train_scales, ld_tscale,
+                             N, k_per_module, U, query, ld_query, query_scales, ld_qscale, Q, nullptr,
+                             0, &tk, qws, sm_count(), status, st));
+    return EOGP_OK;
+  }
+  const int ldd = (N + 3) & ~3;
+  if (N > 0) {
+    const int rc = score_dense(train, ld_train, train_scales, ld_tscale, N, k_per_module, U, mode, query,
+                               ld_query, query_scales, ld_qscale, Q, dense, ldd, qws, p.q_bytes, W, D, st);
+    if (rc != EOGP_OK) return rc;
+  }
+  CUDA_TRY(launch_topk_dense(dense, ldd, Q, N, topk, lst, lsi, st));
+  CUDA_TRY(launch_topk_merge(lst, lsi, topk_dense_slots(N), Q, topk, top_scores, ld_top_scores, top_index,
+                             ld_top_index, st));
   return EOGP_OK;
 }

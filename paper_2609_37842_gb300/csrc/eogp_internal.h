@@ -81,13 +81,34 @@ cudaError_t launch_score_paper(const uint32_t* train, int ldt, const float* ts, 
                                const int* ks, int U, const float* y, int ldy, int Q, float* out,
                                int ldo, cudaStream_t st);
 
-// k_score_tc.cu: CODES scoring on the tensor cores (e4m3 +-1 operands).
-bool score_tc_supported(const int* ks, int U, int Q);
-size_t score_tc_ws_bytes(const int* ks, int U, int Q);
-cudaError_t launch_score_tc(const uint32_t* train, int ldt, const float* ts, int ldts, int N,
-                            const int* ks, int U, const uint32_t* query, int ldq, const float* qs,
-                            int ldqs, int Q, float* out, int ldo, void* ws, int num_sms,
-                            unsigned* status, cudaStream_t st);
+// k_score_tc.cu: CODES (e4m3 +-1 operands) and PAPER (bf16 hi/lo query x bf16 +-1
+// codes) scoring on the tensor cores, dense output or fused top-K.
+constexpr int kTopKMax = 64;  // largest K of the fused top-K
+struct TcTopK {
+  int K;
+  float* lst;  // per-CTA lists [grid][Q][K] (workspace)
+  int* lsi;
+  float* out_s;  // final [Q, K] scores / stored indices
+  int ld_os;
+  int* out_i;
+  int ld_oi;
+};
+bool score_tc_supported(int mode, const int* ks, int U, int Q);
+size_t score_tc_ws_bytes(int mode, const int* ks, int U, int Q);
+int score_tc_grid(int N, int Q, int num_sms);
+bool score_tc_topk_fits(int mode, int Q, int K);
+cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const float* ts, int ldts, int N,
+                            const int* ks, int U, const void* query, int ldq, const float* qs,
+                            int ldqs, int Q, float* out, int ldo, const TcTopK* topk, void* ws,
+                            int num_sms, unsigned* status, cudaStream_t st);
+
+// k_topk.cu: top-K of a dense [Q, N] score matrix into per-slot lists, and the
+// merge of per-slot lists [S][Q][K] (index -1 = empty) into [Q, K].
+int topk_dense_slots(int N);
+cudaError_t launch_topk_dense(const float* scores, int ld, int Q, int N, int K, float* lst, int* lsi,
+                              cudaStream_t st);
+cudaError_t launch_topk_merge(const float* lst, const int* lsi, int S, int Q, int K, float* out_s,
+                              int ld_os, int* out_i, int ld_oi, cudaStream_t st);
 
 // k_simt.cu: C[i][j] = alpha * sum_k A(i,k) B(j,k), A(i,k) = A[i*sai + k*sak], etc.
 cudaError_t launch_simt_gemm(int M, int N, int K, float alpha, const float* A, long long sai,

@@ -1,27 +1,46 @@
-// One-bit scoring on the tensor cores (CODES mode, Sec. 3.3 Eq. onebit_influence
-// with both sides one-bit; App. B.3 scan).
+// Scoring on the tensor cores (Sec. 3.3 Eq. onebit_influence; App. B.3 scan),
+// in two modes and with two outputs.
 //
-// For module u the +-1 inner product d_u = <b_q, b_i> is an integer with
-// |d_u| <= k_u. Both sides are expanded to e4m3 bytes (+1 = 0x38, -1 = 0xB8,
-// exact) and multiplied with tcgen05.mma kind::f8f6f4 into fp32 TMEM: every
-// partial sum is an integer far below 2^24, so d_u is exact. The epilogue then
-// dequantises in the same fixed fp32 order as the popcount kernels,
-//   acc = fl(acc + fl(fl(s_qu * s_iu) * d_u))   in module order,
-// keeping acc in TMEM between modules, so scores are bitwise identical to the
-// popcount path and to the oracle's float32 evaluation.
+// CODES: both sides one-bit. For module u the +-1 inner product d_u = <b_q, b_i>
+//   is an integer with |d_u| <= k_u. Both sides are expanded to e4m3 bytes
+//   (+1 = 0x38, -1 = 0xB8, exact) and multiplied with tcgen05.mma kind::f8f6f4
+//   into fp32 TMEM: every partial sum is an integer far below 2^24, so d_u is
+//   exact. The epilogue dequantises in the same fixed fp32 order as the
+//   popcount kernels, acc = fl(acc + fl(fl(s_qu * s_iu) * d_u)) in module order,
+//   keeping acc in TMEM between modules, so scores are bitwise identical to the
+//   popcount path and to the oracle's float32 evaluation.
+// PAPER: the query stays unquantised (the paper's asymmetric score
+//   sum_u s_iu <y_u, b_iu>). y is split into bf16 hi + lo (y - hi rounded again),
+//   stored bits are expanded to bf16 +-1, and two kind::f16 MMAs (hi, lo) add
+//   into one fp32 accumulator per module: products are exact, the split keeps
+//   y to about 2^-17 relative, and the MMA sums in fp32. The epilogue forms
+//   acc = fl(acc + fl(s_iu * d_u)) in module order.
+//
+// Output: either the dense [Q, N] score matrix, or (TOPK) only each query's K
+// best stored rows. In the TOPK epilogue the last module's scores of a tile
+// are staged 32 query columns at a time in shared memory and the thread that
+// owns a query column merges them into that query's sorted list (score
+// descending, equal scores by lower stored index). A CTA's lists cover the
+// stored rows of its tiles and go to global memory when the CTA moves to the
+// next query tile; a separate kernel merges the per-CTA lists. The Q x N
+// matrix never reaches HBM.
 //
 // Tiles: 128 stored rows (MMA M, operand A) x BNq <= 128 queries (MMA N,
-// operand B), K = 128 code bits per pipeline stage. Queries are expanded once
-// per call into the workspace and fetched by TMA; stored rows are expanded from
+// operand B). Queries are prepared once per call in the workspace (e4m3 bytes,
+// or bf16 hi and lo rows) and fetched by TMA; stored rows are expanded from
 // their bits into shared memory (128-byte swizzled rows) by four warps, so the
 // store is read from HBM as bits. Tiles run query-tile-major: one query tile
 // stays in L2 while the stored codes stream past it.
 //
 // Warps: 0-3 expand stored rows (warp 0 lane 0 also issues the query TMA),
-// 4-7 dequantise (TMEM lane quarters 0-3), 8 owns TMEM and issues the MMAs.
-// TMEM: two 128-column d_u buffers (module u+1 accumulates while module u is
-// dequantised) and a 128-column running score.
+// 4-7 dequantise (TMEM lane quarters 0-3; in TOPK, thread t also owns query
+// column t), 8 owns TMEM and issues the MMAs. TMEM: two 128-column d_u
+// buffers (module u+1 accumulates while module u is dequantised) and a
+// 128-column running score.
+#include <cuda_bf16.h>
+
 #include <algorithm>
+#include <cmath>
 
 #include "eogp_dev.cuh"
 #include "eogp_internal.h"
@@ -32,20 +51,61 @@ namespace {
 
 constexpr int kMaxMods = 1024;
 constexpr int kThreadsTc = 288;
-constexpr int kStages = 4;
 constexpr uint32_t kAB = 16384u;  // 128 rows x 128 bytes
+constexpr int kTbStride = 129;    // staged column stride (floats): conflict-free both ways
 
 struct ScoreTcArgs {
-  int N, Q, U, BNq, n_it, n_tiles, ldt, ldts, ldqs, ldo;
+  int N, Q, U, BNq, n_it, n_tiles, ldt, ldts, ldqs, ldo, K;
   const uint32_t* train;
   const float* ts;
   const float* qs;
   float* out;
+  float* lst;  // TOPK: per-CTA lists [gridDim.x][Q][K]
+  int* lsi;
   unsigned* status;
-  int k[kMaxMods];     // bits per module (multiple of 128)
+  int k[kMaxMods];     // bits per module
   int woff[kMaxMods];  // word offset of module u in a stored row
-  int boff[kMaxMods];  // byte offset of module u in an expanded query row
+  int boff[kMaxMods];  // offset of module u in a prepared query row (bytes CODES, elements PAPER)
 };
+
+template <int MODE>
+struct TcMode;
+template <>
+struct TcMode<EOGP_SCORE_CODES> {
+  static constexpr int kBits = 128;  // code bits per pipeline stage
+  static constexpr int kQBoxes = 1;  // query operand tiles per stage
+};
+template <>
+struct TcMode<EOGP_SCORE_PAPER> {
+  static constexpr int kBits = 64;
+  static constexpr int kQBoxes = 2;  // hi, lo
+};
+
+template <int MODE, bool TOPK>
+constexpr int tc_stages() {
+  return (MODE == EOGP_SCORE_PAPER && TOPK) ? 3 : 4;
+}
+
+template <int MODE>
+constexpr uint32_t tc_stage_bytes() {
+  return kAB * (1 + TcMode<MODE>::kQBoxes);
+}
+
+// Shared-memory carve-up (byte offsets after 1024-byte alignment).
+struct TcSmem {
+  uint32_t sq, bars, tb, lists, total;
+};
+template <int MODE, bool TOPK>
+__host__ __device__ inline TcSmem tc_smem_layout(int BNq, int K) {
+  constexpr int S = tc_stages<MODE, TOPK>();
+  TcSmem l;
+  l.sq = S * tc_stage_bytes<MODE>();
+  l.bars = l.sq + 128 * 4;
+  l.tb = l.bars + (2 * S + 4) * 8 + 16;
+  l.lists = l.tb + (TOPK ? 32 * kTbStride * 4 : 0);
+  l.total = l.lists + (TOPK ? static_cast<uint32_t>(BNq) * K * 8 : 0);
+  return l;
+}
 
 // 8 code bits -> 8 e4m3 bytes (bit j -> byte j: +1 if set, -1 if clear).
 __device__ __forceinline__ uint64_t expand8(uint32_t v) {
@@ -54,22 +114,37 @@ __device__ __forceinline__ uint64_t expand8(uint32_t v) {
   return 0xB8B8B8B8B8B8B8B8ull ^ x;
 }
 
+// 4 code bits -> 4 bf16 values (bit j -> element j: +1 = 0x3F80 if set, -1 = 0xBF80 if
+// clear). Each 16-bit lane isolates its bit at position j, then adding 0x8000 - 2^j
+// carries into bit 15 exactly when the bit is set.
+__device__ __forceinline__ uint64_t expand4_bf16(uint32_t v) {
+  uint64_t x = (static_cast<uint64_t>(v & 0xFu) * 0x0001000100010001ull) & 0x0008000400020001ull;
+  x = (x + 0x7FF87FFC7FFE7FFFull) & 0x8000800080008000ull;
+  return 0xBF80BF80BF80BF80ull ^ x;
+}
+
+template <int MODE, bool TOPK>
 __global__ void __launch_bounds__(kThreadsTc, 1)
-    k_score_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ ScoreTcArgs g) {
+    k_score_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQlo,
+               const __grid_constant__ ScoreTcArgs g) {
+  constexpr int S = tc_stages<MODE, TOPK>();
+  constexpr uint32_t kStage = tc_stage_bytes<MODE>();
+  constexpr int kBits = TcMode<MODE>::kBits;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
+  const TcSmem L = tc_smem_layout<MODE, TOPK>(g.BNq, g.K);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  constexpr uint32_t kStage = 2 * kAB;
-  float* sq = reinterpret_cast<float*>(smem + kStages * kStage);  // [128] query scales of module u
-  uint64_t* full = reinterpret_cast<uint64_t*>(sq + 128);
-  uint64_t* empty = full + kStages;
-  uint64_t* dfull = empty + kStages;
+  float* sq = reinterpret_cast<float*>(smem + L.sq);  // [128] query scales of module u (CODES)
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bars);
+  uint64_t* empty = full + S;
+  uint64_t* dfull = empty + S;
   uint64_t* dempty = dfull + 2;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(dempty + 2);
 
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tmQ);
-    for (int s = 0; s < kStages; ++s) {
+    if (MODE == EOGP_SCORE_PAPER) tma_prefetch_desc(&tmQlo);
+    for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 5);  // TMA transaction arrive + 4 expander warps
       mbar_init(&empty[s], 1);
     }
@@ -97,10 +172,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       const bool rv = i0 + r < g.N;
       const uint32_t* crow = g.train + static_cast<size_t>(rv ? i0 + r : 0) * g.ldt;
       for (int u = 0; u < g.U && ok; ++u) {
-        const int nkb = g.k[u] >> 7;
+        const int nkb = g.k[u] / kBits;
         for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const int s = static_cast<int>(it % kStages);
-          const uint32_t ph = (it / kStages) & 1u;
+          const int s = static_cast<int>(it % S);
+          const uint32_t ph = (it / S) & 1u;
           uint32_t w_ok = 1;
           if (lane == 0) w_ok = mbar_wait(&empty[s], ph ^ 1u, g.status) ? 1u : 0u;
           w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
@@ -110,22 +185,43 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
           }
           uint8_t* st = smem + static_cast<size_t>(s) * kStage;
           if (warp == 0 && lane == 0) {
-            mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(g.BNq) * 128u);
-            tma_load_2d(st + kAB, &tmQ, g.boff[u] + kb * 128, q0, &full[s]);
+            mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(g.BNq) * 128u * TcMode<MODE>::kQBoxes);
+            if (MODE == EOGP_SCORE_CODES) {
+              tma_load_2d(st + kAB, &tmQ, g.boff[u] + kb * 128, q0, &full[s]);
+            } else {
+              tma_load_2d(st + kAB, &tmQ, g.boff[u] + kb * 64, q0, &full[s]);
+              tma_load_2d(st + 2 * kAB, &tmQlo, g.boff[u] + kb * 64, q0, &full[s]);
+            }
           }
-          uint4 bits = make_uint4(0, 0, 0, 0);
-          if (rv) bits = __ldg(reinterpret_cast<const uint4*>(crow + g.woff[u] + kb * 4));
-          const uint32_t wv[4] = {bits.x, bits.y, bits.z, bits.w};
+          if (MODE == EOGP_SCORE_CODES) {
+            uint4 bits = make_uint4(0, 0, 0, 0);
+            if (rv) bits = __ldg(reinterpret_cast<const uint4*>(crow + g.woff[u] + kb * 4));
+            const uint32_t wv[4] = {bits.x, bits.y, bits.z, bits.w};
 #pragma unroll
-          for (int c = 0; c < 8; ++c) {  // 16 bits -> 16 bytes per swizzled 16-byte chunk
-            const uint32_t h = wv[c >> 1] >> ((c & 1) * 16);
-            const uint64_t lo = expand8(h), hi = expand8(h >> 8);
-            uint4 v;
-            v.x = static_cast<uint32_t>(lo);
-            v.y = static_cast<uint32_t>(lo >> 32);
-            v.z = static_cast<uint32_t>(hi);
-            v.w = static_cast<uint32_t>(hi >> 32);
-            *reinterpret_cast<uint4*>(st + row_off + ((c ^ (r & 7)) << 4)) = v;
+            for (int c = 0; c < 8; ++c) {  // 16 bits -> 16 bytes per swizzled 16-byte chunk
+              const uint32_t h = wv[c >> 1] >> ((c & 1) * 16);
+              const uint64_t lo = expand8(h), hi = expand8(h >> 8);
+              uint4 v;
+              v.x = static_cast<uint32_t>(lo);
+              v.y = static_cast<uint32_t>(lo >> 32);
+              v.z = static_cast<uint32_t>(hi);
+              v.w = static_cast<uint32_t>(hi >> 32);
+              *reinterpret_cast<uint4*>(st + row_off + ((c ^ (r & 7)) << 4)) = v;
+            }
+          } else {
+            uint2 bits = make_uint2(0, 0);
+            if (rv) bits = __ldg(reinterpret_cast<const uint2*>(crow + g.woff[u] + kb * 2));
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {  // 8 bits -> 8 bf16 per swizzled 16-byte chunk
+              const uint32_t h = (c < 4 ? bits.x : bits.y) >> ((c & 3) * 8);
+              const uint64_t lo = expand4_bf16(h), hi = expand4_bf16(h >> 4);
+              uint4 v;
+              v.x = static_cast<uint32_t>(lo);
+              v.y = static_cast<uint32_t>(lo >> 32);
+              v.z = static_cast<uint32_t>(hi);
+              v.w = static_cast<uint32_t>(hi >> 32);
+              *reinterpret_cast<uint4*>(st + row_off + ((c ^ (r & 7)) << 4)) = v;
+            }
           }
           fence_proxy_async_smem();
           __syncwarp();
@@ -136,20 +232,44 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   } else if (warp < 8) {
     // ---------------------------------------------------------- dequantise
     const int q4 = warp & 3;
-    const int ep = threadIdx.x - 128;
+    const int ep = threadIdx.x - 128;  // TMEM lane (stored row in the tile); TOPK: query column
     const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
+    float* tb = reinterpret_cast<float*>(smem + L.tb);
+    float* ls = reinterpret_cast<float*>(smem + L.lists) + static_cast<size_t>(ep) * g.K;
+    int* li = reinterpret_cast<int*>(smem + L.lists + static_cast<size_t>(g.BNq) * g.K * 4) +
+              static_cast<size_t>(ep) * g.K;
+    int seg_qt = -1, cnt = 0;
+    float tau = -INFINITY;
+    auto flush = [&]() {
+      const int q = seg_qt * g.BNq + ep;
+      if (ep < g.BNq && q < g.Q) {
+        const size_t o = (static_cast<size_t>(blockIdx.x) * g.Q + q) * g.K;
+        for (int p = 0; p < g.K; ++p) {
+          g.lst[o + p] = p < cnt ? ls[p] : -INFINITY;
+          g.lsi[o + p] = p < cnt ? li[p] : -1;
+        }
+      }
+    };
     uint32_t gm = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < g.n_tiles && ok; tile += gridDim.x) {
       const int qt = tile / g.n_it, ib = tile % g.n_it;
       const int i0 = ib * 128, q0 = qt * g.BNq;
-      const int row = i0 + q4 * 32 + lane;
+      const int row = i0 + ep;
+      if (TOPK && qt != seg_qt) {
+        if (seg_qt >= 0) flush();
+        seg_qt = qt;
+        cnt = 0;
+        tau = -INFINITY;
+      }
       for (int u = 0; u < g.U; ++u, ++gm) {
         const int buf = static_cast<int>(gm & 1u);
         const uint32_t dph = (gm >> 1) & 1u;
-        named_bar_sync(1, 128);  // previous module's readers of sq are done
-        if (ep < g.BNq) sq[ep] = q0 + ep < g.Q ? g.qs[static_cast<size_t>(q0 + ep) * g.ldqs + u] : 0.f;
-        named_bar_sync(1, 128);
+        if (MODE == EOGP_SCORE_CODES) {
+          named_bar_sync(1, 128);  // previous module's readers of sq are done
+          if (ep < g.BNq) sq[ep] = q0 + ep < g.Q ? g.qs[static_cast<size_t>(q0 + ep) * g.ldqs + u] : 0.f;
+          named_bar_sync(1, 128);
+        }
         uint32_t w_ok = 1;
         if (lane == 0) w_ok = mbar_wait(&dfull[buf], dph, g.status) ? 1u : 0u;
         w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
@@ -160,6 +280,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
           break;
         }
         const float si = row < g.N ? g.ts[static_cast<size_t>(row) * g.ldts + u] : 0.f;
+        const bool last = u + 1 == g.U;
         for (int c0 = 0; c0 < g.BNq; c0 += 32) {
           float d[32], a[32];
           tmem_ld32(tmem + lane_base + buf * 128u + c0, d);
@@ -169,14 +290,47 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
           } else {
             tmem_ld32(tmem + lane_base + 256u + c0, a);
           }
+          if (MODE == EOGP_SCORE_CODES) {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) a[j] = __fadd_rn(a[j], __fmul_rn(__fmul_rn(sq[c0 + j], si), d[j]));
-          if (u + 1 < g.U) {
+            for (int j = 0; j < 32; ++j) a[j] = __fadd_rn(a[j], __fmul_rn(__fmul_rn(sq[c0 + j], si), d[j]));
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) a[j] = __fadd_rn(a[j], __fmul_rn(si, d[j]));
+          }
+          if (!last) {
             tmem_st32(tmem + lane_base + 256u + c0, a);
-          } else if (row < g.N) {
-#pragma unroll 8
-            for (int j = 0; j < 32; ++j)
-              if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
+          } else if (!TOPK) {
+            if (row < g.N) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
+            }
+          } else {
+            // Stage these 32 query columns column-major; the warp owning them ranks them.
+#pragma unroll
+            for (int j = 0; j < 32; ++j) tb[j * kTbStride + ep] = a[j];
+            named_bar_sync(3, 128);
+            if ((ep >> 5) == (c0 >> 5) && q0 + ep < g.Q) {
+              const int nr = min(128, g.N - i0);
+              const float* col = tb + lane * kTbStride;
+              for (int r = 0; r < nr; ++r) {
+                const float v = col[r];
+                const bool take = cnt < g.K ? (v == v) : (v > tau);
+                if (take) {
+                  int p = cnt < g.K ? cnt : g.K - 1;
+                  while (p > 0 && ls[p - 1] < v) {
+                    ls[p] = ls[p - 1];
+                    li[p] = li[p - 1];
+                    --p;
+                  }
+                  ls[p] = v;
+                  li[p] = i0 + r;
+                  if (cnt < g.K) ++cnt;
+                  if (cnt == g.K) tau = ls[g.K - 1];
+                }
+              }
+            }
+            named_bar_sync(3, 128);
           }
         }
         tc_fence_before();
@@ -184,10 +338,12 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
         if (lane == 0) mbar_arrive(&dempty[buf]);
       }
     }
+    if (TOPK && seg_qt >= 0) flush();
   } else {
     // ---------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      const uint32_t idesc = idesc_e4m3_f32(128, g.BNq);
+      const uint32_t idesc =
+          MODE == EOGP_SCORE_CODES ? idesc_e4m3_f32(128, g.BNq) : idesc_bf16_f32(128, g.BNq, 0, 0);
       uint32_t it = 0, gm = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < g.n_tiles && ok; tile += gridDim.x) {
@@ -200,10 +356,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
           }
           tc_fence_after();
           const uint32_t d = tmem + buf * 128u;
-          const int nkb = g.k[u] >> 7;
+          const int nkb = g.k[u] / kBits;
           for (int kb = 0; kb < nkb; ++kb, ++it) {
-            const int s = static_cast<int>(it % kStages);
-            const uint32_t ph = (it / kStages) & 1u;
+            const int s = static_cast<int>(it % S);
+            const uint32_t ph = (it / S) & 1u;
             if (!mbar_wait(&full[s], ph, g.status)) {
               ok = false;
               break;
@@ -211,9 +367,16 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
             tc_fence_after();
             const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * kStage);
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              tc_mma_f8(d, sdesc_sw128(sa + kk * 32, 16, 1024), sdesc_sw128(sa + kAB + kk * 32, 16, 1024),
-                        idesc, (kb | kk) != 0 ? 1u : 0u);
+            for (int kk = 0; kk < 4; ++kk) {
+              const uint64_t ad = sdesc_sw128(sa + kk * 32, 16, 1024);
+              const uint32_t acc = (kb | kk) != 0 ? 1u : 0u;
+              if (MODE == EOGP_SCORE_CODES) {
+                tc_mma_f8(d, ad, sdesc_sw128(sa + kAB + kk * 32, 16, 1024), idesc, acc);
+              } else {
+                tc_mma_f16(d, ad, sdesc_sw128(sa + kAB + kk * 32, 16, 1024), idesc, acc);
+                tc_mma_f16(d, ad, sdesc_sw128(sa + 2 * kAB + kk * 32, 16, 1024), idesc, 1u);
+              }
+            }
             tc_commit(&empty[s]);
           }
           tc_commit(&dfull[buf]);
@@ -246,45 +409,93 @@ __global__ void k_expand_queries(const uint32_t* __restrict__ query, int ldq, in
   }
 }
 
-size_t score_tc_smem() {
-  return 1024 + kStages * 2 * kAB + 128 * 4 + (2 * kStages + 4) * 8 + 16;
+// Query coordinates y (fp32) -> bf16 hi = rn(y) and lo = rn(y - hi), dense rows of D.
+__global__ void k_split_queries(const float* __restrict__ y, int ldq, int D,
+                                __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __restrict__ lo) {
+  const int q = blockIdx.y;
+  for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < D; c += gridDim.x * blockDim.x) {
+    const float v = y[static_cast<size_t>(q) * ldq + c];
+    const __nv_bfloat16 h = __float2bfloat16_rn(v);
+    hi[static_cast<size_t>(q) * D + c] = h;
+    lo[static_cast<size_t>(q) * D + c] = __float2bfloat16_rn(v - __bfloat162float(h));
+  }
+}
+
+int bnq_for(int Q) { return std::min(128, (Q + 31) / 32 * 32); }
+
+template <int MODE, bool TOPK>
+cudaError_t launch_tc_kernel(const CUtensorMap& t0, const CUtensorMap& t1, const ScoreTcArgs& g,
+                             int grid, cudaStream_t st) {
+  const size_t smem = 1024 + tc_smem_layout<MODE, TOPK>(g.BNq, g.K).total;
+  cudaError_t e = cudaFuncSetAttribute(k_score_tc<MODE, TOPK>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  k_score_tc<MODE, TOPK><<<grid, kThreadsTc, smem, st>>>(t0, t1, g);
+  return cudaGetLastError();
 }
 
 }  // namespace
 
-bool score_tc_supported(const int* ks, int U, int Q) {
-  if (Q < 64 || Q > 65535 || U < 1 || U > kMaxMods) return false;
-  for (int u = 0; u < U; ++u)
-    if (ks[u] <= 0 || ks[u] % 128) return false;
-  return true;
+bool score_tc_supported(int mode, const int* ks, int U, int Q) {
+  if (U < 1 || U > kMaxMods || Q < 1 || Q > 65535) return false;
+  if (mode == EOGP_SCORE_CODES) {
+    if (Q < 64) return false;  // the popcount kernels are faster for a handful of queries
+    for (int u = 0; u < U; ++u)
+      if (ks[u] <= 0 || ks[u] % 128) return false;
+    return true;
+  }
+  if (mode == EOGP_SCORE_PAPER) {
+    for (int u = 0; u < U; ++u)
+      if (ks[u] <= 0 || ks[u] % 64) return false;
+    return true;
+  }
+  return false;
 }
 
-size_t score_tc_ws_bytes(const int* ks, int U, int Q) {
+size_t score_tc_ws_bytes(int mode, const int* ks, int U, int Q) {
   long long D = 0;
   for (int u = 0; u < U; ++u) D += ks[u];
-  return (static_cast<size_t>(Q) * D + 255) & ~size_t(255);
+  const size_t per = mode == EOGP_SCORE_PAPER ? 4 : 1;  // bf16 hi + lo, or e4m3
+  return (static_cast<size_t>(Q) * D * per + 255) & ~size_t(255);
 }
 
-cudaError_t launch_score_tc(const uint32_t* train, int ldt, const float* ts, int ldts, int N,
-                            const int* ks, int U, const uint32_t* query, int ldq, const float* qs,
-                            int ldqs, int Q, float* out, int ldo, void* ws, int num_sms,
-                            unsigned* status, cudaStream_t st) {
+int score_tc_grid(int N, int Q, int num_sms) {
+  const long long tiles =
+      static_cast<long long>((N + 127) / 128) * ((Q + bnq_for(Q) - 1) / bnq_for(Q));
+  return static_cast<int>(std::max<long long>(1, std::min<long long>(tiles, std::max(1, num_sms))));
+}
+
+bool score_tc_topk_fits(int mode, int Q, int K) {
+  if (K < 1 || K > kTopKMax) return false;
+  const size_t need = 1024 + (mode == EOGP_SCORE_PAPER
+                                  ? tc_smem_layout<EOGP_SCORE_PAPER, true>(bnq_for(Q), K).total
+                                  : tc_smem_layout<EOGP_SCORE_CODES, true>(bnq_for(Q), K).total);
+  return need <= 232448;
+}
+
+cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const float* ts, int ldts, int N,
+                            const int* ks, int U, const void* query, int ldq, const float* qs,
+                            int ldqs, int Q, float* out, int ldo, const TcTopK* topk, void* ws,
+                            int num_sms, unsigned* status, cudaStream_t st) {
   if (N <= 0 || Q <= 0) return cudaSuccess;
   ScoreTcArgs g;  // ~12 KB parameter block, copied at launch
   g.N = N;
   g.Q = Q;
   g.U = U;
-  g.BNq = std::min(128, (Q + 31) / 32 * 32);
+  g.BNq = bnq_for(Q);
   g.n_it = (N + 127) / 128;
   g.n_tiles = g.n_it * ((Q + g.BNq - 1) / g.BNq);
   g.ldt = ldt;
   g.ldts = ldts;
   g.ldqs = ldqs;
   g.ldo = ldo;
+  g.K = topk ? topk->K : 0;
   g.train = train;
   g.ts = ts;
   g.qs = qs;
   g.out = out;
+  g.lst = topk ? topk->lst : nullptr;
+  g.lsi = topk ? topk->lsi : nullptr;
   g.status = status;
   int wo = 0, bo = 0;
   for (int u = 0; u < U; ++u) {
@@ -294,26 +505,49 @@ cudaError_t launch_score_tc(const uint32_t* train, int ldt, const float* ts, int
     wo += ks[u] / 32;
     bo += ks[u];
   }
-  const int row_bytes = bo;
-  uint8_t* qx = static_cast<uint8_t*>(ws);
-  {
-    dim3 grid(std::max(1, std::min((row_bytes / 32 + 255) / 256, 64)), Q);
-    k_expand_queries<<<grid, 256, 0, st>>>(query, ldq, row_bytes, qx);
+  const int D = bo;
+  const int grid = score_tc_grid(N, Q, num_sms);
+  CUtensorMap t0, t1;
+  if (mode == EOGP_SCORE_CODES) {
+    uint8_t* qx = static_cast<uint8_t*>(ws);
+    dim3 eg(std::max(1, std::min((D / 32 + 255) / 256, 64)), Q);
+    k_expand_queries<<<eg, 256, 0, st>>>(static_cast<const uint32_t*>(query), ldq, D, qx);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
+    const uint64_t dims[2] = {static_cast<uint64_t>(D), static_cast<uint64_t>(Q)};
+    const uint64_t strides[1] = {static_cast<uint64_t>(D)};
+    const uint32_t box[2] = {128, static_cast<uint32_t>(g.BNq)};
+    if (make_tmap(&t0, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, qx, dims, strides, box,
+                  CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+    t1 = t0;
+  } else {
+    __nv_bfloat16* hi = static_cast<__nv_bfloat16*>(ws);
+    __nv_bfloat16* lo = hi + static_cast<size_t>(Q) * D;
+    dim3 eg(std::max(1, std::min((D + 255) / 256, 64)), Q);
+    k_split_queries<<<eg, 256, 0, st>>>(static_cast<const float*>(query), ldq, D, hi, lo);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const uint64_t dims[2] = {static_cast<uint64_t>(D), static_cast<uint64_t>(Q)};
+    const uint64_t strides[1] = {static_cast<uint64_t>(D) * 2};
+    const uint32_t box[2] = {64, static_cast<uint32_t>(g.BNq)};
+    if (make_tmap(&t0, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, hi, dims, strides, box,
+                  CU_TENSOR_MAP_SWIZZLE_128B) ||
+        make_tmap(&t1, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, lo, dims, strides, box,
+                  CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
   }
-  CUtensorMap tq;
-  const uint64_t dims[2] = {static_cast<uint64_t>(row_bytes), static_cast<uint64_t>(Q)};
-  const uint64_t strides[1] = {static_cast<uint64_t>(row_bytes)};
-  const uint32_t box[2] = {128, static_cast<uint32_t>(g.BNq)};
-  if (make_tmap(&tq, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, qx, dims, strides, box,
-                CU_TENSOR_MAP_SWIZZLE_128B))
-    return cudaErrorInvalidValue;
-  const size_t smem = score_tc_smem();
-  cudaError_t e = cudaFuncSetAttribute(k_score_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
-  const int grid = std::min(g.n_tiles, std::max(1, num_sms));
-  k_score_tc<<<grid, kThreadsTc, smem, st>>>(tq, g);
-  return cudaGetLastError();
+  if (topk) {
+    // List entries a CTA never fills keep index -1 and are skipped by the merge.
+    cudaError_t e =
+        cudaMemsetAsync(topk->lsi, 0xFF, static_cast<size_t>(grid) * Q * topk->K * sizeof(int), st);
+    if (e != cudaSuccess) return e;
+    e = mode == EOGP_SCORE_CODES ? launch_tc_kernel<EOGP_SCORE_CODES, true>(t0, t1, g, grid, st)
+                                 : launch_tc_kernel<EOGP_SCORE_PAPER, true>(t0, t1, g, grid, st);
+    if (e != cudaSuccess) return e;
+    return launch_topk_merge(topk->lst, topk->lsi, grid, Q, topk->K, topk->out_s, topk->ld_os,
+                             topk->out_i, topk->ld_oi, st);
+  }
+  return mode == EOGP_SCORE_CODES ? launch_tc_kernel<EOGP_SCORE_CODES, false>(t0, t1, g, grid, st)
+                                  : launch_tc_kernel<EOGP_SCORE_PAPER, false>(t0, t1, g, grid, st);
 }

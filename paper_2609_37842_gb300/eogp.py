@@ -20,6 +20,7 @@ OK, EINVAL, EUNSUPPORTED, ECUDA, ETIMEOUT, EWORKSPACE, EDEVICE = 0, -1, -2, -3, 
 F32, BF16 = 0, 1
 OUT_FIRST_STAGE, OUT_COORDS, OUT_CODES = 0, 1, 2
 SCORE_CODES, SCORE_PAPER, SCORE_FP = 0, 1, 2
+TOPK_MAX = 256
 K_ROTATE, K_CONTRACT, K_PROJECT, K_PACK, K_SCORE, K_SIMT = range(6)
 KERNEL_KINDS = {K_ROTATE: "rotate", K_CONTRACT: "contract", K_PROJECT: "project", K_PACK: "pack",
                 K_SCORE: "score", K_SIMT: "simt_f32"}
@@ -75,6 +76,11 @@ EXPORTS = {
     "eogp_score": (c_int, [c_void_p, c_int, c_void_p, c_int, c_int, c_void_p, c_int, c_int,
                            c_void_p, c_int, c_void_p, c_int, c_int, c_void_p, c_int, c_void_p,
                            c_size_t, c_void_p]),
+    "eogp_score_topk_workspace_size": (c_int, [c_int, c_void_p, c_int, c_int, c_int, c_int,
+                                               POINTER(c_size_t)]),
+    "eogp_score_topk": (c_int, [c_void_p, c_int, c_void_p, c_int, c_int, c_void_p, c_int, c_int,
+                                c_void_p, c_int, c_void_p, c_int, c_int, c_int, c_void_p, c_int,
+                                c_void_p, c_int, c_void_p, c_size_t, c_void_p]),
 }
 
 _LIB = None
@@ -346,3 +352,33 @@ def score(train, train_scales, ks: Sequence[int], mode: int, query, query_scales
                             qs_ld, Q, _ptr(out), out.stride(0), _ptr(ws),
                             ws.numel() if ws is not None else 0, _stream(stream)))
     return out
+
+
+def score_topk(train, train_scales, ks: Sequence[int], mode: int, query, topk: int,
+               query_scales=None, ws=None, stream=None):
+    """eogp_score_topk: per query the `topk` best stored rows. Returns
+    (scores [Q, topk] fp32, index [Q, topk] int32), score descending, equal
+    scores by lower row; (-inf, -1) past N."""
+    import torch
+    for t, nm in ((train, "train"), (query, "query"), (train_scales, "train_scales"),
+                  (query_scales, "query_scales")):
+        _rows(t, nm)
+    N = train.shape[0]
+    Q = query.shape[0]
+    dev = query.device
+    karr = (c_int * len(ks))(*[int(k) for k in ks])
+    top_s = torch.empty((Q, topk), dtype=torch.float32, device=dev)
+    top_i = torch.empty((Q, topk), dtype=torch.int32, device=dev)
+    if ws is None:
+        need = c_size_t()
+        _check(lib().eogp_score_topk_workspace_size(N, karr, len(ks), int(mode), Q, int(topk),
+                                                    ctypes.byref(need)))
+        ws = workspace(need.value, dev)
+    ts_ld = train_scales.stride(0) if train_scales is not None else 0
+    qs_ld = query_scales.stride(0) if query_scales is not None else 0
+    _check(lib().eogp_score_topk(_ptr(train), train.stride(0), _ptr(train_scales), ts_ld, N, karr,
+                                 len(ks), int(mode), _ptr(query), query.stride(0),
+                                 _ptr(query_scales), qs_ld, Q, int(topk), _ptr(top_s),
+                                 top_s.stride(0), _ptr(top_i), top_i.stride(0), _ptr(ws), ws.numel(),
+                                 _stream(stream)))
+    return top_s, top_i

@@ -128,3 +128,32 @@ def test_host_argument_checks():
     ks = (ctypes.c_int * 2)(32, 0)
     assert L.eogp_score(16, 2, 16, 2, 4, ks, 2, 0, 16, 2, 16, 2, 4, 16, 4, None, 0, None) == E.EINVAL
     assert L.eogp_compress_workspace_size(None, 1, 0, ctypes.byref(n)) == E.EINVAL
+
+
+def test_topk_host_argument_checks():
+    L = E.lib()
+    import ctypes
+    n = ctypes.c_size_t()
+    ks = (ctypes.c_int * 2)(1024, 1024)
+    for bad_k in (0, E.TOPK_MAX + 1):
+        assert L.eogp_score_topk_workspace_size(100, ks, 2, E.SCORE_CODES, 64, bad_k,
+                                                ctypes.byref(n)) == E.EINVAL
+    assert L.eogp_score_topk_workspace_size(100, ks, 2, E.SCORE_CODES, 64, 10, ctypes.byref(n)) == E.OK
+    assert n.value > 0
+    assert L.eogp_score_topk_workspace_size(100, ks, 2, E.SCORE_CODES, 0, 10, ctypes.byref(n)) == E.OK
+    assert n.value == 0
+    # bad mode, bad topk, missing outputs: rejected before any device work
+    args = [16, 32, 16, 2, 100, ks, 2, 7, 16, 32, 16, 2, 64, 10, 16, 10, 16, 10, 256, 1 << 20, None]
+    assert L.eogp_score_topk(*args) == E.EINVAL
+    args[7] = E.SCORE_CODES
+    args[13] = 0
+    assert L.eogp_score_topk(*args) == E.EINVAL
+    args[13] = 10
+    args[14] = None
+    assert L.eogp_score_topk(*args) == E.EINVAL
+    args[14] = 16
+    args[15] = 5     # ld_top_scores < topk
+    assert L.eogp_score_topk(*args) == E.EINVAL
+    args[15] = 10
+    args[19] = 0     # workspace too small
+    assert L.eogp_score_topk(*args) == E.EWORKSPACE

@@ -341,6 +341,31 @@ def test_norm_preservation():
     assert np.sum(R1 * R2) == pytest.approx(np.sum(G1 * G2), rel=1e-12)
 
 
+def check_topk(Om, seed):
+    """Ranking by brute force: Python's sort of (-score, index) pairs over the
+    non-NaN scores, on rows with planted ties, NaNs, -inf and fewer rows than K."""
+    rng = np.random.default_rng(seed)
+    Q, N, K = 6, 23, 8
+    sc = rng.integers(-4, 5, (Q, N)).astype(np.float64)   # many equal scores
+    sc[1, ::3] = np.nan
+    sc[2, :] = np.nan
+    sc[2, 5] = 1.5
+    sc[3, 7] = -np.inf
+    sc[4] = rng.standard_normal(N)
+    for Kq, rows in ((K, sc), (30, sc[:2])):               # K > N: tail must be (-inf, -1)
+        vals, idx = Om.top_k(rows, Kq)
+        for q in range(rows.shape[0]):
+            pairs = sorted((-rows[q, i], i) for i in range(rows.shape[1]) if not math.isnan(rows[q, i]))
+            want = pairs[:Kq]
+            assert [int(i) for i in idx[q, :len(want)]] == [i for _, i in want]
+            assert list(vals[q, :len(want)]) == [-v for v, _ in want]
+            assert (idx[q, len(want):] == -1).all() and (vals[q, len(want):] == -np.inf).all()
+
+
+def test_topk_brute_force():
+    check_topk(O, 31)
+
+
 def _golden_rows(name):
     with open(os.path.join(GOLDEN, name)) as f:
         return [ln.split() for ln in f if ln.strip() and not ln.startswith("#")]
@@ -422,3 +447,18 @@ def test_planted_bit_order_is_caught(monkeypatch):
     orig = O.pack_bits
     monkeypatch.setattr(O, "pack_bits", lambda b: orig(np.asarray(b)[..., ::-1]))
     assert _fails(check_packing, O, 19)
+
+
+def test_planted_topk_mistakes_are_caught(monkeypatch):
+    orig = O.top_k
+    def later_index_first(scores, K):        # equal scores ranked by higher index
+        v, i = orig(np.asarray(scores)[:, ::-1], K)
+        n = np.asarray(scores).shape[1]
+        return v, np.where(i >= 0, n - 1 - i, -1)
+    monkeypatch.setattr(O, "top_k", later_index_first)
+    assert _fails(check_topk, O, 31)
+
+    def nan_ranks(scores, K):                # NaN treated as the lowest score instead of dropped
+        return orig(np.nan_to_num(np.asarray(scores, np.float64), nan=-1e300), K)
+    monkeypatch.setattr(O, "top_k", nan_ranks)
+    assert _fails(check_topk, O, 31)
