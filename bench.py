@@ -454,6 +454,7 @@ def main():
     B, T, U = args.batch, w.T, len(w.modules)
     words = (w.k + 31) // 32
     peaks, peaks_src = load_peaks()
+    bf16_burst = peaks.get("bf16_tflops") or PEAKS_FALLBACK["bf16_tflops"]
 
     mods = build_stack(w, B, dev, seed=1000 + rank)
     ws_bytes = max(E.compress_workspace_size(md["desc"], B, E.OUT_CODES) for md in mods)
@@ -543,10 +544,45 @@ def main():
         torch.cuda.synchronize()
         E.sync_status()
         sms = e0.elapsed_time(e1) / reps
-        words_total = N * Q * U * words
+        D = U * w.k
+        f8_peak = 2.0 * bf16_burst          # e4m3 dense = 2 x bf16 dense (nominal ratio)
+        alg = 2.0 * N * Q * D               # +-1 multiply-adds of the inner products
         scoring = {"metric": "query x train scores/sec", "value": N * Q / (sms / 1000.0),
-                   "unit": "scores/s", "ms_per_call": sms, "N": N, "Q": Q, "bits": U * w.k,
-                   "mode": "CODES (xor-popcount)", "word_ops_per_s": words_total / (sms / 1000.0)}
+                   "unit": "scores/s", "ms_per_call": sms, "N": N, "Q": Q, "bits": D,
+                   "mode": "CODES (tcgen05 kind::f8f6f4, +-1 e4m3 operands)",
+                   "tensor_TFLOPs": alg / (sms / 1000.0) / 1e12,
+                   "tensor_frac": alg / (sms / 1000.0) / 1e12 / f8_peak,
+                   "tensor_peak": f8_peak, "tensor_peak_source": f"2 x {peaks_src} bf16_tflops (e4m3)"}
+        # paper mode (unquantised queries), dense and with the ranking fused (K = 20)
+        y = torch.randn((Q, D), generator=g, device=dev)
+        wsp = E.workspace(E.score_workspace_size(N, ks, E.SCORE_PAPER, Q), dev)
+
+        def timed(fn, reps=3):
+            fn()
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(reps):
+                fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            E.sync_status()
+            return a.elapsed_time(b) / reps
+
+        pms = timed(lambda: E.score(tc, tsc, ks, E.SCORE_PAPER, y, out=out, ws=wsp))
+        scoring["paper_dense"] = {"ms_per_call": pms, "scores_per_s": N * Q / (pms / 1000.0),
+                                  "tensor_TFLOPs_issued": 2 * alg / (pms / 1000.0) / 1e12,
+                                  "tensor_frac_issued": 2 * alg / (pms / 1000.0) / 1e12 / bf16_burst,
+                                  "note": "bf16 hi + lo query split: 2 MMAs per algorithmic one"}
+        del out
+        K = 20
+        wtc = E.workspace(E.score_topk_workspace_size(N, ks, E.SCORE_CODES, Q, K), dev)
+        wtp = E.workspace(E.score_topk_workspace_size(N, ks, E.SCORE_PAPER, Q, K), dev)
+        cms = timed(lambda: E.score_topk(tc, tsc, ks, E.SCORE_CODES, qc, K, query_scales=qsc, ws=wtc))
+        tms = timed(lambda: E.score_topk(tc, tsc, ks, E.SCORE_PAPER, y, K, ws=wtp))
+        scoring["codes_top20"] = {"ms_per_call": cms, "scores_per_s": N * Q / (cms / 1000.0)}
+        scoring["paper_top20"] = {"ms_per_call": tms, "scores_per_s": N * Q / (tms / 1000.0)}
+        del y, wsp, wtc, wtp
 
     # ---- end to end through the public API with host buffers ----
     # Per module: host -> device copy of (a, s) on a copy stream, then the
@@ -663,10 +699,31 @@ def main():
             E.sync_status()
             qms = e0.elapsed_time(e1)
             byts = len(chunks) * (N * Wsc * 4 + N * 4) + Q * N * 4
-            scan["per_Q"][str(Q)] = {"ms": qms, "scores_per_s": N * Q / (qms / 1000.0),
-                                     "GBps": byts / (qms / 1000.0) / 1e9,
-                                     "frac_of_hbm": byts / (qms / 1000.0) / 1e9 / hbm,
-                                     "word_ops_per_s": N * Q * Wsc / (qms / 1000.0)}
+            ent = {"ms": qms, "scores_per_s": N * Q / (qms / 1000.0),
+                   "GBps": byts / (qms / 1000.0) / 1e9,
+                   "frac_of_hbm": byts / (qms / 1000.0) / 1e9 / hbm}
+            if Q >= 64:   # tensor-core kernel: +-1 multiply-adds against the e4m3 peak
+                tfl = 2.0 * N * ksc * Q / (qms / 1000.0) / 1e12
+                ent.update({"kernel": "k_score_tc", "tensor_TFLOPs": tfl,
+                            "tensor_frac": tfl / (2.0 * bf16_burst)})
+            else:
+                ent.update({"kernel": "k_score_codes_smallq (popcount)",
+                            "word_ops_per_s": N * Q * Wsc / (qms / 1000.0)})
+            if Q >= 1024:  # per-query top 20 in the scoring epilogue: no Q x N output
+                K = 20
+                wt = E.workspace(E.score_topk_workspace_size(N, [ksc], E.SCORE_CODES, Q, K), dev)
+                E.score_topk(tr, tsc, [ksc], E.SCORE_CODES, qc, K, query_scales=qs, ws=wt)
+                torch.cuda.synchronize()
+                e0.record(stream)
+                E.score_topk(tr, tsc, [ksc], E.SCORE_CODES, qc, K, query_scales=qs, ws=wt)
+                e1.record(stream)
+                torch.cuda.synchronize()
+                E.sync_status()
+                kms = e0.elapsed_time(e1)
+                ent["top20"] = {"ms": kms, "scores_per_s": N * Q / (kms / 1000.0),
+                                "output_bytes_avoided": Q * N * 4}
+                del wt
+            scan["per_Q"][str(Q)] = ent
         del tr, out
 
     configs = None

@@ -44,6 +44,7 @@
 
 #include "eogp_dev.cuh"
 #include "eogp_internal.h"
+#include "topk_dev.cuh"
 
 using namespace eogp;
 
@@ -55,7 +56,7 @@ constexpr uint32_t kAB = 16384u;  // 128 rows x 128 bytes
 constexpr int kTbStride = 129;    // staged column stride (floats): conflict-free both ways
 
 struct ScoreTcArgs {
-  int N, Q, U, BNq, n_it, n_tiles, ldt, ldts, ldqs, ldo, K;
+  int N, Q, U, D, BNq, n_it, n_tiles, ldt, ldts, ldqs, ldo, K;
   const uint32_t* train;
   const float* ts;
   const float* qs;
@@ -64,8 +65,6 @@ struct ScoreTcArgs {
   int* lsi;
   unsigned* status;
   int k[kMaxMods];     // bits per module
-  int woff[kMaxMods];  // word offset of module u in a stored row
-  int boff[kMaxMods];  // offset of module u in a prepared query row (bytes CODES, elements PAPER)
 };
 
 template <int MODE>
@@ -74,11 +73,13 @@ template <>
 struct TcMode<EOGP_SCORE_CODES> {
   static constexpr int kBits = 128;  // code bits per pipeline stage
   static constexpr int kQBoxes = 1;  // query operand tiles per stage
+  using Bits = uint4;                // one stage of one stored row
 };
 template <>
 struct TcMode<EOGP_SCORE_PAPER> {
   static constexpr int kBits = 64;
   static constexpr int kQBoxes = 2;  // hi, lo
+  using Bits = uint2;
 };
 
 template <int MODE, bool TOPK>
@@ -123,6 +124,46 @@ __device__ __forceinline__ uint64_t expand4_bf16(uint32_t v) {
   return 0xBF80BF80BF80BF80ull ^ x;
 }
 
+// One stage of one stored row -> its 128-byte swizzled shared-memory row
+// (16-byte chunk c goes to position c ^ (row & 7)).
+__device__ __forceinline__ void expand_stage(uint8_t* dst, int sw, uint4 bits) {  // 128 bits -> e4m3
+  const uint32_t wv[4] = {bits.x, bits.y, bits.z, bits.w};
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const uint32_t h = wv[c >> 1] >> ((c & 1) * 16);
+    const uint64_t lo = expand8(h), hi = expand8(h >> 8);
+    *reinterpret_cast<uint4*>(dst + ((c ^ sw) << 4)) =
+        make_uint4(static_cast<uint32_t>(lo), static_cast<uint32_t>(lo >> 32), static_cast<uint32_t>(hi),
+                   static_cast<uint32_t>(hi >> 32));
+  }
+}
+__device__ __forceinline__ void expand_stage(uint8_t* dst, int sw, uint2 bits) {  // 64 bits -> bf16
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const uint32_t h = (c < 4 ? bits.x : bits.y) >> ((c & 3) * 8);
+    const uint64_t lo = expand4_bf16(h), hi = expand4_bf16(h >> 4);
+    *reinterpret_cast<uint4*>(dst + ((c ^ sw) << 4)) =
+        make_uint4(static_cast<uint32_t>(lo), static_cast<uint32_t>(lo >> 32), static_cast<uint32_t>(hi),
+                   static_cast<uint32_t>(hi >> 32));
+  }
+}
+
+// Tiles of a CTA. Dense output: strided over the grid, so all CTAs work on the
+// same query tile at a time. Ranking: a contiguous run of tiles, so a CTA
+// ranks long runs of stored rows of one query tile (fewer fresh lists).
+template <bool TOPK>
+__device__ __forceinline__ int tile_begin(const ScoreTcArgs& g) {
+  return TOPK ? static_cast<int>(static_cast<long long>(g.n_tiles) * blockIdx.x / gridDim.x) : blockIdx.x;
+}
+template <bool TOPK>
+__device__ __forceinline__ int tile_end(const ScoreTcArgs& g) {
+  return TOPK ? static_cast<int>(static_cast<long long>(g.n_tiles) * (blockIdx.x + 1) / gridDim.x) : g.n_tiles;
+}
+template <bool TOPK>
+__device__ __forceinline__ int tile_step() {
+  return TOPK ? 1 : gridDim.x;
+}
+
 template <int MODE, bool TOPK>
 __global__ void __launch_bounds__(kThreadsTc, 1)
     k_score_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQlo,
@@ -130,6 +171,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   constexpr int S = tc_stages<MODE, TOPK>();
   constexpr uint32_t kStage = tc_stage_bytes<MODE>();
   constexpr int kBits = TcMode<MODE>::kBits;
+  constexpr int kG = 8;  // stages of code bits prefetched at a time
+  using StageBits = typename TcMode<MODE>::Bits;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const TcSmem L = tc_smem_layout<MODE, TOPK>(g.BNq, g.K);
@@ -162,71 +205,57 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
 
   if (warp < 4) {
     // ---------------------------------------------------------- expanders
+    // A stored row's modules are back to back, so pipeline stage j of a tile
+    // reads bits [j kBits, (j+1) kBits) of the row and query columns from
+    // j kBits on. The bits of the next kG stages are loaded into registers
+    // while the current kG stages are expanded, hiding the HBM latency.
     const int r = threadIdx.x;  // stored row within the tile
     const uint32_t row_off = static_cast<uint32_t>((r >> 3) * 1024 + (r & 7) * 128);
+    const int nst = g.D / kBits;
     uint32_t it = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < g.n_tiles && ok; tile += gridDim.x) {
+    for (int tile = tile_begin<TOPK>(g), tstep = tile_step<TOPK>(), tend = tile_end<TOPK>(g);
+         tile < tend && ok; tile += tstep) {
       const int qt = tile / g.n_it, ib = tile % g.n_it;
       const int i0 = ib * 128, q0 = qt * g.BNq;
       const bool rv = i0 + r < g.N;
-      const uint32_t* crow = g.train + static_cast<size_t>(rv ? i0 + r : 0) * g.ldt;
-      for (int u = 0; u < g.U && ok; ++u) {
-        const int nkb = g.k[u] / kBits;
-        for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const int s = static_cast<int>(it % S);
-          const uint32_t ph = (it / S) & 1u;
-          uint32_t w_ok = 1;
-          if (lane == 0) w_ok = mbar_wait(&empty[s], ph ^ 1u, g.status) ? 1u : 0u;
-          w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
-          if (!w_ok) {
-            ok = false;
-            break;
-          }
-          uint8_t* st = smem + static_cast<size_t>(s) * kStage;
-          if (warp == 0 && lane == 0) {
-            mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(g.BNq) * 128u * TcMode<MODE>::kQBoxes);
-            if (MODE == EOGP_SCORE_CODES) {
-              tma_load_2d(st + kAB, &tmQ, g.boff[u] + kb * 128, q0, &full[s]);
+      const StageBits* brow =
+          reinterpret_cast<const StageBits*>(g.train + static_cast<size_t>(rv ? i0 + r : 0) * g.ldt);
+      StageBits cur[kG], nxt[kG];
+#pragma unroll
+      for (int jj = 0; jj < kG; ++jj) cur[jj] = (rv && jj < nst) ? __ldg(brow + jj) : StageBits{};
+      for (int j0 = 0; j0 < nst && ok; j0 += kG) {
+#pragma unroll
+        for (int jj = 0; jj < kG; ++jj)
+          nxt[jj] = (rv && j0 + kG + jj < nst) ? __ldg(brow + j0 + kG + jj) : StageBits{};
+#pragma unroll
+        for (int jj = 0; jj < kG; ++jj) {
+          const int j = j0 + jj;
+          if (j < nst && ok) {
+            const int s = static_cast<int>(it % S);
+            const uint32_t ph = (it / S) & 1u;
+            ++it;
+            uint32_t w_ok = 1;
+            if (lane == 0) w_ok = mbar_wait(&empty[s], ph ^ 1u, g.status) ? 1u : 0u;
+            w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
+            if (!w_ok) {
+              ok = false;
             } else {
-              tma_load_2d(st + kAB, &tmQ, g.boff[u] + kb * 64, q0, &full[s]);
-              tma_load_2d(st + 2 * kAB, &tmQlo, g.boff[u] + kb * 64, q0, &full[s]);
+              uint8_t* st = smem + static_cast<size_t>(s) * kStage;
+              if (warp == 0 && lane == 0) {
+                mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(g.BNq) * 128u * TcMode<MODE>::kQBoxes);
+                tma_load_2d(st + kAB, &tmQ, j * kBits, q0, &full[s]);
+                if (MODE == EOGP_SCORE_PAPER) tma_load_2d(st + 2 * kAB, &tmQlo, j * kBits, q0, &full[s]);
+              }
+              expand_stage(st + row_off, r & 7, cur[jj]);
+              fence_proxy_async_smem();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(&full[s]);
             }
           }
-          if (MODE == EOGP_SCORE_CODES) {
-            uint4 bits = make_uint4(0, 0, 0, 0);
-            if (rv) bits = __ldg(reinterpret_cast<const uint4*>(crow + g.woff[u] + kb * 4));
-            const uint32_t wv[4] = {bits.x, bits.y, bits.z, bits.w};
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {  // 16 bits -> 16 bytes per swizzled 16-byte chunk
-              const uint32_t h = wv[c >> 1] >> ((c & 1) * 16);
-              const uint64_t lo = expand8(h), hi = expand8(h >> 8);
-              uint4 v;
-              v.x = static_cast<uint32_t>(lo);
-              v.y = static_cast<uint32_t>(lo >> 32);
-              v.z = static_cast<uint32_t>(hi);
-              v.w = static_cast<uint32_t>(hi >> 32);
-              *reinterpret_cast<uint4*>(st + row_off + ((c ^ (r & 7)) << 4)) = v;
-            }
-          } else {
-            uint2 bits = make_uint2(0, 0);
-            if (rv) bits = __ldg(reinterpret_cast<const uint2*>(crow + g.woff[u] + kb * 2));
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {  // 8 bits -> 8 bf16 per swizzled 16-byte chunk
-              const uint32_t h = (c < 4 ? bits.x : bits.y) >> ((c & 3) * 8);
-              const uint64_t lo = expand4_bf16(h), hi = expand4_bf16(h >> 4);
-              uint4 v;
-              v.x = static_cast<uint32_t>(lo);
-              v.y = static_cast<uint32_t>(lo >> 32);
-              v.z = static_cast<uint32_t>(hi);
-              v.w = static_cast<uint32_t>(hi >> 32);
-              *reinterpret_cast<uint4*>(st + row_off + ((c ^ (r & 7)) << 4)) = v;
-            }
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&full[s]);
         }
+#pragma unroll
+        for (int jj = 0; jj < kG; ++jj) cur[jj] = nxt[jj];
       }
     }
   } else if (warp < 8) {
@@ -238,29 +267,27 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
     float* ls = reinterpret_cast<float*>(smem + L.lists) + static_cast<size_t>(ep) * g.K;
     int* li = reinterpret_cast<int*>(smem + L.lists + static_cast<size_t>(g.BNq) * g.K * 4) +
               static_cast<size_t>(ep) * g.K;
-    int seg_qt = -1, cnt = 0;
-    float tau = -INFINITY;
+    int seg_qt = -1;
+    TopkState tk;
+    topk_reset(tk);
     auto flush = [&]() {
       const int q = seg_qt * g.BNq + ep;
       if (ep < g.BNq && q < g.Q) {
         const size_t o = (static_cast<size_t>(blockIdx.x) * g.Q + q) * g.K;
-        for (int p = 0; p < g.K; ++p) {
-          g.lst[o + p] = p < cnt ? ls[p] : -INFINITY;
-          g.lsi[o + p] = p < cnt ? li[p] : -1;
-        }
+        topk_write(ls, li, g.K, tk, g.lst + o, g.lsi + o);
       }
     };
     uint32_t gm = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < g.n_tiles && ok; tile += gridDim.x) {
+    for (int tile = tile_begin<TOPK>(g), tstep = tile_step<TOPK>(), tend = tile_end<TOPK>(g);
+         tile < tend && ok; tile += tstep) {
       const int qt = tile / g.n_it, ib = tile % g.n_it;
       const int i0 = ib * 128, q0 = qt * g.BNq;
       const int row = i0 + ep;
       if (TOPK && qt != seg_qt) {
         if (seg_qt >= 0) flush();
         seg_qt = qt;
-        cnt = 0;
-        tau = -INFINITY;
+        topk_reset(tk);
       }
       for (int u = 0; u < g.U; ++u, ++gm) {
         const int buf = static_cast<int>(gm & 1u);
@@ -297,45 +324,31 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
 #pragma unroll
             for (int j = 0; j < 32; ++j) a[j] = __fadd_rn(a[j], __fmul_rn(si, d[j]));
           }
-          if (!last) {
+          if (!last || TOPK) {
             tmem_st32(tmem + lane_base + 256u + c0, a);
-          } else if (!TOPK) {
-            if (row < g.N) {
+          } else if (row < g.N) {
 #pragma unroll
-              for (int j = 0; j < 32; ++j)
-                if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
-            }
-          } else {
-            // Stage these 32 query columns column-major; the warp owning them ranks them.
-#pragma unroll
-            for (int j = 0; j < 32; ++j) tb[j * kTbStride + ep] = a[j];
-            named_bar_sync(3, 128);
-            if ((ep >> 5) == (c0 >> 5) && q0 + ep < g.Q) {
-              const int nr = min(128, g.N - i0);
-              const float* col = tb + lane * kTbStride;
-              for (int r = 0; r < nr; ++r) {
-                const float v = col[r];
-                const bool take = cnt < g.K ? (v == v) : (v > tau);
-                if (take) {
-                  int p = cnt < g.K ? cnt : g.K - 1;
-                  while (p > 0 && ls[p - 1] < v) {
-                    ls[p] = ls[p - 1];
-                    li[p] = li[p - 1];
-                    --p;
-                  }
-                  ls[p] = v;
-                  li[p] = i0 + r;
-                  if (cnt < g.K) ++cnt;
-                  if (cnt == g.K) tau = ls[g.K - 1];
-                }
-              }
-            }
-            named_bar_sync(3, 128);
+            for (int j = 0; j < 32; ++j)
+              if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
           }
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&dempty[buf]);
+        if (lane == 0) mbar_arrive(&dempty[buf]);  // D buffer free: the MMAs run on
+        if (TOPK && last) {
+          // Rank the finished tile from the running-score columns, 32 query columns at
+          // a time: staged column-major, then the warp owning them offers them to its lists.
+          for (int c0 = 0; c0 < g.BNq; c0 += 32) {
+            float a[32];
+            tmem_ld32(tmem + lane_base + 256u + c0, a);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) tb[j * kTbStride + ep] = a[j];
+            named_bar_sync(3, 128);
+            if ((ep >> 5) == (c0 >> 5) && q0 + ep < g.Q)
+              topk_scan(tb + lane * kTbStride, min(128, g.N - i0), i0, ls, li, g.K, tk);
+            named_bar_sync(3, 128);
+          }
+        }
       }
     }
     if (TOPK && seg_qt >= 0) flush();
@@ -346,7 +359,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
           MODE == EOGP_SCORE_CODES ? idesc_e4m3_f32(128, g.BNq) : idesc_bf16_f32(128, g.BNq, 0, 0);
       uint32_t it = 0, gm = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < g.n_tiles && ok; tile += gridDim.x) {
+      for (int tile = tile_begin<TOPK>(g), tstep = tile_step<TOPK>(), tend = tile_end<TOPK>(g);
+         tile < tend && ok; tile += tstep) {
         for (int u = 0; u < g.U && ok; ++u, ++gm) {
           const int buf = static_cast<int>(gm & 1u);
           const uint32_t dph = (gm >> 1) & 1u;
@@ -390,7 +404,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   if (warp == 8) tmem_dealloc(tmem, 512);
 }
 
-// Query codes -> e4m3 bytes: out[q][boff_u + c] = +1 / -1 for bit c of module u.
+// Query codes -> e4m3 bytes: out[q][c] = +1 / -1 for bit c of the concatenated modules.
 __global__ void k_expand_queries(const uint32_t* __restrict__ query, int ldq, int row_bytes,
                                  uint8_t* __restrict__ out) {
   const int q = blockIdx.y;
@@ -478,7 +492,7 @@ cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const floa
                             int ldqs, int Q, float* out, int ldo, const TcTopK* topk, void* ws,
                             int num_sms, unsigned* status, cudaStream_t st) {
   if (N <= 0 || Q <= 0) return cudaSuccess;
-  ScoreTcArgs g;  // ~12 KB parameter block, copied at launch
+  ScoreTcArgs g;  // ~4 KB parameter block, copied at launch
   g.N = N;
   g.Q = Q;
   g.U = U;
@@ -497,15 +511,12 @@ cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const floa
   g.lst = topk ? topk->lst : nullptr;
   g.lsi = topk ? topk->lsi : nullptr;
   g.status = status;
-  int wo = 0, bo = 0;
+  int D = 0;
   for (int u = 0; u < U; ++u) {
     g.k[u] = ks[u];
-    g.woff[u] = wo;
-    g.boff[u] = bo;
-    wo += ks[u] / 32;
-    bo += ks[u];
+    D += ks[u];
   }
-  const int D = bo;
+  g.D = D;
   const int grid = score_tc_grid(N, Q, num_sms);
   CUtensorMap t0, t1;
   if (mode == EOGP_SCORE_CODES) {

@@ -6,7 +6,7 @@
 // Two kernels:
 // * k_topk_dense ranks a dense [Q, N] score matrix: block (slot s, query tile)
 //   owns stored rows [s R, (s+1) R) of 32 queries; 128-row chunks are staged
-//   transposed in shared memory and lane j keeps query j's sorted list there.
+//   transposed in shared memory and lane j keeps query j's list there.
 // * k_topk_merge merges per-slot lists [S][Q][K] (written by k_topk_dense or by
 //   the fused tensor-core scoring epilogue) into the final [Q, K]. Every slot
 //   list is sorted, so the largest K-th entry over the slots is a lower bound
@@ -15,6 +15,7 @@
 #include <cmath>
 
 #include "eogp_internal.h"
+#include "topk_dev.cuh"
 
 namespace {
 
@@ -51,8 +52,8 @@ __global__ void __launch_bounds__(32) k_topk_dense(const float* __restrict__ sc,
   const int nq = min(32, Q - q0);
   const int r_beg = slot * rows_per_slot, r_end = min(N, r_beg + rows_per_slot);
   const bool vec = (ld & 3) == 0 && (reinterpret_cast<uintptr_t>(sc) & 15) == 0;
-  int cnt = 0;
-  float tau = -INFINITY;
+  eogp::TopkState tk;
+  eogp::topk_reset(tk);
   for (int r0 = r_beg; r0 < r_end; r0 += kChunk) {
     const int nr = min(kChunk, r_end - r0);
     for (int j = 0; j < nq; ++j) {
@@ -69,33 +70,12 @@ __global__ void __launch_bounds__(32) k_topk_dense(const float* __restrict__ sc,
       }
     }
     __syncwarp();
-    if (lane < nq) {
-      const float* col = tb + lane * kTs;
-      for (int r = 0; r < nr; ++r) {
-        const float v = col[r];
-        const bool take = cnt < K ? (v == v) : (v > tau);
-        if (take) {
-          int p = cnt < K ? cnt : K - 1;
-          while (p > 0 && ls[p - 1] < v) {
-            ls[p] = ls[p - 1];
-            li[p] = li[p - 1];
-            --p;
-          }
-          ls[p] = v;
-          li[p] = r0 + r;
-          if (cnt < K) ++cnt;
-          if (cnt == K) tau = ls[K - 1];
-        }
-      }
-    }
+    if (lane < nq) eogp::topk_scan(tb + lane * kTs, nr, r0, ls, li, K, tk);
     __syncwarp();
   }
   if (lane < nq) {
     const size_t o = (static_cast<size_t>(slot) * Q + q0 + lane) * K;
-    for (int p = 0; p < K; ++p) {
-      lst[o + p] = p < cnt ? ls[p] : -INFINITY;
-      lsi[o + p] = p < cnt ? li[p] : -1;
-    }
+    eogp::topk_write(ls, li, K, tk, lst + o, lsi + o);
   }
 }
 

@@ -327,6 +327,21 @@ def pack_sign(x, codes=None, scales=None, stream=None):
     return codes, scales
 
 
+def score_workspace_size(N: int, ks: Sequence[int], mode: int, Q: int) -> int:
+    karr = (c_int * len(ks))(*[int(k) for k in ks])
+    need = c_size_t()
+    _check(lib().eogp_score_workspace_size(int(N), karr, len(ks), int(mode), int(Q), ctypes.byref(need)))
+    return need.value
+
+
+def score_topk_workspace_size(N: int, ks: Sequence[int], mode: int, Q: int, topk: int) -> int:
+    karr = (c_int * len(ks))(*[int(k) for k in ks])
+    need = c_size_t()
+    _check(lib().eogp_score_topk_workspace_size(int(N), karr, len(ks), int(mode), int(Q), int(topk),
+                                                ctypes.byref(need)))
+    return need.value
+
+
 def score(train, train_scales, ks: Sequence[int], mode: int, query, query_scales=None, out=None,
           stream=None, ws=None):
     """eogp_score: returns scores [Q, N] fp32. A workspace of the size
