@@ -422,6 +422,10 @@ def main():
     ap.add_argument("--e2e-batch", type=int, default=128,
                     help="examples per e2e step (pinned host staging is sized by it)")
     ap.add_argument("--no-scan", action="store_true")
+    ap.add_argument("--scan-rows", type=int, default=0,
+                    help="stored codes in the scan (default: the 4,194,304 of the scan workload)")
+    ap.add_argument("--scan-qs", default="",
+                    help="comma-separated query counts of the scan (default: 1,64,1024,8192)")
     ap.add_argument("--no-configs", action="store_true",
                     help="skip the OLMo / 32B / tiny-fp32 throughput and the PCA-fit timing")
     ap.add_argument("--modules", type=int, default=0,
@@ -675,14 +679,15 @@ def main():
                 "frac_of_hbm": pbytes / (pms / 1000.0) / 1e9 / hbm}
         del xs, pc, psc
         sc = synth.SCAN
-        N, ksc = sc["N"], sc["k"]
+        N, ksc = (args.scan_rows or sc["N"]), sc["k"]
+        scan_qs = [int(q) for q in args.scan_qs.split(",")] if args.scan_qs else list(sc["Qs"])
         Wsc = ksc // 32
         tr = torch.randint(-2 ** 31, 2 ** 31 - 1, (N, Wsc), generator=g, device=dev, dtype=torch.int32)
         tsc = torch.exp(sc["scale_sigma"] * torch.randn((N, 1), generator=g, device=dev))
         qmax = 1024
         out = torch.empty((qmax, N), dtype=torch.float32, device=dev)
         scan = {"N": N, "bits": ksc, "mode": "CODES", "per_Q": {}}
-        for Q in sc["Qs"]:
+        for Q in scan_qs:
             qc = torch.randint(-2 ** 31, 2 ** 31 - 1, (Q, Wsc), generator=g, device=dev,
                                dtype=torch.int32)
             qs = torch.exp(sc["scale_sigma"] * torch.randn((Q, 1), generator=g, device=dev))
