@@ -588,6 +588,41 @@ def main():
         scoring["paper_top20"] = {"ms_per_call": tms, "scores_per_s": N * Q / (tms / 1000.0)}
         del y, wsp, wtc, wtp
 
+    # ---- EOGP-R: the SRHT second stage in place of P (App. B.2), same stack ----
+    eogp_r = None
+    if not args.no_score:
+        eogp_r = {}
+        for kr in (w.k, 4 * w.k):
+            rdesc = []
+            for u, md in enumerate(mods):
+                plan, VA, VS, _ = md["desc"]._refs[:4]
+                sg, rw = synth.srht_draw(w.m, kr, seed=w.seed, module_index=u)
+                rdesc.append(E.layer_desc(plan, T, kr, VA, VS, None,
+                                          srht_signs=torch.from_numpy(sg).to(dev),
+                                          srht_rows=torch.from_numpy(rw).to(dev)))
+            rwords = (kr + 31) // 32
+            rcodes = torch.empty((B, U * rwords), dtype=torch.int32, device=dev)
+            rws = E.workspace(max(E.compress_workspace_size(d, B, E.OUT_CODES) for d in rdesc), dev)
+
+            def rstep():
+                for u, md in enumerate(mods):
+                    E.compress_layer(rdesc[u], md["a"], md["s"], E.OUT_CODES,
+                                     codes=rcodes[:, u * rwords:(u + 1) * rwords],
+                                     scales=scales[:, u], ws=rws)
+            rstep()
+            torch.cuda.synchronize()
+            a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a_ev.record(stream)
+            for _ in range(3):
+                rstep()
+            b_ev.record(stream)
+            torch.cuda.synchronize()
+            E.sync_status()
+            rms = a_ev.elapsed_time(b_ev) / 3
+            eogp_r[f"k{kr}"] = {"examples_per_s": B / (rms / 1000.0), "ms_per_step": rms,
+                                "bits_per_module": kr}
+            del rdesc, rcodes, rws
+
     # ---- end to end through the public API with host buffers ----
     # Per module: host -> device copy of (a, s) on a copy stream, then the
     # compression on the compute stream once that copy has landed; module u+1's
@@ -759,7 +794,8 @@ def main():
                            "k": w.k, "modules": U, "parallelism": f"replicas x{world}",
                            "l2": "inputs > L2 (B x 151 MB per step)"},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "scoring": scoring,
-                "pack_sign": pack, "scan": scan, "other_workloads": configs, "fit_pca": fit,
+                "pack_sign": pack, "scan": scan, "eogp_r_srht": eogp_r, "other_workloads": configs,
+                "fit_pca": fit,
                 "gpu_launches": launches, "kernels": kern, "clocks": clk}
         print(json.dumps(line))
     if world > 1:

@@ -166,8 +166,14 @@ typedef struct {
   const void* VS;  /* device [nR x d_out]: row r = eigenvector Q_S[:, R[r]]    */
   const void* Pt;  /* device [k x m]: row c = PCA direction c (column c of P,
                       App. B.2) over the canonical retained order; may be NULL
-                      for EOGP_OUT_FIRST_STAGE                                 */
+                      for EOGP_OUT_FIRST_STAGE or with the SRHT below          */
   const eogp_plan* plan;
+  /* EOGP-R (Sec. 3.2 "A scalable alternative to PCA"; App. B.2
+     Eq. app_srht_definition): when Pt is NULL and srht_rows is set, the second
+     stage is x = sqrt(p/k) R H_p D J z (see eogp_srht) instead of P^T z, with
+     k <= p = 2^ceil(log2 m) and m <= EOGP_SRHT_MAX_M.                       */
+  const int8_t* srht_signs;  /* device [m]: diagonal of D (< 0 means -1)      */
+  const int32_t* srht_rows;  /* device [k]: rows of H_p kept by R, in [0, p)   */
 } eogp_layer_desc;
 
 /* Workspace bytes eogp_compress_layer needs for this descriptor, batch B and
@@ -237,6 +243,23 @@ int eogp_fit_pca(const float* Z, int n, int m, int ldz, int k, void* Pt, int ld_
 /* ========================================================================
  * One-bit encoding (Sec. 3.3 Eq. onebit; Alg. 1 "Store packed binary signs")
  * ======================================================================== */
+/* EOGP-R second stage (Sec. 3.2 "A scalable alternative to PCA"; App. B.2
+ * Eq. app_srht_definition), applied to rows z of z [B x ldz] fp32 device:
+ *   x = sqrt(p/k) R H_p D J z,  p = 2^ceil(log2 m),
+ * J zero-pads to p, D = diag(signs) (signs [m] int8 device, < 0 means -1),
+ * H_p is the orthonormal Walsh-Hadamard matrix in Sylvester order
+ * (H_p[r][c] = (-1)^popcount(r & c) / sqrt(p)), R keeps rows[0..k) (int32
+ * device, each in [0, p), distinct; out-of-range rows give 0 and set
+ * EOGP_EDEVICE in the device status word). The random signs and rows are the
+ * caller's: the same realisation must serve stored examples and queries.
+ * Outputs (either may be NULL): x [B x ldx] fp32; codes [B x ld_codes] and
+ * scales[b * ld_scales] as in eogp_pack_sign (sign bits of x, ||x||_1 / k).
+ * Errors: EOGP_EINVAL, EOGP_EUNSUPPORTED (m > EOGP_SRHT_MAX_M), EOGP_ECUDA. */
+#define EOGP_SRHT_MAX_M 32768
+int eogp_srht(const float* z, int B, int m, int ldz, const int8_t* signs, const int32_t* rows, int k,
+              float* x, int ldx, uint32_t* codes, int ld_codes, float* scales, int ld_scales,
+              eogp_stream_t stream);
+
 /* x [B x ldx] fp32 device -> codes [B x ld_codes] uint32 (bit c % 32 of word
  * c / 32 = [x_c >= 0], pad bits 0) and scales[b * ld_scales] = ||x_b||_1 / k
  * (fixed-order reduction: bitwise reproducible). A NaN input sets

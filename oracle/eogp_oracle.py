@@ -33,10 +33,13 @@ Function map:
   score_codes           Sec. 3.3 Eq. onebit_influence with both sides one-bit
   score_paper           Sec. 3.3 Eq. onebit_influence; App. B.3 Eq. app_stored_influence
   score_fp              Sec. 3.1 (influence as an inner product of coordinates)
+  srht                  Sec. 3.2 "A scalable alternative to PCA"; App. B.2 Eq. app_srht_definition
+  top_k                 App. C (per-query ranking of stored examples, NDCG@20)
   payload_bytes         App. E.1, Eq. app_payload
 
-Readings where the paper is silent are listed in the design doc (ties in the top-m
-selection, bit order, sign of zero, PCA sign convention).
+Where the paper is silent, the function that needs a reading states it (ties
+in the top-m selection, bit order, sign of zero, PCA sign convention, ranking
+order, Hadamard ordering).
 """
 from __future__ import annotations
 
@@ -173,6 +176,36 @@ def fit_pca(Z: np.ndarray, k: int, route: str = "auto") -> Tuple[np.ndarray, np.
 def project(z: np.ndarray, P: np.ndarray) -> np.ndarray:
     """x = P^T z for each row z of z [B, m] (Sec. 3.2, Eq. second_stage)."""
     return np.asarray(z, np.float64) @ np.asarray(P, np.float64)
+
+
+def srht_width(m: int) -> int:
+    """Padded width p = 2^ceil(log2 m) of the SRHT (App. B.2, Eq. app_srht_definition)."""
+    p = 1
+    while p < m:
+        p *= 2
+    return p
+
+
+def srht(z: np.ndarray, signs: np.ndarray, rows: np.ndarray) -> np.ndarray:
+    """EOGP-R second stage x = sqrt(p/k) R H_p D J z for each row z of z [B, m]
+    (Sec. 3.2 "A scalable alternative to PCA"; App. B.2 Eq. app_srht_definition).
+
+    J zero-pads to width p = 2^ceil(log2 m); D = diag(signs) (the m signs that
+    meet non-padded coordinates; the others multiply zeros); H_p is the
+    orthonormal Walsh-Hadamard matrix in Sylvester (natural) order,
+    H_p[r, c] = (-1)^popcount(r & c) / sqrt(p), the ordering the paper leaves
+    unstated; R keeps rows `rows` (k distinct indices in [0, p)) in the given
+    order. The random signs and rows are inputs: the same realisation serves
+    stored examples and queries. H_p is formed explicitly (a library matrix)."""
+    import scipy.linalg
+    z = np.asarray(z, np.float64)
+    B, m = z.shape
+    p = srht_width(m)
+    k = len(rows)
+    zp = np.zeros((B, p))
+    zp[:, :m] = z * np.asarray(signs, np.float64)[None, :m]
+    H = scipy.linalg.hadamard(p).astype(np.float64) / np.sqrt(p)
+    return np.sqrt(p / k) * (zp @ H.T)[:, np.asarray(rows, np.int64)]
 
 
 # --------------------------------------------------------------------------

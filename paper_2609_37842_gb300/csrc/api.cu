@@ -466,6 +466,9 @@ int proj_splits(int B, int k, int m) {
   return tc_gemm_splits_used(m, std::max(1, want));
 }
 
+// EOGP-R descriptor: the SRHT replaces the PCA projection.
+bool uses_srht(const eogp_layer_desc* L) { return !L->Pt && L->srht_rows; }
+
 int make_layout(const eogp_layer_desc* L, int B, int mode, Layout* o) {
   const eogp_plan* P = L->plan;
   const size_t M = static_cast<size_t>(B) * L->T;
@@ -486,15 +489,17 @@ int make_layout(const eogp_layer_desc* L, int B, int mode, Layout* o) {
       o->ldzb = round_up(L->m, 64);
       o->zhi = take(static_cast<size_t>(B) * o->ldzb * 2);
       o->zlo = take(static_cast<size_t>(B) * o->ldzb * 2);
-      o->ldp = round_up(L->k, 16);
-      o->splits = proj_splits(B, L->k, L->m);
-      o->part = take(static_cast<size_t>(o->splits) * B * o->ldp * 4);
+      if (!uses_srht(L)) {
+        o->ldp = round_up(L->k, 16);
+        o->splits = proj_splits(B, L->k, L->m);
+        o->part = take(static_cast<size_t>(o->splits) * B * o->ldp * 4);
+      }
     }
   } else {
     o->at = take(M * P->nC() * 4);
     o->st = take(M * P->nR() * 4);
     if (mode != EOGP_OUT_FIRST_STAGE) o->z = take(static_cast<size_t>(B) * L->m * 4);
-    if (mode == EOGP_OUT_CODES) o->x = take(static_cast<size_t>(B) * L->k * 4);
+    if (mode == EOGP_OUT_CODES && !uses_srht(L)) o->x = take(static_cast<size_t>(B) * L->k * 4);
   }
   o->total = std::max<size_t>(off, 256);
   return EOGP_OK;
@@ -512,8 +517,14 @@ int check_desc(const eogp_layer_desc* L, int B, int mode) {
   if (mode < EOGP_OUT_FIRST_STAGE || mode > EOGP_OUT_CODES) return set_error(EOGP_EINVAL, "bad out_mode");
   if (L->dtype != EOGP_F32 && L->dtype != EOGP_BF16) return set_error(EOGP_EINVAL, "bad dtype");
   if (mode != EOGP_OUT_FIRST_STAGE) {
-    if (L->k < 1 || L->k > L->m) return set_error(EOGP_EINVAL, "k must be in [1, m]");
-    if (!L->Pt) return set_error(EOGP_EINVAL, "Pt is NULL");
+    if (uses_srht(L)) {
+      if (L->m > EOGP_SRHT_MAX_M) return set_error(EOGP_EUNSUPPORTED, "SRHT needs m <= %d", EOGP_SRHT_MAX_M);
+      if (L->k < 1 || L->k > srht_width(L->m)) return set_error(EOGP_EINVAL, "SRHT k must be in [1, p]");
+      if (!L->srht_signs) return set_error(EOGP_EINVAL, "srht_signs is NULL");
+    } else {
+      if (L->k < 1 || L->k > L->m) return set_error(EOGP_EINVAL, "k must be in [1, m]");
+      if (!L->Pt) return set_error(EOGP_EINVAL, "Pt is NULL (and no SRHT given)");
+    }
   }
   if (!L->VA || !L->VS) return set_error(EOGP_EINVAL, "VA / VS is NULL");
   if (L->dtype == EOGP_BF16) {
@@ -594,6 +605,15 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
                                   status, st));
     }
     if (fs) return EOGP_OK;
+    if (uses_srht(L)) {
+      // EOGP-R: x = sqrt(p/k) R H_p D J z, with the sign/scale pack in the same kernel.
+      ProfScope ps(EOGP_K_PROJECT, st);
+      const bool cd = out_mode == EOGP_OUT_CODES;
+      CUDA_TRY(launch_srht(w + lo.zhi, w + lo.zlo, true, lo.ldzb, B, L->m, L->srht_signs, L->srht_rows,
+                           L->k, cd ? nullptr : out, ld_out, cd ? codes : nullptr, ld_codes,
+                           cd ? scales : nullptr, ld_scales, status, st));
+      return EOGP_OK;
+    }
     // x = P^T z (Eq. second_stage), split over K; then sum + sign/pack (Eq. onebit).
     float* part = reinterpret_cast<float*>(w + lo.part);
     const size_t slab = static_cast<size_t>(B) * lo.ldp;
@@ -628,6 +648,13 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
   CUDA_TRY(launch_contract_f32(at, nC, stt, nR, B, L->T, L->m, P->d_posR, P->d_posC, P->d_scale, z,
                                ldz, st));
   if (out_mode == EOGP_OUT_FIRST_STAGE) return EOGP_OK;
+  if (uses_srht(L)) {
+    const bool cd = out_mode == EOGP_OUT_CODES;
+    CUDA_TRY(launch_srht(z, nullptr, false, ldz, B, L->m, L->srht_signs, L->srht_rows, L->k,
+                         cd ? nullptr : out, ld_out, cd ? codes : nullptr, ld_codes,
+                         cd ? scales : nullptr, ld_scales, status, st));
+    return EOGP_OK;
+  }
   float* x = out_mode == EOGP_OUT_COORDS ? out : reinterpret_cast<float*>(w + lo.x);
   const int ldx = out_mode == EOGP_OUT_COORDS ? ld_out : L->k;
   CUDA_TRY(launch_simt_gemm(B, L->k, L->m, 1.f, z, ldz, 1, static_cast<const float*>(L->Pt), L->m, 1,
@@ -635,6 +662,30 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
   if (out_mode == EOGP_OUT_CODES)
     CUDA_TRY(launch_pack(x, 1, 0, ldx, B, L->k, nullptr, 0, codes, ld_codes, scales, ld_scales,
                          status, st));
+  return EOGP_OK;
+}
+
+// ================================================================ SRHT
+
+extern "C" int eogp_srht(const float* z, int B, int m, int ldz, const int8_t* signs, const int32_t* rows,
+                         int k, float* x, int ldx, uint32_t* codes, int ld_codes, float* scales,
+                         int ld_scales, eogp_stream_t stream) {
+  clear_error();
+  if (B < 0 || m < 1) return set_error(EOGP_EINVAL, "need B >= 0, m >= 1");
+  if (m > EOGP_SRHT_MAX_M) return set_error(EOGP_EUNSUPPORTED, "SRHT needs m <= %d", EOGP_SRHT_MAX_M);
+  if (k < 1 || k > srht_width(m)) return set_error(EOGP_EINVAL, "k must be in [1, p = %d]", srht_width(m));
+  if (B == 0) return EOGP_OK;
+  if (!z || !signs || !rows) return set_error(EOGP_EINVAL, "NULL argument");
+  if (ldz < m) return set_error(EOGP_EINVAL, "ldz < m");
+  if (x && ldx < k) return set_error(EOGP_EINVAL, "ldx < k");
+  if (codes && (!scales || ld_codes < (k + 31) / 32 || ld_scales < 1))
+    return set_error(EOGP_EINVAL, "codes need scales and ld_codes >= ceil(k/32)");
+  unsigned* status = status_word();
+  if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  ProfScope ps(EOGP_K_PROJECT, st);
+  CUDA_TRY(launch_srht(z, nullptr, false, ldz, B, m, signs, rows, k, x, ldx, codes, ld_codes, scales,
+                       ld_scales, status, st));
   return EOGP_OK;
 }
 

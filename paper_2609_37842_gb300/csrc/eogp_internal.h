@@ -110,6 +110,14 @@ cudaError_t launch_topk_dense(const float* scores, int ld, int Q, int N, int K, 
 cudaError_t launch_topk_merge(const float* lst, const int* lsi, int S, int Q, int K, float* out_s,
                               int ld_os, int* out_i, int ld_oi, cudaStream_t st);
 
+// k_srht.cu: EOGP-R second stage, one CTA per row (z fp32, or bf16 hi + lo when hilo).
+int srht_width(int m);
+size_t srht_smem_bytes(int m);
+cudaError_t launch_srht(const void* z0, const void* z1, bool hilo, int ldz, int B, int m,
+                        const int8_t* signs, const int32_t* rows, int k, float* x, int ldx,
+                        uint32_t* codes, int ld_codes, float* scales, int ld_scales, unsigned* status,
+                        cudaStream_t st);
+
 // k_simt.cu: C[i][j] = alpha * sum_k A(i,k) B(j,k), A(i,k) = A[i*sai + k*sak], etc.
 cudaError_t launch_simt_gemm(int M, int N, int K, float alpha, const float* A, long long sai,
                              long long sak, const float* Bm, long long sbj, long long sbk,

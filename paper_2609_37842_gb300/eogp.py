@@ -21,6 +21,7 @@ F32, BF16 = 0, 1
 OUT_FIRST_STAGE, OUT_COORDS, OUT_CODES = 0, 1, 2
 SCORE_CODES, SCORE_PAPER, SCORE_FP = 0, 1, 2
 TOPK_MAX = 256
+SRHT_MAX_M = 32768
 K_ROTATE, K_CONTRACT, K_PROJECT, K_PACK, K_SCORE, K_SIMT = range(6)
 KERNEL_KINDS = {K_ROTATE: "rotate", K_CONTRACT: "contract", K_PROJECT: "project", K_PACK: "pack",
                 K_SCORE: "score", K_SIMT: "simt_f32"}
@@ -43,7 +44,7 @@ class PlanInfo(ctypes.Structure):
 class LayerDesc(ctypes.Structure):
     _fields_ = [("d_in", c_int), ("d_out", c_int), ("T", c_int), ("m", c_int), ("k", c_int),
                 ("dtype", c_int), ("VA", c_void_p), ("VS", c_void_p), ("Pt", c_void_p),
-                ("plan", c_void_p)]
+                ("plan", c_void_p), ("srht_signs", c_void_p), ("srht_rows", c_void_p)]
 
 
 EXPORTS = {
@@ -70,6 +71,8 @@ EXPORTS = {
     "eogp_fit_pca_workspace_size": (c_int, [c_int, c_int, c_int, POINTER(c_size_t)]),
     "eogp_fit_pca": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int,
                              c_void_p, c_void_p, c_size_t, c_void_p]),
+    "eogp_srht": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_void_p, c_int, c_void_p, c_int,
+                          c_void_p, c_int, c_void_p, c_int, c_void_p]),
     "eogp_pack_sign": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_int, c_void_p, c_int,
                                c_void_p]),
     "eogp_score_workspace_size": (c_int, [c_int, c_void_p, c_int, c_int, c_int, POINTER(c_size_t)]),
@@ -231,16 +234,18 @@ class Plan:
 
 
 # ------------------------------------------------------------- compression
-def layer_desc(plan: Plan, T: int, k: int, VA, VS, Pt=None) -> LayerDesc:
+def layer_desc(plan: Plan, T: int, k: int, VA, VS, Pt=None, srht_signs=None,
+               srht_rows=None) -> LayerDesc:
     """Descriptor of one module. It keeps references to the plan and tensors so
-    their device memory outlives the descriptor."""
+    their device memory outlives the descriptor. With Pt None and srht_rows
+    given (int32 [k]; srht_signs int8 [m]), the second stage is the SRHT."""
     inf = plan.info()
     _dense(VA, "VA")
     _dense(VS, "VS")
     _dense(Pt, "Pt")
     d = LayerDesc(inf.d_in, inf.d_out, int(T), inf.m, int(k), _dtype_code(VA), _ptr(VA),
-                  _ptr(VS), _ptr(Pt), plan.handle)
-    d._refs = (plan, VA, VS, Pt)
+                  _ptr(VS), _ptr(Pt), plan.handle, _ptr(srht_signs), _ptr(srht_rows))
+    d._refs = (plan, VA, VS, Pt, srht_signs, srht_rows)
     return d
 
 
@@ -312,6 +317,30 @@ def fit_pca(Z, k: int, pt_dtype: int = F32, ws=None, stream=None):
 
 
 # --------------------------------------------------------------- pack, score
+def srht(z, signs, rows, x=None, codes=None, scales=None, want_x=True, want_codes=False,
+         stream=None):
+    """eogp_srht on z [B, m] fp32: returns x [B, k] and/or (codes, scales)."""
+    import torch
+    _rows(z, "z")
+    B, m = z.shape
+    k = rows.shape[0]
+    if want_x and x is None:
+        x = torch.empty((B, k), dtype=torch.float32, device=z.device)
+    if want_codes:
+        if codes is None:
+            codes = torch.empty((B, (k + 31) // 32), dtype=torch.int32, device=z.device)
+        if scales is None:
+            scales = torch.empty((B,), dtype=torch.float32, device=z.device)
+    _check(lib().eogp_srht(_ptr(z), B, m, z.stride(0), _ptr(signs), _ptr(rows), k,
+                           _ptr(x) if want_x else None, x.stride(0) if want_x else 0,
+                           _ptr(codes) if want_codes else None, codes.stride(0) if want_codes else 0,
+                           _ptr(scales) if want_codes else None,
+                           scales.stride(0) if want_codes else 0, _stream(stream)))
+    if want_x and want_codes:
+        return x, codes, scales
+    return x if want_x else (codes, scales)
+
+
 def pack_sign(x, codes=None, scales=None, stream=None):
     """Sign bits and ||x||_1/k of each row of x [B, k] (fp32, device)."""
     import torch

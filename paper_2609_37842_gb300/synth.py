@@ -21,7 +21,7 @@ import numpy as np
 
 # Role ids used to derive independent seed streams.
 ROLE_A, ROLE_S, ROLE_QA, ROLE_QS, ROLE_QUERY_A, ROLE_QUERY_S, ROLE_FIT_A, ROLE_FIT_S, \
-    ROLE_CODES, ROLE_SCALES, ROLE_P, ROLE_Z, ROLE_CHANNEL = range(13)
+    ROLE_CODES, ROLE_SCALES, ROLE_P, ROLE_Z, ROLE_CHANNEL, ROLE_SRHT = range(14)
 
 
 @dataclasses.dataclass(frozen=True)
@@ -248,6 +248,19 @@ def first_stage_like(n: int, m: int, seed: int, decay: float = 0.7) -> np.ndarra
     if mix is not None:
         z = z @ mix.T
     return z.astype(np.float32)
+
+
+def srht_draw(m: int, k: int, seed: int, module_index: int = 0) -> Tuple[np.ndarray, np.ndarray]:
+    """The random parts of one SRHT realisation: m signs (+1 / -1, int8) and k
+    distinct rows of the padded width p = 2^ceil(log2 m), drawn uniformly
+    without replacement and listed in ascending order (int32)."""
+    r = rng_for(seed, ROLE_SRHT, module_index)
+    p = 1
+    while p < m:
+        p *= 2
+    signs = np.where(r.integers(0, 2, m) == 1, 1, -1).astype(np.int8)
+    rows = np.sort(r.choice(p, size=k, replace=False)).astype(np.int32)
+    return signs, rows
 
 
 def torch_layer_inputs(w: Workload, module_index: int, n: int, device, generator):

@@ -1,6 +1,6 @@
 """GPU parity: every ABI call against the CPU oracle on identical seeded inputs.
 
-Tolerances (spec rules, written out here):
+Tolerances (the parity rules, written out here):
   * pre-sign coordinates z and x: per row ||x_gpu - x_oracle|| / ||x_oracle||
     <= 1e-5 for fp32 inputs, <= 2e-3 for bf16 inputs;
   * sign bits: bit-exact except coordinates with |x_oracle| < 1e-4 ||x_oracle||

@@ -366,6 +366,39 @@ def test_topk_brute_force():
     check_topk(O, 31)
 
 
+def check_srht(Om, seed):
+    """SRHT pins: the Hadamard entries against (-1)^popcount(r & c) by brute
+    force; k = p with unit signs is the orthonormal H, so applying it twice is
+    the identity and norms are kept; the sqrt(p/k) normalisation makes
+    E ||S z||^2 = ||z||^2 over random row subsets (exact average over all
+    subsets of size 1 for a tiny p); zero padding ignores the padded signs."""
+    rng = np.random.default_rng(seed)
+    for m in (1, 5, 8, 13):
+        p = Om.srht_width(m)
+        assert p >= m and p & (p - 1) == 0 and (p == 1 or p // 2 < m)
+    p = 8
+    z = rng.standard_normal((3, p))
+    x = Om.srht(z, np.ones(p), np.arange(p))
+    H = np.array([[(-1) ** bin(r & c).count("1") for c in range(p)] for r in range(p)]) / math.sqrt(p)
+    np.testing.assert_allclose(x, z @ H.T, atol=1e-14, rtol=0)
+    np.testing.assert_allclose(Om.srht(x, np.ones(p), np.arange(p)), z, atol=1e-13, rtol=0)
+    np.testing.assert_allclose(np.linalg.norm(x, axis=1), np.linalg.norm(z, axis=1), rtol=1e-13)
+    # average of ||S z||^2 over every single-row selection equals ||z||^2
+    sg = rng.choice([-1.0, 1.0], p)
+    avg = np.mean([np.sum(Om.srht(z, sg, [r]) ** 2, axis=1) for r in range(p)], axis=0)
+    np.testing.assert_allclose(avg, np.sum(z ** 2, axis=1), rtol=1e-12)
+    # m = 6 pads to p = 8; the signs are applied before padding, rows keep their order
+    z6 = rng.standard_normal((2, 6))
+    sg6 = rng.choice([-1.0, 1.0], 6)
+    rows = np.array([5, 0, 3])
+    want = math.sqrt(8 / 3) * (np.concatenate([z6 * sg6, np.zeros((2, 2))], 1) @ H.T)[:, rows]
+    np.testing.assert_allclose(Om.srht(z6, sg6, rows), want, atol=1e-13, rtol=0)
+
+
+def test_srht():
+    check_srht(O, 37)
+
+
 def _golden_rows(name):
     with open(os.path.join(GOLDEN, name)) as f:
         return [ln.split() for ln in f if ln.strip() and not ln.startswith("#")]
@@ -462,3 +495,11 @@ def test_planted_topk_mistakes_are_caught(monkeypatch):
         return orig(np.nan_to_num(np.asarray(scores, np.float64), nan=-1e300), K)
     monkeypatch.setattr(O, "top_k", nan_ranks)
     assert _fails(check_topk, O, 31)
+
+
+def test_planted_srht_mistakes_are_caught(monkeypatch):
+    orig = O.srht
+    monkeypatch.setattr(O, "srht", lambda z, sg, rows: orig(z, sg, rows) * math.sqrt(len(rows) / O.srht_width(np.asarray(z).shape[1])))
+    assert _fails(check_srht, O, 37)          # normalisation dropped
+    monkeypatch.setattr(O, "srht", lambda z, sg, rows: orig(z, -np.asarray(sg, np.float64), rows)[:, ::-1])
+    assert _fails(check_srht, O, 37)          # rows reversed
