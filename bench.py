@@ -390,6 +390,39 @@ def bench_config(name, B, steps, warmup, dev, stream_bases=False):
     return out
 
 
+def bench_ekfac(dev, d_in, d_out, T, B, reps=3):
+    """EK-FAC eigenvalue correction over the full coordinate block of one module:
+    examples/s and TFLOP/s (algorithmic: full rotations 2 B T (d_in^2 + d_out^2)
+    plus the contraction 2 B T d_in d_out)."""
+    import torch
+    from paper_2609_37842_gb300 import eogp as E
+    from paper_2609_37842_gb300 import synth
+    g = torch.Generator(device=dev)
+    g.manual_seed(13)
+    gh = torch.Generator()
+    gh.manual_seed(13)
+    VA = synth.torch_eigvec_rows(d_in, d_in, dev, gh, torch.bfloat16)
+    VS = synth.torch_eigvec_rows(d_out, d_out, dev, gh, torch.bfloat16)
+    a = torch.randn((B, T, d_in), generator=g, device=dev).to(torch.bfloat16)
+    s = (0.1 * torch.randn((B, T, d_out), generator=g, device=dev)).to(torch.bfloat16)
+    desc = E.ekfac_desc(T, VA, VS)
+    sumsq = torch.zeros((d_out, d_in), dtype=torch.float64, device=dev)
+    ws = E.workspace(E.ekfac_workspace_size(desc, B), dev)
+    E.ekfac_accumulate(desc, a, s, sumsq=sumsq, ws=ws)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        E.ekfac_accumulate(desc, a, s, sumsq=sumsq, accumulate=True, ws=ws)
+    e1.record()
+    torch.cuda.synchronize()
+    E.sync_status()
+    ms = e0.elapsed_time(e1) / reps
+    flops = 2.0 * B * T * (d_in * d_in + d_out * d_out + d_in * d_out)
+    return {"shape": f"{d_in}->{d_out}", "T": T, "batch": B, "ms_per_call": ms,
+            "examples_per_s": B / (ms / 1000.0), "alg_TFLOPs": flops / (ms / 1000.0) / 1e12}
+
+
 def bench_fit(dev, n=10000, m=4096, k=1024):
     import torch
     from paper_2609_37842_gb300 import eogp as E
@@ -777,6 +810,8 @@ def main():
             "olmo2_32b_gate_bf16": bench_config("olmo2_32b_gate_bf16", 64, 5, 3, dev),
         }
         fit = bench_fit(dev)
+        configs["ekfac_correction"] = [bench_ekfac(dev, 768, 3072, 512, 32),
+                                       bench_ekfac(dev, 2048, 8192, 2048, 4)]
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:

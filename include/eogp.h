@@ -223,6 +223,36 @@ int eogp_compress_layer_static(const eogp_layer_desc* L, const void* a, const vo
                                float* scales, int ld_scales, eogp_stream_t stream);
 
 /* ========================================================================
+ * EK-FAC eigenvalue correction (Sec. 2.2 "EK-FAC approximation": the mean
+ * square of each coordinate of the gradients expressed in the K-FAC eigenbasis;
+ * App. C.2: averaged over examples, using sequence-level gradients)
+ * ======================================================================== */
+typedef struct {
+  int d_in, d_out; /* module shape                                             */
+  int T;           /* tokens per example                                       */
+  int dtype;       /* EOGP_F32 or EOGP_BF16: type of a, s, VA, VS              */
+  const void* VA;  /* device [d_in x d_in]: row i = eigenvector Q_A[:, i]      */
+  const void* VS;  /* device [d_out x d_out]: row j = eigenvector Q_S[:, j]    */
+} eogp_ekfac_desc;
+
+int eogp_ekfac_workspace_size(const eogp_ekfac_desc* D, int B, size_t* bytes);
+
+/* For the B examples of a [B x T x d_in], s [B x T x d_out] (dense, device):
+ *   sumsq[j * ld + i] (+)= sum_b ((Q_S^T G_b Q_A)[j][i])^2,  G_b = sum_t s_t a_t^T,
+ * over the full d_out x d_in coordinate block (fp64 device array, ld >= d_in;
+ * added to when `accumulate` is nonzero, overwritten otherwise). The corrected
+ * eigenvalues are sumsq / (examples seen); pass them to eogp_plan_layer as
+ * the full Lambda table. The per-example coordinates are formed as in
+ * eogp_compress_layer (bf16: hi/lo intermediates, 3 MMAs per step), their
+ * squares summed in fp32 over runs of examples and the runs added in fp64 in a
+ * fixed order (bitwise reproducible).
+ * BF16 requires d_in, d_out multiples of 8 and 16-byte aligned a, s, VA, VS.
+ * Errors: EOGP_EINVAL, EOGP_EUNSUPPORTED, EOGP_EWORKSPACE, EOGP_ECUDA. */
+int eogp_ekfac_accumulate(const eogp_ekfac_desc* D, const void* a, const void* s, int B,
+                          double* sumsq, int ld, int accumulate, void* ws, size_t ws_bytes,
+                          eogp_stream_t stream);
+
+/* ========================================================================
  * PCA fit (App. B.2 "PCA fitting"; Alg. 1 "fit P_u by uncentered PCA")
  * ======================================================================== */
 int eogp_fit_pca_workspace_size(int n, int m, int k, size_t* bytes);

@@ -25,6 +25,7 @@ Function map:
   select_retained       Sec. 3.2 (Eq. sigma_ekfac and the text after it), Alg. 1
   per_example_gradient  Sec. 2.2 (K-FAC factors from a and delta)
   rotate                Sec. 2.2 (apply Q_A (x) Q_S through its two factors)
+  ekfac_sumsq           Sec. 2.2 "EK-FAC approximation"; App. C.2 (corrected eigenvalues)
   first_stage           Sec. 3.2, Eq. first_stage
   fit_pca               App. B.2 "PCA fitting", Alg. 1
   project               Sec. 3.2, Eq. second_stage
@@ -104,6 +105,19 @@ def rotate(G: np.ndarray, Q_A: np.ndarray, Q_S: np.ndarray) -> np.ndarray:
     Q_A = np.asarray(Q_A, np.float64)
     Q_S = np.asarray(Q_S, np.float64)
     return Q_S.T @ np.asarray(G, np.float64) @ Q_A
+
+
+def ekfac_sumsq(a: np.ndarray, s: np.ndarray, Q_A: np.ndarray, Q_S: np.ndarray) -> np.ndarray:
+    """Sum over examples of the squared eigenbasis coordinates,
+    sum_b (Q_S^T G_b Q_A)[j, i]^2 with G_b = sum_t s_t a_t^T (d_out x d_in).
+    Divided by the number of examples this is the EK-FAC corrected eigenvalue
+    table (Sec. 2.2 "EK-FAC approximation": mean square of each coordinate of
+    the gradients in the K-FAC eigenbasis; App. C.2: over examples, with
+    sequence-level gradients)."""
+    out = np.zeros((np.asarray(Q_S).shape[1], np.asarray(Q_A).shape[1]))
+    for b in range(np.asarray(a).shape[0]):
+        out += rotate(per_example_gradient(a[b], s[b]), Q_A, Q_S) ** 2
+    return out
 
 
 def first_stage(a: np.ndarray, s: np.ndarray, Q_A: np.ndarray, Q_S: np.ndarray,

@@ -665,6 +665,127 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
   return EOGP_OK;
 }
 
+// ================================================================ EK-FAC correction
+
+namespace {
+
+constexpr int kEkfacStages = 3;
+
+struct EkfacLayout {
+  int ldA = 0, ldS = 0, n_chunks = 1;
+  size_t at_hi = 0, at_lo = 0, st_hi = 0, st_lo = 0, part = 0;  // bf16
+  size_t at = 0, st = 0, g = 0;                                 // fp32
+  size_t total = 0;
+};
+
+int ekfac_check(const eogp_ekfac_desc* D, int B) {
+  if (!D) return set_error(EOGP_EINVAL, "descriptor is NULL");
+  if (D->d_in < 1 || D->d_out < 1 || D->T < 1 || B < 0) return set_error(EOGP_EINVAL, "bad sizes");
+  if (D->dtype != EOGP_F32 && D->dtype != EOGP_BF16) return set_error(EOGP_EINVAL, "bad dtype");
+  if (!D->VA || !D->VS) return set_error(EOGP_EINVAL, "VA / VS is NULL");
+  if (D->dtype == EOGP_BF16) {
+    if (D->d_in % 8 || D->d_out % 8) return set_error(EOGP_EUNSUPPORTED, "bf16 path needs d_in, d_out multiples of 8");
+    if (!aligned16(D->VA) || !aligned16(D->VS)) return set_error(EOGP_EINVAL, "bf16 operands must be 16-byte aligned");
+    if (static_cast<long long>(B) * D->T > 0x7FFFFFFFLL) return set_error(EOGP_EUNSUPPORTED, "B*T too large");
+  }
+  return EOGP_OK;
+}
+
+EkfacLayout ekfac_layout(const eogp_ekfac_desc* D, int B) {
+  EkfacLayout o;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off += al256(bytes);
+    return at;
+  };
+  const size_t M = static_cast<size_t>(B) * D->T;
+  if (D->dtype == EOGP_BF16) {
+    o.ldA = round_up(D->d_in, 128);
+    o.ldS = round_up(D->d_out, 128);
+    o.at_hi = take(M * o.ldA * 2);
+    o.at_lo = take(M * o.ldA * 2);
+    o.st_hi = take(M * o.ldS * 2);
+    o.st_lo = take(M * o.ldS * 2);
+    const int n_tiles = (o.ldA / 128) * (o.ldS / 128);
+    o.n_chunks = ekfac_chunks(std::max(1, B), n_tiles, sm_count());
+    o.part = take(static_cast<size_t>(o.n_chunks) * D->d_out * D->d_in * 4);
+  } else {
+    o.at = take(M * D->d_in * 4);
+    o.st = take(M * D->d_out * 4);
+    o.g = take(static_cast<size_t>(D->d_out) * D->d_in * 4);
+  }
+  o.total = std::max<size_t>(off, 256);
+  return o;
+}
+
+}  // namespace
+
+extern "C" int eogp_ekfac_workspace_size(const eogp_ekfac_desc* D, int B, size_t* bytes) {
+  clear_error();
+  if (!bytes) return set_error(EOGP_EINVAL, "bytes is NULL");
+  if (int rc = ekfac_check(D, B)) return rc;
+  *bytes = ekfac_layout(D, B).total;
+  return EOGP_OK;
+}
+
+extern "C" int eogp_ekfac_accumulate(const eogp_ekfac_desc* D, const void* a, const void* s, int B,
+                                     double* sumsq, int ld, int accumulate, void* ws, size_t ws_bytes,
+                                     eogp_stream_t stream) {
+  clear_error();
+  if (int rc = ekfac_check(D, B)) return rc;
+  if (!sumsq || ld < D->d_in) return set_error(EOGP_EINVAL, "sumsq is NULL or ld < d_in");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (B == 0) {
+    if (!accumulate) CUDA_TRY(cudaMemset2DAsync(sumsq, static_cast<size_t>(ld) * 8, 0,
+                                                static_cast<size_t>(D->d_in) * 8, D->d_out, st));
+    return EOGP_OK;
+  }
+  if (!a || !s) return set_error(EOGP_EINVAL, "a / s is NULL");
+  const EkfacLayout lo = ekfac_layout(D, B);
+  if (!ws || ws_bytes < lo.total)
+    return set_error(EOGP_EWORKSPACE, "workspace of %zu bytes needed, %zu given", lo.total, ws_bytes);
+  if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
+  unsigned* status = status_word();
+  if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
+  char* w = static_cast<char*>(ws);
+  const int M = B * D->T;
+  if (D->dtype == EOGP_BF16) {
+    if (!aligned16(a) || !aligned16(s)) return set_error(EOGP_EINVAL, "a / s must be 16-byte aligned");
+    {
+      ProfScope ps(EOGP_K_ROTATE, st);
+      CUDA_TRY(launch_tc_rotate(M, D->d_in, a, D->d_in, D->VA, D->d_in, D->d_in, w + lo.at_hi,
+                                w + lo.at_lo, lo.ldA, D->T, sm_count(), status, st));
+    }
+    {
+      ProfScope ps(EOGP_K_ROTATE, st);
+      CUDA_TRY(launch_tc_rotate(M, D->d_out, s, D->d_out, D->VS, D->d_out, D->d_out, w + lo.st_hi,
+                                w + lo.st_lo, lo.ldS, D->T, sm_count(), status, st));
+    }
+    ProfScope ps(EOGP_K_CONTRACT, st);
+    CUDA_TRY(launch_tc_ekfac(w + lo.st_hi, w + lo.st_lo, lo.ldS, w + lo.at_hi, w + lo.at_lo, lo.ldA, B,
+                             D->T, D->d_out, D->d_in, reinterpret_cast<float*>(w + lo.part), lo.n_chunks,
+                             sumsq, ld, accumulate, kEkfacStages, sm_count(), status, st));
+    return EOGP_OK;
+  }
+  ProfScope ps(EOGP_K_SIMT, st);
+  float* at = reinterpret_cast<float*>(w + lo.at);
+  float* stt = reinterpret_cast<float*>(w + lo.st);
+  float* G = reinterpret_cast<float*>(w + lo.g);
+  CUDA_TRY(launch_simt_gemm(M, D->d_in, D->d_in, 1.f, static_cast<const float*>(a), D->d_in, 1,
+                            static_cast<const float*>(D->VA), D->d_in, 1, at, D->d_in, st));
+  CUDA_TRY(launch_simt_gemm(M, D->d_out, D->d_out, 1.f, static_cast<const float*>(s), D->d_out, 1,
+                            static_cast<const float*>(D->VS), D->d_out, 1, stt, D->d_out, st));
+  for (int b = 0; b < B; ++b) {
+    // G~_b[j][i] = sum_t S~[b T + t][j] A~[b T + t][i]
+    const float* sb = stt + static_cast<size_t>(b) * D->T * D->d_out;
+    const float* ab = at + static_cast<size_t>(b) * D->T * D->d_in;
+    CUDA_TRY(launch_simt_gemm(D->d_out, D->d_in, D->T, 1.f, sb, 1, D->d_out, ab, 1, D->d_in, G, D->d_in, st));
+    CUDA_TRY(launch_sq_accum(G, D->d_out, D->d_in, sumsq, ld, (accumulate || b > 0) ? 1 : 0, st));
+  }
+  return EOGP_OK;
+}
+
 // ================================================================ SRHT
 
 extern "C" int eogp_srht(const float* z, int B, int m, int ldz, const int8_t* signs, const int32_t* rows,

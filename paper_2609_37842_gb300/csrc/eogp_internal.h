@@ -110,6 +110,16 @@ cudaError_t launch_topk_dense(const float* scores, int ld, int Q, int N, int K, 
 cudaError_t launch_topk_merge(const float* lst, const int* lsi, int S, int Q, int K, float* out_s,
                               int ld_os, int* out_i, int ld_oi, cudaStream_t st);
 
+// EK-FAC eigenvalue correction (k_tc.cu, bf16; k_simt.cu, fp32).
+size_t ekfac_smem_bytes(int stages);
+int ekfac_chunks(int B, int n_tiles, int num_sms);
+cudaError_t launch_tc_ekfac(const void* St_hi, const void* St_lo, int ldS, const void* At_hi,
+                            const void* At_lo, int ldA, int B, int T, int d_out, int d_in, float* part,
+                            int n_chunks, double* sumsq, int ld, int accumulate, int stages, int num_sms,
+                            unsigned* status, cudaStream_t st);
+cudaError_t launch_sq_accum(const float* G, int rows, int cols, double* sumsq, int ld, int accumulate,
+                            cudaStream_t st);
+
 // k_srht.cu: EOGP-R second stage, one CTA per row (z fp32, or bf16 hi + lo when hilo).
 int srht_width(int m);
 size_t srht_smem_bytes(int m);

@@ -7,6 +7,8 @@
 //  k_contract_f32: one thread per (example, retained coordinate r):
 //    z[b][r] = scale[r] * sum_t S~[b,t][posR[r]] * A~[b,t][posC[r]]
 //    (Eq. first_stage through the Kronecker identity of Sec. 2.2).
+#include <algorithm>
+
 #include "eogp_dev.cuh"
 #include "eogp_internal.h"
 
@@ -124,5 +126,28 @@ cudaError_t launch_gather_rows(const void* src, int ld_src, int elem_bytes, cons
   else
     k_gather_rows<uint16_t><<<n_rows, 256, 0, st>>>(static_cast<const uint16_t*>(src), ld_src, idx,
                                                     row_len, static_cast<uint16_t*>(dst));
+  return cudaGetLastError();
+}
+
+namespace {
+// sumsq[j * ld + i] = (accumulate ? sumsq : 0) + G[j][i]^2 in fp64 (G dense [rows][cols]).
+__global__ void k_sq_accum(const float* __restrict__ G, int rows, int cols, double* __restrict__ sumsq,
+                           int ld, int accumulate) {
+  const long long n = static_cast<long long>(rows) * cols;
+  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < n;
+       e += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const double g = static_cast<double>(G[e]);
+    const size_t o = static_cast<size_t>(e / cols) * ld + e % cols;
+    sumsq[o] = accumulate ? sumsq[o] + g * g : g * g;
+  }
+}
+}  // namespace
+
+cudaError_t launch_sq_accum(const float* G, int rows, int cols, double* sumsq, int ld, int accumulate,
+                            cudaStream_t st) {
+  const long long n = static_cast<long long>(rows) * cols;
+  if (n <= 0) return cudaSuccess;
+  const unsigned blocks = static_cast<unsigned>(std::min<long long>((n + 255) / 256, 4096));
+  k_sq_accum<<<blocks, 256, 0, st>>>(G, rows, cols, sumsq, ld, accumulate);
   return cudaGetLastError();
 }

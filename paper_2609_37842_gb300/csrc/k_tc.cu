@@ -372,6 +372,203 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) tmem_dealloc(tmem, 256);
 }
 
+// k_tc_ekfac -- EK-FAC eigenvalue correction (Sec. 2.2 "EK-FAC approximation":
+// the mean square of each coordinate of the gradients in the K-FAC eigenbasis,
+// App. C.2: over examples, sequence-level gradients). For one 128 x 128 tile
+// (rt, ct) of the full d_out x d_in coordinate block and a run of examples,
+// G~_b[tile] is formed exactly as in k_tc_contract (3 MMAs per K step over the
+// tokens) and its squares are summed over the run in TMEM (columns 256..383),
+// so each item writes one fp32 partial tile. Items are chunk-major
+// (item = chunk * n_tiles + tile): CTAs running together read the same
+// examples' operands through L2.
+struct EkfacArgs {
+  int T, stages, n_rt, n_ct, n_tiles, n_items, bpc, B, nblkS, nblkA, d_out, d_in;
+  float* part;  // [n_chunks][d_out][d_in]
+  unsigned* status;
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_tc_ekfac(const __grid_constant__ CUtensorMap tmShi, const __grid_constant__ CUtensorMap tmSlo,
+               const __grid_constant__ CUtensorMap tmAhi, const __grid_constant__ CUtensorMap tmAlo,
+               const EkfacArgs g) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(g.stages) * kCStage);
+  uint64_t* empty = full + g.stages;
+  uint64_t* tfull = empty + g.stages;
+  uint64_t* tempty = tfull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  const int nkb = (g.T + 63) / 64;
+
+  if (threadIdx.x == 0) {
+    tma_prefetch_desc(&tmShi);
+    tma_prefetch_desc(&tmSlo);
+    tma_prefetch_desc(&tmAhi);
+    tma_prefetch_desc(&tmAlo);
+    for (int s = 0; s < g.stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 4);
+    }
+    fence_barrier_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < g.n_items && ok; item += gridDim.x) {
+        const int chunk = item / g.n_tiles, tile = item % g.n_tiles;
+        const int rt = tile / g.n_ct, ct = tile % g.n_ct;
+        const int b1 = min(g.B, (chunk + 1) * g.bpc);
+        for (int b = chunk * g.bpc; b < b1 && ok; ++b) {
+          const int zs = b * g.nblkS + rt, za = b * g.nblkA + ct;
+          for (int kb = 0; kb < nkb; ++kb, ++it) {
+            const int s = static_cast<int>(it % g.stages);
+            const uint32_t ph = (it / g.stages) & 1u;
+            if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) {
+              ok = false;
+              break;
+            }
+            uint8_t* st = smem + static_cast<size_t>(s) * kCStage;
+            mbar_arrive_expect_tx(&full[s], kCStage);
+            const int t0 = kb * 64;
+            tma_load_3d(st + 0 * kOpBytes, &tmShi, 0, t0, zs, &full[s]);
+            tma_load_3d(st + 0 * kOpBytes + 8192, &tmShi, 64, t0, zs, &full[s]);
+            tma_load_3d(st + 1 * kOpBytes, &tmSlo, 0, t0, zs, &full[s]);
+            tma_load_3d(st + 1 * kOpBytes + 8192, &tmSlo, 64, t0, zs, &full[s]);
+            tma_load_3d(st + 2 * kOpBytes, &tmAhi, 0, t0, za, &full[s]);
+            tma_load_3d(st + 2 * kOpBytes + 8192, &tmAhi, 64, t0, za, &full[s]);
+            tma_load_3d(st + 3 * kOpBytes, &tmAlo, 0, t0, za, &full[s]);
+            tma_load_3d(st + 3 * kOpBytes + 8192, &tmAlo, 64, t0, za, &full[s]);
+          }
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(128, 128, 1, 1);
+      uint32_t it = 0;
+      int i = 0;  // examples issued by this CTA (selects the TMEM buffer)
+      bool ok = true;
+      for (int item = blockIdx.x; item < g.n_items && ok; item += gridDim.x) {
+        const int chunk = item / g.n_tiles;
+        const int b1 = min(g.B, (chunk + 1) * g.bpc);
+        for (int b = chunk * g.bpc; b < b1 && ok; ++b, ++i) {
+          const int buf = i & 1;
+          const uint32_t aph = static_cast<uint32_t>(i >> 1) & 1u;
+          if (!mbar_wait(&tempty[buf], aph ^ 1u, g.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d = tmem + buf * 128u;
+          for (int kb = 0; kb < nkb; ++kb, ++it) {
+            const int s = static_cast<int>(it % g.stages);
+            const uint32_t ph = (it / g.stages) & 1u;
+            if (!mbar_wait(&full[s], ph, g.status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * kCStage);
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk) {
+              const uint32_t o = kk * 2048u;  // 16 token rows of 128 bytes
+              const uint64_t sh = sdesc_sw128(sa + 0 * kOpBytes + o, 8192, 1024);
+              const uint64_t sl = sdesc_sw128(sa + 1 * kOpBytes + o, 8192, 1024);
+              const uint64_t ah = sdesc_sw128(sa + 2 * kOpBytes + o, 8192, 1024);
+              const uint64_t al = sdesc_sw128(sa + 3 * kOpBytes + o, 8192, 1024);
+              tc_mma_f16(d, sh, ah, idesc, (kb | kk) != 0 ? 1u : 0u);
+              tc_mma_f16(d, sh, al, idesc, 1u);
+              tc_mma_f16(d, sl, ah, idesc, 1u);
+            }
+            tc_commit(&empty[s]);
+          }
+          tc_commit(&tfull[buf]);
+        }
+      }
+    }
+    __syncwarp();
+  } else {
+    const int q = warp & 3;
+    const uint32_t lane_base = static_cast<uint32_t>(q * 32) << 16;
+    const int row_in = q * 32 + lane;
+    int i = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < g.n_items && ok; item += gridDim.x) {
+      const int chunk = item / g.n_tiles, tile = item % g.n_tiles;
+      const int rt = tile / g.n_ct, ct = tile % g.n_ct;
+      const int b0 = chunk * g.bpc, b1 = min(g.B, (chunk + 1) * g.bpc);
+      for (int b = b0; b < b1; ++b, ++i) {
+        const int buf = i & 1;
+        const uint32_t aph = static_cast<uint32_t>(i >> 1) & 1u;
+        uint32_t w_ok = 1;
+        if (lane == 0) w_ok = mbar_wait(&tfull[buf], aph, g.status) ? 1u : 0u;
+        w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
+        __syncwarp();
+        tc_fence_after();
+        if (!__syncthreads_and_named(w_ok)) {
+          ok = false;
+          break;
+        }
+        for (int j = 0; j < 4; ++j) {
+          float v[32], acc[32];
+          tmem_ld32(tmem + lane_base + buf * 128u + 32 * j, v);
+          if (b == b0) {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) acc[c] = __fmul_rn(v[c], v[c]);
+          } else {
+            tmem_ld32(tmem + lane_base + 256u + 32 * j, acc);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) acc[c] = __fadd_rn(acc[c], __fmul_rn(v[c], v[c]));
+          }
+          if (b + 1 < b1) {
+            tmem_st32(tmem + lane_base + 256u + 32 * j, acc);
+          } else {
+            const int row = rt * 128 + row_in, col0 = ct * 128 + 32 * j;
+            if (row < g.d_out) {
+              float* dst = g.part + (static_cast<size_t>(chunk) * g.d_out + row) * g.d_in + col0;
+#pragma unroll
+              for (int c = 0; c < 32; ++c)
+                if (col0 + c < g.d_in) dst[c] = acc[c];
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_relaxed(&tempty[buf]);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+// sumsq[j * ld + i] (+)= sum over chunks c of part[c][j][i], chunks in order (fp64).
+__global__ void k_ekfac_finalize(const float* __restrict__ part, int n_chunks, int d_out, int d_in,
+                                 double* __restrict__ sumsq, int ld, int accumulate) {
+  const size_t n = static_cast<size_t>(d_out) * d_in;
+  for (size_t e = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; e < n;
+       e += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    double t = 0.0;
+    for (int c = 0; c < n_chunks; ++c) t += static_cast<double>(part[static_cast<size_t>(c) * n + e]);
+    const size_t o = (e / d_in) * static_cast<size_t>(ld) + e % d_in;
+    sumsq[o] = accumulate ? sumsq[o] + t : t;
+  }
+}
+
 size_t gemm_smem_bytes(int BN, int stages, int nA) {
   return 1024 + static_cast<size_t>(stages) * (nA * kABytes + BN * 128u) + (2 * stages + 1) * 8 + 16;
 }
@@ -906,5 +1103,55 @@ cudaError_t launch_tc_contract(const void* St_hi, const void* St_lo, int ldS, co
   if (e != cudaSuccess) return e;
   const int grid = std::min(g.n_items, std::max(1, num_sms));
   k_tc_contract<<<grid, kThreads, smem, st>>>(tSh, tSl, tAh, tAl, g);
+  return cudaGetLastError();
+}
+
+size_t ekfac_smem_bytes(int stages) {
+  return 1024 + static_cast<size_t>(stages) * kCStage + (2 * stages + 4) * 8 + 16;
+}
+
+int ekfac_chunks(int B, int n_tiles, int num_sms) {
+  // Enough items for about two per SM, each chunk as long as possible.
+  const int want_items = 2 * std::max(1, num_sms);
+  int nch = std::max(1, std::min(B, (want_items + n_tiles - 1) / n_tiles));
+  const int bpc = (B + nch - 1) / nch;
+  return (B + bpc - 1) / bpc;
+}
+
+cudaError_t launch_tc_ekfac(const void* St_hi, const void* St_lo, int ldS, const void* At_hi,
+                            const void* At_lo, int ldA, int B, int T, int d_out, int d_in, float* part,
+                            int n_chunks, double* sumsq, int ld, int accumulate, int stages, int num_sms,
+                            unsigned* status, cudaStream_t st) {
+  if (B <= 0) return cudaSuccess;
+  CUtensorMap tSh, tSl, tAh, tAl;
+  const uint64_t nS = static_cast<uint64_t>(B) * (ldS / 128), nA = static_cast<uint64_t>(B) * (ldA / 128);
+  if (tmap_bf16_blocked(&tSh, St_hi, T, nS) || tmap_bf16_blocked(&tSl, St_lo, T, nS) ||
+      tmap_bf16_blocked(&tAh, At_hi, T, nA) || tmap_bf16_blocked(&tAl, At_lo, T, nA))
+    return cudaErrorInvalidValue;
+  EkfacArgs g;
+  g.T = T;
+  g.stages = stages;
+  g.n_rt = (d_out + 127) / 128;
+  g.n_ct = (d_in + 127) / 128;
+  g.n_tiles = g.n_rt * g.n_ct;
+  g.bpc = (B + n_chunks - 1) / n_chunks;
+  g.n_items = g.n_tiles * ((B + g.bpc - 1) / g.bpc);
+  g.B = B;
+  g.nblkS = ldS / 128;
+  g.nblkA = ldA / 128;
+  g.d_out = d_out;
+  g.d_in = d_in;
+  g.part = part;
+  g.status = status;
+  const size_t smem = ekfac_smem_bytes(stages);
+  cudaError_t e = cudaFuncSetAttribute(k_tc_ekfac, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  const int grid = std::min(g.n_items, std::max(1, num_sms));
+  k_tc_ekfac<<<grid, kThreads, smem, st>>>(tSh, tSl, tAh, tAl, g);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_ekfac_finalize<<<std::max(1, num_sms) * 4, 256, 0, st>>>(part, (B + g.bpc - 1) / g.bpc, d_out, d_in,
+                                                            sumsq, ld, accumulate);
   return cudaGetLastError();
 }

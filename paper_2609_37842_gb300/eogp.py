@@ -47,6 +47,11 @@ class LayerDesc(ctypes.Structure):
                 ("plan", c_void_p), ("srht_signs", c_void_p), ("srht_rows", c_void_p)]
 
 
+class EkfacDesc(ctypes.Structure):
+    _fields_ = [("d_in", c_int), ("d_out", c_int), ("T", c_int), ("dtype", c_int),
+                ("VA", c_void_p), ("VS", c_void_p)]
+
+
 EXPORTS = {
     # name: (restype, argtypes)
     "eogp_last_error": (ctypes.c_char_p, []),
@@ -68,6 +73,9 @@ EXPORTS = {
     "eogp_compress_layer_static": (c_int, [POINTER(LayerDesc), c_void_p, c_void_p, c_int, c_int,
                                            c_void_p, c_int, c_void_p, c_int, c_void_p, c_int,
                                            c_void_p]),
+    "eogp_ekfac_workspace_size": (c_int, [POINTER(EkfacDesc), c_int, POINTER(c_size_t)]),
+    "eogp_ekfac_accumulate": (c_int, [POINTER(EkfacDesc), c_void_p, c_void_p, c_int, c_void_p, c_int,
+                                      c_int, c_void_p, c_size_t, c_void_p]),
     "eogp_fit_pca_workspace_size": (c_int, [c_int, c_int, c_int, POINTER(c_size_t)]),
     "eogp_fit_pca": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int,
                              c_void_p, c_void_p, c_size_t, c_void_p]),
@@ -295,6 +303,41 @@ def compress_layer(desc: LayerDesc, a, s, out_mode: int, out=None, codes=None, s
 
 
 # ------------------------------------------------------------------ fit PCA
+def ekfac_desc(T: int, VA, VS) -> EkfacDesc:
+    """EK-FAC correction descriptor: VA [d_in, d_in], VS [d_out, d_out] with the
+    eigenvectors as rows (full bases). Keeps references to the tensors."""
+    _dense(VA, "VA")
+    _dense(VS, "VS")
+    d = EkfacDesc(VA.shape[1], VS.shape[1], int(T), _dtype_code(VA), _ptr(VA), _ptr(VS))
+    d._refs = (VA, VS)
+    return d
+
+
+def ekfac_workspace_size(desc: EkfacDesc, B: int) -> int:
+    n = c_size_t()
+    _check(lib().eogp_ekfac_workspace_size(ctypes.byref(desc), int(B), ctypes.byref(n)))
+    return n.value
+
+
+def ekfac_accumulate(desc: EkfacDesc, a, s, sumsq=None, accumulate: bool = False, ws=None,
+                     stream=None):
+    """eogp_ekfac_accumulate: sumsq [d_out, d_in] fp64 (+)= sum_b (Q_S^T G_b Q_A)^2."""
+    import torch
+    _dense(a, "a")
+    _dense(s, "s")
+    B = a.shape[0]
+    dev = a.device
+    if sumsq is None:
+        sumsq = torch.zeros((desc.d_out, desc.d_in), dtype=torch.float64, device=dev)
+    _rows(sumsq, "sumsq")
+    if ws is None:
+        ws = workspace(ekfac_workspace_size(desc, B), dev)
+    _check(lib().eogp_ekfac_accumulate(ctypes.byref(desc), _ptr(a), _ptr(s), B, _ptr(sumsq),
+                                       sumsq.stride(0), 1 if accumulate else 0, _ptr(ws), ws.numel(),
+                                       _stream(stream)))
+    return sumsq
+
+
 def fit_pca_workspace_size(n: int, m: int, k: int) -> int:
     v = c_size_t()
     _check(lib().eogp_fit_pca_workspace_size(int(n), int(m), int(k), ctypes.byref(v)))

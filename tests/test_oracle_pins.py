@@ -399,6 +399,30 @@ def test_srht():
     check_srht(O, 37)
 
 
+def check_ekfac(Om, seed):
+    """EK-FAC correction pins: the squared coordinates of vec(G_b) under the
+    dense Kronecker basis (Q_A (x) Q_S)^T, summed over examples; their total
+    equals sum_b ||G_b||_F^2 (the basis is orthonormal); one token of one
+    example gives the outer product of the squared rotated factors."""
+    rng = np.random.default_rng(seed)
+    B, T, d_in, d_out = 3, 4, 5, 6
+    QA, QS = haar(d_in, rng), haar(d_out, rng)
+    a, s = rng.standard_normal((B, T, d_in)), rng.standard_normal((B, T, d_out))
+    got = Om.ekfac_sumsq(a, s, QA, QS)
+    K = np.kron(QA, QS)
+    want = sum((K.T @ vec(sum(np.outer(s[b, t], a[b, t]) for t in range(T)))) ** 2 for b in range(B))
+    np.testing.assert_allclose(vec(got), want, rtol=1e-12, atol=1e-14)
+    tot = sum(np.sum(sum(np.outer(s[b, t], a[b, t]) for t in range(T)) ** 2) for b in range(B))
+    assert got.sum() == pytest.approx(tot, rel=1e-12)
+    one = Om.ekfac_sumsq(a[:1, :1], s[:1, :1], QA, QS)
+    np.testing.assert_allclose(one, np.outer((QS.T @ s[0, 0]) ** 2, (QA.T @ a[0, 0]) ** 2),
+                               rtol=1e-12, atol=1e-15)
+
+
+def test_ekfac_correction():
+    check_ekfac(O, 41)
+
+
 def _golden_rows(name):
     with open(os.path.join(GOLDEN, name)) as f:
         return [ln.split() for ln in f if ln.strip() and not ln.startswith("#")]
@@ -503,3 +527,11 @@ def test_planted_srht_mistakes_are_caught(monkeypatch):
     assert _fails(check_srht, O, 37)          # normalisation dropped
     monkeypatch.setattr(O, "srht", lambda z, sg, rows: orig(z, -np.asarray(sg, np.float64), rows)[:, ::-1])
     assert _fails(check_srht, O, 37)          # rows reversed
+
+
+def test_planted_ekfac_mistakes_are_caught(monkeypatch):
+    orig = O.ekfac_sumsq
+    monkeypatch.setattr(O, "ekfac_sumsq", lambda a, s, QA, QS: orig(a, s, QA, QS) / np.asarray(a).shape[0])
+    assert _fails(check_ekfac, O, 41)         # mean instead of sum
+    monkeypatch.setattr(O, "ekfac_sumsq", lambda a, s, QA, QS: orig(np.asarray(a)[:, ::-1], s, QA, QS))
+    assert _fails(check_ekfac, O, 41)         # tokens of a and s paired wrongly
