@@ -174,6 +174,16 @@ typedef struct {
      k <= p = 2^ceil(log2 m) and m <= EOGP_SRHT_MAX_M.                       */
   const int8_t* srht_signs;  /* device [m]: diagonal of D (< 0 means -1)      */
   const int32_t* srht_rows;  /* device [k]: rows of H_p kept by R, in [0, p)   */
+  /* Real-workload plumbing (App. C.1): */
+  const float* bias_A;  /* device [nC] fp32, or NULL. Non-NULL: the module has a
+                           bias (GPT-2 attributes biases), treated as a constant-1
+                           input channel appended after the d_in activations: the
+                           plan and Q_A are over d_in + 1 inputs, VA holds the
+                           first d_in components of the retained eigenvectors and
+                           bias_A[r] = Q_A[d_in][C[r]], their bias-channel component */
+  const int32_t* lengths;  /* device [B] or NULL: example b keeps tokens
+                           t < lengths[b] (0 <= lengths[b] <= T); later positions
+                           are padding and contribute nothing (as s_t = 0)        */
 } eogp_layer_desc;
 
 /* Workspace bytes eogp_compress_layer needs for this descriptor, batch B and

@@ -23,6 +23,8 @@ Function map:
   kfac_eigenvalues      Sec. 2.2 (eigenvalues of A (x) S)
   damping               App. C.2, Eq. app_module_damping
   select_retained       Sec. 3.2 (Eq. sigma_ekfac and the text after it), Alg. 1
+  with_bias_channel     App. C.1 (biases as a constant-1 input channel)
+  mask_tokens           App. C.1 (variable-length examples padded to T)
   per_example_gradient  Sec. 2.2 (K-FAC factors from a and delta)
   rotate                Sec. 2.2 (apply Q_A (x) Q_S through its two factors)
   ekfac_sumsq           Sec. 2.2 "EK-FAC approximation"; App. C.2 (corrected eigenvalues)
@@ -89,6 +91,24 @@ def select_retained(Lam: np.ndarray, m: int) -> Tuple[np.ndarray, np.ndarray]:
 # --------------------------------------------------------------------------
 # First stage
 # --------------------------------------------------------------------------
+
+def with_bias_channel(a: np.ndarray) -> np.ndarray:
+    """Activations with a constant-1 channel appended (App. C.1: GPT-2's biases
+    are attributed; a bias is the weight of an input that is always 1, so the
+    bias gradient sum_t s_t is the last column of G)."""
+    a = np.asarray(a, np.float64)
+    return np.concatenate([a, np.ones(a.shape[:-1] + (1,))], axis=-1)
+
+
+def mask_tokens(s: np.ndarray, lengths) -> np.ndarray:
+    """Output gradients with the padding positions t >= lengths[b] of each
+    example zeroed, so only the example's own tokens enter G_b (App. C.1:
+    examples are conversations of at most 2048 tokens)."""
+    s = np.array(s, np.float64)
+    for b, n in enumerate(lengths):
+        s[b, int(n):] = 0.0
+    return s
+
 
 def per_example_gradient(a_b: np.ndarray, s_b: np.ndarray) -> np.ndarray:
     """G = sum_t s_t a_t^T, a d_out x d_in matrix, from one example's activations

@@ -509,9 +509,11 @@ int check_desc(const eogp_layer_desc* L, int B, int mode) {
   if (!L) return set_error(EOGP_EINVAL, "descriptor is NULL");
   if (!L->plan) return set_error(EOGP_EINVAL, "descriptor has no plan");
   const eogp_plan* P = L->plan;
-  if (L->d_in != P->d_in || L->d_out != P->d_out || L->m != P->m)
-    return set_error(EOGP_EINVAL, "descriptor shape (%d, %d, m=%d) differs from the plan (%d, %d, m=%d)",
-                     L->d_in, L->d_out, L->m, P->d_in, P->d_out, P->m);
+  const int bias = L->bias_A ? 1 : 0;
+  if (L->d_in + bias != P->d_in || L->d_out != P->d_out || L->m != P->m)
+    return set_error(EOGP_EINVAL,
+                     "descriptor shape (%d%s, %d, m=%d) differs from the plan (%d, %d, m=%d)", L->d_in,
+                     bias ? " + bias" : "", L->d_out, L->m, P->d_in, P->d_out, P->m);
   if (L->T < 1) return set_error(EOGP_EINVAL, "T must be >= 1");
   if (B < 0) return set_error(EOGP_EINVAL, "B must be >= 0");
   if (mode < EOGP_OUT_FIRST_STAGE || mode > EOGP_OUT_CODES) return set_error(EOGP_EINVAL, "bad out_mode");
@@ -588,12 +590,12 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
     {
       ProfScope ps(EOGP_K_ROTATE, st);
       CUDA_TRY(launch_tc_rotate(M, L->d_in, a, L->d_in, L->VA, L->d_in, P->nC(), at_hi, at_lo,
-                                lo.ldA, L->T, sm_count(), status, st));
+                                lo.ldA, L->T, L->bias_A, nullptr, sm_count(), status, st));
     }
     {
       ProfScope ps(EOGP_K_ROTATE, st);
       CUDA_TRY(launch_tc_rotate(M, L->d_out, s, L->d_out, L->VS, L->d_out, P->nR(), st_hi, st_lo,
-                                lo.ldS, L->T, sm_count(), status, st));
+                                lo.ldS, L->T, nullptr, L->lengths, sm_count(), status, st));
     }
     // Per-example contraction over tokens + scale/gather into z (Eq. first_stage).
     const bool fs = out_mode == EOGP_OUT_FIRST_STAGE;
@@ -643,6 +645,8 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
                             L->d_in, 1, at, nC, st));
   CUDA_TRY(launch_simt_gemm(M, nR, L->d_out, 1.f, sf, L->d_out, 1, static_cast<const float*>(L->VS),
                             L->d_out, 1, stt, nR, st));
+  CUDA_TRY(launch_rows_fixup(at, M, nC, nC, L->T, L->bias_A, nullptr, st));
+  CUDA_TRY(launch_rows_fixup(stt, M, nR, nR, L->T, nullptr, L->lengths, st));
   float* z = out_mode == EOGP_OUT_FIRST_STAGE ? out : reinterpret_cast<float*>(w + lo.z);
   const int ldz = out_mode == EOGP_OUT_FIRST_STAGE ? ld_out : L->m;
   CUDA_TRY(launch_contract_f32(at, nC, stt, nR, B, L->T, L->m, P->d_posR, P->d_posC, P->d_scale, z,
@@ -755,12 +759,12 @@ extern "C" int eogp_ekfac_accumulate(const eogp_ekfac_desc* D, const void* a, co
     {
       ProfScope ps(EOGP_K_ROTATE, st);
       CUDA_TRY(launch_tc_rotate(M, D->d_in, a, D->d_in, D->VA, D->d_in, D->d_in, w + lo.at_hi,
-                                w + lo.at_lo, lo.ldA, D->T, sm_count(), status, st));
+                                w + lo.at_lo, lo.ldA, D->T, nullptr, nullptr, sm_count(), status, st));
     }
     {
       ProfScope ps(EOGP_K_ROTATE, st);
       CUDA_TRY(launch_tc_rotate(M, D->d_out, s, D->d_out, D->VS, D->d_out, D->d_out, w + lo.st_hi,
-                                w + lo.st_lo, lo.ldS, D->T, sm_count(), status, st));
+                                w + lo.st_lo, lo.ldS, D->T, nullptr, nullptr, sm_count(), status, st));
     }
     ProfScope ps(EOGP_K_CONTRACT, st);
     CUDA_TRY(launch_tc_ekfac(w + lo.st_hi, w + lo.st_lo, lo.ldS, w + lo.at_hi, w + lo.at_lo, lo.ldA, B,

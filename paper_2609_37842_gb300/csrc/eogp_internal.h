@@ -117,6 +117,8 @@ cudaError_t launch_tc_ekfac(const void* St_hi, const void* St_lo, int ldS, const
                             const void* At_lo, int ldA, int B, int T, int d_out, int d_in, float* part,
                             int n_chunks, double* sumsq, int ld, int accumulate, int stages, int num_sms,
                             unsigned* status, cudaStream_t st);
+cudaError_t launch_rows_fixup(float* X, int M, int n, int ld, int T, const float* bias,
+                              const int32_t* lengths, cudaStream_t st);
 cudaError_t launch_sq_accum(const float* G, int rows, int cols, double* sumsq, int ld, int accumulate,
                             cudaStream_t st);
 
@@ -156,8 +158,8 @@ cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, 
 // (a multiple of 128), rows M = B * T, written in the blocked layout
 // [B][ldo / 128][T][128] that launch_tc_contract reads.
 cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W, int ldw, int Wrows,
-                             void* hi, void* lo, int ldo, int T, int num_sms, unsigned* status,
-                             cudaStream_t st);
+                             void* hi, void* lo, int ldo, int T, const float* bias,
+                             const int32_t* lengths, int num_sms, unsigned* status, cudaStream_t st);
 // Number of K splits launch_tc_gemm actually uses for a requested count.
 int tc_gemm_splits_used(int K, int splits);
 // Per-example tile-sparse contraction over tokens with the scale-and-gather epilogue.

@@ -151,3 +151,31 @@ cudaError_t launch_sq_accum(const float* G, int rows, int cols, double* sumsq, i
   k_sq_accum<<<blocks, 256, 0, st>>>(G, rows, cols, sumsq, ld, accumulate);
   return cudaGetLastError();
 }
+
+namespace {
+// Row fix-ups of a rotated token matrix X [M x n] (row = b * T + t): add the
+// bias-channel term bias[c], or zero the rows of tokens t >= lengths[b].
+__global__ void k_rows_fixup(float* __restrict__ X, int M, int n, int ld, int T, const float* __restrict__ bias,
+                             const int32_t* __restrict__ lengths) {
+  const long long tot = static_cast<long long>(M) * n;
+  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < tot;
+       e += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int row = static_cast<int>(e / n), c = static_cast<int>(e % n);
+    float* p = X + static_cast<size_t>(row) * ld + c;
+    if (lengths && row % T >= lengths[row / T]) {
+      *p = 0.f;
+    } else if (bias) {
+      *p += bias[c];
+    }
+  }
+}
+}  // namespace
+
+cudaError_t launch_rows_fixup(float* X, int M, int n, int ld, int T, const float* bias,
+                              const int32_t* lengths, cudaStream_t st) {
+  const long long tot = static_cast<long long>(M) * n;
+  if (tot <= 0 || (!bias && !lengths)) return cudaSuccess;
+  const unsigned blocks = static_cast<unsigned>(std::min<long long>((tot + 255) / 256, 8192));
+  k_rows_fixup<<<blocks, 256, 0, st>>>(X, M, n, ld, T, bias, lengths);
+  return cudaGetLastError();
+}

@@ -589,11 +589,29 @@ size_t contract_smem_bytes(int stages) {
 // element (row = b*T + t, col) sits at ((b * (ldo/128) + col/128) * T + t) * 128
 // + col % 128, so one 128-column block of one example is T*256 contiguous bytes.
 struct RotArgs {
-  int M, K, BN, stages, nN, n_tiles, ldo, T;
+  int M, K, BN, stages, nN, n_tiles, ldo, T, nbias;
   __nv_bfloat16* hi;
   __nv_bfloat16* lo;
+  const float* bias;        // per output column (the constant-1 input channel), or null
+  const int32_t* lengths;   // tokens kept per example (later tokens give 0), or null
   unsigned* status;
 };
+
+// Bias channel and token lengths, applied to one 32-column chunk of one output
+// row before the hi/lo split.
+__device__ __forceinline__ void rot_fixup(const RotArgs& g, int row, int col, float (&v)[32]) {
+  if (g.bias) {
+#pragma unroll
+    for (int e = 0; e < 32; ++e) v[e] += col + e < g.nbias ? __ldg(g.bias + col + e) : 0.f;
+  }
+  if (g.lengths) {
+    const int bex = row / g.T;
+    if (row - bex * g.T >= __ldg(g.lengths + bex)) {
+#pragma unroll
+      for (int e = 0; e < 32; ++e) v[e] = 0.f;
+    }
+  }
+}
 
 __global__ void __launch_bounds__(kThreads, 1)
     k_tc_rotate(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
@@ -704,6 +722,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld32(tb + c, v);
         const int col = n0 + c;
         if (row < g.M && col < g.ldo) {
+          rot_fixup(g, row, col, v);
           uint32_t h[16], l[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
@@ -869,6 +888,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         tmem_ld32(tb + c, v);
         const int col = n0 + c;
         if (row < g.M && col < g.ldo) {
+          rot_fixup(g, row, col, v);
           uint32_t h[16], l[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
@@ -1008,8 +1028,8 @@ int rotate_bn(int ldo) {
 }
 
 cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W, int ldw, int Wrows,
-                             void* hi, void* lo, int ldo, int T, int num_sms, unsigned* status,
-                             cudaStream_t st) {
+                             void* hi, void* lo, int ldo, int T, const float* bias,
+                             const int32_t* lengths, int num_sms, unsigned* status, cudaStream_t st) {
   if (M <= 0) return cudaSuccess;
   const int BN = rotate_bn(ldo);
   // As many pipeline stages as fit in 227 KB of shared memory (at most 8);
@@ -1037,6 +1057,9 @@ cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W
   g.T = T;
   g.hi = static_cast<__nv_bfloat16*>(hi);
   g.lo = static_cast<__nv_bfloat16*>(lo);
+  g.bias = bias;
+  g.nbias = Wrows;
+  g.lengths = lengths;
   g.status = status;
   if (rotate_pairs(K) && BN % 32 == 0) {
     // CTA pairs: tiles of 256 rows, W split in halves of BN / 2 rows.

@@ -78,7 +78,7 @@ def test_gpt2_stack_in_bench_launch_configuration():
     for u in (0, 1, 2, 3, 47):    # c_attn, attn.c_proj, c_fc, mlp.c_proj (first block), last module
         md = mods[u]
         desc = md["desc"]
-        plan, VA, VS, Pt = desc._refs
+        plan, VA, VS, Pt = desc._refs[:4]
         x = E.compress_layer(desc, md["a"], md["s"], E.OUT_COORDS, ws=ws)
         E.sync_status()
         R, C = plan.sets()

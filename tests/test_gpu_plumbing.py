@@ -1,0 +1,90 @@
+"""GPU parity of the real-workload plumbing of the compression call against
+the oracle: a module bias as a constant-1 input channel (App. C.1, GPT-2
+attributes biases) and variable-length examples padded to T (App. C.1,
+conversations of at most 2048 tokens), separately and together, on the bf16
+tensor-core path (within 2e-3 per row) and the fp32 path (within 1e-5).
+"""
+import numpy as np
+import pytest
+
+from oracle import eogp_oracle as O
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from paper_2609_37842_gb300 import eogp as E  # noqa: E402
+from paper_2609_37842_gb300 import synth  # noqa: E402
+
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_37842_gb300 import build
+    build.build()
+    E.lib()
+    yield
+    torch.cuda.empty_cache()
+
+
+def dev(a, dt=None):
+    t = torch.from_numpy(np.ascontiguousarray(a)).to(DEV)
+    return t.to(dt) if dt is not None else t
+
+
+def row_rel(got, want):
+    return np.linalg.norm(got - want, axis=1) / np.linalg.norm(want, axis=1)
+
+
+@pytest.mark.parametrize("dtype,d_in,d_out,T,B,m,k,bias,lens,tol", [
+    ("bf16", 768, 768, 100, 4, 4096, 1024, True, False, 2e-3),
+    ("bf16", 256, 384, 128, 5, 2000, 300, False, True, 2e-3),
+    ("bf16", 768, 2304, 130, 3, 4096, 1024, True, True, 2e-3),
+    ("f32", 64, 64, 16, 6, 512, 128, True, True, 1e-5),
+])
+def test_bias_and_lengths(dtype, d_in, d_out, T, B, m, k, bias, lens, tol):
+    rng = np.random.default_rng(d_in + T + B)
+    rnd = (lambda v: synth.round_to(v, dtype))
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    d_eff = d_in + (1 if bias else 0)
+    QA, QS = rnd(synth.haar_orthogonal(d_eff, rng)), rnd(synth.haar_orthogonal(d_out, rng))
+    lamA, lamS = synth.power_spectrum(d_eff, 1.2), synth.power_spectrum(d_out, 1.2)
+    a = rnd(rng.standard_normal((B, T, d_in)))
+    s = rnd(rng.standard_normal((B, T, d_out)) * 0.1)
+    lengths = rng.integers(1, T + 1, B).astype(np.int32) if lens else None
+    if lens:
+        lengths[0] = T          # one full example, and one cut very short
+        lengths[-1] = 1
+    Pt = rnd(synth.haar_orthogonal(m, rng, k).T)
+    plan = E.Plan.from_factors(lamS, lamA, m, 0.1)
+    R, C = plan.sets()
+    VA_full = QA.T[C]                       # [nC, d_eff]: retained eigenvectors as rows
+    VA = np.ascontiguousarray(VA_full[:, :d_in], dtype=np.float32)
+    bias_A = np.ascontiguousarray(VA_full[:, d_in], dtype=np.float32) if bias else None
+    VS = np.ascontiguousarray(QS.T[R], dtype=np.float32)
+    desc = E.layer_desc(plan, T, k, dev(VA, tdt), dev(VS, tdt), dev(Pt.astype(np.float32), tdt),
+                        bias_A=dev(bias_A) if bias else None,
+                        lengths=dev(lengths) if lens else None)
+    ad, sd = dev(a.astype(np.float32), tdt), dev(s.astype(np.float32), tdt)
+    x = E.compress_layer(desc, ad, sd, E.OUT_COORDS)
+    codes, scales = E.compress_layer(desc, ad, sd, E.OUT_CODES)
+    E.sync_status()
+    a_or = O.with_bias_channel(a) if bias else a
+    s_or = O.mask_tokens(s, lengths) if lens else s
+    Lam = O.kfac_eigenvalues(lamS, lamA)
+    z_or = O.first_stage(a_or, s_or, QA, QS, Lam, O.damping(Lam, 0.1), m)
+    x_or = O.project(z_or, Pt.astype(np.float64).T)
+    rel = row_rel(x.cpu().numpy().astype(np.float64), x_or)
+    print(f"max row rel err {rel.max():.2e}")
+    assert rel.max() <= tol
+    bits, sc = O.onebit(x_or)
+    got = O.unpack_bits(codes.cpu().numpy().view(np.uint32), k)
+    small = np.abs(x_or) < 1e-4 * np.linalg.norm(x_or, axis=1, keepdims=True)
+    assert not ((got != bits) & ~small).any()
+    np.testing.assert_allclose(scales.cpu().numpy(), sc, rtol=max(tol, 1e-5))
+    if bias:   # the bias channel changes the result (the term is really used)
+        z_nob = O.first_stage(np.concatenate([a, np.zeros(a.shape[:-1] + (1,))], -1), s_or, QA, QS,
+                              Lam, O.damping(Lam, 0.1), m)
+        assert row_rel(O.project(z_nob, Pt.astype(np.float64).T), x_or).min() > 10 * rel.max()

@@ -423,6 +423,28 @@ def test_ekfac_correction():
     check_ekfac(O, 41)
 
 
+def check_plumbing(Om, seed):
+    """Bias channel: the last column of G for [a; 1] is sum_t s_t and the other
+    columns are G for a. Token lengths: G_b from the masked s equals the sum
+    over the example's own tokens only."""
+    rng = np.random.default_rng(seed)
+    T, d_in, d_out = 6, 4, 3
+    a, s = rng.standard_normal((2, T, d_in)), rng.standard_normal((2, T, d_out))
+    ab = Om.with_bias_channel(a)
+    assert ab.shape == (2, T, d_in + 1) and (ab[..., -1] == 1).all() and (ab[..., :-1] == a).all()
+    G = Om.per_example_gradient(ab[0], s[0])
+    np.testing.assert_allclose(G[:, -1], s[0].sum(0), rtol=1e-13)
+    np.testing.assert_allclose(G[:, :-1], Om.per_example_gradient(a[0], s[0]), rtol=1e-13)
+    sm = Om.mask_tokens(s, [4, 0])
+    want = sum(np.outer(s[0, t], a[0, t]) for t in range(4))
+    np.testing.assert_allclose(Om.per_example_gradient(a[0], sm[0]), want, rtol=1e-13)
+    assert not Om.per_example_gradient(a[1], sm[1]).any()
+
+
+def test_bias_channel_and_token_lengths():
+    check_plumbing(O, 43)
+
+
 def _golden_rows(name):
     with open(os.path.join(GOLDEN, name)) as f:
         return [ln.split() for ln in f if ln.strip() and not ln.startswith("#")]
@@ -535,3 +557,13 @@ def test_planted_ekfac_mistakes_are_caught(monkeypatch):
     assert _fails(check_ekfac, O, 41)         # mean instead of sum
     monkeypatch.setattr(O, "ekfac_sumsq", lambda a, s, QA, QS: orig(np.asarray(a)[:, ::-1], s, QA, QS))
     assert _fails(check_ekfac, O, 41)         # tokens of a and s paired wrongly
+
+
+def test_planted_plumbing_mistakes_are_caught(monkeypatch):
+    orig = O.mask_tokens
+    monkeypatch.setattr(O, "mask_tokens", lambda s, n: orig(s, [int(x) + 1 for x in n]))
+    assert _fails(check_plumbing, O, 43)      # off-by-one length
+    monkeypatch.setattr(O, "mask_tokens", orig)
+    ob = O.with_bias_channel
+    monkeypatch.setattr(O, "with_bias_channel", lambda a: ob(a)[..., ::-1])
+    assert _fails(check_plumbing, O, 43)      # bias channel first instead of last
