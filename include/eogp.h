@@ -344,6 +344,29 @@ int eogp_score(const void* train, int ld_train, const float* train_scales, int l
                const float* query_scales, int ld_qscale, int Q, float* scores, int ld_scores,
                void* ws, size_t ws_bytes, eogp_stream_t stream);
 
+/* ---- store records (App. E.1, Eq. app_payload) --------------------------
+ * Per example, for each module u in order: ceil(k_u / 8) bytes of signs
+ * (coordinate c at bit c % 8 of byte c / 8) followed by the module's scale as
+ * an IEEE half (round to nearest even, little-endian): sum_u (ceil(k_u/8) + 2)
+ * bytes, the paper's per-example payload. The paper does not fix the order of
+ * signs and scale inside a module's record; signs come first here. */
+int eogp_payload_bytes(const int* k_per_module, int U, size_t* bytes_per_example);
+
+/* codes [N x ld_codes] uint32 (modules at their word offsets, as eogp_score
+ * reads them) and scales [N x ld_scales] fp32, device -> payload [N x
+ * ld_payload] bytes, device (ld_payload >= eogp_payload_bytes). Pad bits of
+ * a partial last byte are written as 0.
+ * Errors: EOGP_EINVAL, EOGP_ECUDA. */
+int eogp_payload_pack(const uint32_t* codes, int ld_codes, const float* scales, int ld_scales, int N,
+                      const int* k_per_module, int U, uint8_t* payload, size_t ld_payload,
+                      eogp_stream_t stream);
+
+/* Inverse of eogp_payload_pack: payload -> codes (pad bits and pad words 0)
+ * and scales (the stored halves, exactly), device.
+ * Errors: EOGP_EINVAL, EOGP_ECUDA. */
+int eogp_payload_unpack(const uint8_t* payload, size_t ld_payload, int N, const int* k_per_module, int U,
+                        uint32_t* codes, int ld_codes, float* scales, int ld_scales, eogp_stream_t stream);
+
 /* ---- ranking (App. C: stored examples ranked per query by score, descending;
  * NDCG@20 reads the first 20) ------------------------------------------- */
 #define EOGP_TOPK_MAX 256

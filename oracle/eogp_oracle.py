@@ -39,6 +39,7 @@ Function map:
   srht                  Sec. 3.2 "A scalable alternative to PCA"; App. B.2 Eq. app_srht_definition
   top_k                 App. C (per-query ranking of stored examples, NDCG@20)
   payload_bytes         App. E.1, Eq. app_payload
+  to_payload/from_payload  App. E.1 (per-module sign bytes + FP16 scale records)
 
 Where the paper is silent, the function that needs a reading states it (ties
 in the top-m selection, bit order, sign of zero, PCA sign convention, ranking
@@ -392,6 +393,38 @@ def top_k(scores: np.ndarray, K: int) -> Tuple[np.ndarray, np.ndarray]:
 def payload_bytes(ks: Sequence[int], scale_bytes: int = 2) -> int:
     """Per-example payload sum_u (ceil(k_u / 8) + 2) bytes (App. E.1, Eq. app_payload)."""
     return int(sum((k + 7) // 8 + scale_bytes for k in ks))
+
+
+def to_payload(codes: np.ndarray, scales: np.ndarray, ks: Sequence[int]) -> np.ndarray:
+    """Per-example store records (App. E.1, Eq. app_payload): for each module in
+    order, its ceil(k_u / 8) bytes of signs packed byte by byte (coordinate c at
+    bit c % 8 of byte c / 8) followed by its scale as an IEEE half (round to
+    nearest even, little-endian). The order of signs and scale inside a module's
+    record is not stated in the paper; signs first is the reading taken here.
+    codes [N, W] uint32 (module u at its word offset), scales [N, U] ->
+    uint8 [N, payload_bytes(ks)]."""
+    off = module_word_offsets(ks)
+    parts = []
+    for u, k in enumerate(ks):
+        bits = unpack_bits(np.asarray(codes)[:, off[u]:off[u + 1]], k)
+        parts.append(np.packbits(bits.astype(np.uint8), axis=1, bitorder="little"))
+        half = np.asarray(scales, np.float32)[:, u].astype(np.float16)
+        parts.append(half.astype("<f2").view(np.uint8).reshape(-1, 2))
+    return np.concatenate(parts, axis=1)
+
+
+def from_payload(payload: np.ndarray, ks: Sequence[int]) -> Tuple[np.ndarray, np.ndarray]:
+    """Inverse of to_payload: (codes [N, W] uint32 with zero pad bits, scales
+    [N, U] float32 holding the stored halves exactly)."""
+    payload = np.asarray(payload, np.uint8)
+    mods, scl, o = [], [], 0
+    for k in ks:
+        nb = (k + 7) // 8
+        bits = np.unpackbits(payload[:, o:o + nb], axis=1, bitorder="little")[:, :k].astype(bool)
+        mods.append(bits)
+        scl.append(payload[:, o + nb:o + nb + 2].copy().view("<f2").astype(np.float32)[:, 0])
+        o += nb + 2
+    return pack_concat(mods), np.stack(scl, axis=1)
 
 
 def correction_bytes(m: int, k: int) -> int:

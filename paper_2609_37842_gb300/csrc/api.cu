@@ -790,6 +790,59 @@ extern "C" int eogp_ekfac_accumulate(const eogp_ekfac_desc* D, const void* a, co
   return EOGP_OK;
 }
 
+// ================================================================ store records
+
+static int payload_args_ok(const int* ks, int U, long long* W) {
+  *W = 0;
+  if (!ks || U < 1 || U > 1024) return set_error(EOGP_EINVAL, "need 1 <= U <= 1024 modules");
+  for (int u = 0; u < U; ++u) {
+    if (ks[u] < 1) return set_error(EOGP_EINVAL, "k_per_module must be >= 1");
+    *W += (ks[u] + 31) / 32;
+  }
+  return EOGP_OK;
+}
+
+extern "C" int eogp_payload_bytes(const int* k_per_module, int U, size_t* bytes_per_example) {
+  clear_error();
+  long long W;
+  if (!bytes_per_example) return set_error(EOGP_EINVAL, "bytes_per_example is NULL");
+  if (int rc = payload_args_ok(k_per_module, U, &W)) return rc;
+  *bytes_per_example = payload_row_bytes(k_per_module, U);
+  return EOGP_OK;
+}
+
+extern "C" int eogp_payload_pack(const uint32_t* codes, int ld_codes, const float* scales, int ld_scales, int N,
+                                 const int* k_per_module, int U, uint8_t* payload, size_t ld_payload,
+                                 eogp_stream_t stream) {
+  clear_error();
+  long long W;
+  if (int rc = payload_args_ok(k_per_module, U, &W)) return rc;
+  if (N < 0) return set_error(EOGP_EINVAL, "N must be >= 0");
+  if (N == 0) return EOGP_OK;
+  if (!codes || !scales || !payload) return set_error(EOGP_EINVAL, "NULL argument");
+  if (ld_codes < W || ld_scales < U || ld_payload < payload_row_bytes(k_per_module, U))
+    return set_error(EOGP_EINVAL, "leading dimension too small");
+  CUDA_TRY(launch_payload_pack(codes, ld_codes, scales, ld_scales, N, k_per_module, U, payload, ld_payload,
+                               reinterpret_cast<cudaStream_t>(stream)));
+  return EOGP_OK;
+}
+
+extern "C" int eogp_payload_unpack(const uint8_t* payload, size_t ld_payload, int N, const int* k_per_module,
+                                   int U, uint32_t* codes, int ld_codes, float* scales, int ld_scales,
+                                   eogp_stream_t stream) {
+  clear_error();
+  long long W;
+  if (int rc = payload_args_ok(k_per_module, U, &W)) return rc;
+  if (N < 0) return set_error(EOGP_EINVAL, "N must be >= 0");
+  if (N == 0) return EOGP_OK;
+  if (!codes || !scales || !payload) return set_error(EOGP_EINVAL, "NULL argument");
+  if (ld_codes < W || ld_scales < U || ld_payload < payload_row_bytes(k_per_module, U))
+    return set_error(EOGP_EINVAL, "leading dimension too small");
+  CUDA_TRY(launch_payload_unpack(payload, ld_payload, N, k_per_module, U, codes, ld_codes, scales, ld_scales,
+                                 reinterpret_cast<cudaStream_t>(stream)));
+  return EOGP_OK;
+}
+
 // ================================================================ SRHT
 
 extern "C" int eogp_srht(const float* z, int B, int m, int ldz, const int8_t* signs, const int32_t* rows,

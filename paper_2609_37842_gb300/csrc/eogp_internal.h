@@ -122,6 +122,13 @@ cudaError_t launch_rows_fixup(float* X, int M, int n, int ld, int T, const float
 cudaError_t launch_sq_accum(const float* G, int rows, int cols, double* sumsq, int ld, int accumulate,
                             cudaStream_t st);
 
+// k_payload.cu: store records (per-module sign bytes + FP16 scale).
+size_t payload_row_bytes(const int* ks, int U);
+cudaError_t launch_payload_pack(const uint32_t* codes, int ld_codes, const float* scales, int ld_scales, int N,
+                                const int* ks, int U, uint8_t* out, size_t ld_out, cudaStream_t st);
+cudaError_t launch_payload_unpack(const uint8_t* in, size_t ld_in, int N, const int* ks, int U, uint32_t* codes,
+                                  int ld_codes, float* scales, int ld_scales, cudaStream_t st);
+
 // k_srht.cu: EOGP-R second stage, one CTA per row (z fp32, or bf16 hi + lo when hilo).
 int srht_width(int m);
 size_t srht_smem_bytes(int m);

@@ -80,6 +80,11 @@ EXPORTS = {
     "eogp_fit_pca_workspace_size": (c_int, [c_int, c_int, c_int, POINTER(c_size_t)]),
     "eogp_fit_pca": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int,
                              c_void_p, c_void_p, c_size_t, c_void_p]),
+    "eogp_payload_bytes": (c_int, [c_void_p, c_int, POINTER(c_size_t)]),
+    "eogp_payload_pack": (c_int, [c_void_p, c_int, c_void_p, c_int, c_int, c_void_p, c_int, c_void_p,
+                                  c_size_t, c_void_p]),
+    "eogp_payload_unpack": (c_int, [c_void_p, c_size_t, c_int, c_void_p, c_int, c_void_p, c_int,
+                                    c_void_p, c_int, c_void_p]),
     "eogp_srht": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_void_p, c_int, c_void_p, c_int,
                           c_void_p, c_int, c_void_p, c_int, c_void_p]),
     "eogp_pack_sign": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_int, c_void_p, c_int,
@@ -475,3 +480,55 @@ def score_topk(train, train_scales, ks: Sequence[int], mode: int, query, topk: i
                                  top_s.stride(0), _ptr(top_i), top_i.stride(0), _ptr(ws), ws.numel(),
                                  _stream(stream)))
     return top_s, top_i
+
+
+def payload_bytes(ks: Sequence[int]) -> int:
+    karr = (c_int * len(ks))(*[int(k) for k in ks])
+    n = c_size_t()
+    _check(lib().eogp_payload_bytes(karr, len(ks), ctypes.byref(n)))
+    return n.value
+
+
+def payload_pack(codes, scales, ks: Sequence[int], out=None, stream=None):
+    """Store records [N, payload_bytes(ks)] uint8 (device) from codes and scales."""
+    import torch
+    _rows(codes, "codes")
+    _rows(scales, "scales")
+    N = codes.shape[0]
+    karr = (c_int * len(ks))(*[int(k) for k in ks])
+    if out is None:
+        out = torch.empty((N, payload_bytes(ks)), dtype=torch.uint8, device=codes.device)
+    sc = scales if scales.dim() == 2 else scales[:, None]
+    _check(lib().eogp_payload_pack(_ptr(codes), codes.stride(0), _ptr(sc), sc.stride(0), N, karr, len(ks),
+                                   _ptr(out), out.stride(0), _stream(stream)))
+    return out
+
+
+def payload_unpack(payload, ks: Sequence[int], stream=None):
+    """(codes [N, W] int32, scales [N, U] fp32) from store records (device)."""
+    import torch
+    _rows(payload, "payload")
+    N = payload.shape[0]
+    karr = (c_int * len(ks))(*[int(k) for k in ks])
+    W = sum((int(k) + 31) // 32 for k in ks)
+    codes = torch.empty((N, W), dtype=torch.int32, device=payload.device)
+    scales = torch.empty((N, len(ks)), dtype=torch.float32, device=payload.device)
+    _check(lib().eogp_payload_unpack(_ptr(payload), payload.stride(0), N, karr, len(ks), _ptr(codes),
+                                     codes.stride(0), _ptr(scales), scales.stride(0), _stream(stream)))
+    return codes, scales
+
+
+def write_store(path: str, payload) -> None:
+    """Write store records (rows of payload_pack) to a file, back to back."""
+    with open(path, "wb") as f:
+        f.write(payload.cpu().numpy().tobytes())
+
+
+def read_store(path: str, ks: Sequence[int], device) -> "torch.Tensor":
+    """Read a file of store records back as a [N, payload_bytes(ks)] uint8 tensor."""
+    import torch
+    rb = payload_bytes(ks)
+    raw = np.fromfile(path, dtype=np.uint8)
+    if raw.size % rb:
+        raise ValueError(f"{path}: {raw.size} bytes is not a whole number of {rb}-byte records")
+    return torch.from_numpy(raw.reshape(-1, rb)).to(device)

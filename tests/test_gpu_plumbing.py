@@ -88,3 +88,33 @@ def test_bias_and_lengths(dtype, d_in, d_out, T, B, m, k, bias, lens, tol):
         z_nob = O.first_stage(np.concatenate([a, np.zeros(a.shape[:-1] + (1,))], -1), s_or, QA, QS,
                               Lam, O.damping(Lam, 0.1), m)
         assert row_rel(O.project(z_nob, Pt.astype(np.float64).T), x_or).min() > 10 * rel.max()
+
+
+@pytest.mark.parametrize("N,ks", [(37, [13, 32, 70]), (300, [1024] * 48), (1, [1])])
+def test_store_records(N, ks, tmp_path):
+    """Store records (App. E.1): bytes equal the oracle's, the round trip gives the
+    codes back and the scales rounded to half precision, and a file written and
+    read back scores exactly like the records it came from."""
+    rng = np.random.default_rng(N + len(ks))
+    codes = O.pack_concat([rng.integers(0, 2, (N, k)).astype(bool) for k in ks])
+    scales = rng.lognormal(0, 0.5, (N, len(ks))).astype(np.float32)
+    cd, sd = dev(codes.view(np.int32)), dev(scales)
+    pay = E.payload_pack(cd, sd, ks)
+    E.sync_status()
+    want = O.to_payload(codes, scales, ks)
+    assert pay.shape[1] == O.payload_bytes(ks)
+    np.testing.assert_array_equal(pay.cpu().numpy(), want)
+    c2, s2 = E.payload_unpack(pay, ks)
+    E.sync_status()
+    wc, ws = O.from_payload(want, ks)
+    np.testing.assert_array_equal(c2.cpu().numpy().view(np.uint32), wc)
+    np.testing.assert_array_equal(s2.cpu().numpy(), ws)
+    path = str(tmp_path / "store.bin")
+    E.write_store(path, pay)
+    back = E.read_store(path, ks, DEV)
+    assert torch.equal(back, pay)
+    if all(k % 32 == 0 for k in ks):
+        q = min(N, 5)
+        sc = E.score(c2, s2, ks, E.SCORE_CODES, c2[:q], s2[:q])
+        E.sync_status()
+        np.testing.assert_array_equal(sc.cpu().numpy(), O.score_codes_f32(wc, ws, ks, wc[:q], ws[:q]))

@@ -457,6 +457,37 @@ def test_payload_matches_tab_cost():
     assert O.payload_bytes([2048]) == 258
 
 
+def check_payload(Om, seed):
+    """Store records: the size of Eq. app_payload (pinned to Tab. cost above), the
+    byte order of the signs written out by hand, the half-precision scale
+    (round to nearest even) and the round trip."""
+    rng = np.random.default_rng(seed)
+    ks = [13, 32, 70]
+    bits = [rng.integers(0, 2, (4, k)).astype(bool) for k in ks]
+    codes = Om.pack_concat(bits)
+    scales = np.array([[1.0, 1 + 2 ** -11, 1 + 3 * 2 ** -11]] * 4, np.float32)
+    pay = Om.to_payload(codes, scales, ks)
+    assert pay.shape == (4, Om.payload_bytes(ks))
+    o = 0
+    for u, k in enumerate(ks):
+        nb = (k + 7) // 8
+        for e in range(4):
+            for c in range(k):
+                assert ((int(pay[e, o + c // 8]) >> (c % 8)) & 1) == int(bits[u][e, c])
+            assert int(pay[e, o + (k - 1) // 8]) >> ((k - 1) % 8 + 1) == 0   # pad bits are 0
+        halfbits = int(pay[0, o + nb]) | (int(pay[0, o + nb + 1]) << 8)
+        want = {0: 0x3C00, 1: 0x3C00, 2: 0x3C02}[u]   # 1, tie to even -> 1, 1 + 2^-9
+        assert halfbits == want
+        o += nb + 2
+    c2, s2 = Om.from_payload(pay, ks)
+    np.testing.assert_array_equal(c2, codes)
+    np.testing.assert_array_equal(s2, scales.astype(np.float16).astype(np.float32))
+
+
+def test_payload_records():
+    check_payload(O, 47)
+
+
 def test_correction_storage_matches_paper():
     for m, k, mods, gb, tol in _golden_rows("correction_storage.txt"):
         tot = O.correction_bytes(int(m), int(k)) * int(mods) / 1e9
@@ -567,3 +598,17 @@ def test_planted_plumbing_mistakes_are_caught(monkeypatch):
     ob = O.with_bias_channel
     monkeypatch.setattr(O, "with_bias_channel", lambda a: ob(a)[..., ::-1])
     assert _fails(check_plumbing, O, 43)      # bias channel first instead of last
+
+
+def test_planted_payload_mistake_is_caught(monkeypatch):
+    orig = O.to_payload
+    def big_endian_half(codes, scales, ks):
+        pay = orig(codes, scales, ks).copy()
+        o = 0
+        for k in ks:
+            nb = (k + 7) // 8
+            pay[:, [o + nb, o + nb + 1]] = pay[:, [o + nb + 1, o + nb]]
+            o += nb + 2
+        return pay
+    monkeypatch.setattr(O, "to_payload", big_endian_half)
+    assert _fails(check_payload, O, 47)
