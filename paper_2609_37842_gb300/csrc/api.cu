@@ -1027,24 +1027,27 @@ extern "C" int eogp_score(const void* train, int ld_train, const float* train_sc
 struct TopkPlan {
   bool fused;
   int slots;
-  size_t q_bytes, dense_bytes, list_bytes, total;
+  size_t q_bytes, dense_bytes, list_bytes, buf_bytes, scr_bytes, total;
 };
 
 static TopkPlan topk_plan(int N, const int* ks, int U, int mode, int Q, int K) {
   TopkPlan p{};
   const bool tc_ok = (mode == EOGP_SCORE_CODES || mode == EOGP_SCORE_PAPER) &&
                      score_tc_supported(mode, ks, U, Q);
-  p.fused = tc_ok && score_tc_topk_fits(mode, Q, K);
+  p.fused = tc_ok && score_tc_topk_fits(mode, U, Q, K);
   p.q_bytes = tc_ok ? score_tc_ws_bytes(mode, ks, U, Q) : 0;
   if (p.fused) {
-    p.slots = score_tc_grid(N, Q, sm_count());
+    p.slots = score_tc_grid(mode, U, N, Q, K, sm_count());
     p.dense_bytes = 0;
   } else {
     p.slots = topk_dense_slots(N);
     p.dense_bytes = al256(static_cast<size_t>(Q) * ((static_cast<size_t>(N) + 3) & ~size_t(3)) * 4);
   }
   p.list_bytes = al256(static_cast<size_t>(p.slots) * Q * K * 4);
-  p.total = al256(p.q_bytes) + p.dense_bytes + 2 * p.list_bytes;
+  p.buf_bytes = p.fused ? al256(score_tc_list_buf_bytes(mode, U, Q, K, p.slots)) : 0;
+  p.scr_bytes = p.fused ? al256(score_tc_scratch_bytes(mode, U, Q, K, p.slots)) : 0;
+  p.total = al256(p.q_bytes) + p.dense_bytes + 2 * p.list_bytes + 2 * p.buf_bytes +
+            (p.fused ? al256(static_cast<size_t>(Q) * 4) : 0) + p.scr_bytes;
   return p;
 }
 
@@ -1086,6 +1089,12 @@ extern "C" int eogp_score_topk(const void* train, int ld_train, const float* tra
   float* dense = reinterpret_cast<float*>(w + al256(p.q_bytes));
   float* lst = reinterpret_cast<float*>(w + al256(p.q_bytes) + p.dense_bytes);
   int* lsi = reinterpret_cast<int*>(w + al256(p.q_bytes) + p.dense_bytes + p.list_bytes);
+  float* bufs = reinterpret_cast<float*>(w + al256(p.q_bytes) + p.dense_bytes + 2 * p.list_bytes);
+  int* bufi = reinterpret_cast<int*>(w + al256(p.q_bytes) + p.dense_bytes + 2 * p.list_bytes + p.buf_bytes);
+  unsigned* gtau = reinterpret_cast<unsigned*>(w + al256(p.q_bytes) + p.dense_bytes + 2 * p.list_bytes +
+                                               2 * p.buf_bytes);
+  float* scr = reinterpret_cast<float*>(w + al256(p.q_bytes) + p.dense_bytes + 2 * p.list_bytes +
+                                        2 * p.buf_bytes + al256(static_cast<size_t>(Q) * 4));
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   ProfScope ps(EOGP_K_SCORE, st);
   if (p.fused && N > 0) {
@@ -1100,7 +1109,7 @@ extern "C" int eogp_score_topk(const void* train, int ld_train, const float* tra
                                               : "fused top-K needs 8-byte aligned code rows (ld_train % 2 == 0)");
     unsigned* status = status_word();
     if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
-    TcTopK tk{topk, lst, lsi, top_scores, ld_top_scores, top_index, ld_top_index};
+    TcTopK tk{topk, lst, lsi, bufs, bufi, gtau, scr, top_scores, ld_top_scores, top_index, ld_top_index};
     CUDA_TRY(launch_score_tc(mode, static_cast<const uint32_t*>(train), ld_train, train_scales, ld_tscale,
                              N, k_per_module, U, query, ld_query, query_scales, ld_qscale, Q, nullptr,
                              0, &tk, qws, sm_count(), status, st));

@@ -83,11 +83,16 @@ cudaError_t launch_score_paper(const uint32_t* train, int ldt, const float* ts, 
 
 // k_score_tc.cu: CODES (e4m3 +-1 operands) and PAPER (bf16 hi/lo query x bf16 +-1
 // codes) scoring on the tensor cores, dense output or fused top-K.
-constexpr int kTopKMax = 64;  // largest K of the fused top-K
+constexpr int kTopKMax = 32;  // largest K of the fused top-K (kTopKBuf - 32)
+constexpr int kTopKBuf = 64;  // running list buffer per query column of the fused top-K
 struct TcTopK {
   int K;
   float* lst;  // per-CTA lists [grid][Q][K] (workspace)
   int* lsi;
+  float* bufs;  // running list buffers [grid][queries per tile][kTopKBuf] (workspace)
+  int* bufi;
+  unsigned* gtau;  // [Q] shared thresholds (workspace)
+  float* scr;      // per-CTA score scratch (workspace)
   float* out_s;  // final [Q, K] scores / stored indices
   int ld_os;
   int* out_i;
@@ -95,8 +100,10 @@ struct TcTopK {
 };
 bool score_tc_supported(int mode, const int* ks, int U, int Q);
 size_t score_tc_ws_bytes(int mode, const int* ks, int U, int Q);
-int score_tc_grid(int N, int Q, int num_sms);
-bool score_tc_topk_fits(int mode, int Q, int K);
+int score_tc_grid(int mode, int U, int N, int Q, int K, int num_sms);
+bool score_tc_topk_fits(int mode, int U, int Q, int K);
+size_t score_tc_list_buf_bytes(int mode, int U, int Q, int K, int grid);  // each of bufs, bufi
+size_t score_tc_scratch_bytes(int mode, int U, int Q, int K, int grid);
 cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const float* ts, int ldts, int N,
                             const int* ks, int U, const void* query, int ldq, const float* qs,
                             int ldqs, int Q, float* out, int ldo, const TcTopK* topk, void* ws,

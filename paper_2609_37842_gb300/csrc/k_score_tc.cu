@@ -18,11 +18,11 @@
 //
 // Output: either the dense [Q, N] score matrix, or (TOPK) only each query's K
 // best stored rows. In the TOPK epilogue the last module's scores of a tile
-// are staged 32 query columns at a time in shared memory and the thread that
-// owns a query column merges them into that query's sorted list (score
-// descending, equal scores by lower stored index). A CTA's lists cover the
-// stored rows of its tiles and go to global memory when the CTA moves to the
-// next query tile; a separate kernel merges the per-CTA lists. The Q x N
+// are compared, 32 query columns at a time, with each column's threshold;
+// chunks holding a candidate are staged in shared memory and a warp per column
+// appends the candidates to that query's list (topk_dev.cuh). A CTA's lists
+// cover the stored rows of its tiles and are written out when the CTA moves to
+// the next query tile; a separate kernel merges the per-CTA lists. The Q x N
 // matrix never reaches HBM.
 //
 // Tiles: 128 stored rows (MMA M, operand A) x BNq <= 128 queries (MMA N,
@@ -51,9 +51,12 @@ using namespace eogp;
 namespace {
 
 constexpr int kMaxMods = 1024;
-constexpr int kThreadsTc = 288;
-constexpr uint32_t kAB = 16384u;  // 128 rows x 128 bytes
-constexpr int kTbStride = 129;    // staged column stride (floats): conflict-free both ways
+constexpr int kExpWarps = 8;                        // expander warps (two per stored row)
+constexpr int kThreadsTc = (kExpWarps + 4 + 1) * 32;  // + 4 dequantise warps + 1 MMA warp
+constexpr int kDqWarp0 = kExpWarps;                 // first dequantise warp
+constexpr int kMmaWarp = kExpWarps + 4;
+constexpr uint32_t kAB = 16384u;                    // 128 rows x 128 bytes
+constexpr int kFusedCap = kTopKBuf;                 // list buffer per query column (K <= 32, 2 per lane)
 
 struct ScoreTcArgs {
   int N, Q, U, D, BNq, n_it, n_tiles, ldt, ldts, ldqs, ldo, K;
@@ -63,8 +66,12 @@ struct ScoreTcArgs {
   float* out;
   float* lst;  // TOPK: per-CTA lists [gridDim.x][Q][K]
   int* lsi;
+  float* bufs;  // TOPK: running list buffers [gridDim.x][BNq][kFusedCap] (global, L2-resident)
+  int* bufi;
+  unsigned* gtau;  // TOPK: per query, order key of the best threshold any CTA's list reached
+  float* scr;      // TOPK: per-CTA scratch of one tile's scores [gridDim.x][BN][128] (L2-resident)
   unsigned* status;
-  int k[kMaxMods];     // bits per module
+  int k[kMaxMods];  // bits per module
 };
 
 template <int MODE>
@@ -73,46 +80,54 @@ template <>
 struct TcMode<EOGP_SCORE_CODES> {
   static constexpr int kBits = 128;  // code bits per pipeline stage
   static constexpr int kQBoxes = 1;  // query operand tiles per stage
-  using Bits = uint4;                // one stage of one stored row
+  using HalfBits = uint2;            // one stage of half a stored row
 };
 template <>
 struct TcMode<EOGP_SCORE_PAPER> {
   static constexpr int kBits = 64;
   static constexpr int kQBoxes = 2;  // hi, lo
-  using Bits = uint2;
+  using HalfBits = uint32_t;
 };
 
-template <int MODE, bool TOPK>
-constexpr int tc_stages() {
-  return (MODE == EOGP_SCORE_PAPER && TOPK) ? 3 : 4;
+// BN: queries per tile (MMA N). 256 only for CODES with one module (no running
+// score is needed, so the two accumulators take all 512 TMEM columns).
+template <int MODE, int BN>
+constexpr uint32_t tc_stage_bytes() {
+  return kAB + static_cast<uint32_t>(BN) * 128u * TcMode<MODE>::kQBoxes;
 }
 
-template <int MODE>
-constexpr uint32_t tc_stage_bytes() {
-  return kAB * (1 + TcMode<MODE>::kQBoxes);
+template <int MODE, bool TOPK, int BN>
+constexpr int tc_stages() {
+  return 4;
 }
 
 // Shared-memory carve-up (byte offsets after 1024-byte alignment).
 struct TcSmem {
-  uint32_t sq, bars, tb, lists, total;
+  uint32_t sq, bars, lists, total;
 };
-template <int MODE, bool TOPK>
+template <int MODE, bool TOPK, int BN>
 __host__ __device__ inline TcSmem tc_smem_layout(int BNq, int K) {
-  constexpr int S = tc_stages<MODE, TOPK>();
+  constexpr int S = tc_stages<MODE, TOPK, BN>();
   TcSmem l;
-  l.sq = S * tc_stage_bytes<MODE>();
-  l.bars = l.sq + 128 * 4;
-  l.tb = l.bars + (2 * S + 4) * 8 + 16;
-  l.lists = l.tb + (TOPK ? 32 * kTbStride * 4 : 0);
-  l.total = l.lists + (TOPK ? static_cast<uint32_t>(BNq) * K * 8 : 0);
+  l.sq = S * tc_stage_bytes<MODE, BN>();
+  l.bars = l.sq + BN * 4;
+  l.lists = l.bars + (2 * S + 4) * 8 + 16;
+  // per-column held count, own threshold and shared threshold (the list buffers
+  // themselves are in global memory)
+  l.total = l.lists + (TOPK ? BN * 12 + 8 * 4 * 4 : 0);
   return l;
 }
 
-// 8 code bits -> 8 e4m3 bytes (bit j -> byte j: +1 if set, -1 if clear).
+// 4 code bits -> 4 e4m3 bytes (bit j -> byte j: +1 = 0x38 if set, -1 = 0xB8 if
+// clear): the multiply places bit j at bit 8j + 7 (the four shifted copies of
+// the nibble never overlap, so there are no carries).
+__device__ __forceinline__ uint32_t e4m3x4(uint32_t nib) {
+  return ((nib * 0x10204080u) & 0x80808080u) ^ 0xB8B8B8B8u;
+}
+
+// 8 code bits -> 8 e4m3 bytes (query expansion).
 __device__ __forceinline__ uint64_t expand8(uint32_t v) {
-  uint64_t x = (static_cast<uint64_t>(v & 0xFFu) * 0x0101010101010101ull) & 0x8040201008040201ull;
-  x = (x + 0x7F7F7F7F7F7F7F7Full) & 0x8080808080808080ull;  // 0x80 where the bit is set
-  return 0xB8B8B8B8B8B8B8B8ull ^ x;
+  return static_cast<uint64_t>(e4m3x4(v & 0xFu)) | (static_cast<uint64_t>(e4m3x4((v >> 4) & 0xFu)) << 32);
 }
 
 // 4 code bits -> 4 bf16 values (bit j -> element j: +1 = 0x3F80 if set, -1 = 0xBF80 if
@@ -124,25 +139,23 @@ __device__ __forceinline__ uint64_t expand4_bf16(uint32_t v) {
   return 0xBF80BF80BF80BF80ull ^ x;
 }
 
-// One stage of one stored row -> its 128-byte swizzled shared-memory row
-// (16-byte chunk c goes to position c ^ (row & 7)).
-__device__ __forceinline__ void expand_stage(uint8_t* dst, int sw, uint4 bits) {  // 128 bits -> e4m3
-  const uint32_t wv[4] = {bits.x, bits.y, bits.z, bits.w};
+// Half a stage of one stored row -> 4 of its 8 swizzled 16-byte chunks
+// (chunk c goes to position c ^ (row & 7)); `half` selects chunks 4 half .. +3.
+__device__ __forceinline__ void expand_half(uint8_t* row, int sw, int half, uint2 bits) {  // 64 bits -> e4m3
 #pragma unroll
-  for (int c = 0; c < 8; ++c) {
-    const uint32_t h = wv[c >> 1] >> ((c & 1) * 16);
-    const uint64_t lo = expand8(h), hi = expand8(h >> 8);
-    *reinterpret_cast<uint4*>(dst + ((c ^ sw) << 4)) =
-        make_uint4(static_cast<uint32_t>(lo), static_cast<uint32_t>(lo >> 32), static_cast<uint32_t>(hi),
-                   static_cast<uint32_t>(hi >> 32));
+  for (int cc = 0; cc < 4; ++cc) {
+    const uint32_t h = (cc < 2 ? bits.x : bits.y) >> ((cc & 1) * 16);
+    *reinterpret_cast<uint4*>(row + (((4 * half + cc) ^ sw) << 4)) =
+        make_uint4(e4m3x4(h & 0xFu), e4m3x4((h >> 4) & 0xFu), e4m3x4((h >> 8) & 0xFu),
+                   e4m3x4((h >> 12) & 0xFu));
   }
 }
-__device__ __forceinline__ void expand_stage(uint8_t* dst, int sw, uint2 bits) {  // 64 bits -> bf16
+__device__ __forceinline__ void expand_half(uint8_t* row, int sw, int half, uint32_t bits) {  // 32 bits -> bf16
 #pragma unroll
-  for (int c = 0; c < 8; ++c) {
-    const uint32_t h = (c < 4 ? bits.x : bits.y) >> ((c & 3) * 8);
+  for (int cc = 0; cc < 4; ++cc) {
+    const uint32_t h = bits >> (cc * 8);
     const uint64_t lo = expand4_bf16(h), hi = expand4_bf16(h >> 4);
-    *reinterpret_cast<uint4*>(dst + ((c ^ sw) << 4)) =
+    *reinterpret_cast<uint4*>(row + (((4 * half + cc) ^ sw) << 4)) =
         make_uint4(static_cast<uint32_t>(lo), static_cast<uint32_t>(lo >> 32), static_cast<uint32_t>(hi),
                    static_cast<uint32_t>(hi >> 32));
   }
@@ -164,20 +177,21 @@ __device__ __forceinline__ int tile_step() {
   return TOPK ? 1 : gridDim.x;
 }
 
-template <int MODE, bool TOPK>
+template <int MODE, bool TOPK, int BN>
 __global__ void __launch_bounds__(kThreadsTc, 1)
     k_score_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQlo,
                const __grid_constant__ ScoreTcArgs g) {
-  constexpr int S = tc_stages<MODE, TOPK>();
-  constexpr uint32_t kStage = tc_stage_bytes<MODE>();
+  constexpr int S = tc_stages<MODE, TOPK, BN>();
+  constexpr uint32_t kStage = tc_stage_bytes<MODE, BN>();
   constexpr int kBits = TcMode<MODE>::kBits;
   constexpr int kG = 8;  // stages of code bits prefetched at a time
-  using StageBits = typename TcMode<MODE>::Bits;
+  constexpr uint32_t kAcc = 2u * BN;  // running-score columns (BN == 128 only)
+  using HalfBits = typename TcMode<MODE>::HalfBits;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  const TcSmem L = tc_smem_layout<MODE, TOPK>(g.BNq, g.K);
+  const TcSmem L = tc_smem_layout<MODE, TOPK, BN>(g.BNq, g.K);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  float* sq = reinterpret_cast<float*>(smem + L.sq);  // [128] query scales of module u (CODES)
+  float* sq = reinterpret_cast<float*>(smem + L.sq);  // [BN] query scales of module u (CODES)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bars);
   uint64_t* empty = full + S;
   uint64_t* dfull = empty + S;
@@ -188,7 +202,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
     tma_prefetch_desc(&tmQ);
     if (MODE == EOGP_SCORE_PAPER) tma_prefetch_desc(&tmQlo);
     for (int s = 0; s < S; ++s) {
-      mbar_init(&full[s], 5);  // TMA transaction arrive + 4 expander warps
+      mbar_init(&full[s], 1 + kExpWarps);  // TMA transaction arrive + the expander warps
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -197,19 +211,20 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
     }
     fence_barrier_init();
   }
-  if (warp == 8) tmem_alloc(tslot, 512);
+  if (warp == kMmaWarp) tmem_alloc(tslot, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
-  if (warp < 4) {
+  if (warp < kExpWarps) {
     // ---------------------------------------------------------- expanders
     // A stored row's modules are back to back, so pipeline stage j of a tile
     // reads bits [j kBits, (j+1) kBits) of the row and query columns from
-    // j kBits on. The bits of the next kG stages are loaded into registers
-    // while the current kG stages are expanded, hiding the HBM latency.
-    const int r = threadIdx.x;  // stored row within the tile
+    // j kBits on. Two threads share a row (a half stage each). The bits of the
+    // next kG stages are loaded into registers while the current kG stages are
+    // expanded, hiding the HBM latency.
+    const int r = threadIdx.x & 127, half = threadIdx.x >> 7;  // stored row, half of its stage
     const uint32_t row_off = static_cast<uint32_t>((r >> 3) * 1024 + (r & 7) * 128);
     const int nst = g.D / kBits;
     uint32_t it = 0;
@@ -219,15 +234,15 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       const int qt = tile / g.n_it, ib = tile % g.n_it;
       const int i0 = ib * 128, q0 = qt * g.BNq;
       const bool rv = i0 + r < g.N;
-      const StageBits* brow =
-          reinterpret_cast<const StageBits*>(g.train + static_cast<size_t>(rv ? i0 + r : 0) * g.ldt);
-      StageBits cur[kG], nxt[kG];
+      const HalfBits* brow =
+          reinterpret_cast<const HalfBits*>(g.train + static_cast<size_t>(rv ? i0 + r : 0) * g.ldt) + half;
+      HalfBits cur[kG], nxt[kG];
 #pragma unroll
-      for (int jj = 0; jj < kG; ++jj) cur[jj] = (rv && jj < nst) ? __ldg(brow + jj) : StageBits{};
+      for (int jj = 0; jj < kG; ++jj) cur[jj] = (rv && jj < nst) ? __ldg(brow + 2 * jj) : HalfBits{};
       for (int j0 = 0; j0 < nst && ok; j0 += kG) {
 #pragma unroll
         for (int jj = 0; jj < kG; ++jj)
-          nxt[jj] = (rv && j0 + kG + jj < nst) ? __ldg(brow + j0 + kG + jj) : StageBits{};
+          nxt[jj] = (rv && j0 + kG + jj < nst) ? __ldg(brow + 2 * (j0 + kG + jj)) : HalfBits{};
 #pragma unroll
         for (int jj = 0; jj < kG; ++jj) {
           const int j = j0 + jj;
@@ -245,9 +260,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
               if (warp == 0 && lane == 0) {
                 mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(g.BNq) * 128u * TcMode<MODE>::kQBoxes);
                 tma_load_2d(st + kAB, &tmQ, j * kBits, q0, &full[s]);
-                if (MODE == EOGP_SCORE_PAPER) tma_load_2d(st + 2 * kAB, &tmQlo, j * kBits, q0, &full[s]);
+                if (MODE == EOGP_SCORE_PAPER)
+                  tma_load_2d(st + kAB + static_cast<uint32_t>(BN) * 128u, &tmQlo, j * kBits, q0, &full[s]);
               }
-              expand_stage(st + row_off, r & 7, cur[jj]);
+              expand_half(st + row_off, r & 7, half, cur[jj]);
               fence_proxy_async_smem();
               __syncwarp();
               if (lane == 0) mbar_arrive(&full[s]);
@@ -258,24 +274,82 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
         for (int jj = 0; jj < kG; ++jj) cur[jj] = nxt[jj];
       }
     }
-  } else if (warp < 8) {
+  } else if (warp < kMmaWarp) {
     // ---------------------------------------------------------- dequantise
     const int q4 = warp & 3;
-    const int ep = threadIdx.x - 128;  // TMEM lane (stored row in the tile); TOPK: query column
+    const int ep = threadIdx.x - 32 * kDqWarp0;  // TMEM lane (stored row in the tile)
     const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
-    float* tb = reinterpret_cast<float*>(smem + L.tb);
-    float* ls = reinterpret_cast<float*>(smem + L.lists) + static_cast<size_t>(ep) * g.K;
-    int* li = reinterpret_cast<int*>(smem + L.lists + static_cast<size_t>(g.BNq) * g.K * 4) +
-              static_cast<size_t>(ep) * g.K;
+    float* lsb = g.bufs + static_cast<size_t>(blockIdx.x) * g.BNq * kFusedCap;
+    int* lib = g.bufi + static_cast<size_t>(blockIdx.x) * g.BNq * kFusedCap;
+    int* cntb = reinterpret_cast<int*>(smem + L.lists);
+    float* taub = reinterpret_cast<float*>(cntb + BN);
+    float* gtb = taub + BN;  // shared thresholds of this query tile, refreshed per tile
+    uint32_t* cmask = reinterpret_cast<uint32_t*>(gtb + BN);  // [BN / 32][4] per-warp column masks
+    int q0_cur = 0;
+    auto list_of = [&](int col) {
+      return WarpTopk{lsb + static_cast<size_t>(col) * kFusedCap, lib + static_cast<size_t>(col) * kFusedCap,
+                      cntb + col, taub + col, g.K, g.gtau + q0_cur + col};
+    };
+    const int dw = ep >> 5;  // dequantise warp 0..3
     int seg_qt = -1;
-    TopkState tk;
-    topk_reset(tk);
+    // Lists of the finished query tile to global memory; warp dw writes columns dw, dw + 4, ...
     auto flush = [&]() {
-      const int q = seg_qt * g.BNq + ep;
-      if (ep < g.BNq && q < g.Q) {
-        const size_t o = (static_cast<size_t>(blockIdx.x) * g.Q + q) * g.K;
-        topk_write(ls, li, g.K, tk, g.lst + o, g.lsi + o);
+      for (int col = dw; col < g.BNq; col += 4) {
+        const int q = seg_qt * g.BNq + col;
+        if (q < g.Q) {
+          const size_t off = (static_cast<size_t>(blockIdx.x) * g.Q + q) * g.K;
+          topk_warp_write<2>(list_of(col), lane, g.lst + off, g.lsi + off);
+        }
       }
+    };
+    // Ranks one chunk of 32 query columns (values a[] of this thread's stored row):
+    // if no value beats its column's threshold (the usual case once the lists
+    // have filled), nothing is staged; otherwise the chunk is staged column-major
+    // and warp dw offers 8 of the columns to their lists.
+    // Last module of a tile, per chunk of 32 query columns: keep the scores in this
+    // CTA's scratch (column-major) and note which columns hold a row that can
+    // enter the column's list (one bit per column, per warp).
+    float* scr = g.scr + static_cast<size_t>(blockIdx.x) * BN * 128;
+    auto screen_chunk = [&](int c0, int q0, int row, const float (&a)[32]) {
+      uint32_t bits = 0;
+      if (row < g.N) {
+        const float4* t4 = reinterpret_cast<const float4*>(taub + c0);
+        const float4* g4 = reinterpret_cast<const float4*>(gtb + c0);
+#pragma unroll
+        for (int j4 = 0; j4 < 8; ++j4) {
+          const float4 t = t4[j4], u = g4[j4];
+          const float tj[4] = {t.x, t.y, t.z, t.w}, uj[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float x = a[4 * j4 + e];
+            const bool live = q0 + c0 + 4 * j4 + e < g.Q;
+            bits |= (live && x >= uj[e] && (tj[e] != tj[e] ? x == x : x > tj[e])) ? (1u << (4 * j4 + e)) : 0u;
+          }
+        }
+      }
+      const uint32_t wbits = __reduce_or_sync(0xffffffffu, bits);
+      if (lane == 0) cmask[(c0 >> 5) * 4 + dw] = wbits;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) scr[static_cast<size_t>(c0 + j) * 128 + ep] = a[j];
+    };
+    // After the D buffer is released: the flagged columns, dealt round-robin to
+    // the four warps, offered to their lists from the scratch.
+    auto rank_tile = [&](int q0, int i0) {
+      named_bar_sync(3, 128);  // scratch and masks of every warp visible
+      const int nr = min(128, g.N - i0);
+      int n = 0;
+      for (int c0 = 0; c0 < g.BNq; c0 += 32) {
+        const uint32_t* cm = cmask + (c0 >> 5) * 4;
+        uint32_t colmask = cm[0] | cm[1] | cm[2] | cm[3];
+        for (; colmask; ++n) {
+          const int cc = __ffs(colmask) - 1;
+          colmask &= colmask - 1;
+          if ((n & 3) == dw)
+            topk_warp_offer<2>(scr + static_cast<size_t>(c0 + cc) * 128, nr, i0, list_of(c0 + cc), lane,
+                               gtb[c0 + cc]);
+        }
+      }
+      named_bar_sync(3, 128);  // lists settled before the next tile screens or flushes
     };
     uint32_t gm = 0;
     bool ok = true;
@@ -285,16 +359,31 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       const int i0 = ib * 128, q0 = qt * g.BNq;
       const int row = i0 + ep;
       if (TOPK && qt != seg_qt) {
-        if (seg_qt >= 0) flush();
+        if (seg_qt >= 0) {
+          flush();
+          named_bar_sync(3, 128);  // every list written before any is reset
+        }
         seg_qt = qt;
-        topk_reset(tk);
+        q0_cur = q0;
+        for (int col = ep; col < BN; col += 128) {
+          cntb[col] = 0;
+          taub[col] = NAN;
+        }
+        named_bar_sync(3, 128);
+      }
+      if (TOPK) {
+        // Thresholds other CTAs' lists of these queries have reached (read before the
+        // last module's ranking, after the barriers of the module loop).
+        for (int col = ep; col < BN; col += 128)
+          gtb[col] = q0 + col < g.Q ? topk_unkey32(__ldcg(g.gtau + q0 + col)) : INFINITY;
       }
       for (int u = 0; u < g.U; ++u, ++gm) {
         const int buf = static_cast<int>(gm & 1u);
         const uint32_t dph = (gm >> 1) & 1u;
         if (MODE == EOGP_SCORE_CODES) {
           named_bar_sync(1, 128);  // previous module's readers of sq are done
-          if (ep < g.BNq) sq[ep] = q0 + ep < g.Q ? g.qs[static_cast<size_t>(q0 + ep) * g.ldqs + u] : 0.f;
+          for (int c = ep; c < g.BNq; c += 128)
+            sq[c] = q0 + c < g.Q ? g.qs[static_cast<size_t>(q0 + c) * g.ldqs + u] : 0.f;
           named_bar_sync(1, 128);
         }
         uint32_t w_ok = 1;
@@ -310,12 +399,12 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
         const bool last = u + 1 == g.U;
         for (int c0 = 0; c0 < g.BNq; c0 += 32) {
           float d[32], a[32];
-          tmem_ld32(tmem + lane_base + buf * 128u + c0, d);
+          tmem_ld32(tmem + lane_base + buf * static_cast<uint32_t>(BN) + c0, d);
           if (u == 0) {
 #pragma unroll
             for (int j = 0; j < 32; ++j) a[j] = 0.f;
           } else {
-            tmem_ld32(tmem + lane_base + 256u + c0, a);
+            tmem_ld32(tmem + lane_base + kAcc + c0, a);
           }
           if (MODE == EOGP_SCORE_CODES) {
 #pragma unroll
@@ -324,31 +413,22 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
 #pragma unroll
             for (int j = 0; j < 32; ++j) a[j] = __fadd_rn(a[j], __fmul_rn(si, d[j]));
           }
-          if (!last || TOPK) {
-            tmem_st32(tmem + lane_base + 256u + c0, a);
-          } else if (row < g.N) {
+          if (!last) {
+            tmem_st32(tmem + lane_base + kAcc + c0, a);
+          } else if (!TOPK) {
+            if (row < g.N) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j)
-              if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
+              for (int j = 0; j < 32; ++j)
+                if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
+            }
+          } else {
+            screen_chunk(c0, q0, row, a);
           }
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&dempty[buf]);  // D buffer free: the MMAs run on
-        if (TOPK && last) {
-          // Rank the finished tile from the running-score columns, 32 query columns at
-          // a time: staged column-major, then the warp owning them offers them to its lists.
-          for (int c0 = 0; c0 < g.BNq; c0 += 32) {
-            float a[32];
-            tmem_ld32(tmem + lane_base + 256u + c0, a);
-#pragma unroll
-            for (int j = 0; j < 32; ++j) tb[j * kTbStride + ep] = a[j];
-            named_bar_sync(3, 128);
-            if ((ep >> 5) == (c0 >> 5) && q0 + ep < g.Q)
-              topk_scan(tb + lane * kTbStride, min(128, g.N - i0), i0, ls, li, g.K, tk);
-            named_bar_sync(3, 128);
-          }
-        }
+        if (TOPK && last) rank_tile(q0, i0);
       }
     }
     if (TOPK && seg_qt >= 0) flush();
@@ -360,7 +440,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       uint32_t it = 0, gm = 0;
       bool ok = true;
       for (int tile = tile_begin<TOPK>(g), tstep = tile_step<TOPK>(), tend = tile_end<TOPK>(g);
-         tile < tend && ok; tile += tstep) {
+           tile < tend && ok; tile += tstep) {
         for (int u = 0; u < g.U && ok; ++u, ++gm) {
           const int buf = static_cast<int>(gm & 1u);
           const uint32_t dph = (gm >> 1) & 1u;
@@ -369,7 +449,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t d = tmem + buf * 128u;
+          const uint32_t d = tmem + buf * static_cast<uint32_t>(BN);
           const int nkb = g.k[u] / kBits;
           for (int kb = 0; kb < nkb; ++kb, ++it) {
             const int s = static_cast<int>(it % S);
@@ -388,7 +468,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
                 tc_mma_f8(d, ad, sdesc_sw128(sa + kAB + kk * 32, 16, 1024), idesc, acc);
               } else {
                 tc_mma_f16(d, ad, sdesc_sw128(sa + kAB + kk * 32, 16, 1024), idesc, acc);
-                tc_mma_f16(d, ad, sdesc_sw128(sa + 2 * kAB + kk * 32, 16, 1024), idesc, 1u);
+                tc_mma_f16(d, ad, sdesc_sw128(sa + kAB + BN * 128u + kk * 32, 16, 1024), idesc, 1u);
               }
             }
             tc_commit(&empty[s]);
@@ -401,7 +481,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 8) tmem_dealloc(tmem, 512);
+  if (warp == kMmaWarp) tmem_dealloc(tmem, 512);
 }
 
 // Query codes -> e4m3 bytes: out[q][c] = +1 / -1 for bit c of the concatenated modules.
@@ -435,17 +515,39 @@ __global__ void k_split_queries(const float* __restrict__ y, int ldq, int D,
   }
 }
 
-int bnq_for(int Q) { return std::min(128, (Q + 31) / 32 * 32); }
+template <int MODE, bool TOPK, int BN>
+size_t tc_smem_need(int BNq, int K) {
+  return 1024 + tc_smem_layout<MODE, TOPK, BN>(BNq, K).total;
+}
 
-template <int MODE, bool TOPK>
+// Queries per tile: 256 for CODES with one module and enough queries (when the
+// shared memory allows), else 128.
+int tc_bn(int mode, int U, int Q, int K) {
+  if (mode == EOGP_SCORE_CODES && U == 1 && Q >= 256 &&
+      (K == 0 || tc_smem_need<EOGP_SCORE_CODES, true, 256>(256, K) <= 232448))
+    return 256;
+  return 128;
+}
+
+int bnq_for(int Q, int BN) { return std::min(BN, (Q + 31) / 32 * 32); }
+
+template <int MODE, bool TOPK, int BN>
 cudaError_t launch_tc_kernel(const CUtensorMap& t0, const CUtensorMap& t1, const ScoreTcArgs& g,
                              int grid, cudaStream_t st) {
-  const size_t smem = 1024 + tc_smem_layout<MODE, TOPK>(g.BNq, g.K).total;
-  cudaError_t e = cudaFuncSetAttribute(k_score_tc<MODE, TOPK>,
+  const size_t smem = tc_smem_need<MODE, TOPK, BN>(g.BNq, g.K);
+  cudaError_t e = cudaFuncSetAttribute(k_score_tc<MODE, TOPK, BN>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  k_score_tc<MODE, TOPK><<<grid, kThreadsTc, smem, st>>>(t0, t1, g);
+  k_score_tc<MODE, TOPK, BN><<<grid, kThreadsTc, smem, st>>>(t0, t1, g);
   return cudaGetLastError();
+}
+
+template <bool TOPK>
+cudaError_t dispatch_tc(int mode, int BN, const CUtensorMap& t0, const CUtensorMap& t1, const ScoreTcArgs& g,
+                        int grid, cudaStream_t st) {
+  if (mode == EOGP_SCORE_PAPER) return launch_tc_kernel<EOGP_SCORE_PAPER, TOPK, 128>(t0, t1, g, grid, st);
+  if (BN == 256) return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 256>(t0, t1, g, grid, st);
+  return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 128>(t0, t1, g, grid, st);
 }
 
 }  // namespace
@@ -466,6 +568,15 @@ bool score_tc_supported(int mode, const int* ks, int U, int Q) {
   return false;
 }
 
+size_t score_tc_list_buf_bytes(int mode, int U, int Q, int K, int grid) {
+  const int bq = bnq_for(Q, tc_bn(mode, U, Q, K));
+  return static_cast<size_t>(grid) * bq * kFusedCap * 4;  // each of scores and indices
+}
+
+size_t score_tc_scratch_bytes(int mode, int U, int Q, int K, int grid) {
+  return static_cast<size_t>(grid) * tc_bn(mode, U, Q, K) * 128 * 4;
+}
+
 size_t score_tc_ws_bytes(int mode, const int* ks, int U, int Q) {
   long long D = 0;
   for (int u = 0; u < U; ++u) D += ks[u];
@@ -473,17 +584,19 @@ size_t score_tc_ws_bytes(int mode, const int* ks, int U, int Q) {
   return (static_cast<size_t>(Q) * D * per + 255) & ~size_t(255);
 }
 
-int score_tc_grid(int N, int Q, int num_sms) {
-  const long long tiles =
-      static_cast<long long>((N + 127) / 128) * ((Q + bnq_for(Q) - 1) / bnq_for(Q));
+int score_tc_grid(int mode, int U, int N, int Q, int K, int num_sms) {
+  const int bq = bnq_for(Q, tc_bn(mode, U, Q, K));
+  const long long tiles = static_cast<long long>((N + 127) / 128) * ((Q + bq - 1) / bq);
   return static_cast<int>(std::max<long long>(1, std::min<long long>(tiles, std::max(1, num_sms))));
 }
 
-bool score_tc_topk_fits(int mode, int Q, int K) {
+bool score_tc_topk_fits(int mode, int U, int Q, int K) {
   if (K < 1 || K > kTopKMax) return false;
-  const size_t need = 1024 + (mode == EOGP_SCORE_PAPER
-                                  ? tc_smem_layout<EOGP_SCORE_PAPER, true>(bnq_for(Q), K).total
-                                  : tc_smem_layout<EOGP_SCORE_CODES, true>(bnq_for(Q), K).total);
+  const int BN = tc_bn(mode, U, Q, K);
+  const int bq = bnq_for(Q, BN);
+  const size_t need = mode == EOGP_SCORE_PAPER ? tc_smem_need<EOGP_SCORE_PAPER, true, 128>(bq, K)
+                      : BN == 256              ? tc_smem_need<EOGP_SCORE_CODES, true, 256>(bq, K)
+                                               : tc_smem_need<EOGP_SCORE_CODES, true, 128>(bq, K);
   return need <= 232448;
 }
 
@@ -496,7 +609,8 @@ cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const floa
   g.N = N;
   g.Q = Q;
   g.U = U;
-  g.BNq = bnq_for(Q);
+  const int BN = tc_bn(mode, U, Q, topk ? topk->K : 0);
+  g.BNq = bnq_for(Q, BN);
   g.n_it = (N + 127) / 128;
   g.n_tiles = g.n_it * ((Q + g.BNq - 1) / g.BNq);
   g.ldt = ldt;
@@ -510,6 +624,10 @@ cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const floa
   g.out = out;
   g.lst = topk ? topk->lst : nullptr;
   g.lsi = topk ? topk->lsi : nullptr;
+  g.bufs = topk ? topk->bufs : nullptr;
+  g.bufi = topk ? topk->bufi : nullptr;
+  g.gtau = topk ? topk->gtau : nullptr;
+  g.scr = topk ? topk->scr : nullptr;
   g.status = status;
   int D = 0;
   for (int u = 0; u < U; ++u) {
@@ -517,7 +635,7 @@ cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const floa
     D += ks[u];
   }
   g.D = D;
-  const int grid = score_tc_grid(N, Q, num_sms);
+  const int grid = score_tc_grid(mode, U, N, Q, topk ? topk->K : 0, num_sms);
   CUtensorMap t0, t1;
   if (mode == EOGP_SCORE_CODES) {
     uint8_t* qx = static_cast<uint8_t*>(ws);
@@ -553,12 +671,12 @@ cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const floa
     cudaError_t e =
         cudaMemsetAsync(topk->lsi, 0xFF, static_cast<size_t>(grid) * Q * topk->K * sizeof(int), st);
     if (e != cudaSuccess) return e;
-    e = mode == EOGP_SCORE_CODES ? launch_tc_kernel<EOGP_SCORE_CODES, true>(t0, t1, g, grid, st)
-                                 : launch_tc_kernel<EOGP_SCORE_PAPER, true>(t0, t1, g, grid, st);
+    e = cudaMemsetAsync(topk->gtau, 0, static_cast<size_t>(Q) * sizeof(unsigned), st);  // key 0: none yet
+    if (e != cudaSuccess) return e;
+    e = dispatch_tc<true>(mode, BN, t0, t1, g, grid, st);
     if (e != cudaSuccess) return e;
     return launch_topk_merge(topk->lst, topk->lsi, grid, Q, topk->K, topk->out_s, topk->ld_os,
                              topk->out_i, topk->ld_oi, st);
   }
-  return mode == EOGP_SCORE_CODES ? launch_tc_kernel<EOGP_SCORE_CODES, false>(t0, t1, g, grid, st)
-                                  : launch_tc_kernel<EOGP_SCORE_PAPER, false>(t0, t1, g, grid, st);
+  return dispatch_tc<false>(mode, BN, t0, t1, g, grid, st);
 }

@@ -6,7 +6,8 @@
 // Two kernels:
 // * k_topk_dense ranks a dense [Q, N] score matrix: block (slot s, query tile)
 //   owns stored rows [s R, (s+1) R) of 32 queries; 128-row chunks are staged
-//   transposed in shared memory and lane j keeps query j's list there.
+//   transposed in shared memory and the warp offers each query's column to
+//   that query's list.
 // * k_topk_merge merges per-slot lists [S][Q][K] (written by k_topk_dense or by
 //   the fused tensor-core scoring epilogue) into the final [Q, K]. Every slot
 //   list is sorted, so the largest K-th entry over the slots is a lower bound
@@ -40,20 +41,27 @@ __device__ __forceinline__ int key_index(unsigned long long key) {
   return static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(key));
 }
 
+template <int E>
 __global__ void __launch_bounds__(32) k_topk_dense(const float* __restrict__ sc, int ld, int Q, int N,
                                                    int K, int rows_per_slot, float* __restrict__ lst,
                                                    int* __restrict__ lsi) {
+  constexpr int kCap = 32 * E;
   extern __shared__ float sm[];
-  float* tb = sm;                                         // [32 queries][kTs]
-  float* ls = sm + 32 * kTs + static_cast<size_t>(threadIdx.x) * K;  // this lane's list
-  int* li = reinterpret_cast<int*>(sm + 32 * kTs + 32 * K) + static_cast<size_t>(threadIdx.x) * K;
+  float* tb = sm;                                     // [32 queries][kTs]
+  float* ls = sm + 32 * kTs;                          // [32][kCap]
+  int* li = reinterpret_cast<int*>(ls + 32 * kCap);   // [32][kCap]
+  int* cnt = li + 32 * kCap;                          // [32]
+  float* tau = reinterpret_cast<float*>(cnt + 32);    // [32]
   const int lane = threadIdx.x;
   const int slot = blockIdx.x, q0 = blockIdx.y * 32;
   const int nq = min(32, Q - q0);
   const int r_beg = slot * rows_per_slot, r_end = min(N, r_beg + rows_per_slot);
   const bool vec = (ld & 3) == 0 && (reinterpret_cast<uintptr_t>(sc) & 15) == 0;
-  eogp::TopkState tk;
-  eogp::topk_reset(tk);
+  auto list_of = [&](int j) {
+    return eogp::WarpTopk{ls + static_cast<size_t>(j) * kCap, li + static_cast<size_t>(j) * kCap, cnt + j, tau + j,
+                          K, nullptr};
+  };
+  for (int j = 0; j < nq; ++j) eogp::topk_warp_reset(list_of(j), lane);
   for (int r0 = r_beg; r0 < r_end; r0 += kChunk) {
     const int nr = min(kChunk, r_end - r0);
     for (int j = 0; j < nq; ++j) {
@@ -70,12 +78,12 @@ __global__ void __launch_bounds__(32) k_topk_dense(const float* __restrict__ sc,
       }
     }
     __syncwarp();
-    if (lane < nq) eogp::topk_scan(tb + lane * kTs, nr, r0, ls, li, K, tk);
+    for (int j = 0; j < nq; ++j) eogp::topk_warp_offer<E>(tb + j * kTs, nr, r0, list_of(j), lane);
     __syncwarp();
   }
-  if (lane < nq) {
-    const size_t o = (static_cast<size_t>(slot) * Q + q0 + lane) * K;
-    eogp::topk_write(ls, li, K, tk, lst + o, lsi + o);
+  for (int j = 0; j < nq; ++j) {
+    const size_t o = (static_cast<size_t>(slot) * Q + q0 + j) * K;
+    eogp::topk_warp_write<E>(list_of(j), lane, lst + o, lsi + o);
   }
 }
 
@@ -162,19 +170,30 @@ int topk_dense_slots(int N) {
   return std::max(1, (N + R - 1) / R);
 }
 
-cudaError_t launch_topk_dense(const float* scores, int ld, int Q, int N, int K, float* lst, int* lsi,
-                              cudaStream_t st) {
-  if (Q <= 0) return cudaSuccess;
+template <int E>
+cudaError_t launch_topk_dense_e(const float* scores, int ld, int Q, int N, int K, float* lst, int* lsi,
+                                cudaStream_t st) {
   const int S = topk_dense_slots(N);
-  const size_t smem = (32 * kTs + 32 * static_cast<size_t>(K) * 2) * 4;
+  const size_t smem = (32 * kTs + 32 * static_cast<size_t>(32 * E) * 2 + 64) * 4;
   if (smem > 48 * 1024) {
-    const cudaError_t e = cudaFuncSetAttribute(k_topk_dense, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    const cudaError_t e = cudaFuncSetAttribute(k_topk_dense<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                static_cast<int>(smem));
     if (e != cudaSuccess) return e;
   }
   dim3 grid(S, (Q + 31) / 32);
-  k_topk_dense<<<grid, 32, smem, st>>>(scores, ld, Q, N, K, rows_per_slot(N), lst, lsi);
+  k_topk_dense<E><<<grid, 32, smem, st>>>(scores, ld, Q, N, K, rows_per_slot(N), lst, lsi);
   return cudaGetLastError();
+}
+
+cudaError_t launch_topk_dense(const float* scores, int ld, int Q, int N, int K, float* lst, int* lsi,
+                              cudaStream_t st) {
+  if (Q <= 0) return cudaSuccess;
+  switch (eogp::topk_entries_per_lane(K)) {
+    case 2: return launch_topk_dense_e<2>(scores, ld, Q, N, K, lst, lsi, st);
+    case 4: return launch_topk_dense_e<4>(scores, ld, Q, N, K, lst, lsi, st);
+    case 8: return launch_topk_dense_e<8>(scores, ld, Q, N, K, lst, lsi, st);
+    default: return launch_topk_dense_e<16>(scores, ld, Q, N, K, lst, lsi, st);
+  }
 }
 
 cudaError_t launch_topk_merge(const float* lst, const int* lsi, int S, int Q, int K, float* out_s,

@@ -7,7 +7,7 @@
   reproducible, so the lists must match exactly (values and indices, including
   planted equal scores); PAPER / FP lists are checked for validity within the
   score tolerance (several lists are correct when scores differ by less).
-* The fused path (ranking inside the tensor-core epilogue, K <= 64), the dense
+* The fused path (ranking inside the tensor-core epilogue, K <= 32), the dense
   path (Q < 64 CODES, FP, K > 64) and the edge cases N < K and N = 0.
 * Full scan scale (4,194,304 stored 16,384-bit codes, Q = 1024): the fused
   lists equal the oracle ranking of the dense scores of sampled queries.
@@ -107,10 +107,12 @@ def codes_case(N, Q, ks, seed, dup=True):
     return tc, ts, qc, qs
 
 
-@pytest.mark.parametrize("N,Q,ks,K", [(1000, 70, [128, 256], 10), (5000, 130, [1024, 1024], 64),
-                                      (300, 64, [128], 1), (50, 64, [128], 64),
-                                      (20000, 200, [512], 20)])
+@pytest.mark.parametrize("N,Q,ks,K", [(1000, 70, [128, 256], 10), (5000, 130, [1024, 1024], 32),
+                                      (300, 64, [128], 1), (20, 64, [128], 32),
+                                      (20000, 200, [512], 20), (30000, 300, [1024], 20),
+                                      (5000, 130, [1024, 1024], 64)])
 def test_topk_codes_fused_exact(N, Q, ks, K):
+    """K <= 32 ranks inside the tensor-core epilogue; K = 64 takes the dense path."""
     tc, ts, qc, qs = codes_case(N, Q, ks, N + K)
     vals, idx = E.score_topk(dev(tc), dev(ts), ks, E.SCORE_CODES, dev(qc), K, query_scales=dev(qs))
     E.sync_status()
