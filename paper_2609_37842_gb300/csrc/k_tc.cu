@@ -597,19 +597,67 @@ struct RotArgs {
   unsigned* status;
 };
 
-// Bias channel and token lengths, applied to one 32-column chunk of one output
+// Bias channel and token lengths, applied to one W-column chunk of one output
 // row before the hi/lo split.
-__device__ __forceinline__ void rot_fixup(const RotArgs& g, int row, int col, float (&v)[32]) {
+template <int W>
+__device__ __forceinline__ void rot_fixup(const RotArgs& g, int row, int col, float (&v)[W]) {
   if (g.bias) {
 #pragma unroll
-    for (int e = 0; e < 32; ++e) v[e] += col + e < g.nbias ? __ldg(g.bias + col + e) : 0.f;
+    for (int e = 0; e < W; ++e) v[e] += col + e < g.nbias ? __ldg(g.bias + col + e) : 0.f;
   }
   if (g.lengths) {
     const int bex = row / g.T;
     if (row - bex * g.T >= __ldg(g.lengths + bex)) {
 #pragma unroll
-      for (int e = 0; e < 32; ++e) v[e] = 0.f;
+      for (int e = 0; e < W; ++e) v[e] = 0.f;
     }
+  }
+}
+
+// One W-column chunk (W = 32 or 16) of one output row: fix-ups, hi/lo split,
+// 32-byte stores into the blocked layout (element (row = b T + t, col) at
+// ((b (ldo / 128) + col / 128) T + t) 128 + col % 128).
+template <int W>
+__device__ __forceinline__ void rot_store(const RotArgs& g, int row, int col, float (&v)[W]) {
+  rot_fixup<W>(g, row, col, v);
+  uint32_t h[W / 2], l[W / 2];
+#pragma unroll
+  for (int e = 0; e < W / 2; ++e) {
+    const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * e]);
+    const __nv_bfloat16 h1 = __float2bfloat16_rn(v[2 * e + 1]);
+    h[e] = pack_bf16x2(h0, h1);
+    l[e] = pack_bf16x2(__float2bfloat16_rn(v[2 * e] - __bfloat162float(h0)),
+                       __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1)));
+  }
+  const int bex = row / g.T, tok = row - bex * g.T;
+  // 16-column pieces: tiles start on multiples of 16, so a piece never crosses a
+  // 128-column block (a 32-column chunk may, and is placed piece by piece).
+#pragma unroll
+  for (int q = 0; q < W / 16; ++q) {
+    const int cq = col + 16 * q;
+    const size_t off = ((static_cast<size_t>(bex) * (g.ldo >> 7) + (cq >> 7)) * g.T + tok) * 128 + (cq & 127);
+    uint32_t w[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) w[e] = h[8 * q + e];
+    st_global_v8(g.hi + off, w);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) w[e] = l[8 * q + e];
+    st_global_v8(g.lo + off, w);
+  }
+}
+
+// Drains one accumulator row of a BN-column tile (BN a multiple of 16).
+__device__ __forceinline__ void rot_drain(const RotArgs& g, uint32_t tb, int row, int n0) {
+  int c = 0;
+  for (; c + 32 <= g.BN; c += 32) {
+    float v[32];
+    tmem_ld32(tb + c, v);
+    if (row < g.M && n0 + c < g.ldo) rot_store<32>(g, row, n0 + c, v);
+  }
+  if (c < g.BN) {
+    float v[16];
+    tmem_ld16(tb + c, v);
+    if (row < g.M && n0 + c < g.ldo) rot_store<16>(g, row, n0 + c, v);
   }
 }
 
@@ -717,39 +765,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int m0 = (t / g.nN) * 128, n0 = (t % g.nN) * g.BN;
       const int row = m0 + q * 32 + lane;
       const uint32_t tb = tmem + buf * bstride + (static_cast<uint32_t>(q * 32) << 16);
-      for (int c = 0; c < g.BN; c += 32) {
-        float v[32];
-        tmem_ld32(tb + c, v);
-        const int col = n0 + c;
-        if (row < g.M && col < g.ldo) {
-          rot_fixup(g, row, col, v);
-          uint32_t h[16], l[16];
-#pragma unroll
-          for (int e = 0; e < 16; ++e) {
-            const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * e]);
-            const __nv_bfloat16 h1 = __float2bfloat16_rn(v[2 * e + 1]);
-            h[e] = pack_bf16x2(h0, h1);
-            l[e] = pack_bf16x2(__float2bfloat16_rn(v[2 * e] - __bfloat162float(h0)),
-                               __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1)));
-          }
-          const int bex = row / g.T, tok = row - bex * g.T;
-          const size_t off =
-              ((static_cast<size_t>(bex) * (g.ldo >> 7) + (col >> 7)) * g.T + tok) * 128 + (col & 127);
-          uint32_t w[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) w[e] = h[e];
-          st_global_v8(g.hi + off, w);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) w[e] = h[8 + e];
-          st_global_v8(g.hi + off + 16, w);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) w[e] = l[e];
-          st_global_v8(g.lo + off, w);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) w[e] = l[8 + e];
-          st_global_v8(g.lo + off + 16, w);
-        }
-      }
+      rot_drain(g, tb, row, n0);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_relaxed(&tempty[buf]);
@@ -883,39 +899,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int m0 = (t / g.nN) * 256 + static_cast<int>(rank) * 128, n0 = (t % g.nN) * g.BN;
       const int row = m0 + q * 32 + lane;
       const uint32_t tb = tmem + buf * bstride + (static_cast<uint32_t>(q * 32) << 16);
-      for (int c = 0; c < g.BN; c += 32) {
-        float v[32];
-        tmem_ld32(tb + c, v);
-        const int col = n0 + c;
-        if (row < g.M && col < g.ldo) {
-          rot_fixup(g, row, col, v);
-          uint32_t h[16], l[16];
-#pragma unroll
-          for (int e = 0; e < 16; ++e) {
-            const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * e]);
-            const __nv_bfloat16 h1 = __float2bfloat16_rn(v[2 * e + 1]);
-            h[e] = pack_bf16x2(h0, h1);
-            l[e] = pack_bf16x2(__float2bfloat16_rn(v[2 * e] - __bfloat162float(h0)),
-                               __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1)));
-          }
-          const int bex = row / g.T, tok = row - bex * g.T;
-          const size_t off =
-              ((static_cast<size_t>(bex) * (g.ldo >> 7) + (col >> 7)) * g.T + tok) * 128 + (col & 127);
-          uint32_t w[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) w[e] = h[e];
-          st_global_v8(g.hi + off, w);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) w[e] = h[8 + e];
-          st_global_v8(g.hi + off + 16, w);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) w[e] = l[e];
-          st_global_v8(g.lo + off, w);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) w[e] = l[8 + e];
-          st_global_v8(g.lo + off + 16, w);
-        }
-      }
+      rot_drain(g, tb, row, n0);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_relaxed_cluster(mapa_shared(smem_u32(&tempty[buf]), 0));
@@ -1007,17 +991,21 @@ static bool rotate_pairs(int K) {
   return K <= 1536;
 }
 
-int rotate_bn(int ldo) {
+// N tile width for `n` output columns: as few tiles of at most 256 columns as
+// is cheapest, each a multiple of `gran` (16: tcgen05 N granularity for one
+// CTA; 32 for CTA pairs, whose halves must be multiples of 16), counting a
+// fixed per-tile overhead of 32 columns. EOGP_ROT_BN overrides for sweeps.
+int rotate_bn(int n, int gran) {
   static int forced = -1;
   if (forced < 0) {
     const char* e = getenv("EOGP_ROT_BN");
     forced = e ? atoi(e) : 0;
   }
-  if (forced > 0 && forced % 32 == 0 && forced <= 256) return forced;
-  const int n0 = (ldo + 255) / 256;
+  if (forced > 0 && forced % gran == 0 && forced <= 256) return forced;
+  const int n0 = (n + 255) / 256;
   int best = 0, best_cost = 1 << 30;
   for (int nN = n0; nN <= n0 + 1; ++nN) {
-    const int bn = ((ldo + nN - 1) / nN + 31) / 32 * 32;
+    const int bn = ((n + nN - 1) / nN + gran - 1) / gran * gran;
     const int cost = nN * bn + 32 * nN;
     if (cost < best_cost) {
       best_cost = cost;
@@ -1031,7 +1019,8 @@ cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W
                              void* hi, void* lo, int ldo, int T, const float* bias,
                              const int32_t* lengths, int num_sms, unsigned* status, cudaStream_t st) {
   if (M <= 0) return cudaSuccess;
-  const int BN = rotate_bn(ldo);
+  const bool pairs = rotate_pairs(K);
+  const int BN = rotate_bn(Wrows, pairs ? 32 : 16);
   // As many pipeline stages as fit in 227 KB of shared memory (at most 8);
   // EOGP_ROT_STAGES overrides for tuning sweeps.
   static int forced_stages = -1;
@@ -1051,7 +1040,7 @@ cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W
   g.K = K;
   g.BN = BN;
   g.stages = stages;
-  g.nN = (ldo + BN - 1) / BN;
+  g.nN = (Wrows + BN - 1) / BN;  // columns past the last tile (padding up to ldo) are not written
   g.n_tiles = ((M + 127) / 128) * g.nN;
   g.ldo = ldo;
   g.T = T;
@@ -1061,7 +1050,7 @@ cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W
   g.nbias = Wrows;
   g.lengths = lengths;
   g.status = status;
-  if (rotate_pairs(K) && BN % 32 == 0) {
+  if (pairs) {
     // CTA pairs: tiles of 256 rows, W split in halves of BN / 2 rows.
     CUtensorMap tWh;
     if (tmap_bf16_2d(&tWh, W, K, Wrows, ldw, 64, BN / 2)) return cudaErrorInvalidValue;
