@@ -42,7 +42,7 @@ METRIC = "training examples compressed/sec per layer stack"
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # dram__bytes_read.sum + dram__bytes_write.sum per rotation launch from the committed
 # ncu capture (profiles/), or None when the kernel changed after the capture.
-ROTATE_TRAFFIC_BYTES = 692.1e6  # mean over one transformer block (8 launches) at B = 256
+ROTATE_TRAFFIC_BYTES = 1424.9e6  # mean over one transformer block (8 launches) at B = 512
 
 
 def load_peaks():
@@ -445,7 +445,7 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--batch", type=int, default=256)
+    ap.add_argument("--batch", type=int, default=512)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -550,11 +550,30 @@ def main():
     peak = peaks.get("bf16_tflops_sustained") or PEAKS_FALLBACK["bf16_tflops_sustained"]
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": (achieved / peak) if achieved else None,
-                # captured on the full stack's block structure at B = 256 only
-                "traffic": ROTATE_TRAFFIC_BYTES if (B == 256 and U % 4 == 0) else None,
+                # captured on the full stack's block structure at the default batch only
+                "traffic": ROTATE_TRAFFIC_BYTES if (B == 512 and U % 4 == 0) else None,
                 "kernel": "k_tc_rotate / k_tc_rotate2 (Kronecker rotations)",
                 "peak_source": f"{peaks_src} bf16_tflops_sustained",
                 "flops_per_launch": flops_per_launch}
+
+    # ---- context: cuBLAS bf16 on the largest rotation shape (not on the path) ----
+    ref_gemm = None
+    if rank == 0 and not args.no_score:
+        kmax = max(md["d_in"] for md in mods)
+        A = torch.randn((B * T, kmax), device=dev, dtype=torch.bfloat16)
+        Wt = torch.randn((640, kmax), device=dev, dtype=torch.bfloat16)
+        A @ Wt.t()
+        torch.cuda.synchronize()
+        a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a_ev.record(stream)
+        for _ in range(3):
+            A @ Wt.t()
+        b_ev.record(stream)
+        torch.cuda.synchronize()
+        gms = a_ev.elapsed_time(b_ev) / 3
+        ref_gemm = {"what": f"cuBLAS bf16 [{B * T} x {kmax}] x [{kmax} x 640] -> bf16 (context only)",
+                    "ms": gms, "TFLOPs": 2.0 * B * T * kmax * 640 / (gms / 1000.0) / 1e12}
+        del A, Wt
 
     # ---- scoring: Q = 1024 one-bit queries x N = 16384 stored codes ----
     scoring = None
@@ -829,7 +848,8 @@ def main():
                            "k": w.k, "modules": U, "parallelism": f"replicas x{world}",
                            "l2": "inputs > L2 (B x 151 MB per step)"},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "scoring": scoring,
-                "pack_sign": pack, "scan": scan, "eogp_r_srht": eogp_r, "other_workloads": configs,
+                "pack_sign": pack, "scan": scan, "eogp_r_srht": eogp_r, "reference_gemm": ref_gemm,
+                "other_workloads": configs,
                 "fit_pca": fit,
                 "gpu_launches": launches, "kernels": kern, "clocks": clk}
         print(json.dumps(line))

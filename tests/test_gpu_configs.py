@@ -1,7 +1,7 @@
 """GPU parity on every workload shape at full size, on sampled outputs.
 
 * GPT-2 stack: the compression in the exact launch configuration bench.py
-  times (B = 128 examples per call, T = 512, m = 4096, k = 1024, device-side
+  times (B = 512 examples per call, T = 512, m = 4096, k = 1024, device-side
   inputs), checked on sampled examples of one module of each shape.
 * OLMo 2 1B / 7B shapes and the 32B gate projection (T = 2048, m = 8192,
   k = 2048): a few examples per distinct module shape.
@@ -65,7 +65,7 @@ def check_x_codes(x_gpu, codes_gpu, scales_gpu, x_or, k):
 def test_gpt2_stack_in_bench_launch_configuration():
     import bench
     w = synth.WORKLOADS["gpt2_small_bf16"]
-    B = 128
+    B = 512
     dev = torch.device(DEV)
     mods = bench.build_stack(w, B, dev, seed=1000)
     ws = E.workspace(max(E.compress_workspace_size(md["desc"], B, E.OUT_CODES) for md in mods), dev)
@@ -74,7 +74,7 @@ def test_gpt2_stack_in_bench_launch_configuration():
     scales = torch.empty((B, len(mods)), dtype=torch.float32, device=dev)
     bench.compress_step(mods, E, codes, scales, ws, words)
     E.sync_status()
-    examples = [0, 77, 127]
+    examples = [0, 301, 511]
     for u in (0, 1, 2, 3, 47):    # c_attn, attn.c_proj, c_fc, mlp.c_proj (first block), last module
         md = mods[u]
         desc = md["desc"]
