@@ -556,6 +556,14 @@ def main():
                 "peak_source": f"{peaks_src} bf16_tflops_sustained",
                 "flops_per_launch": flops_per_launch}
 
+    # ---- measured e4m3 tensor-core and popcount rates (scoring rooflines) ----
+    probes = None
+    if rank == 0 and not args.no_score:
+        f8, pc = E.measure_peaks()
+        probes = {"e4m3_tflops": f8, "popc_words_per_s": pc,
+                  "what": "eogp_measure_peaks: back-to-back kind::f8f6f4 MMAs from shared memory; "
+                          "XOR + popcount chains on every core"}
+
     # ---- context: cuBLAS bf16 on the largest rotation shape (not on the path) ----
     ref_gemm = None
     if rank == 0 and not args.no_score:
@@ -601,14 +609,15 @@ def main():
         E.sync_status()
         sms = e0.elapsed_time(e1) / reps
         D = U * w.k
-        f8_peak = 2.0 * bf16_burst          # e4m3 dense = 2 x bf16 dense (nominal ratio)
+        f8_peak = probes["e4m3_tflops"] if probes else 2.0 * bf16_burst
         alg = 2.0 * N * Q * D               # +-1 multiply-adds of the inner products
         scoring = {"metric": "query x train scores/sec", "value": N * Q / (sms / 1000.0),
                    "unit": "scores/s", "ms_per_call": sms, "N": N, "Q": Q, "bits": D,
                    "mode": "CODES (tcgen05 kind::f8f6f4, +-1 e4m3 operands)",
                    "tensor_TFLOPs": alg / (sms / 1000.0) / 1e12,
                    "tensor_frac": alg / (sms / 1000.0) / 1e12 / f8_peak,
-                   "tensor_peak": f8_peak, "tensor_peak_source": f"2 x {peaks_src} bf16_tflops (e4m3)"}
+                   "tensor_peak": f8_peak,
+                   "tensor_peak_source": "eogp_measure_peaks e4m3" if probes else f"2 x {peaks_src} bf16_tflops"}
         # paper mode (unquantised queries), dense and with the ranking fused (K = 20)
         y = torch.randn((Q, D), generator=g, device=dev)
         wsp = E.workspace(E.score_workspace_size(N, ks, E.SCORE_PAPER, Q), dev)
@@ -797,10 +806,14 @@ def main():
             if Q >= 64:   # tensor-core kernel: +-1 multiply-adds against the e4m3 peak
                 tfl = 2.0 * N * ksc * Q / (qms / 1000.0) / 1e12
                 ent.update({"kernel": "k_score_tc", "tensor_TFLOPs": tfl,
-                            "tensor_frac": tfl / (2.0 * bf16_burst)})
+                            "tensor_frac": tfl / (probes["e4m3_tflops"] if probes else 2.0 * bf16_burst),
+                            "tensor_peak_source": "eogp_measure_peaks e4m3" if probes
+                            else "2 x measured bf16 burst"})
             else:
-                ent.update({"kernel": "k_score_codes_smallq (popcount)",
-                            "word_ops_per_s": N * Q * Wsc / (qms / 1000.0)})
+                wops = N * Q * Wsc / (qms / 1000.0)
+                ent.update({"kernel": "k_score_codes_smallq (popcount)", "word_ops_per_s": wops})
+                if probes:
+                    ent["popc_frac"] = wops / probes["popc_words_per_s"]
             if Q >= 1024:  # per-query top 20 in the scoring epilogue: no Q x N output
                 K = 20
                 wt = E.workspace(E.score_topk_workspace_size(N, [ksc], E.SCORE_CODES, Q, K), dev)
@@ -849,6 +862,7 @@ def main():
                            "l2": "inputs > L2 (B x 151 MB per step)"},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "scoring": scoring,
                 "pack_sign": pack, "scan": scan, "eogp_r_srht": eogp_r, "reference_gemm": ref_gemm,
+                "measured_rates": probes,
                 "other_workloads": configs,
                 "fit_pca": fit,
                 "gpu_launches": launches, "kernels": kern, "clocks": clk}

@@ -96,6 +96,14 @@ int eogp_sync_status(eogp_stream_t stream);
 int eogp_profile_enable(int on);
 int eogp_profile_read(int kind, int* launches, double* total_ms, int reset);
 
+/* Throughput probes for the scoring rooflines (no counterpart in the paper: a
+ * library convenience). Measures on the current device, synchronously: the dense
+ * tcgen05 kind::f8f6f4 e4m3 rate (TFLOP/s, back-to-back M = 128, N = 256, K = 32
+ * MMAs from shared memory, one CTA per SM) and the CUDA-core XOR + popcount rate
+ * (32-bit words per second). Either output may be NULL.
+ * Errors: EOGP_ECUDA, EOGP_ETIMEOUT. */
+int eogp_measure_peaks(double* e4m3_tflops, double* popc_words_per_s);
+
 /* ========================================================================
  * Retained-set plan (host; once per module)
  *

@@ -843,6 +843,24 @@ extern "C" int eogp_payload_unpack(const uint8_t* payload, size_t ld_payload, in
   return EOGP_OK;
 }
 
+// ================================================================ probes
+
+extern "C" int eogp_measure_peaks(double* e4m3_tflops, double* popc_words_per_s) {
+  clear_error();
+  unsigned* status = status_word();
+  if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
+  unsigned* sink = nullptr;
+  CUDA_TRY(cudaMalloc(reinterpret_cast<void**>(&sink), sizeof(unsigned)));
+  double f8 = 0.0, pc = 0.0;
+  const cudaError_t e = run_peak_probes(sm_count(), status, sink, &f8, &pc, nullptr);
+  cudaFree(sink);
+  if (e != cudaSuccess) return set_error(EOGP_ECUDA, "%s", cudaGetErrorString(e));
+  if (int rc = eogp_sync_status(nullptr)) return rc;
+  if (e4m3_tflops) *e4m3_tflops = f8;
+  if (popc_words_per_s) *popc_words_per_s = pc;
+  return EOGP_OK;
+}
+
 // ================================================================ SRHT
 
 extern "C" int eogp_srht(const float* z, int B, int m, int ldz, const int8_t* signs, const int32_t* rows,

@@ -136,6 +136,10 @@ cudaError_t launch_payload_pack(const uint32_t* codes, int ld_codes, const float
 cudaError_t launch_payload_unpack(const uint8_t* in, size_t ld_in, int N, const int* ks, int U, uint32_t* codes,
                                   int ld_codes, float* scales, int ld_scales, cudaStream_t st);
 
+// k_peaks.cu: e4m3 tensor-core and XOR + popcount throughput probes.
+cudaError_t run_peak_probes(int num_sms, unsigned* status, unsigned* sink, double* f8_tflops,
+                            double* popc_words_per_s, cudaStream_t st);
+
 // k_srht.cu: EOGP-R second stage, one CTA per row (z fp32, or bf16 hi + lo when hilo).
 int srht_width(int m);
 size_t srht_smem_bytes(int m);

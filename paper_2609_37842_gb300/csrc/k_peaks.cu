@@ -1,0 +1,125 @@
+// Throughput probes for the scoring rooflines: the dense e4m3 tensor-core rate
+// of tcgen05.mma kind::f8f6f4 (the +-1 scoring MMA) and the integer
+// XOR + popcount rate of the CUDA cores (the popcount scoring kernels). Neither
+// is among the measured copy / bf16 GEMM peaks.
+//
+// MMA probe: one CTA per SM; one thread issues back-to-back M = 128, N = 256,
+// K = 32 MMAs from two fixed shared-memory operand tiles into alternating TMEM
+// accumulators, committing to an mbarrier every 64 MMAs and waiting (bounded)
+// one batch behind. POPC probe: every thread runs 8 independent XOR + POPC +
+// ADD chains; the sums are written so the work is kept.
+#include "eogp_dev.cuh"
+#include "eogp_internal.h"
+
+using namespace eogp;
+
+namespace {
+
+constexpr int kBatch = 64;
+
+__global__ void __launch_bounds__(128, 1) k_peak_f8(int batches, unsigned* status, unsigned* sink) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* A = smem;          // 128 rows x 128 bytes
+  uint8_t* B = smem + 16384;  // 256 rows x 128 bytes
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 16384 + 32768);
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 2);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int i = threadIdx.x; i < (16384 + 32768) / 16; i += blockDim.x)
+    reinterpret_cast<uint4*>(smem)[i] = make_uint4(0x38383838u, 0xB8B8B8B8u, 0x38383838u, 0xB8B8B8B8u);
+  if (threadIdx.x == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    fence_barrier_init();
+  }
+  fence_proxy_async_smem();
+  if (warp == 0) tmem_alloc(tslot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tslot;
+  if (warp == 0 && lane == 0) {
+    const uint32_t idesc = idesc_e4m3_f32(128, 256);
+    const uint32_t sa = smem_u32(A), sb = smem_u32(B);
+    for (int b = 0; b < batches; ++b) {
+      const int buf = b & 1;
+      if (b >= 2 && !mbar_wait(&bar[buf], ((b >> 1) - 1) & 1u, status)) break;
+      tc_fence_after();
+#pragma unroll 4
+      for (int i = 0; i < kBatch; ++i) {
+        const int kk = i & 3;
+        tc_mma_f8(tmem + buf * 256u, sdesc_sw128(sa + kk * 32, 16, 1024), sdesc_sw128(sb + kk * 32, 16, 1024),
+                  idesc, i != 0 ? 1u : 0u);
+      }
+      tc_commit(&bar[buf]);
+    }
+    // drain the last two batches
+    for (int b = batches > 2 ? batches - 2 : 0; b < batches; ++b)
+      if (!mbar_wait(&bar[b & 1], (b >> 1) & 1u, status)) break;
+  }
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    float v[16];
+    tmem_ld16(tmem + (static_cast<uint32_t>(lane) << 16), v);  // keep the result observable
+    if (lane == 0 && v[0] == 12345.f) atomicAdd(sink, 1u);
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+__global__ void __launch_bounds__(256) k_peak_popc(int iters, unsigned* sink) {
+  uint32_t x[8], acc[8];
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    x[c] = (threadIdx.x + 1u) * 2654435761u + c * 40503u + blockIdx.x;
+    acc[c] = 0;
+  }
+  for (int i = 0; i < iters; ++i) {
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      x[c] ^= 0x9E3779B9u + static_cast<uint32_t>(i);
+      acc[c] += __popc(x[c]);
+    }
+  }
+  uint32_t t = 0;
+#pragma unroll
+  for (int c = 0; c < 8; ++c) t += acc[c];
+  if (t == 0xFFFFFFFFu) atomicAdd(sink, t);
+}
+
+}  // namespace
+
+cudaError_t run_peak_probes(int num_sms, unsigned* status, unsigned* sink, double* f8_tflops,
+                            double* popc_words_per_s, cudaStream_t st) {
+  cudaEvent_t e0, e1, e2;
+  cudaEventCreate(&e0);
+  cudaEventCreate(&e1);
+  cudaEventCreate(&e2);
+  // more than half of an SM's shared memory: one CTA (and one TMEM allocation) per SM
+  const size_t smem = 140 * 1024;
+  cudaError_t e = cudaFuncSetAttribute(k_peak_f8, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  const int batches = 4096;
+  k_peak_f8<<<num_sms, 128, smem, st>>>(8, status, sink);  // warm-up
+  cudaEventRecord(e0, st);
+  k_peak_f8<<<num_sms, 128, smem, st>>>(batches, status, sink);
+  cudaEventRecord(e1, st);
+  const int iters = 1 << 15;
+  const int blocks = num_sms * 8;
+  k_peak_popc<<<blocks, 256, 0, st>>>(iters, sink);
+  cudaEventRecord(e2, st);
+  e = cudaEventSynchronize(e2);
+  if (e != cudaSuccess) return e;
+  float ms1 = 0.f, ms2 = 0.f;
+  cudaEventElapsedTime(&ms1, e0, e1);
+  cudaEventElapsedTime(&ms2, e1, e2);
+  cudaEventDestroy(e0);
+  cudaEventDestroy(e1);
+  cudaEventDestroy(e2);
+  const double flops = 2.0 * 128 * 256 * 32 * static_cast<double>(kBatch) * batches * num_sms;
+  *f8_tflops = flops / (ms1 / 1000.0) / 1e12;
+  *popc_words_per_s = static_cast<double>(blocks) * 256 * 8 * iters / (ms2 / 1000.0);
+  return cudaGetLastError();
+}
