@@ -168,6 +168,8 @@ def cpu_sample(w, n_examples, seed=1):
         shapes.setdefault((mod.d_in, mod.d_out), []).append(u)
     rng = np.random.default_rng(seed)
     total = 0.0
+    per_shape = {}
+    flops = 0.0
     for (d_in, d_out), us in shapes.items():
         u = us[0]
         QA = synth.round_bf16(synth.haar_orthogonal(d_in, rng))
@@ -181,10 +183,39 @@ def cpu_sample(w, n_examples, seed=1):
         O.compress_layer(a, s, QA, QS, Lam, lam, w.m, P)
         dt = (time.perf_counter() - t0) / n_examples
         total += dt * len(us)
+        per_shape[f"{d_in}->{d_out}"] = 1.0 / dt
+        # the oracle's dense work per example: G (2 T d_out d_in), Q_S^T G Q_A
+        # (2 d_out d_in (d_in + d_out)), P^T z (2 m k)
+        flops += len(us) * (2.0 * w.T * d_out * d_in + 2.0 * d_out * d_in * (d_in + d_out) +
+                            2.0 * w.m * w.k)
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
     desc = (f"{n_examples} example(s) x one module of each of the {len(shapes)} distinct shapes, "
             f"scaled by the shape counts to the {len(w.modules)}-module stack")
+    cpu_sample.details = {"examples_per_s_per_shape": per_shape,
+                          "oracle_GFLOPs": flops / total / 1e9 if total else None}
     return total, cores, desc
+
+
+def cpu_score_sample(seconds=3.0):
+    """Oracle one-bit scores/s (float32 evaluation order) on the GPT-2 query shape
+    (48 modules of 1024 bits): repeated batches of 64 stored rows x 4 queries for
+    about `seconds` of scoring (input generation not timed)."""
+    import numpy as np
+    from oracle import eogp_oracle as O
+    rng = np.random.default_rng(3)
+    ks = [1024] * 48
+    Q, n = 4, 64
+    qc = O.pack_concat([rng.integers(0, 2, (Q, k)).astype(bool) for k in ks])
+    qs = rng.lognormal(0, 0.5, (Q, len(ks))).astype(np.float32)
+    done, busy = 0, 0.0
+    while busy < seconds:
+        tc = O.pack_concat([rng.integers(0, 2, (n, k)).astype(bool) for k in ks])
+        ts = rng.lognormal(0, 0.5, (n, len(ks))).astype(np.float32)
+        t1 = time.perf_counter()
+        O.score_codes_f32(tc, ts, ks, qc, qs)
+        busy += time.perf_counter() - t1
+        done += n * Q
+    return done / busy
 
 
 def run_reference(args):
@@ -849,7 +880,9 @@ def main():
     if rank == 0 and not args.no_cpu_baseline:
         sec, cores, desc = cpu_sample(w, 1)
         cpu = {"value": 1.0 / sec, "unit": "examples/s", "cores": cores, "kind": "oracle",
-               "sample": desc}
+               "sample": desc, **cpu_sample.details,
+               "oracle_scores_per_s": cpu_score_sample(),
+               "scores_sample": "64 stored rows x 4 one-bit queries of 48 x 1024 bits, repeated for ~3 s"}
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": world,
