@@ -288,6 +288,22 @@ int eogp_fit_pca_workspace_size(int n, int m, int k, size_t* bytes);
 int eogp_fit_pca(const float* Z, int n, int m, int ldz, int k, void* Pt, int ld_pt, int pt_dtype,
                  float* eig, void* ws, size_t ws_bytes, eogp_stream_t stream);
 
+/* The same fit split for data spread over several processes or GPUs (the
+ * covariance route of App. B.2: P from Z^T Z / n). Each holder of rows adds its
+ * part of the second moment, the parts are summed (one reduction of an m x m
+ * fp64 matrix, e.g. over a process group), and the fit runs on the sum.
+ *   eogp_second_moment: C [m x ldc] fp64 device (+)= sum_r z_r z_r^T over the n
+ *     rows of Z [n x ldz] fp32 device (overwritten when accumulate == 0).
+ *   eogp_fit_pca_from_moment: Pt, eig as eogp_fit_pca for the matrix C / n_total
+ *     (n_total = rows summed into C); workspace from
+ *     eogp_fit_pca_from_moment_workspace_size; m <= 12288; blocks the host.
+ * Errors: EOGP_EINVAL, EOGP_EUNSUPPORTED, EOGP_EWORKSPACE, EOGP_ECUDA. */
+int eogp_second_moment(const float* Z, int n, int m, int ldz, double* C, int ldc, int accumulate,
+                       eogp_stream_t stream);
+int eogp_fit_pca_from_moment_workspace_size(int m, int k, size_t* bytes);
+int eogp_fit_pca_from_moment(const double* C, int m, int ldc, int n_total, int k, void* Pt, int ld_pt,
+                             int pt_dtype, float* eig, void* ws, size_t ws_bytes, eogp_stream_t stream);
+
 /* ========================================================================
  * One-bit encoding (Sec. 3.3 Eq. onebit; Alg. 1 "Store packed binary signs")
  * ======================================================================== */

@@ -30,6 +30,7 @@ Function map:
   ekfac_sumsq           Sec. 2.2 "EK-FAC approximation"; App. C.2 (corrected eigenvalues)
   first_stage           Sec. 3.2, Eq. first_stage
   fit_pca               App. B.2 "PCA fitting", Alg. 1
+  fit_pca_from_moment   App. B.2 (covariance route from a summed second moment)
   project               Sec. 3.2, Eq. second_stage
   onebit                Sec. 3.3, Eq. onebit; App. A.3 Eq. app_onebit_scale
   pack_bits/unpack_bits App. E.1 (per-module byte packing, Eq. app_payload)
@@ -206,6 +207,15 @@ def fit_pca(Z: np.ndarray, k: int, route: str = "auto") -> Tuple[np.ndarray, np.
     else:
         raise ValueError(route)
     return canonical_signs(P), mu
+
+
+def fit_pca_from_moment(C: np.ndarray, n: int, k: int) -> Tuple[np.ndarray, np.ndarray]:
+    """fit_pca's covariance route (App. B.2) from a second moment already summed
+    over all n rows, C = sum_r z_r z_r^T (e.g. added up over shards): the top-k
+    eigenvectors of C / n with the canonical signs, and their eigenvalues."""
+    w, V = np.linalg.eigh(np.asarray(C, np.float64) / n)
+    idx = np.argsort(-w, kind="stable")[:k]
+    return canonical_signs(V[:, idx]), w[idx]
 
 
 def project(z: np.ndarray, P: np.ndarray) -> np.ndarray:

@@ -896,16 +896,7 @@ extern "C" int eogp_fit_pca_workspace_size(int n, int m, int k, size_t* bytes) {
   return EOGP_OK;
 }
 
-extern "C" int eogp_fit_pca(const float* Z, int n, int m, int ldz, int k, void* Pt, int ld_pt,
-                            int pt_dtype, float* eig, void* ws, size_t ws_bytes, eogp_stream_t stream) {
-  clear_error();
-  size_t need = 0;
-  if (int rc = eogp_fit_pca_workspace_size(n, m, k, &need)) return rc;
-  if (!Z || !Pt || !eig) return set_error(EOGP_EINVAL, "NULL argument");
-  if (ldz < m || ld_pt < m) return set_error(EOGP_EINVAL, "ldz / ld_pt must be >= m");
-  if (pt_dtype != EOGP_F32 && pt_dtype != EOGP_BF16) return set_error(EOGP_EINVAL, "bad pt_dtype");
-  if (!ws || ws_bytes < need) return set_error(EOGP_EWORKSPACE, "workspace of %zu bytes needed", need);
-  if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
+static PcaWs carve_pca_ws(void* ws, int n, int m, int k) {
   const int nn = std::min(n, m);
   char* w = static_cast<char*>(ws);
   size_t off = 0;
@@ -922,8 +913,56 @@ extern "C" int eogp_fit_pca(const float* Z, int n, int m, int ldz, int k, void* 
   pw.sel = reinterpret_cast<int*>(take(static_cast<size_t>(k) * 4));
   pw.red = reinterpret_cast<double*>(take(4 * 8));
   pw.Pr = n < m ? reinterpret_cast<double*>(take(static_cast<size_t>(k) * m * 8)) : nullptr;
-  return fit_pca_device(Z, n, m, ldz, k, Pt, ld_pt, pt_dtype, eig, pw, status_word(),
+  return pw;
+}
+
+extern "C" int eogp_fit_pca(const float* Z, int n, int m, int ldz, int k, void* Pt, int ld_pt,
+                            int pt_dtype, float* eig, void* ws, size_t ws_bytes, eogp_stream_t stream) {
+  clear_error();
+  size_t need = 0;
+  if (int rc = eogp_fit_pca_workspace_size(n, m, k, &need)) return rc;
+  if (!Z || !Pt || !eig) return set_error(EOGP_EINVAL, "NULL argument");
+  if (ldz < m || ld_pt < m) return set_error(EOGP_EINVAL, "ldz / ld_pt must be >= m");
+  if (pt_dtype != EOGP_F32 && pt_dtype != EOGP_BF16) return set_error(EOGP_EINVAL, "bad pt_dtype");
+  if (!ws || ws_bytes < need) return set_error(EOGP_EWORKSPACE, "workspace of %zu bytes needed", need);
+  if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
+  return fit_pca_device(Z, n, m, ldz, k, Pt, ld_pt, pt_dtype, eig, carve_pca_ws(ws, n, m, k), status_word(),
                         reinterpret_cast<cudaStream_t>(stream));
+}
+
+extern "C" int eogp_second_moment(const float* Z, int n, int m, int ldz, double* C, int ldc, int accumulate,
+                                  eogp_stream_t stream) {
+  clear_error();
+  if (n < 0 || m < 1) return set_error(EOGP_EINVAL, "need n >= 0, m >= 1");
+  if (!C || ldc < m) return set_error(EOGP_EINVAL, "C is NULL or ldc < m");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (n == 0) {
+    if (!accumulate) CUDA_TRY(cudaMemset2DAsync(C, static_cast<size_t>(ldc) * 8, 0, static_cast<size_t>(m) * 8, m, st));
+    return EOGP_OK;
+  }
+  if (!Z || ldz < m) return set_error(EOGP_EINVAL, "Z is NULL or ldz < m");
+  CUDA_TRY(second_moment_device(Z, n, m, ldz, C, ldc, accumulate, st));
+  return EOGP_OK;
+}
+
+extern "C" int eogp_fit_pca_from_moment_workspace_size(int m, int k, size_t* bytes) {
+  return eogp_fit_pca_workspace_size(m, m, k, bytes);
+}
+
+extern "C" int eogp_fit_pca_from_moment(const double* C, int m, int ldc, int n_total, int k, void* Pt,
+                                        int ld_pt, int pt_dtype, float* eig, void* ws, size_t ws_bytes,
+                                        eogp_stream_t stream) {
+  clear_error();
+  size_t need = 0;
+  if (int rc = eogp_fit_pca_workspace_size(m, m, k, &need)) return rc;
+  if (n_total < 1) return set_error(EOGP_EINVAL, "n_total must be >= 1");
+  if (!C || !Pt || !eig) return set_error(EOGP_EINVAL, "NULL argument");
+  if (ldc < m || ld_pt < m) return set_error(EOGP_EINVAL, "ldc / ld_pt must be >= m");
+  if (pt_dtype != EOGP_F32 && pt_dtype != EOGP_BF16) return set_error(EOGP_EINVAL, "bad pt_dtype");
+  if (!ws || ws_bytes < need) return set_error(EOGP_EWORKSPACE, "workspace of %zu bytes needed", need);
+  if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
+  return fit_pca_device(nullptr, n_total, m, m, k, Pt, ld_pt, pt_dtype, eig, carve_pca_ws(ws, m, m, k),
+                        status_word(), reinterpret_cast<cudaStream_t>(stream), C, ldc);
 }
 
 // ============================================================== pack, score

@@ -196,6 +196,11 @@ struct PcaWs {
   double* red;   // [4] reduction scratch
   double* Pr;    // [k x m] raw directions (Gram route)
 };
+// C_in (optional): a summed second moment sum_r z_r z_r^T [m x ldc] of n rows in
+// place of Z (covariance route; Z is then unused).
 int fit_pca_device(const float* Z, int n, int m, int ldz, int k, void* Pt, int ld_pt, int pt_dtype,
-                   float* eig, PcaWs ws, unsigned* status, cudaStream_t st);
+                   float* eig, PcaWs ws, unsigned* status, cudaStream_t st, const double* C_in = nullptr,
+                   int ldc = 0);
+cudaError_t second_moment_device(const float* Z, int n, int m, int ldz, double* C, int ldc, int accumulate,
+                                 cudaStream_t st);
 size_t fit_pca_ws_bytes(int n, int m, int k);

@@ -43,7 +43,7 @@ __device__ __forceinline__ void jac_pair(int s, int kidx, int np, int& p, int& q
 // C[i][j] = alpha * sum_k A(i,k) B(j,k) with A(i,k) = A[i*sai + k*sak] (fp32 in,
 // fp64 accumulate and out). 32 x 32 tile per block, 2 x 2 per thread.
 template <typename TA>
-__global__ void __launch_bounds__(256) k_gemm_f64acc(int M, int N, int K, double alpha,
+__global__ void __launch_bounds__(256) k_gemm_f64acc(int M, int N, int K, double alpha, int accumulate,
                                                      const TA* __restrict__ A, long long sai,
                                                      long long sak, const float* __restrict__ B,
                                                      long long sbj, long long sbk,
@@ -87,7 +87,7 @@ __global__ void __launch_bounds__(256) k_gemm_f64acc(int M, int N, int K, double
 #pragma unroll
     for (int y = 0; y < 2; ++y) {
       const int j = j0 + tx + 16 * y;
-      if (j < N) C[i * ldc + j] = alpha * acc[x][y];
+      if (j < N) C[i * ldc + j] = accumulate ? C[i * ldc + j] + alpha * acc[x][y] : alpha * acc[x][y];
     }
   }
 }
@@ -95,10 +95,18 @@ __global__ void __launch_bounds__(256) k_gemm_f64acc(int M, int N, int K, double
 template <typename TA>
 cudaError_t gemm_f64acc(int M, int N, int K, double alpha, const TA* A, long long sai, long long sak,
                         const float* B, long long sbj, long long sbk, double* C, long long ldc,
-                        cudaStream_t st) {
+                        cudaStream_t st, int accumulate = 0) {
   dim3 grid((N + 31) / 32, (M + 31) / 32);
-  k_gemm_f64acc<TA><<<grid, 256, 0, st>>>(M, N, K, alpha, A, sai, sak, B, sbj, sbk, C, ldc);
+  k_gemm_f64acc<TA><<<grid, 256, 0, st>>>(M, N, K, alpha, accumulate, A, sai, sak, B, sbj, sbk, C, ldc);
   return cudaGetLastError();
+}
+
+// A[i][j] = scale * C[i][j] (dense n x n copy of a strided fp64 matrix)
+__global__ void k_scale_copy(const double* __restrict__ C, int ldc, int n, double scale, double* __restrict__ A) {
+  const long long tot = static_cast<long long>(n) * n;
+  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < tot;
+       e += static_cast<long long>(gridDim.x) * blockDim.x)
+    A[e] = scale * C[(e / n) * ldc + e % n];
 }
 
 __global__ void k_eye(double* V, int n) {
@@ -311,9 +319,10 @@ size_t fit_pca_ws_bytes(int n, int m, int k) {
 }
 
 int fit_pca_device(const float* Z, int n, int m, int ldz, int k, void* Pt, int ld_pt, int pt_dtype,
-                   float* eig, PcaWs ws, unsigned* status, cudaStream_t st) {
+                   float* eig, PcaWs ws, unsigned* status, cudaStream_t st, const double* C_in,
+                   int ldc) {
   (void)status;
-  const bool gram = n < m;
+  const bool gram = !C_in && n < m;
   const int nn = gram ? n : m;
   const int np = nn + (nn & 1);
   cudaError_t e;
@@ -327,6 +336,11 @@ int fit_pca_device(const float* Z, int n, int m, int ldz, int k, void* Pt, int l
   if (gram) {
     // A = Z Z^T (n x n)
     PCA_TRY(gemm_f64acc<float>(n, n, m, 1.0, Z, ldz, 1, Z, ldz, 1, ws.A, n, st));
+  } else if (C_in) {
+    // A = C / n from a second moment summed elsewhere (e.g. over shards)
+    k_scale_copy<<<static_cast<unsigned>((static_cast<long long>(m) * m + 255) / 256), 256, 0, st>>>(
+        C_in, ldc, m, 1.0 / n, ws.A);
+    PCA_TRY(cudaGetLastError());
   } else {
     // A = Z^T Z / n (m x m): A(i,j) = sum_r Z[r][i] Z[r][j]
     PCA_TRY(gemm_f64acc<float>(m, m, n, 1.0 / n, Z, 1, ldz, Z, 1, ldz, ws.A, m, st));
@@ -378,4 +392,11 @@ int fit_pca_device(const float* Z, int n, int m, int ldz, int k, void* Pt, int l
   }
 #undef PCA_TRY
   return EOGP_OK;
+}
+
+cudaError_t second_moment_device(const float* Z, int n, int m, int ldz, double* C, int ldc, int accumulate,
+                                 cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  // C(i,j) (+)= sum_r Z[r][i] Z[r][j]
+  return gemm_f64acc<float>(m, m, n, 1.0, Z, 1, ldz, Z, 1, ldz, C, ldc, st, accumulate);
 }

@@ -88,6 +88,10 @@ EXPORTS = {
                                     c_void_p, c_int, c_void_p]),
     "eogp_srht": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_void_p, c_int, c_void_p, c_int,
                           c_void_p, c_int, c_void_p, c_int, c_void_p]),
+    "eogp_second_moment": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_int, c_int, c_void_p]),
+    "eogp_fit_pca_from_moment_workspace_size": (c_int, [c_int, c_int, POINTER(c_size_t)]),
+    "eogp_fit_pca_from_moment": (c_int, [c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int,
+                                         c_void_p, c_void_p, c_size_t, c_void_p]),
     "eogp_pack_sign": (c_int, [c_void_p, c_int, c_int, c_int, c_void_p, c_int, c_void_p, c_int,
                                c_void_p]),
     "eogp_score_workspace_size": (c_int, [c_int, c_void_p, c_int, c_int, c_int, POINTER(c_size_t)]),
@@ -541,3 +545,31 @@ def measure_peaks() -> Tuple[float, float]:
     pc = c_double()
     _check(lib().eogp_measure_peaks(ctypes.byref(f8), ctypes.byref(pc)))
     return f8.value, pc.value
+
+
+def second_moment(Z, C=None, accumulate: bool = False, stream=None):
+    """eogp_second_moment: C [m, m] fp64 (+)= Z^T Z for Z [n, m] fp32 (device)."""
+    import torch
+    _rows(Z, "Z")
+    n, m = Z.shape
+    if C is None:
+        C = torch.zeros((m, m), dtype=torch.float64, device=Z.device)
+    _rows(C, "C")
+    _check(lib().eogp_second_moment(_ptr(Z), n, m, Z.stride(0), _ptr(C), C.stride(0), 1 if accumulate else 0,
+                                    _stream(stream)))
+    return C
+
+
+def fit_pca_from_moment(C, n_total: int, k: int, pt_dtype: int = F32, stream=None):
+    """eogp_fit_pca_from_moment: (Pt [k, m], eig [k]) for the summed second moment C of n_total rows."""
+    import torch
+    _rows(C, "C")
+    m = C.shape[0]
+    need = c_size_t()
+    _check(lib().eogp_fit_pca_from_moment_workspace_size(m, int(k), ctypes.byref(need)))
+    ws = workspace(need.value, C.device)
+    Pt = torch.empty((k, m), dtype=torch.float32 if pt_dtype == F32 else torch.bfloat16, device=C.device)
+    eig = torch.empty((k,), dtype=torch.float32, device=C.device)
+    _check(lib().eogp_fit_pca_from_moment(_ptr(C), m, C.stride(0), int(n_total), int(k), _ptr(Pt), Pt.stride(0),
+                                          int(pt_dtype), _ptr(eig), _ptr(ws), ws.numel(), _stream(stream)))
+    return Pt, eig

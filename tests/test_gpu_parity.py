@@ -293,6 +293,26 @@ def test_fit_pca(n, m, k):
     subspace_checks(Pt.cpu().numpy(), eig.cpu().numpy(), Z, k)
 
 
+@pytest.mark.parametrize("n,m,k", [(1000, 300, 64), (900, 512, 128)])
+def test_fit_pca_from_summed_moments(n, m, k):
+    """The sharded fit: second moments of three row shards added on the device
+    (accumulate) and the fit from the sum match the oracle like a direct fit."""
+    Z = synth.first_stage_like(n, m, seed=n + 2 * m)
+    Zd = torch.from_numpy(Z).to(DEV)
+    cuts = [0, n // 3, (2 * n) // 3, n]
+    C = None
+    for a, b in zip(cuts[:-1], cuts[1:]):
+        C = E.second_moment(Zd[a:b], C=C, accumulate=C is not None)
+    E.sync_status()
+    want = Z.astype(np.float64).T @ Z.astype(np.float64)
+    np.testing.assert_allclose(C.cpu().numpy(), want, rtol=1e-10, atol=1e-9 * np.abs(want).max())
+    Pt, eig = E.fit_pca_from_moment(C, n, k)
+    E.sync_status()
+    subspace_checks(Pt.cpu().numpy(), eig.cpu().numpy(), Z, k)
+    P_or, mu_or = O.fit_pca_from_moment(want, n, k)
+    np.testing.assert_allclose(eig.cpu().numpy(), mu_or, rtol=1e-3)
+
+
 # ------------------------------------------------------------------- errors
 
 def test_workspace_too_small_is_rejected():

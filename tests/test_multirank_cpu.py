@@ -2,7 +2,9 @@
 
 Each rank scores its contiguous shard of a synthetic store with the oracle;
 the gathered scores must equal the unsharded scores exactly, and the job-level
-timing reduction (max over ranks) must match bench.py's rule."""
+timing reduction (max over ranks) must match bench.py's rule. The sharded PCA
+fit (one all-reduce of the second moment) is run with the oracle's arithmetic
+in place of the device calls and must equal the fit on all rows."""
 import os
 import socket
 
@@ -41,6 +43,13 @@ def _worker(rank, world, port, out_dir):
     lo, hi = shard_range(N, rank, world)
     local = O.score_codes_f32(tc[lo:hi], ts[lo:hi], ks, qc, qs).T   # rows = stored examples
     allrows = all_gather_rows(torch.from_numpy(np.ascontiguousarray(local)), N, world)
+    # sharded PCA fit: each rank's rows, one reduction of the second moment
+    from paper_2609_37842_gb300.shard import fit_pca_sharded
+    Z = np.random.default_rng(9).standard_normal((41, 10)) * np.linspace(2, 0.3, 10)[None, :]
+    zlo, zhi = shard_range(41, rank, world)
+    Pt_sh, mu_sh = fit_pca_sharded(torch.from_numpy(Z[zlo:zhi]), 4,
+                                   moment_fn=lambda z: torch.from_numpy(z.numpy().T @ z.numpy()),
+                                   fit_fn=lambda C, n, k: O.fit_pca_from_moment(C.numpy(), n, k))
     # per-rank step time -> job time = max over ranks (bench.py's rule)
     t = torch.tensor([10.0 + rank])
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -48,6 +57,8 @@ def _worker(rank, world, port, out_dir):
         np.save(os.path.join(out_dir, "sharded.npy"), allrows.numpy().T)
         np.save(os.path.join(out_dir, "full.npy"), O.score_codes_f32(tc, ts, ks, qc, qs))
         np.save(os.path.join(out_dir, "tmax.npy"), t.numpy())
+        np.save(os.path.join(out_dir, "pca_sharded.npy"), Pt_sh)
+        np.save(os.path.join(out_dir, "pca_full.npy"), O.fit_pca(Z, 4, route="cov")[0])
     dist.barrier()
     dist.destroy_process_group()
 
@@ -60,6 +71,8 @@ def test_sharded_scores_equal_unsharded(tmp_path):
     full = np.load(tmp_path / "full.npy")
     np.testing.assert_array_equal(sharded, full)
     assert float(np.load(tmp_path / "tmax.npy")[0]) == 11.0
+    np.testing.assert_allclose(np.load(tmp_path / "pca_sharded.npy"), np.load(tmp_path / "pca_full.npy"),
+                               atol=1e-10)
 
 
 def test_shard_range_covers_exactly():

@@ -445,6 +445,25 @@ def test_bias_channel_and_token_lengths():
     check_plumbing(O, 43)
 
 
+def check_sharded_fit(Om, seed):
+    """Summing the shards' second moments and fitting from the sum equals the
+    fit on all rows (covariance route), with either shard order."""
+    rng = np.random.default_rng(seed)
+    Z = rng.standard_normal((50, 12)) * np.linspace(3, 0.2, 12)[None, :]
+    parts = [Z[:17], Z[17:31], Z[31:]]
+    C = sum(p.T @ p for p in parts)
+    P, mu = Om.fit_pca_from_moment(C, 50, 5)
+    P0, mu0 = Om.fit_pca(Z, 5, route="cov")
+    np.testing.assert_allclose(mu, mu0, rtol=1e-12)
+    np.testing.assert_allclose(P, P0, atol=1e-10)
+    P2, _ = Om.fit_pca_from_moment(sum(p.T @ p for p in parts[::-1]), 50, 5)
+    np.testing.assert_allclose(P2, P0, atol=1e-10)
+
+
+def test_sharded_pca_fit():
+    check_sharded_fit(O, 53)
+
+
 def _golden_rows(name):
     with open(os.path.join(GOLDEN, name)) as f:
         return [ln.split() for ln in f if ln.strip() and not ln.startswith("#")]
@@ -612,3 +631,9 @@ def test_planted_payload_mistake_is_caught(monkeypatch):
         return pay
     monkeypatch.setattr(O, "to_payload", big_endian_half)
     assert _fails(check_payload, O, 47)
+
+
+def test_planted_sharded_fit_mistake_is_caught(monkeypatch):
+    orig = O.fit_pca_from_moment
+    monkeypatch.setattr(O, "fit_pca_from_moment", lambda C, n, k: orig(C, 1, k))   # sum, not mean
+    assert _fails(check_sharded_fit, O, 53)
