@@ -192,6 +192,13 @@ typedef struct {
   const int32_t* lengths;  /* device [B] or NULL: example b keeps tokens
                            t < lengths[b] (0 <= lengths[b] <= T); later positions
                            are padding and contribute nothing (as s_t = 0)        */
+  int bases_on_host;    /* nonzero: VA and VS are host pointers (page-locked for
+                           asynchronous copies); each call copies them into its
+                           workspace with cudaMemcpyAsync on its stream before the
+                           rotations (eigenbases too large to keep resident).
+                           A caller that overlaps these copies with the previous
+                           layer's compute stages them itself and passes device
+                           pointers instead.                                      */
 } eogp_layer_desc;
 
 /* Workspace bytes eogp_compress_layer needs for this descriptor, batch B and

@@ -447,6 +447,7 @@ extern "C" int eogp_plan_gather_rows(const eogp_plan* plan, int which, int dtype
 namespace {
 
 struct Layout {
+  size_t va = 0, vs = 0;  // device copies of host eigenbases (bases_on_host)
   // bf16 path
   int ldA = 0, ldS = 0, ldzb = 0, ldp = 0, splits = 1;
   size_t at_hi = 0, at_lo = 0, st_hi = 0, st_lo = 0, zhi = 0, zlo = 0, part = 0;
@@ -478,6 +479,11 @@ int make_layout(const eogp_layer_desc* L, int B, int mode, Layout* o) {
     off += al256(bytes);
     return at;
   };
+  if (L->bases_on_host) {
+    const size_t esz = L->dtype == EOGP_F32 ? 4 : 2;
+    o->va = take(static_cast<size_t>(P->nC()) * L->d_in * esz);
+    o->vs = take(static_cast<size_t>(P->nR()) * L->d_out * esz);
+  }
   if (L->dtype == EOGP_BF16) {
     o->ldA = round_up(std::max(1, P->nC()), 128);
     o->ldS = round_up(std::max(1, P->nR()), 128);
@@ -532,7 +538,7 @@ int check_desc(const eogp_layer_desc* L, int B, int mode) {
   if (L->dtype == EOGP_BF16) {
     if (L->d_in % 8 || L->d_out % 8 || L->m % 8)
       return set_error(EOGP_EUNSUPPORTED, "bf16 path needs d_in, d_out, m multiples of 8");
-    if (!aligned16(L->VA) || !aligned16(L->VS) || (L->Pt && !aligned16(L->Pt)))
+    if ((!L->bases_on_host && (!aligned16(L->VA) || !aligned16(L->VS))) || (L->Pt && !aligned16(L->Pt)))
       return set_error(EOGP_EINVAL, "bf16 operands must be 16-byte aligned");
     if (static_cast<long long>(B) * L->T > 0x7FFFFFFFLL) return set_error(EOGP_EUNSUPPORTED, "B*T too large");
   }
@@ -579,6 +585,17 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
   if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
   char* w = static_cast<char*>(ws);
   const int M = B * L->T;
+  const void* VA = L->VA;
+  const void* VS = L->VS;
+  if (L->bases_on_host) {
+    const size_t esz = L->dtype == EOGP_F32 ? 4 : 2;
+    CUDA_TRY(cudaMemcpyAsync(w + lo.va, L->VA, static_cast<size_t>(P->nC()) * L->d_in * esz,
+                             cudaMemcpyHostToDevice, st));
+    CUDA_TRY(cudaMemcpyAsync(w + lo.vs, L->VS, static_cast<size_t>(P->nR()) * L->d_out * esz,
+                             cudaMemcpyHostToDevice, st));
+    VA = w + lo.va;
+    VS = w + lo.vs;
+  }
 
   if (L->dtype == EOGP_BF16) {
     if (!aligned16(a) || !aligned16(s)) return set_error(EOGP_EINVAL, "a / s must be 16-byte aligned");
@@ -589,12 +606,12 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
     // Kronecker rotations restricted to the retained columns C / rows R (Sec. 2.2).
     {
       ProfScope ps(EOGP_K_ROTATE, st);
-      CUDA_TRY(launch_tc_rotate(M, L->d_in, a, L->d_in, L->VA, L->d_in, P->nC(), at_hi, at_lo,
+      CUDA_TRY(launch_tc_rotate(M, L->d_in, a, L->d_in, VA, L->d_in, P->nC(), at_hi, at_lo,
                                 lo.ldA, L->T, L->bias_A, nullptr, sm_count(), status, st));
     }
     {
       ProfScope ps(EOGP_K_ROTATE, st);
-      CUDA_TRY(launch_tc_rotate(M, L->d_out, s, L->d_out, L->VS, L->d_out, P->nR(), st_hi, st_lo,
+      CUDA_TRY(launch_tc_rotate(M, L->d_out, s, L->d_out, VS, L->d_out, P->nR(), st_hi, st_lo,
                                 lo.ldS, L->T, nullptr, L->lengths, sm_count(), status, st));
     }
     // Per-example contraction over tokens + scale/gather into z (Eq. first_stage).
@@ -641,9 +658,9 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
   float* at = reinterpret_cast<float*>(w + lo.at);
   float* stt = reinterpret_cast<float*>(w + lo.st);
   const int nC = P->nC(), nR = P->nR();
-  CUDA_TRY(launch_simt_gemm(M, nC, L->d_in, 1.f, af, L->d_in, 1, static_cast<const float*>(L->VA),
+  CUDA_TRY(launch_simt_gemm(M, nC, L->d_in, 1.f, af, L->d_in, 1, static_cast<const float*>(VA),
                             L->d_in, 1, at, nC, st));
-  CUDA_TRY(launch_simt_gemm(M, nR, L->d_out, 1.f, sf, L->d_out, 1, static_cast<const float*>(L->VS),
+  CUDA_TRY(launch_simt_gemm(M, nR, L->d_out, 1.f, sf, L->d_out, 1, static_cast<const float*>(VS),
                             L->d_out, 1, stt, nR, st));
   CUDA_TRY(launch_rows_fixup(at, M, nC, nC, L->T, L->bias_A, nullptr, st));
   CUDA_TRY(launch_rows_fixup(stt, M, nR, nR, L->T, nullptr, L->lengths, st));

@@ -45,7 +45,7 @@ class LayerDesc(ctypes.Structure):
     _fields_ = [("d_in", c_int), ("d_out", c_int), ("T", c_int), ("m", c_int), ("k", c_int),
                 ("dtype", c_int), ("VA", c_void_p), ("VS", c_void_p), ("Pt", c_void_p),
                 ("plan", c_void_p), ("srht_signs", c_void_p), ("srht_rows", c_void_p),
-                ("bias_A", c_void_p), ("lengths", c_void_p)]
+                ("bias_A", c_void_p), ("lengths", c_void_p), ("bases_on_host", c_int)]
 
 
 class EkfacDesc(ctypes.Structure):
@@ -260,15 +260,19 @@ def layer_desc(plan: Plan, T: int, k: int, VA, VS, Pt=None, srht_signs=None,
     given (int32 [k]; srht_signs int8 [m]), the second stage is the SRHT.
     bias_A (fp32 [nC]): the module's bias as a constant-1 input channel (the
     plan is over d_in + 1 inputs; VA [nC, d_in]). lengths (int32 [B]): tokens
-    kept per example for the calls that use this descriptor."""
+    kept per example for the calls that use this descriptor. VA and VS may be
+    host tensors (pinned): each call then copies them to its workspace."""
     inf = plan.info()
     _dense(VA, "VA")
     _dense(VS, "VS")
     _dense(Pt, "Pt")
     d_in = inf.d_in - (1 if bias_A is not None else 0)
+    on_host = not VA.is_cuda
+    if on_host != (not VS.is_cuda):
+        raise ValueError("VA and VS must both be on the device or both in host memory")
     d = LayerDesc(d_in, inf.d_out, int(T), inf.m, int(k), _dtype_code(VA), _ptr(VA),
                   _ptr(VS), _ptr(Pt), plan.handle, _ptr(srht_signs), _ptr(srht_rows),
-                  _ptr(bias_A), _ptr(lengths))
+                  _ptr(bias_A), _ptr(lengths), 1 if on_host else 0)
     d._refs = (plan, VA, VS, Pt, srht_signs, srht_rows, bias_A, lengths)
     return d
 

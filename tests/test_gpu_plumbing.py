@@ -118,3 +118,27 @@ def test_store_records(N, ks, tmp_path):
         sc = E.score(c2, s2, ks, E.SCORE_CODES, c2[:q], s2[:q])
         E.sync_status()
         np.testing.assert_array_equal(sc.cpu().numpy(), O.score_codes_f32(wc, ws, ks, wc[:q], ws[:q]))
+
+
+def test_host_resident_eigenbases_give_identical_codes():
+    """Eigenvector rows in page-locked host memory (copied by each call) give the
+    same results, bit for bit, as device-resident ones."""
+    rng = np.random.default_rng(13)
+    d_in, d_out, T, B, m, k = 768, 768, 64, 3, 4096, 1024
+    QA = synth.round_to(synth.haar_orthogonal(d_in, rng), "bf16")
+    QS = synth.round_to(synth.haar_orthogonal(d_out, rng), "bf16")
+    plan = E.Plan.from_factors(synth.power_spectrum(d_out, 1.2), synth.power_spectrum(d_in, 1.2), m, 0.1)
+    R, C = plan.sets()
+    VA = torch.from_numpy(np.ascontiguousarray(QA.T[C], dtype=np.float32)).to(torch.bfloat16)
+    VS = torch.from_numpy(np.ascontiguousarray(QS.T[R], dtype=np.float32)).to(torch.bfloat16)
+    Pt = dev(synth.round_to(synth.haar_orthogonal(m, rng, k).T, "bf16").astype(np.float32), torch.bfloat16)
+    a = dev(synth.round_to(rng.standard_normal((B, T, d_in)), "bf16").astype(np.float32), torch.bfloat16)
+    s = dev(synth.round_to(rng.standard_normal((B, T, d_out)) * 0.1, "bf16").astype(np.float32), torch.bfloat16)
+    d_dev = E.layer_desc(plan, T, k, VA.to(DEV), VS.to(DEV), Pt)
+    d_host = E.layer_desc(plan, T, k, VA.pin_memory(), VS.pin_memory(), Pt)
+    c1, s1 = E.compress_layer(d_dev, a, s, E.OUT_CODES)
+    c2, s2 = E.compress_layer(d_host, a, s, E.OUT_CODES)
+    x1 = E.compress_layer(d_dev, a, s, E.OUT_COORDS)
+    x2 = E.compress_layer(d_host, a, s, E.OUT_COORDS)
+    E.sync_status()
+    assert torch.equal(c1, c2) and torch.equal(s1, s2) and torch.equal(x1, x2)
