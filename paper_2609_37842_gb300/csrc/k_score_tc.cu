@@ -25,18 +25,20 @@
 // the next query tile; a separate kernel merges the per-CTA lists. The Q x N
 // matrix never reaches HBM.
 //
-// Tiles: 128 stored rows (MMA M, operand A) x BNq <= 128 queries (MMA N,
-// operand B). Queries are prepared once per call in the workspace (e4m3 bytes,
-// or bf16 hi and lo rows) and fetched by TMA; stored rows are expanded from
-// their bits into shared memory (128-byte swizzled rows) by four warps, so the
-// store is read from HBM as bits. Tiles run query-tile-major: one query tile
-// stays in L2 while the stored codes stream past it.
+// Tiles: 128 stored rows (MMA M, operand A) x BNq queries (MMA N, operand B),
+// BNq <= 256 for CODES with one module, else <= 128. Queries are prepared once
+// per call in the workspace (e4m3 bytes, or bf16 hi and lo rows) and fetched
+// by TMA; stored rows are expanded from their bits into shared memory
+// (128-byte swizzled rows) by eight warps, so the store is read from HBM as
+// bits. Dense output runs tiles query-tile-major: one query tile stays in L2
+// while the stored codes stream past it.
 //
-// Warps: 0-3 expand stored rows (warp 0 lane 0 also issues the query TMA),
-// 4-7 dequantise (TMEM lane quarters 0-3; in TOPK, thread t also owns query
-// column t), 8 owns TMEM and issues the MMAs. TMEM: two 128-column d_u
-// buffers (module u+1 accumulates while module u is dequantised) and a
-// 128-column running score.
+// Warps: 0-7 expand stored rows, two threads per row (warp 0 lane 0 also
+// issues the query TMA), 8-11 dequantise (TMEM lane quarters 0-3; in TOPK
+// the four warps share the ranking), 12 owns TMEM and issues the MMAs. TMEM:
+// with 128 queries per tile, three 128-column d_u buffers (modules u+1 and
+// u+2 accumulate while module u is dequantised) and a 128-column running
+// score; with 256, two 256-column buffers and no running score.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -96,9 +98,27 @@ constexpr uint32_t tc_stage_bytes() {
   return kAB + static_cast<uint32_t>(BN) * 128u * TcMode<MODE>::kQBoxes;
 }
 
+// Pipeline stages: six when a stage is 32 KB (one-bit queries, 128 per tile),
+// else four (48 KB stages).
 template <int MODE, bool TOPK, int BN>
 constexpr int tc_stages() {
-  return 4;
+  return (MODE == EOGP_SCORE_CODES && BN == 128) ? 6 : 4;
+}
+
+
+// Stages the expanders fill per synchronisation round (one wait, proxy fence
+// and arrive round): two with six stages, so that the MMAs always have at
+// least four stages to work on, else one.
+template <int MODE, bool TOPK, int BN>
+constexpr int tc_group() {
+  return tc_stages<MODE, TOPK, BN>() >= 6 ? 2 : 1;
+}
+
+// Accumulator buffers d_u in TMEM (BN columns each): three of 128 columns plus
+// the 128-column running score, or two of 256 (one module, no running score).
+template <int BN>
+constexpr int tc_dbufs() {
+  return BN == 128 ? 3 : 2;
 }
 
 // Shared-memory carve-up (byte offsets after 1024-byte alignment).
@@ -110,8 +130,8 @@ __host__ __device__ inline TcSmem tc_smem_layout(int BNq, int K) {
   constexpr int S = tc_stages<MODE, TOPK, BN>();
   TcSmem l;
   l.sq = S * tc_stage_bytes<MODE, BN>();
-  l.bars = l.sq + BN * 4;
-  l.lists = l.bars + (2 * S + 4) * 8 + 16;
+  l.bars = l.sq + 2 * BN * 4;  // query scales, double-buffered by module
+  l.lists = l.bars + (2 * S + 2 * tc_dbufs<BN>()) * 8 + 16;
   // per-column held count, own threshold and shared threshold (the list buffers
   // themselves are in global memory)
   l.total = l.lists + (TOPK ? BN * 12 + 8 * 4 * 4 : 0);
@@ -184,19 +204,22 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   constexpr int S = tc_stages<MODE, TOPK, BN>();
   constexpr uint32_t kStage = tc_stage_bytes<MODE, BN>();
   constexpr int kBits = TcMode<MODE>::kBits;
-  constexpr int kG = 8;  // stages of code bits prefetched at a time
-  constexpr uint32_t kAcc = 2u * BN;  // running-score columns (BN == 128 only)
+  constexpr int ND = tc_dbufs<BN>();
+  constexpr uint32_t kAcc = static_cast<uint32_t>(ND * BN);  // running-score columns (BN == 128 only)
   using HalfBits = typename TcMode<MODE>::HalfBits;
+  constexpr int kG = 8;  // stages of code bits prefetched at a time
+  constexpr int kP = tc_group<MODE, TOPK, BN>();
+  static_assert(kG % kP == 0, "prefetch groups hold whole expansion rounds");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const TcSmem L = tc_smem_layout<MODE, TOPK, BN>(g.BNq, g.K);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  float* sq = reinterpret_cast<float*>(smem + L.sq);  // [BN] query scales of module u (CODES)
+  float* sq = reinterpret_cast<float*>(smem + L.sq);  // [2][BN] query scales of module u (CODES)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bars);
   uint64_t* empty = full + S;
   uint64_t* dfull = empty + S;
-  uint64_t* dempty = dfull + 2;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(dempty + 2);
+  uint64_t* dempty = dfull + ND;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(dempty + ND);
 
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tmQ);
@@ -205,7 +228,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       mbar_init(&full[s], 1 + kExpWarps);  // TMA transaction arrive + the expander warps
       mbar_init(&empty[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < ND; ++b) {
       mbar_init(&dfull[b], 1);
       mbar_init(&dempty[b], 4);
     }
@@ -223,7 +246,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
     // reads bits [j kBits, (j+1) kBits) of the row and query columns from
     // j kBits on. Two threads share a row (a half stage each). The bits of the
     // next kG stages are loaded into registers while the current kG stages are
-    // expanded, hiding the HBM latency.
+    // expanded, hiding the HBM latency. With six stages (one-bit queries, 128
+    // per tile) two stages are filled per wait, proxy fence and arrive round.
     const int r = threadIdx.x & 127, half = threadIdx.x >> 7;  // stored row, half of its stage
     const uint32_t row_off = static_cast<uint32_t>((r >> 3) * 1024 + (r & 7) * 128);
     const int nst = g.D / kBits;
@@ -243,30 +267,73 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
 #pragma unroll
         for (int jj = 0; jj < kG; ++jj)
           nxt[jj] = (rv && j0 + kG + jj < nst) ? __ldg(brow + 2 * (j0 + kG + jj)) : HalfBits{};
+        if constexpr (kP == 1) {
 #pragma unroll
-        for (int jj = 0; jj < kG; ++jj) {
-          const int j = j0 + jj;
-          if (j < nst && ok) {
-            const int s = static_cast<int>(it % S);
-            const uint32_t ph = (it / S) & 1u;
-            ++it;
-            uint32_t w_ok = 1;
-            if (lane == 0) w_ok = mbar_wait(&empty[s], ph ^ 1u, g.status) ? 1u : 0u;
-            w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
-            if (!w_ok) {
-              ok = false;
-            } else {
-              uint8_t* st = smem + static_cast<size_t>(s) * kStage;
-              if (warp == 0 && lane == 0) {
-                mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(g.BNq) * 128u * TcMode<MODE>::kQBoxes);
-                tma_load_2d(st + kAB, &tmQ, j * kBits, q0, &full[s]);
-                if (MODE == EOGP_SCORE_PAPER)
-                  tma_load_2d(st + kAB + static_cast<uint32_t>(BN) * 128u, &tmQlo, j * kBits, q0, &full[s]);
+          for (int jj = 0; jj < kG; ++jj) {
+            const int j = j0 + jj;
+            if (j < nst && ok) {
+              const int s = static_cast<int>(it % S);
+              const uint32_t ph = (it / S) & 1u;
+              ++it;
+              uint32_t w_ok = 1;
+              if (lane == 0) w_ok = mbar_wait(&empty[s], ph ^ 1u, g.status) ? 1u : 0u;
+              w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
+              if (!w_ok) {
+                ok = false;
+              } else {
+                uint8_t* st = smem + static_cast<size_t>(s) * kStage;
+                if (warp == 0 && lane == 0) {
+                  mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(g.BNq) * 128u * TcMode<MODE>::kQBoxes);
+                  tma_load_2d(st + kAB, &tmQ, j * kBits, q0, &full[s]);
+                  if (MODE == EOGP_SCORE_PAPER)
+                    tma_load_2d(st + kAB + static_cast<uint32_t>(BN) * 128u, &tmQlo, j * kBits, q0, &full[s]);
+                }
+                expand_half(st + row_off, r & 7, half, cur[jj]);
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&full[s]);
               }
-              expand_half(st + row_off, r & 7, half, cur[jj]);
-              fence_proxy_async_smem();
-              __syncwarp();
-              if (lane == 0) mbar_arrive(&full[s]);
+            }
+          }
+        } else {
+          static_assert(MODE == EOGP_SCORE_CODES, "two-stage rounds load one query operand per stage");
+#pragma unroll
+          for (int jj = 0; jj < kG; jj += 2) {
+            const int j = j0 + jj;
+            if (j < nst && ok) {
+              const bool two = j + 1 < nst;
+              const int s0 = static_cast<int>(it % S), s1 = static_cast<int>((it + 1) % S);
+              const uint32_t ph0 = (it / S) & 1u, ph1 = ((it + 1) / S) & 1u;
+              it += two ? 2 : 1;
+              uint32_t w_ok = 1;
+              if (lane == 0) {
+                w_ok = mbar_wait(&empty[s0], ph0 ^ 1u, g.status) ? 1u : 0u;
+                if (w_ok && two) w_ok = mbar_wait(&empty[s1], ph1 ^ 1u, g.status) ? 1u : 0u;
+              }
+              w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
+              if (!w_ok) {
+                ok = false;
+              } else {
+                uint8_t* st0 = smem + static_cast<size_t>(s0) * kStage;
+                uint8_t* st1 = smem + static_cast<size_t>(s1) * kStage;
+                if (warp == 0 && lane == 0) {
+                  const uint32_t qbytes = static_cast<uint32_t>(g.BNq) * 128u * TcMode<MODE>::kQBoxes;
+                  mbar_arrive_expect_tx(&full[s0], qbytes);
+                  tma_load_2d(st0 + kAB, &tmQ, j * kBits, q0, &full[s0]);
+                  if (two) {
+                    mbar_arrive_expect_tx(&full[s1], qbytes);
+                    tma_load_2d(st1 + kAB, &tmQ, (j + 1) * kBits, q0, &full[s1]);
+                  }
+                }
+                expand_half(st0 + row_off, r & 7, half, cur[jj]);
+                if (two) expand_half(st1 + row_off, r & 7, half, cur[jj + 1]);
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                  mbar_arrive(&full[s0]);
+                  if (two) mbar_arrive(&full[s1]);
+                }
+              }
             }
           }
         }
@@ -377,52 +444,107 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
         for (int col = ep; col < BN; col += 128)
           gtb[col] = q0 + col < g.Q ? topk_unkey32(__ldcg(g.gtau + q0 + col)) : INFINITY;
       }
+      // Scales of module u + 1 are loaded while module u is dequantised. The
+      // query scales go through shared memory (buffer gm & 1): buffer gm & 1 was
+      // last read in module gm - 2, which every thread finished before the
+      // barrier of module gm - 1.
+      constexpr int kSqPer = BN / 128;
+      float si_next = row < g.N ? g.ts[static_cast<size_t>(row) * g.ldts] : 0.f;
+      float sq_next[kSqPer];
+#pragma unroll
+      for (int e = 0; e < kSqPer; ++e) {
+        const int c = ep + 128 * e;
+        sq_next[e] = (MODE == EOGP_SCORE_CODES && c < g.BNq && q0 + c < g.Q)
+                         ? g.qs[static_cast<size_t>(q0 + c) * g.ldqs] : 0.f;
+      }
       for (int u = 0; u < g.U; ++u, ++gm) {
-        const int buf = static_cast<int>(gm & 1u);
-        const uint32_t dph = (gm >> 1) & 1u;
+        const int buf = static_cast<int>(gm % ND);
+        const uint32_t dph = (gm / ND) & 1u;
+        const float si = si_next;
+        float* sqb = sq + (gm & 1u) * BN;
         if (MODE == EOGP_SCORE_CODES) {
-          named_bar_sync(1, 128);  // previous module's readers of sq are done
-          for (int c = ep; c < g.BNq; c += 128)
-            sq[c] = q0 + c < g.Q ? g.qs[static_cast<size_t>(q0 + c) * g.ldqs + u] : 0.f;
-          named_bar_sync(1, 128);
+#pragma unroll
+          for (int e = 0; e < kSqPer; ++e) sqb[ep + 128 * e] = sq_next[e];
+        }
+        if (u + 1 < g.U) {
+          si_next = row < g.N ? g.ts[static_cast<size_t>(row) * g.ldts + u + 1] : 0.f;
+#pragma unroll
+          for (int e = 0; e < kSqPer; ++e) {
+            const int c = ep + 128 * e;
+            sq_next[e] = (MODE == EOGP_SCORE_CODES && c < g.BNq && q0 + c < g.Q)
+                             ? g.qs[static_cast<size_t>(q0 + c) * g.ldqs + u + 1] : 0.f;
+          }
         }
         uint32_t w_ok = 1;
         if (lane == 0) w_ok = mbar_wait(&dfull[buf], dph, g.status) ? 1u : 0u;
         w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
         __syncwarp();
         tc_fence_after();
-        if (!__syncthreads_and_named(w_ok)) {
+        if (!__syncthreads_and_named(w_ok)) {  // also publishes sqb
           ok = false;
           break;
         }
-        const float si = row < g.N ? g.ts[static_cast<size_t>(row) * g.ldts + u] : 0.f;
         const bool last = u + 1 == g.U;
-        for (int c0 = 0; c0 < g.BNq; c0 += 32) {
-          float d[32], a[32];
-          tmem_ld32(tmem + lane_base + buf * static_cast<uint32_t>(BN) + c0, d);
-          if (u == 0) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) a[j] = 0.f;
+        const uint32_t dcol = tmem + lane_base + buf * static_cast<uint32_t>(BN);
+        const uint32_t acol = tmem + lane_base + kAcc;
+        // the module's term: fl(fl(s_q s_i) d) (CODES) or fl(s_i d) (PAPER)
+        auto term = [&](int c, uint32_t dv) {
+          return MODE == EOGP_SCORE_CODES ? __fmul_rn(__fmul_rn(sqb[c], si), __uint_as_float(dv))
+                                          : __fmul_rn(si, __uint_as_float(dv));
+        };
+        if (!last) {
+          // Running score, 16 columns at a time: the TMEM loads of the next chunk
+          // are in flight while this one is combined and stored back.
+          uint32_t dr[16], ar[16];
+          tmem_ld16_issue(dcol, dr);
+          if (u > 0) {
+            tmem_ld16_issue(acol, ar);
           } else {
-            tmem_ld32(tmem + lane_base + kAcc + c0, a);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) ar[j] = 0u;
           }
-          if (MODE == EOGP_SCORE_CODES) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) a[j] = __fadd_rn(a[j], __fmul_rn(__fmul_rn(sq[c0 + j], si), d[j]));
-          } else {
+          for (int ci = 0; ci < BN / 16; ++ci) {
+            const int c0 = 16 * ci;
+            if (c0 < g.BNq) {
+              tmem_wait_ld(dr);
+              tmem_wait_ld(ar);
+              uint32_t o[16];
 #pragma unroll
-            for (int j = 0; j < 32; ++j) a[j] = __fadd_rn(a[j], __fmul_rn(si, d[j]));
-          }
-          if (!last) {
-            tmem_st32(tmem + lane_base + kAcc + c0, a);
-          } else if (!TOPK) {
-            if (row < g.N) {
-#pragma unroll
-              for (int j = 0; j < 32; ++j)
-                if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
+              for (int j = 0; j < 16; ++j)
+                o[j] = __float_as_uint(__fadd_rn(__uint_as_float(ar[j]), term(c0 + j, dr[j])));
+              if (c0 + 16 < g.BNq) {
+                tmem_ld16_issue(dcol + c0 + 16, dr);
+                if (u > 0) tmem_ld16_issue(acol + c0 + 16, ar);
+              }
+              tmem_st16_issue(acol + c0, o);
             }
-          } else {
-            screen_chunk(c0, q0, row, a);
+          }
+          tmem_wait_st();  // stored before the next module reads them
+        } else {
+          for (int c0 = 0; c0 < g.BNq; c0 += 32) {
+            uint32_t dr[32], ar[32];
+            tmem_ld32_issue(dcol + c0, dr);
+            if (u > 0) {
+              tmem_ld32_issue(acol + c0, ar);
+            } else {
+#pragma unroll
+              for (int j = 0; j < 32; ++j) ar[j] = 0u;
+            }
+            tmem_wait_ld(dr);
+            tmem_wait_ld(ar);
+            float a[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) a[j] = __fadd_rn(__uint_as_float(ar[j]), term(c0 + j, dr[j]));
+            if (!TOPK) {
+              if (row < g.N) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                  if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
+              }
+            } else {
+              screen_chunk(c0, q0, row, a);
+            }
           }
         }
         tc_fence_before();
@@ -442,8 +564,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       for (int tile = tile_begin<TOPK>(g), tstep = tile_step<TOPK>(), tend = tile_end<TOPK>(g);
            tile < tend && ok; tile += tstep) {
         for (int u = 0; u < g.U && ok; ++u, ++gm) {
-          const int buf = static_cast<int>(gm & 1u);
-          const uint32_t dph = (gm >> 1) & 1u;
+          const int buf = static_cast<int>(gm % ND);
+          const uint32_t dph = (gm / ND) & 1u;
           if (!mbar_wait(&dempty[buf], dph ^ 1u, g.status)) {
             ok = false;
             break;
