@@ -228,6 +228,41 @@ int eogp_compress_layer(const eogp_layer_desc* L, const void* a, const void* s, 
                         float* scales, int ld_scales, void* ws, size_t ws_bytes,
                         eogp_stream_t stream);
 
+/* Page-locked host memory for inputs that eogp_compress_layer_host (or the
+ * caller) copies to the device: an anonymous mapping aligned to and advised for
+ * transparent huge pages, registered with cudaHostRegister. Measured on GB300
+ * systems, host-to-device copies from it ran at the link rate (~211 GB/s) in
+ * every trial, where cudaHostAlloc'd buffers varied from ~80 to ~210 GB/s
+ * between allocations. The size is rounded up to whole huge pages; the memory
+ * is zero-filled. eogp_host_free takes only the pointer (NULL is a no-op).
+ * A library convenience with no counterpart in the paper.
+ * Errors: EOGP_EINVAL (bytes == 0, ptr NULL, mapping failed, pointer not from
+ * eogp_host_alloc), EOGP_ECUDA (registration failed, e.g. no device). */
+int eogp_host_alloc(size_t bytes, void** ptr);
+int eogp_host_free(void* ptr);
+
+/* Same computation and outputs as eogp_compress_layer, with the inputs a and s
+ * in host memory (page-locked, so that the copies run asynchronously): the
+ * batch is compressed `chunk` examples at a time (0: about 64 MB of a and s
+ * per chunk). Each chunk is copied into the workspace with cudaMemcpyAsync on
+ * a copy stream the call creates, double-buffered, so the copy of chunk c + 1
+ * overlaps the compute of chunk c on `stream`; the compute of every chunk is
+ * queued on `stream`, which therefore orders all of the call's work, and the
+ * call releases its copy stream and events itself. `descriptor->lengths` (if
+ * any) is a device array of all B examples. With bases_on_host the eigenbases
+ * are copied once per call, not per chunk. a and s must stay valid and
+ * unchanged until `stream` reaches the point of the call. A library
+ * convenience for inputs that live in host memory: the paper times store
+ * construction including its host-to-device transfers (App. E.3) but gives no
+ * interface for it.
+ * Errors: as eogp_compress_layer; EOGP_EINVAL for chunk < 0. */
+int eogp_compress_host_workspace_size(const eogp_layer_desc* L, int B, int chunk, int out_mode,
+                                      size_t* bytes);
+int eogp_compress_layer_host(const eogp_layer_desc* L, const void* a, const void* s, int B, int chunk,
+                             int out_mode, float* out, int ld_out, uint32_t* codes, int ld_codes,
+                             float* scales, int ld_scales, void* ws, size_t ws_bytes,
+                             eogp_stream_t stream);
+
 /* Same computation and outputs as eogp_compress_layer, for callers that cannot
  * allocate device memory (a plugin whose host framework owns every device
  * allocation, a service confined to a memory budget fixed at start-up, a C

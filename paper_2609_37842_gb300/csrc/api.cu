@@ -686,6 +686,150 @@ extern "C" int eogp_compress_layer(const eogp_layer_desc* L, const void* a, cons
   return EOGP_OK;
 }
 
+// ================================================================ host-resident inputs
+
+namespace {
+
+// Examples per chunk when the caller passes 0: about 64 MB of a and s.
+int host_chunk(const eogp_layer_desc* L, int B, int chunk) {
+  if (chunk > 0) return std::min(chunk, std::max(B, 1));
+  const size_t esz = L->dtype == EOGP_F32 ? 4 : 2;
+  const size_t per = static_cast<size_t>(L->T) * (L->d_in + L->d_out) * esz;
+  const size_t c = std::max<size_t>(1, (size_t(64) << 20) / std::max<size_t>(per, 1));
+  return static_cast<int>(std::min<size_t>(c, std::max(B, 1)));
+}
+
+struct HostLayout {
+  int chunk = 1;
+  size_t a_bytes = 0, s_bytes = 0;  // one chunk's a and s
+  size_t stage[2] = {0, 0};         // double-buffered staging of a chunk's a then s
+  size_t va = 0, vs = 0;            // device copies of host eigenbases
+  size_t comp = 0, comp_bytes = 0;  // eogp_compress_layer workspace for one chunk
+  size_t total = 0;
+};
+
+HostLayout host_layout(const eogp_layer_desc* L, int B, int chunk, int mode) {
+  HostLayout h;
+  h.chunk = host_chunk(L, B, chunk);
+  const size_t esz = L->dtype == EOGP_F32 ? 4 : 2;
+  h.a_bytes = static_cast<size_t>(h.chunk) * L->T * L->d_in * esz;
+  h.s_bytes = static_cast<size_t>(h.chunk) * L->T * L->d_out * esz;
+  size_t off = 0;
+  for (int i = 0; i < 2; ++i) {
+    h.stage[i] = off;
+    off += al256(h.a_bytes) + al256(h.s_bytes);
+  }
+  if (L->bases_on_host) {
+    h.va = off;
+    off += al256(static_cast<size_t>(L->plan->nC()) * L->d_in * esz);
+    h.vs = off;
+    off += al256(static_cast<size_t>(L->plan->nR()) * L->d_out * esz);
+  }
+  eogp_layer_desc d = *L;
+  d.bases_on_host = 0;  // the chunks read the device copies
+  Layout lo;
+  make_layout(&d, h.chunk, mode, &lo);
+  h.comp = off;
+  h.comp_bytes = lo.total;
+  h.total = off + lo.total;
+  return h;
+}
+
+// Stream and events of one host-input call, released when it returns (the
+// runtime frees them once the work queued on them has completed).
+struct HostCallRes {
+  cudaStream_t cs = nullptr;
+  cudaEvent_t entry = nullptr, landed[2] = {nullptr, nullptr}, done[2] = {nullptr, nullptr};
+  ~HostCallRes() {
+    for (cudaEvent_t e : {entry, landed[0], landed[1], done[0], done[1]})
+      if (e) cudaEventDestroy(e);
+    if (cs) cudaStreamDestroy(cs);
+  }
+};
+
+}  // namespace
+
+extern "C" int eogp_compress_host_workspace_size(const eogp_layer_desc* L, int B, int chunk,
+                                                 int out_mode, size_t* bytes) {
+  clear_error();
+  if (!bytes) return set_error(EOGP_EINVAL, "bytes is NULL");
+  if (chunk < 0) return set_error(EOGP_EINVAL, "chunk must be >= 0");
+  if (int rc = check_desc(L, B, out_mode)) return rc;
+  *bytes = host_layout(L, B, chunk, out_mode).total;
+  return EOGP_OK;
+}
+
+extern "C" int eogp_compress_layer_host(const eogp_layer_desc* L, const void* a, const void* s, int B,
+                                        int chunk, int out_mode, float* out, int ld_out, uint32_t* codes,
+                                        int ld_codes, float* scales, int ld_scales, void* ws,
+                                        size_t ws_bytes, eogp_stream_t stream) {
+  clear_error();
+  if (chunk < 0) return set_error(EOGP_EINVAL, "chunk must be >= 0");
+  if (int rc = check_desc(L, B, out_mode)) return rc;
+  if (B == 0) return EOGP_OK;
+  if (!a || !s) return set_error(EOGP_EINVAL, "a / s is NULL");
+  if (out_mode == EOGP_OUT_CODES) {
+    if (!codes || !scales) return set_error(EOGP_EINVAL, "codes / scales is NULL");
+  } else if (!out) {
+    return set_error(EOGP_EINVAL, "out is NULL");
+  }
+  const HostLayout h = host_layout(L, B, chunk, out_mode);
+  if (!ws || ws_bytes < h.total)
+    return set_error(EOGP_EWORKSPACE, "workspace of %zu bytes needed, %zu given", h.total, ws_bytes);
+  if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
+  if (int rc = check_device(L->plan)) return rc;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  const size_t esz = L->dtype == EOGP_F32 ? 4 : 2;
+  const size_t a_row = static_cast<size_t>(L->T) * L->d_in * esz;   // bytes of one example's a
+  const size_t s_row = static_cast<size_t>(L->T) * L->d_out * esz;
+  HostCallRes r;
+  CUDA_TRY(cudaStreamCreateWithFlags(&r.cs, cudaStreamNonBlocking));
+  CUDA_TRY(cudaEventCreateWithFlags(&r.entry, cudaEventDisableTiming));
+  for (int i = 0; i < 2; ++i) {
+    CUDA_TRY(cudaEventCreateWithFlags(&r.landed[i], cudaEventDisableTiming));
+    CUDA_TRY(cudaEventCreateWithFlags(&r.done[i], cudaEventDisableTiming));
+  }
+  // Work already queued on `stream` (an earlier call) may still read the staging
+  // buffers: the first copies wait for it.
+  CUDA_TRY(cudaEventRecord(r.entry, st));
+  CUDA_TRY(cudaStreamWaitEvent(r.cs, r.entry, 0));
+  eogp_layer_desc d = *L;
+  if (L->bases_on_host) {
+    CUDA_TRY(cudaMemcpyAsync(w + h.va, L->VA, static_cast<size_t>(L->plan->nC()) * L->d_in * esz,
+                             cudaMemcpyDefault, r.cs));
+    CUDA_TRY(cudaMemcpyAsync(w + h.vs, L->VS, static_cast<size_t>(L->plan->nR()) * L->d_out * esz,
+                             cudaMemcpyDefault, r.cs));
+    d.VA = w + h.va;
+    d.VS = w + h.vs;
+    d.bases_on_host = 0;
+  }
+  const int n_chunks = (B + h.chunk - 1) / h.chunk;
+  for (int c = 0; c < n_chunks; ++c) {
+    const int b0 = c * h.chunk, nb = std::min(h.chunk, B - b0), buf = c & 1;
+    char* sa = w + h.stage[buf];
+    char* ss = sa + al256(h.a_bytes);
+    // Copy stream: the staging buffer is free once chunk c - 2 has been computed.
+    if (c >= 2) CUDA_TRY(cudaStreamWaitEvent(r.cs, r.done[buf], 0));
+    CUDA_TRY(cudaMemcpyAsync(sa, static_cast<const char*>(a) + b0 * a_row, nb * a_row,
+                             cudaMemcpyDefault, r.cs));
+    CUDA_TRY(cudaMemcpyAsync(ss, static_cast<const char*>(s) + b0 * s_row, nb * s_row,
+                             cudaMemcpyDefault, r.cs));
+    CUDA_TRY(cudaEventRecord(r.landed[buf], r.cs));
+    // Compute stream: chunk c once its inputs have landed.
+    CUDA_TRY(cudaStreamWaitEvent(st, r.landed[buf], 0));
+    d.lengths = L->lengths ? L->lengths + b0 : nullptr;
+    const bool cd = out_mode == EOGP_OUT_CODES;
+    if (int rc = eogp_compress_layer(&d, sa, ss, nb, out_mode, cd ? nullptr : out + static_cast<size_t>(b0) * ld_out,
+                                     ld_out, cd ? codes + static_cast<size_t>(b0) * ld_codes : nullptr, ld_codes,
+                                     cd ? scales + static_cast<size_t>(b0) * ld_scales : nullptr, ld_scales,
+                                     w + h.comp, h.comp_bytes, stream))
+      return rc;
+    CUDA_TRY(cudaEventRecord(r.done[buf], st));
+  }
+  return EOGP_OK;
+}
+
 // ================================================================ EK-FAC correction
 
 namespace {

@@ -75,6 +75,13 @@ EXPORTS = {
     "eogp_compress_layer_static": (c_int, [POINTER(LayerDesc), c_void_p, c_void_p, c_int, c_int,
                                            c_void_p, c_int, c_void_p, c_int, c_void_p, c_int,
                                            c_void_p]),
+    "eogp_host_alloc": (c_int, [c_size_t, POINTER(c_void_p)]),
+    "eogp_host_free": (c_int, [c_void_p]),
+    "eogp_compress_host_workspace_size": (c_int, [POINTER(LayerDesc), c_int, c_int, c_int,
+                                                  POINTER(c_size_t)]),
+    "eogp_compress_layer_host": (c_int, [POINTER(LayerDesc), c_void_p, c_void_p, c_int, c_int, c_int,
+                                         c_void_p, c_int, c_void_p, c_int, c_void_p, c_int, c_void_p,
+                                         c_size_t, c_void_p]),
     "eogp_ekfac_workspace_size": (c_int, [POINTER(EkfacDesc), c_int, POINTER(c_size_t)]),
     "eogp_ekfac_accumulate": (c_int, [POINTER(EkfacDesc), c_void_p, c_void_p, c_int, c_void_p, c_int,
                                       c_int, c_void_p, c_size_t, c_void_p]),
@@ -319,6 +326,67 @@ def compress_layer(desc: LayerDesc, a, s, out_mode: int, out=None, codes=None, s
     _check(lib().eogp_compress_layer(ctypes.byref(desc), _ptr(a), _ptr(s), B, out_mode, _ptr(out),
                                      out.stride(0), None, 0, None, 0, _ptr(ws), ws.numel(),
                                      _stream(stream)))
+    return out
+
+
+def host_empty(shape, dtype):
+    """A CPU tensor of `shape` / `dtype` in eogp_host_alloc memory (page-locked,
+    huge-page backed, zero-filled); the memory is released with the tensor."""
+    import numpy as np
+    import torch
+    import weakref
+    nel = 1
+    for d in shape:
+        nel *= int(d)
+    esz = torch.empty((), dtype=dtype).element_size()
+    nbytes = max(1, nel * esz)
+    p = c_void_p()
+    _check(lib().eogp_host_alloc(nbytes, ctypes.byref(p)))
+    buf = (ctypes.c_uint8 * nbytes).from_address(p.value)
+    t = torch.from_numpy(np.frombuffer(buf, dtype=np.uint8)[:nel * esz]).view(dtype).view(*shape)
+    weakref.finalize(buf, lib().eogp_host_free, p.value)
+    t._eogp_host_buf = buf   # the finalizer runs once no tensor view holds the buffer
+    return t
+
+
+def compress_host_workspace_size(desc: LayerDesc, B: int, out_mode: int, chunk: int = 0) -> int:
+    n = c_size_t()
+    _check(lib().eogp_compress_host_workspace_size(ctypes.byref(desc), int(B), int(chunk),
+                                                   int(out_mode), ctypes.byref(n)))
+    return n.value
+
+
+def compress_layer_host(desc: LayerDesc, a, s, out_mode: int, device, chunk: int = 0, out=None,
+                        codes=None, scales=None, ws=None, stream=None):
+    """eogp_compress_layer_host: a [B, T, d_in], s [B, T, d_out] in (page-locked)
+    host memory, copied chunk by chunk by the call itself; outputs on `device`
+    as for compress_layer."""
+    import torch
+    _dense(a, "a")
+    _dense(s, "s")
+    _rows(out, "out")
+    _rows(codes, "codes")
+    if a.is_cuda or s.is_cuda:
+        raise ValueError("compress_layer_host takes host tensors (use compress_layer for device ones)")
+    B = a.shape[0]
+    if ws is None:
+        ws = workspace(compress_host_workspace_size(desc, B, out_mode, chunk), device)
+    if out_mode == OUT_CODES:
+        if codes is None:
+            codes = torch.empty((B, (desc.k + 31) // 32), dtype=torch.int32, device=device)
+        if scales is None:
+            scales = torch.empty((B,), dtype=torch.float32, device=device)
+        _check(lib().eogp_compress_layer_host(ctypes.byref(desc), _ptr(a), _ptr(s), B, int(chunk),
+                                              out_mode, None, 0, _ptr(codes), codes.stride(0),
+                                              _ptr(scales), scales.stride(0), _ptr(ws), ws.numel(),
+                                              _stream(stream)))
+        return codes, scales
+    width = desc.m if out_mode == OUT_FIRST_STAGE else desc.k
+    if out is None:
+        out = torch.empty((B, width), dtype=torch.float32, device=device)
+    _check(lib().eogp_compress_layer_host(ctypes.byref(desc), _ptr(a), _ptr(s), B, int(chunk), out_mode,
+                                          _ptr(out), out.stride(0), None, 0, None, 0, _ptr(ws),
+                                          ws.numel(), _stream(stream)))
     return out
 
 

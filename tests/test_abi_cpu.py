@@ -157,3 +157,47 @@ def test_topk_host_argument_checks():
     args[15] = 10
     args[19] = 0     # workspace too small
     assert L.eogp_score_topk(*args) == E.EWORKSPACE
+
+
+def test_host_input_call_argument_checks():
+    """eogp_compress_layer_host / _workspace_size: argument checks that run before
+    any device work (no GPU needed)."""
+    import ctypes
+    lam = np.arange(1, 9, dtype=np.float64) ** -1.0
+    plan = E.Plan.from_factors(lam, lam, 10, 0.1)
+    desc = E.LayerDesc(8, 8, 64, 10, 4, E.F32, 16, 16, 16, plan.handle)   # T = 64: 2 KB of a per example
+    L = E.lib()
+    n1, n2, n0 = ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_size_t()
+    assert L.eogp_compress_host_workspace_size(ctypes.byref(desc), 6, 1, E.OUT_CODES, ctypes.byref(n1)) == E.OK
+    assert L.eogp_compress_host_workspace_size(ctypes.byref(desc), 6, 2, E.OUT_CODES, ctypes.byref(n2)) == E.OK
+    assert L.eogp_compress_host_workspace_size(ctypes.byref(desc), 6, 0, E.OUT_CODES, ctypes.byref(n0)) == E.OK
+    assert 0 < n1.value < n2.value <= n0.value   # bigger chunks stage more; the default takes all 6
+    assert L.eogp_compress_host_workspace_size(ctypes.byref(desc), 6, -1, E.OUT_CODES,
+                                               ctypes.byref(n1)) == E.EINVAL
+    assert L.eogp_compress_host_workspace_size(None, 6, 0, E.OUT_CODES, ctypes.byref(n1)) == E.EINVAL
+    args = [ctypes.byref(desc), 16, 16, 2, 0, E.OUT_CODES, None, 0, 16, 1, 16, 1, 256, n0.value, None]
+    assert L.eogp_compress_layer_host(*args) == E.EINVAL          # host-only plan
+    args[4] = -1
+    assert L.eogp_compress_layer_host(*args) == E.EINVAL          # negative chunk
+    args[4], args[3] = 0, 0
+    assert L.eogp_compress_layer_host(*args) == E.OK              # empty batch: nothing to do
+    args[3], args[12] = 2, None
+    assert L.eogp_compress_layer_host(*args) == E.EWORKSPACE
+
+
+def test_host_alloc_argument_checks():
+    """eogp_host_alloc / eogp_host_free: argument checks, and clean failure (or
+    success, with a GPU present) of the registration."""
+    import ctypes
+    L = E.lib()
+    p = ctypes.c_void_p()
+    assert L.eogp_host_alloc(0, ctypes.byref(p)) == E.EINVAL and not p.value
+    assert L.eogp_host_alloc(4096, None) == E.EINVAL
+    assert L.eogp_host_free(None) == E.OK
+    assert L.eogp_host_free(ctypes.c_void_p(4096)) == E.EINVAL   # not from eogp_host_alloc
+    rc = L.eogp_host_alloc(4096, ctypes.byref(p))
+    if rc == E.OK:          # a device is present: the region is usable and released
+        ctypes.memset(p.value, 7, 4096)
+        assert L.eogp_host_free(p) == E.OK
+    else:                   # no device: registration fails and nothing is handed out
+        assert rc == E.ECUDA and not p.value

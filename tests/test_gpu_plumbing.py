@@ -142,3 +142,75 @@ def test_host_resident_eigenbases_give_identical_codes():
     x2 = E.compress_layer(d_host, a, s, E.OUT_COORDS)
     E.sync_status()
     assert torch.equal(c1, c2) and torch.equal(s1, s2) and torch.equal(x1, x2)
+
+
+@pytest.mark.parametrize("dtype,d_in,d_out,T,B,m,k,chunk,bias,lens,host_bases", [
+    ("bf16", 768, 2304, 64, 7, 4096, 1024, 3, True, True, False),
+    ("bf16", 768, 768, 64, 5, 4096, 1024, 0, False, False, True),
+    ("bf16", 256, 384, 128, 4, 2000, 300, 1, False, True, True),
+    ("f32", 64, 64, 16, 9, 512, 128, 4, True, False, False),
+])
+def test_host_inputs_match_device_inputs(dtype, d_in, d_out, T, B, m, k, chunk, bias, lens, host_bases):
+    """eogp_compress_layer_host (inputs in page-locked host memory, copied chunk by
+    chunk by the call) gives the results of eogp_compress_layer on the same
+    inputs in device memory, bit for bit, in every output mode: ragged last
+    chunk, per-example lengths offset per chunk, bias channel, host eigenbases."""
+    rng = np.random.default_rng(d_in + B + chunk)
+    rnd = (lambda v: synth.round_to(v, dtype))
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    d_eff = d_in + (1 if bias else 0)
+    QA, QS = rnd(synth.haar_orthogonal(d_eff, rng)), rnd(synth.haar_orthogonal(d_out, rng))
+    plan = E.Plan.from_factors(synth.power_spectrum(d_out, 1.2), synth.power_spectrum(d_eff, 1.2), m, 0.1)
+    R, C = plan.sets()
+    VA_full = QA.T[C]
+    VA = torch.from_numpy(np.ascontiguousarray(VA_full[:, :d_in], dtype=np.float32)).to(tdt)
+    VS = torch.from_numpy(np.ascontiguousarray(QS.T[R], dtype=np.float32)).to(tdt)
+    if host_bases:
+        VA, VS = VA.pin_memory(), VS.pin_memory()
+    else:
+        VA, VS = VA.to(DEV), VS.to(DEV)
+    bias_A = dev(np.ascontiguousarray(VA_full[:, d_in], dtype=np.float32)) if bias else None
+    lengths = None
+    if lens:
+        lv = rng.integers(1, T + 1, B).astype(np.int32)
+        lv[0] = T
+        lengths = dev(lv)
+    Pt = dev(rnd(synth.haar_orthogonal(m, rng, k).T).astype(np.float32), tdt)
+    desc = E.layer_desc(plan, T, k, VA, VS, Pt, bias_A=bias_A, lengths=lengths)
+    a = torch.from_numpy(rnd(rng.standard_normal((B, T, d_in))).astype(np.float32)).to(tdt)
+    s = torch.from_numpy(rnd(rng.standard_normal((B, T, d_out)) * 0.1).astype(np.float32)).to(tdt)
+    if chunk == 3:      # inputs in eogp_host_alloc memory
+        ah, sh = E.host_empty(a.shape, tdt), E.host_empty(s.shape, tdt)
+        ah.copy_(a)
+        sh.copy_(s)
+    else:
+        ah, sh = a.pin_memory(), s.pin_memory()
+    ad, sd = a.to(DEV), s.to(DEV)
+    c1, s1 = E.compress_layer(desc, ad, sd, E.OUT_CODES)
+    c2, s2 = E.compress_layer_host(desc, ah, sh, E.OUT_CODES, DEV, chunk=chunk)
+    for mode in (E.OUT_COORDS, E.OUT_FIRST_STAGE):
+        x1 = E.compress_layer(desc, ad, sd, mode)
+        x2 = E.compress_layer_host(desc, ah, sh, mode, DEV, chunk=chunk)
+        torch.cuda.synchronize()
+        assert torch.equal(x1, x2), mode
+    E.sync_status()
+    assert torch.equal(c1, c2) and torch.equal(s1, s2)
+
+
+def test_host_empty_memory_round_trip():
+    """eogp_host_alloc memory (through host_empty): zero-filled, writable, copies
+    to and from the device asynchronously, and is released with the tensor."""
+    import gc
+    t = E.host_empty((3, 1000, 7), torch.bfloat16)
+    assert t.shape == (3, 1000, 7) and t.dtype == torch.bfloat16 and not t.is_cuda
+    assert int(t.abs().sum()) == 0
+    src = torch.randn(3, 1000, 7).to(torch.bfloat16)
+    t.copy_(src)
+    d = torch.empty_like(t, device=DEV)
+    d.copy_(t, non_blocking=True)
+    back = E.host_empty(t.shape, torch.bfloat16)
+    back.copy_(d, non_blocking=True)
+    torch.cuda.synchronize()
+    assert torch.equal(back, src)
+    del t, back
+    gc.collect()
