@@ -248,7 +248,9 @@ int eogp_host_free(void* ptr);
  * a copy stream the call creates, double-buffered, so the copy of chunk c + 1
  * overlaps the compute of chunk c on `stream`; the compute of every chunk is
  * queued on `stream`, which therefore orders all of the call's work, and the
- * call releases its copy stream and events itself. `descriptor->lengths` (if
+ * call releases its copy stream and events itself. The first copies wait for
+ * the work already queued on `stream` (the workspace may be memory that such
+ * work still uses, as with a stream-ordered allocator). `descriptor->lengths` (if
  * any) is a device array of all B examples. With bases_on_host the eigenbases
  * are copied once per call, not per chunk. a and s must stay valid and
  * unchanged until `stream` reaches the point of the call. A library
