@@ -5,6 +5,9 @@
   inputs), checked on sampled examples of one module of each shape.
 * OLMo 2 1B / 7B shapes and the 32B gate projection (T = 2048, m = 8192,
   k = 2048): a few examples per distinct module shape.
+* GPT-2 query scoring: Q = 1024 one-bit queries of 48 modules x 1024 bits
+  (the bench's query workload) against 300 stored codes, every score bit for
+  bit, dense and with the top-20 ranking fused.
 * Scoring sweep: 4,194,304 stored 16,384-bit codes, Q in {1, 64, 1024, 8192};
   sampled stored rows are checked bit for bit.
 * PCA fit at the GPT-2 size (10,000 fitting rows, m = 4096, k = 1024).
@@ -201,3 +204,30 @@ def test_fit_pca_gpt2_size():
     np.testing.assert_allclose(eig.cpu().numpy(), mu[:k], rtol=1e-3)
     assert np.abs(P.T @ P - np.eye(k)).max() <= 1e-4
     assert np.trace(P.T @ C @ P) == pytest.approx(mu[:k].sum(), rel=1e-4)
+
+
+# ------------------------------------------------------ GPT-2 query scoring
+
+def test_gpt2_query_scoring_all_scores():
+    """Q = 1024 queries x 48 modules x 1024 bits (the bench's query workload: the
+    running score kept in TMEM across modules) against N = 300 stored codes (a
+    ragged last row tile): every score equals the oracle's float32 evaluation
+    bit for bit, and the fused top-20 equals the oracle ranking."""
+    rng = np.random.default_rng(48)
+    ks = [1024] * 48
+    N, Q = 300, 1024
+    W = sum(ks) // 32
+    tc = rng.integers(0, 2**32, (N, W), dtype=np.uint64).astype(np.uint32)
+    qc = rng.integers(0, 2**32, (Q, W), dtype=np.uint64).astype(np.uint32)
+    ts = rng.lognormal(0, 0.5, (N, 48)).astype(np.float32)
+    qs = rng.lognormal(0, 0.5, (Q, 48)).astype(np.float32)
+    d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(DEV)
+    tcd, qcd = d(tc.view(np.int32)), d(qc.view(np.int32))
+    got = E.score(tcd, d(ts), ks, E.SCORE_CODES, qcd, d(qs))
+    vals, idx = E.score_topk(tcd, d(ts), ks, E.SCORE_CODES, qcd, 20, query_scales=d(qs))
+    E.sync_status()
+    want = O.score_codes_f32(tc, ts, ks, qc, qs)
+    np.testing.assert_array_equal(got.cpu().numpy(), want)
+    want_v, want_i = O.top_k(want, 20)
+    np.testing.assert_array_equal(idx.cpu().numpy(), want_i)
+    np.testing.assert_array_equal(vals.cpu().numpy().astype(np.float64), want_v)

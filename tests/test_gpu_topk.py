@@ -110,6 +110,7 @@ def codes_case(N, Q, ks, seed, dup=True):
 @pytest.mark.parametrize("N,Q,ks,K", [(1000, 70, [128, 256], 10), (5000, 130, [1024, 1024], 32),
                                       (300, 64, [128], 1), (20, 64, [128], 32),
                                       (20000, 200, [512], 20), (30000, 300, [1024], 20),
+                                      (3000, 300, [512, 1024, 128], 20),   # several modules, two query tiles
                                       (5000, 130, [1024, 1024], 64)])
 def test_topk_codes_fused_exact(N, Q, ks, K):
     """K <= 32 ranks inside the tensor-core epilogue; K = 64 takes the dense path."""
