@@ -992,9 +992,10 @@ static bool rotate_pairs(int K) {
 }
 
 // N tile width for `n` output columns: as few tiles of at most 256 columns as
-// is cheapest, each a multiple of `gran` (16: tcgen05 N granularity for one
-// CTA; 32 for CTA pairs, whose halves must be multiples of 16), counting a
-// fixed per-tile overhead of 32 columns. EOGP_ROT_BN overrides for sweeps.
+// is cheapest, each a multiple of `gran` (16: the tcgen05 N granularity, for one
+// CTA and for CTA pairs, whose halves of N / 2 rows are whole 8-row swizzle
+// atoms), counting a fixed per-tile overhead of 32 columns. EOGP_ROT_BN
+// overrides for sweeps.
 int rotate_bn(int n, int gran) {
   static int forced = -1;
   if (forced < 0) {
@@ -1020,7 +1021,7 @@ cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W
                              const int32_t* lengths, int num_sms, unsigned* status, cudaStream_t st) {
   if (M <= 0) return cudaSuccess;
   const bool pairs = rotate_pairs(K);
-  const int BN = rotate_bn(Wrows, pairs ? 32 : 16);
+  const int BN = rotate_bn(Wrows, 16);
   // As many pipeline stages as fit in 227 KB of shared memory (at most 8);
   // EOGP_ROT_STAGES overrides for tuning sweeps.
   static int forced_stages = -1;
