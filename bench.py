@@ -492,6 +492,9 @@ def main():
                     help="stored codes in the scan (default: the 4,194,304 of the scan workload)")
     ap.add_argument("--scan-qs", default="",
                     help="comma-separated query counts of the scan (default: 1,64,1024,8192)")
+    ap.add_argument("--only-ekfac", action="store_true",
+                    help="time only the EK-FAC correction (GPT-2 c_fc and OLMo-1B gate modules); "
+                         "the case profiles/ captures for k_tc_ekfac")
     ap.add_argument("--no-configs", action="store_true",
                     help="skip the OLMo / 32B / tiny-fp32 throughput and the PCA-fit timing")
     ap.add_argument("--modules", type=int, default=0,
@@ -517,6 +520,11 @@ def main():
     from paper_2609_37842_gb300 import eogp as E
     from paper_2609_37842_gb300 import synth
 
+    if args.only_ekfac:
+        ek = [bench_ekfac(dev, 768, 3072, 512, 32), bench_ekfac(dev, 2048, 8192, 2048, 4)]
+        if rank == 0:
+            print(json.dumps({"ekfac_correction": ek}))
+        return
     w = synth.WORKLOADS[WORKLOAD]
     if args.modules:
         import dataclasses

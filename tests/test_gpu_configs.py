@@ -208,7 +208,7 @@ def test_fit_pca_gpt2_size():
 
 # ------------------------------------------------------ GPT-2 query scoring
 
-def test_gpt2_query_scoring_all_scores():
+def test_gpt2_query_scoring_all_scores(monkeypatch):
     """Q = 1024 queries x 48 modules x 1024 bits (the bench's query workload: the
     running score kept in TMEM across modules) against N = 300 stored codes (a
     ragged last row tile): every score equals the oracle's float32 evaluation
@@ -224,10 +224,13 @@ def test_gpt2_query_scoring_all_scores():
     d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(DEV)
     tcd, qcd = d(tc.view(np.int32)), d(qc.view(np.int32))
     got = E.score(tcd, d(ts), ks, E.SCORE_CODES, qcd, d(qs))
-    vals, idx = E.score_topk(tcd, d(ts), ks, E.SCORE_CODES, qcd, 20, query_scales=d(qs))
     E.sync_status()
     want = O.score_codes_f32(tc, ts, ks, qc, qs)
     np.testing.assert_array_equal(got.cpu().numpy(), want)
     want_v, want_i = O.top_k(want, 20)
-    np.testing.assert_array_equal(idx.cpu().numpy(), want_i)
-    np.testing.assert_array_equal(vals.cpu().numpy().astype(np.float64), want_v)
+    for fused in ("1", "0"):     # ranking fused into the scoring kernel, and the dense path
+        monkeypatch.setenv("EOGP_TOPK_FUSED", fused)
+        vals, idx = E.score_topk(tcd, d(ts), ks, E.SCORE_CODES, qcd, 20, query_scales=d(qs))
+        E.sync_status()
+        np.testing.assert_array_equal(idx.cpu().numpy(), want_i)
+        np.testing.assert_array_equal(vals.cpu().numpy().astype(np.float64), want_v)

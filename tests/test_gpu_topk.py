@@ -7,8 +7,11 @@
   reproducible, so the lists must match exactly (values and indices, including
   planted equal scores); PAPER / FP lists are checked for validity within the
   score tolerance (several lists are correct when scores differ by less).
-* The fused path (ranking inside the tensor-core epilogue, K <= 32), the dense
-  path (Q < 64 CODES, FP, K > 64) and the edge cases N < K and N = 0.
+* The fused path (ranking inside the tensor-core epilogue, K <= 32, the
+  library's choice whenever it applies), the dense path (dense scores then a
+  selection pass: Q < 64 CODES, FP, K > 32, and any request with
+  EOGP_TOPK_FUSED=0, which the tests use to run both paths on the same cases)
+  and the edge cases N < K and N = 0.
 * Full scan scale (4,194,304 stored 16,384-bit codes, Q = 1024): the fused
   lists equal the oracle ranking of the dense scores of sampled queries.
 """
@@ -112,8 +115,11 @@ def codes_case(N, Q, ks, seed, dup=True):
                                       (20000, 200, [512], 20), (30000, 300, [1024], 20),
                                       (3000, 300, [512, 1024, 128], 20),   # several modules, two query tiles
                                       (5000, 130, [1024, 1024], 64)])
-def test_topk_codes_fused_exact(N, Q, ks, K):
-    """K <= 32 ranks inside the tensor-core epilogue; K = 64 takes the dense path."""
+@pytest.mark.parametrize("fused", ["1", "0"])
+def test_topk_codes_fused_exact(N, Q, ks, K, fused, monkeypatch):
+    """K <= 32 ranks inside the tensor-core epilogue when fused; K = 64 always
+    takes the dense path. Both paths give the oracle's lists exactly."""
+    monkeypatch.setenv("EOGP_TOPK_FUSED", fused)
     tc, ts, qc, qs = codes_case(N, Q, ks, N + K)
     vals, idx = E.score_topk(dev(tc), dev(ts), ks, E.SCORE_CODES, dev(qc), K, query_scales=dev(qs))
     E.sync_status()
@@ -135,7 +141,9 @@ def test_topk_codes_dense_exact(N, Q, ks, K):
 
 @pytest.mark.parametrize("N,Q,ks,K", [(1500, 70, [64, 128], 20), (4000, 3, [256], 10),
                                       (600, 130, [128], 100)])
-def test_topk_paper_valid(N, Q, ks, K):
+@pytest.mark.parametrize("fused", ["1", "0"])
+def test_topk_paper_valid(N, Q, ks, K, fused, monkeypatch):
+    monkeypatch.setenv("EOGP_TOPK_FUSED", fused)
     rng = np.random.default_rng(N + Q + K)
     tc = rand_store(rng, N, ks)
     ts = rng.lognormal(0, 0.5, (N, len(ks))).astype(np.float32)
