@@ -1243,17 +1243,19 @@ extern "C" int eogp_score(const void* train, int ld_train, const float* train_sc
 // Workspace plan of eogp_score_topk: fused (tensor-core scoring with the ranking in
 // its epilogue) or dense (scores into the workspace, then a ranking kernel).
 struct TopkPlan {
-  bool fused;
+  bool fused, select;
   int slots;
   size_t q_bytes, dense_bytes, list_bytes, buf_bytes, scr_bytes, total;
 };
 
-// The ranking is fused into the tensor-core scoring kernel whenever that kernel
-// supports the request (measured faster than dense scores plus a selection pass
-// at every size tried: 2.4 against 2.9 ms for the GPT-2 query workload, 61
-// against 97 ms for 1024 queries over the 4.2M-code store). EOGP_TOPK_FUSED = 0
-// forces the dense path (tests); it is read at every call, so the workspace
-// query and the call must see the same setting.
+// Paths: up to topk_select_max_n() stored rows, dense scores (tensor cores
+// where they apply) and a radix select per query row (k_topk_select); beyond,
+// the ranking is fused into the tensor-core scoring kernel when it supports the
+// request (the Q x N matrix then never reaches HBM), else dense scores, per-slot
+// lists and a merge. Measured on the GPT-2 query workload (N = 16384, Q = 1024,
+// top 20): fused 2.4 ms, dense + per-slot lists 2.9 ms. EOGP_TOPK_FUSED = 1 / 0
+// forces the fused / a dense path (tests); it is read at every call, so the
+// workspace query and the call must see the same setting.
 static int topk_fused_override() {
   const char* e = getenv("EOGP_TOPK_FUSED");
   return e ? atoi(e) : -1;
@@ -1263,13 +1265,16 @@ static TopkPlan topk_plan(int N, const int* ks, int U, int mode, int Q, int K) {
   TopkPlan p{};
   const bool tc_ok = (mode == EOGP_SCORE_CODES || mode == EOGP_SCORE_PAPER) &&
                      score_tc_supported(mode, ks, U, Q);
-  p.fused = tc_ok && score_tc_topk_fits(mode, U, Q, K) && topk_fused_override() != 0;
+  const int force = topk_fused_override();
+  p.fused = tc_ok && score_tc_topk_fits(mode, U, Q, K) && force != 0 &&
+            (force == 1 || N > topk_select_max_n());
+  p.select = !p.fused && N <= topk_select_max_n();
   p.q_bytes = tc_ok ? score_tc_ws_bytes(mode, ks, U, Q) : 0;
   if (p.fused) {
     p.slots = score_tc_grid(mode, U, N, Q, K, sm_count());
     p.dense_bytes = 0;
   } else {
-    p.slots = topk_dense_slots(N);
+    p.slots = p.select ? 0 : topk_dense_slots(N);
     p.dense_bytes = al256(static_cast<size_t>(Q) * ((static_cast<size_t>(N) + 3) & ~size_t(3)) * 4);
   }
   p.list_bytes = al256(static_cast<size_t>(p.slots) * Q * K * 4);
@@ -1349,6 +1354,10 @@ extern "C" int eogp_score_topk(const void* train, int ld_train, const float* tra
     const int rc = score_dense(train, ld_train, train_scales, ld_tscale, N, k_per_module, U, mode, query,
                                ld_query, query_scales, ld_qscale, Q, dense, ldd, qws, p.q_bytes, W, D, st);
     if (rc != EOGP_OK) return rc;
+  }
+  if (p.select) {
+    CUDA_TRY(launch_topk_select(dense, ldd, Q, N, topk, top_scores, ld_top_scores, top_index, ld_top_index, st));
+    return EOGP_OK;
   }
   CUDA_TRY(launch_topk_dense(dense, ldd, Q, N, topk, lst, lsi, st));
   CUDA_TRY(launch_topk_merge(lst, lsi, topk_dense_slots(N), Q, topk, top_scores, ld_top_scores, top_index,

@@ -112,6 +112,12 @@ cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const floa
 // k_topk.cu: top-K of a dense [Q, N] score matrix into per-slot lists, and the
 // merge of per-slot lists [S][Q][K] (index -1 = empty) into [Q, K].
 int topk_dense_slots(int N);
+// Largest N k_topk_select ranks (one row per block, held in shared memory).
+int topk_select_max_n();
+// Per query the K best of a dense [Q, N] score row, written to the final
+// outputs (N <= topk_select_max_n(), K <= EOGP_TOPK_MAX).
+cudaError_t launch_topk_select(const float* scores, int ld, int Q, int N, int K, float* out_s, int ld_os,
+                               int* out_i, int ld_oi, cudaStream_t st);
 cudaError_t launch_topk_dense(const float* scores, int ld, int Q, int N, int K, float* lst, int* lsi,
                               cudaStream_t st);
 cudaError_t launch_topk_merge(const float* lst, const int* lsi, int S, int Q, int K, float* out_s,

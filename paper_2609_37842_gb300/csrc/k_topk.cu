@@ -3,7 +3,14 @@
 // Order: score descending, equal scores by lower stored index; NaN scores
 // never rank; missing places are (-inf, -1).
 //
-// Two kernels:
+// Three kernels:
+// * k_topk_select ranks one row of a dense [Q, N] score matrix per block when
+//   the row fits in shared memory (N <= kSelectMaxN): the K-th largest score
+//   is found exactly as the largest order-preserving 32-bit key t with at
+//   least K keys >= t, built bit by bit from the top (block-wide counting
+//   passes over the row held in shared memory, no atomics); the K winners are
+//   gathered (the equal-to-threshold ones in index order, so the lowest indices
+//   win ties) and sorted.
 // * k_topk_dense ranks a dense [Q, N] score matrix: block (slot s, query tile)
 //   owns stored rows [s R, (s+1) R) of 32 queries; 128-row chunks are staged
 //   transposed in shared memory and the warp offers each query's column to
@@ -24,10 +31,12 @@ constexpr int kChunk = 128;
 constexpr int kTs = kChunk + 1;  // staged row stride (floats)
 constexpr int kMaxSlots = 512;
 constexpr int kMergeCap = 4096;  // keys sorted at once by the merge
+constexpr int kSelectMaxN = 49152;  // rows k_topk_select holds in shared memory (192 KB)
 
-// Order-preserving 64-bit key: larger key = larger score, then lower index.
+// Order-preserving 64-bit key: larger key = larger score, then lower index
+// (-0 and +0 are the same score).
 __device__ __forceinline__ unsigned long long make_key(float s, int idx) {
-  const uint32_t b = __float_as_uint(s);
+  const uint32_t b = __float_as_uint(s == 0.f ? 0.f : s);
   const uint32_t o = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
   return (static_cast<unsigned long long>(o) << 32) | (0xFFFFFFFFu - static_cast<uint32_t>(idx));
 }
@@ -84,6 +93,122 @@ __global__ void __launch_bounds__(32) k_topk_dense(const float* __restrict__ sc,
   for (int j = 0; j < nq; ++j) {
     const size_t o = (static_cast<size_t>(slot) * Q + q0 + j) * K;
     eogp::topk_warp_write<E>(list_of(j), lane, lst + o, lsi + o);
+  }
+}
+
+constexpr int kSelThreads = 512;
+constexpr int kSelWarps = kSelThreads / 32;
+
+// 32-bit order key of a score: larger score, larger key; -0 and +0 equal; NaN
+// maps to 0, below every score (no non-NaN float maps to 0).
+__device__ __forceinline__ uint32_t sel_key(float s) {
+  if (s != s) return 0u;
+  const uint32_t b = __float_as_uint(s == 0.f ? 0.f : s);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+// Number of keys of this block's row that are >= t (block-uniform result).
+// red is double-buffered by `parity` so consecutive calls need one barrier.
+__device__ __forceinline__ uint32_t count_ge(const uint32_t* skey, int N, uint32_t t, uint32_t* red,
+                                             int parity) {
+  uint32_t c = 0;
+  for (int i = threadIdx.x; i < N; i += kSelThreads) c += skey[i] >= t ? 1u : 0u;
+  c = __reduce_add_sync(0xffffffffu, c);
+  if ((threadIdx.x & 31) == 0) red[parity * kSelWarps + (threadIdx.x >> 5)] = c;
+  __syncthreads();
+  uint32_t tot = 0;
+#pragma unroll
+  for (int w = 0; w < kSelWarps; ++w) tot += red[parity * kSelWarps + w];
+  return tot;
+}
+
+__global__ void __launch_bounds__(kSelThreads) k_topk_select(const float* __restrict__ sc, int ld, int N,
+                                                             int K, float* __restrict__ out_s, int ld_os,
+                                                             int* __restrict__ out_i, int ld_oi) {
+  extern __shared__ uint32_t skey[];  // [N] keys of this query's row
+  __shared__ uint32_t red[2 * kSelWarps];
+  __shared__ uint32_t weq[kSelWarps];
+  __shared__ unsigned long long cand[EOGP_TOPK_MAX];
+  __shared__ uint32_t s_ngt;
+  const int q = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const float* row = sc + static_cast<size_t>(q) * ld;
+  for (int i = tid; i < N; i += kSelThreads) skey[i] = sel_key(row[i]);
+  if (tid == 0) s_ngt = 0;
+  __syncthreads();
+  // Valid (non-NaN) scores are the keys >= 1.
+  int parity = 0;
+  const uint32_t nv = count_ge(skey, N, 1u, red, parity);
+  parity ^= 1;
+  const int Kv = static_cast<int>(min(static_cast<uint32_t>(K), nv));
+  if (Kv > 0) {
+    // T = the Kv-th largest key: the largest t with at least Kv keys >= t, built
+    // bit by bit from the top.
+    uint32_t T = 0;
+    for (int bit = 31; bit >= 0; --bit) {
+      const uint32_t c = T | (1u << bit);
+      if (count_ge(skey, N, c, red, parity) >= static_cast<uint32_t>(Kv)) T = c;
+      parity ^= 1;
+    }
+    const uint32_t ngt = T == 0xFFFFFFFFu ? 0u : count_ge(skey, N, T + 1u, red, parity);
+    parity ^= 1;
+    const uint32_t rem = static_cast<uint32_t>(Kv) - ngt;  // keys equal to T that rank, >= 1
+    // Gather. Keys above T (ngt of them) in any order; keys equal to T in index
+    // order, so that the rem lowest indices win: warp w scans the contiguous
+    // segment [w seg, (w+1) seg) twice (count, then place).
+    const int seg = ((N + kSelWarps - 1) / kSelWarps + 31) & ~31;
+    const int b0 = warp * seg, b1 = min(N, b0 + seg);
+    uint32_t mine = 0;
+    for (int base = b0; base < b1; base += 32) {
+      const int i = base + lane;
+      mine += __popc(__ballot_sync(0xffffffffu, i < b1 && skey[i] == T));
+    }
+    if (lane == 0) weq[warp] = mine;
+    __syncthreads();
+    uint32_t before = 0;
+    for (int w = 0; w < warp; ++w) before += weq[w];
+    for (int base = b0; base < b1; base += 32) {
+      const int i = base + lane;
+      const uint32_t k = i < b1 ? skey[i] : 0u;
+      const unsigned long long ck =
+          (static_cast<unsigned long long>(k) << 32) | (0xFFFFFFFFu - static_cast<uint32_t>(i));
+      if (k > T) cand[atomicAdd(&s_ngt, 1u)] = ck;
+      const unsigned b = __ballot_sync(0xffffffffu, i < b1 && k == T);
+      const uint32_t pos = before + static_cast<uint32_t>(__popc(b & ((1u << lane) - 1u)));
+      if (((b >> lane) & 1u) && pos < rem) cand[ngt + pos] = ck;
+      before += static_cast<uint32_t>(__popc(b));
+    }
+    __syncthreads();
+    // Sort the Kv winners: descending key = score descending, then lower index.
+    int P = 1;
+    while (P < Kv) P <<= 1;
+    for (int i = Kv + tid; i < P; i += kSelThreads) cand[i] = 0ull;
+    __syncthreads();
+    for (int k2 = 2; k2 <= P; k2 <<= 1) {
+      for (int j = k2 >> 1; j > 0; j >>= 1) {
+        for (int i = tid; i < P; i += kSelThreads) {
+          const int ixj = i ^ j;
+          if (ixj > i) {
+            const unsigned long long a = cand[i], b2 = cand[ixj];
+            const bool desc = (i & k2) == 0;
+            if (desc ? (a < b2) : (a > b2)) {
+              cand[i] = b2;
+              cand[ixj] = a;
+            }
+          }
+        }
+        __syncthreads();
+      }
+    }
+  }
+  for (int p = tid; p < K; p += kSelThreads) {
+    float v = -INFINITY;
+    int ix = -1;
+    if (p < Kv) {
+      ix = static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(cand[p]));
+      v = row[ix];  // the stored score itself (keys merge -0 into +0)
+    }
+    out_s[static_cast<size_t>(q) * ld_os + p] = v;
+    out_i[static_cast<size_t>(q) * ld_oi + p] = ix;
   }
 }
 
@@ -194,6 +319,22 @@ cudaError_t launch_topk_dense(const float* scores, int ld, int Q, int N, int K, 
     case 8: return launch_topk_dense_e<8>(scores, ld, Q, N, K, lst, lsi, st);
     default: return launch_topk_dense_e<16>(scores, ld, Q, N, K, lst, lsi, st);
   }
+}
+
+int topk_select_max_n() { return kSelectMaxN; }
+
+cudaError_t launch_topk_select(const float* scores, int ld, int Q, int N, int K, float* out_s, int ld_os,
+                               int* out_i, int ld_oi, cudaStream_t st) {
+  if (Q <= 0) return cudaSuccess;
+  if (N > kSelectMaxN || K > EOGP_TOPK_MAX) return cudaErrorInvalidValue;
+  const size_t smem = static_cast<size_t>(std::max(N, 1)) * 4;
+  if (smem > 48 * 1024) {
+    const cudaError_t e = cudaFuncSetAttribute(k_topk_select, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  k_topk_select<<<Q, kSelThreads, smem, st>>>(scores, ld, N, K, out_s, ld_os, out_i, ld_oi);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_topk_merge(const float* lst, const int* lsi, int S, int Q, int K, float* out_s,

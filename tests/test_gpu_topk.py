@@ -7,11 +7,11 @@
   reproducible, so the lists must match exactly (values and indices, including
   planted equal scores); PAPER / FP lists are checked for validity within the
   score tolerance (several lists are correct when scores differ by less).
-* The fused path (ranking inside the tensor-core epilogue, K <= 32, the
-  library's choice whenever it applies), the dense path (dense scores then a
-  selection pass: Q < 64 CODES, FP, K > 32, and any request with
-  EOGP_TOPK_FUSED=0, which the tests use to run both paths on the same cases)
-  and the edge cases N < K and N = 0.
+* The three paths: up to 49,152 stored rows, dense scores and a radix select
+  per query row (the library's choice there); beyond, the ranking fused into
+  the tensor-core epilogue (K <= 32), else dense scores, per-slot lists and a
+  merge. EOGP_TOPK_FUSED=1 / 0 forces the fused / a dense path, which the
+  tests use to run both on the same cases; edge cases N < K and N = 0, ties.
 * Full scan scale (4,194,304 stored 16,384-bit codes, Q = 1024): the fused
   lists equal the oracle ranking of the dense scores of sampled queries.
 """
@@ -129,7 +129,9 @@ def test_topk_codes_fused_exact(N, Q, ks, K, fused, monkeypatch):
 
 
 @pytest.mark.parametrize("N,Q,ks,K", [(3000, 5, [128, 64], 16), (4000, 70, [256], 100),
-                                      (700, 33, [1024], 256)])
+                                      (700, 33, [1024], 256),
+                                      (60000, 33, [128], 100),      # beyond the select: slot lists + merge
+                                      (50000, 70, [256, 128], 40)])
 def test_topk_codes_dense_exact(N, Q, ks, K):
     tc, ts, qc, qs = codes_case(N, Q, ks, N + K + 1)
     vals, idx = E.score_topk(dev(tc), dev(ts), ks, E.SCORE_CODES, dev(qc), K, query_scales=dev(qs))
