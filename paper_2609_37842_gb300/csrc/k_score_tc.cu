@@ -43,6 +43,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 
 #include "eogp_dev.cuh"
 #include "eogp_internal.h"
@@ -93,45 +94,63 @@ struct TcMode<EOGP_SCORE_PAPER> {
 
 // BN: queries per tile (MMA N). 256 only for CODES with one module (no running
 // score is needed, so the two accumulators take all 512 TMEM columns).
-template <int MODE, int BN>
+// AT: the expanded stored rows (operand A) go to tensor memory instead of
+// shared memory (CODES): a pipeline stage is then only the query operand in
+// shared memory plus a 32-column A slot in TMEM, and the tensor cores read A
+// from TMEM (tcgen05.mma with [a-tmem]), taking the A writes and reads off the
+// shared-memory bandwidth the query operand's TMA writes and MMA reads use.
+template <int MODE, int BN, bool AT>
 constexpr uint32_t tc_stage_bytes() {
-  return kAB + static_cast<uint32_t>(BN) * 128u * TcMode<MODE>::kQBoxes;
+  return (AT ? 0u : kAB) + static_cast<uint32_t>(BN) * 128u * TcMode<MODE>::kQBoxes;
+}
+template <bool AT>
+constexpr uint32_t tc_b_offset() {
+  return AT ? 0u : kAB;
 }
 
-// Pipeline stages: six when a stage is 32 KB (one-bit queries, 128 per tile),
-// else four (48 KB stages).
-template <int MODE, bool TOPK, int BN>
+// Pipeline stages. Shared-memory A: six when a stage is 32 KB (one-bit
+// queries, 128 per tile), else four (48 KB stages). TMEM A: six 32 KB query
+// stages with 256 queries per tile (A slots in TMEM columns 256-447), four with
+// 128 (A slots in columns 384-511).
+template <int MODE, bool TOPK, int BN, bool AT>
 constexpr int tc_stages() {
-  return (MODE == EOGP_SCORE_CODES && BN == 128) ? 6 : 4;
+  return AT ? (BN == 256 ? 6 : 4) : ((MODE == EOGP_SCORE_CODES && BN == 128) ? 6 : 4);
 }
 
-
-// Stages the expanders fill per synchronisation round (one wait, proxy fence
-// and arrive round): two with six stages, so that the MMAs always have at
-// least four stages to work on, else one.
-template <int MODE, bool TOPK, int BN>
+// Stages the expanders fill per synchronisation round (one wait, fence and
+// arrive round): two with six stages, so that the MMAs always have at least
+// four stages to work on, else one.
+template <int MODE, bool TOPK, int BN, bool AT>
 constexpr int tc_group() {
-  return tc_stages<MODE, TOPK, BN>() >= 6 ? 2 : 1;
+  return tc_stages<MODE, TOPK, BN, AT>() >= 6 ? 2 : 1;
 }
 
-// Accumulator buffers d_u in TMEM (BN columns each): three of 128 columns plus
-// the 128-column running score, or two of 256 (one module, no running score).
-template <int BN>
+// Accumulator buffers d_u in TMEM (BN columns each). Shared-memory A: three of
+// 128 columns plus the 128-column running score, or two of 256 (one module, no
+// running score). TMEM A: two of 128 plus the running score, or one of 256.
+template <int BN, bool AT>
 constexpr int tc_dbufs() {
-  return BN == 128 ? 3 : 2;
+  return AT ? (BN == 128 ? 2 : 1) : (BN == 128 ? 3 : 2);
+}
+constexpr int kMaxDbufs = 3;
+
+// First TMEM column of A slot s (TMEM A), after the accumulators.
+template <int BN>
+__device__ __forceinline__ uint32_t tc_acol(int s) {
+  return static_cast<uint32_t>((BN == 256 ? 256 : 384) + 32 * s);
 }
 
 // Shared-memory carve-up (byte offsets after 1024-byte alignment).
 struct TcSmem {
   uint32_t sq, bars, lists, total;
 };
-template <int MODE, bool TOPK, int BN>
+template <int MODE, bool TOPK, int BN, bool AT>
 __host__ __device__ inline TcSmem tc_smem_layout(int BNq, int K) {
-  constexpr int S = tc_stages<MODE, TOPK, BN>();
+  constexpr int S = tc_stages<MODE, TOPK, BN, AT>();
   TcSmem l;
-  l.sq = S * tc_stage_bytes<MODE, BN>();
+  l.sq = S * tc_stage_bytes<MODE, BN, AT>();
   l.bars = l.sq + 2 * BN * 4;  // query scales, double-buffered by module
-  l.lists = l.bars + (2 * S + 2 * tc_dbufs<BN>()) * 8 + 16;
+  l.lists = l.bars + (2 * S + 2 * kMaxDbufs) * 8 + 16;
   // per-column held count, own threshold and shared threshold (the list buffers
   // themselves are in global memory)
   l.total = l.lists + (TOPK ? BN * 12 + 8 * 4 * 4 : 0);
@@ -181,6 +200,19 @@ __device__ __forceinline__ void expand_half(uint8_t* row, int sw, int half, uint
   }
 }
 
+// Half a stage of one stored row -> 16 TMEM columns of e4m3 (column n holds
+// elements 4n..4n+3 of the half: bits 4n..4n+3), stored without waiting.
+__device__ __forceinline__ void expand_half_tmem(uint32_t taddr, uint2 bits) {
+  uint32_t v[16];
+#pragma unroll
+  for (int n = 0; n < 8; ++n) {
+    v[n] = e4m3x4((bits.x >> (4 * n)) & 0xFu);
+    v[8 + n] = e4m3x4((bits.y >> (4 * n)) & 0xFu);
+  }
+  tmem_st16_issue(taddr, v);
+}
+__device__ __forceinline__ void expand_half_tmem(uint32_t, uint32_t) {}  // bf16: shared memory only
+
 // Tiles of a CTA. Dense output: strided over the grid, so all CTAs work on the
 // same query tile at a time. Ranking: a contiguous run of tiles, so a CTA
 // ranks long runs of stored rows of one query tile (fewer fresh lists).
@@ -197,22 +229,25 @@ __device__ __forceinline__ int tile_step() {
   return TOPK ? 1 : gridDim.x;
 }
 
-template <int MODE, bool TOPK, int BN>
+template <int MODE, bool TOPK, int BN, bool AT>
 __global__ void __launch_bounds__(kThreadsTc, 1)
     k_score_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQlo,
                const __grid_constant__ ScoreTcArgs g) {
-  constexpr int S = tc_stages<MODE, TOPK, BN>();
-  constexpr uint32_t kStage = tc_stage_bytes<MODE, BN>();
+  static_assert(!AT || MODE == EOGP_SCORE_CODES, "operand A in TMEM is the e4m3 (one-bit) path");
+  constexpr int S = tc_stages<MODE, TOPK, BN, AT>();
+  constexpr uint32_t kStage = tc_stage_bytes<MODE, BN, AT>();
+  constexpr uint32_t kBOff = tc_b_offset<AT>();
   constexpr int kBits = TcMode<MODE>::kBits;
-  constexpr int ND = tc_dbufs<BN>();
-  constexpr uint32_t kAcc = static_cast<uint32_t>(ND * BN);  // running-score columns (BN == 128 only)
+  constexpr int ND = tc_dbufs<BN, AT>();
+  // running-score columns: only 128-query tiles keep one (several modules)
+  constexpr uint32_t kAcc = static_cast<uint32_t>(ND * BN);
   using HalfBits = typename TcMode<MODE>::HalfBits;
   constexpr int kG = 8;  // stages of code bits prefetched at a time
-  constexpr int kP = tc_group<MODE, TOPK, BN>();
+  constexpr int kP = tc_group<MODE, TOPK, BN, AT>();
   static_assert(kG % kP == 0, "prefetch groups hold whole expansion rounds");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  const TcSmem L = tc_smem_layout<MODE, TOPK, BN>(g.BNq, g.K);
+  const TcSmem L = tc_smem_layout<MODE, TOPK, BN, AT>(g.BNq, g.K);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   float* sq = reinterpret_cast<float*>(smem + L.sq);  // [2][BN] query scales of module u (CODES)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bars);
@@ -250,6 +285,27 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
     // per tile) two stages are filled per wait, proxy fence and arrive round.
     const int r = threadIdx.x & 127, half = threadIdx.x >> 7;  // stored row, half of its stage
     const uint32_t row_off = static_cast<uint32_t>((r >> 3) * 1024 + (r & 7) * 128);
+    // TMEM A: this thread's row is TMEM lane r (warp w holds lanes 32 (w % 4) ..),
+    // its half stage 16 columns of the stage's A slot.
+    const uint32_t a_lane = tmem + (static_cast<uint32_t>(r & ~31) << 16) + 16u * static_cast<uint32_t>(half);
+    auto put = [&](int s, uint8_t* st, HalfBits bits) {
+      if constexpr (AT) {
+        tc_fence_after();  // the MMAs that read the slot before (released through empty[s]) are done
+        expand_half_tmem(a_lane + tc_acol<BN>(s), bits);
+      } else {
+        expand_half(st + row_off, r & 7, half, bits);
+      }
+    };
+    // the half stages written so far become visible to the MMA issuer once the
+    // warp's lane 0 arrives on the stage's barrier
+    auto publish = [&]() {
+      if constexpr (AT) {
+        tmem_wait_st();
+        tc_fence_before();
+      } else {
+        fence_proxy_async_smem();
+      }
+    };
     const int nst = g.D / kBits;
     uint32_t it = 0;
     bool ok = true;
@@ -284,12 +340,12 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
                 uint8_t* st = smem + static_cast<size_t>(s) * kStage;
                 if (warp == 0 && lane == 0) {
                   mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(g.BNq) * 128u * TcMode<MODE>::kQBoxes);
-                  tma_load_2d(st + kAB, &tmQ, j * kBits, q0, &full[s]);
+                  tma_load_2d(st + kBOff, &tmQ, j * kBits, q0, &full[s]);
                   if (MODE == EOGP_SCORE_PAPER)
-                    tma_load_2d(st + kAB + static_cast<uint32_t>(BN) * 128u, &tmQlo, j * kBits, q0, &full[s]);
+                    tma_load_2d(st + kBOff + static_cast<uint32_t>(BN) * 128u, &tmQlo, j * kBits, q0, &full[s]);
                 }
-                expand_half(st + row_off, r & 7, half, cur[jj]);
-                fence_proxy_async_smem();
+                put(s, st, cur[jj]);
+                publish();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&full[s]);
               }
@@ -319,15 +375,15 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
                 if (warp == 0 && lane == 0) {
                   const uint32_t qbytes = static_cast<uint32_t>(g.BNq) * 128u * TcMode<MODE>::kQBoxes;
                   mbar_arrive_expect_tx(&full[s0], qbytes);
-                  tma_load_2d(st0 + kAB, &tmQ, j * kBits, q0, &full[s0]);
+                  tma_load_2d(st0 + kBOff, &tmQ, j * kBits, q0, &full[s0]);
                   if (two) {
                     mbar_arrive_expect_tx(&full[s1], qbytes);
-                    tma_load_2d(st1 + kAB, &tmQ, (j + 1) * kBits, q0, &full[s1]);
+                    tma_load_2d(st1 + kBOff, &tmQ, (j + 1) * kBits, q0, &full[s1]);
                   }
                 }
-                expand_half(st0 + row_off, r & 7, half, cur[jj]);
-                if (two) expand_half(st1 + row_off, r & 7, half, cur[jj + 1]);
-                fence_proxy_async_smem();
+                put(s0, st0, cur[jj]);
+                if (two) put(s1, st1, cur[jj + 1]);
+                publish();
                 __syncwarp();
                 if (lane == 0) {
                   mbar_arrive(&full[s0]);
@@ -586,7 +642,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
             for (int kk = 0; kk < 4; ++kk) {
               const uint64_t ad = sdesc_sw128(sa + kk * 32, 16, 1024);
               const uint32_t acc = (kb | kk) != 0 ? 1u : 0u;
-              if (MODE == EOGP_SCORE_CODES) {
+              if constexpr (AT) {
+                tc_mma_f8_ta(d, tmem + tc_acol<BN>(s) + 8u * kk, sdesc_sw128(sa + kk * 32, 16, 1024), idesc, acc);
+              } else if (MODE == EOGP_SCORE_CODES) {
                 tc_mma_f8(d, ad, sdesc_sw128(sa + kAB + kk * 32, 16, 1024), idesc, acc);
               } else {
                 tc_mma_f16(d, ad, sdesc_sw128(sa + kAB + kk * 32, 16, 1024), idesc, acc);
@@ -637,15 +695,28 @@ __global__ void k_split_queries(const float* __restrict__ y, int ldq, int D,
   }
 }
 
-template <int MODE, bool TOPK, int BN>
+template <int MODE, bool TOPK, int BN, bool AT = false>
 size_t tc_smem_need(int BNq, int K) {
-  return 1024 + tc_smem_layout<MODE, TOPK, BN>(BNq, K).total;
+  return 1024 + tc_smem_layout<MODE, TOPK, BN, AT>(BNq, K).total;
+}
+
+// Operand A of the one-bit (CODES) kernel in TMEM unless EOGP_SCORE_AT = 0
+// (shared memory, for comparisons; read at every call).
+bool tc_a_in_tmem(int mode) {
+  if (mode != EOGP_SCORE_CODES) return false;
+  const char* e = getenv("EOGP_SCORE_AT");
+  return !(e && atoi(e) == 0);
 }
 
 // Queries per tile: 256 for CODES with one module and enough queries (when the
-// shared memory allows), else 128.
+// shared memory allows), else 128. (Measured with operand A in TMEM on the
+// 4.2M-code scan at Q = 1024: 48.0 ms with 256-query tiles and one accumulator,
+// 63.2 ms with 192-query tiles and two: the expansion is repeated per query
+// tile.) EOGP_SCORE_BN = 128 forces 128 (comparisons).
 int tc_bn(int mode, int U, int Q, int K) {
-  if (mode == EOGP_SCORE_CODES && U == 1 && Q >= 256 &&
+  const char* e = getenv("EOGP_SCORE_BN");
+  const bool force128 = e && atoi(e) == 128;
+  if (mode == EOGP_SCORE_CODES && U == 1 && Q >= 256 && !force128 &&
       (K == 0 || tc_smem_need<EOGP_SCORE_CODES, true, 256>(256, K) <= 232448))
     return 256;
   return 128;
@@ -653,23 +724,28 @@ int tc_bn(int mode, int U, int Q, int K) {
 
 int bnq_for(int Q, int BN) { return std::min(BN, (Q + 31) / 32 * 32); }
 
-template <int MODE, bool TOPK, int BN>
+template <int MODE, bool TOPK, int BN, bool AT>
 cudaError_t launch_tc_kernel(const CUtensorMap& t0, const CUtensorMap& t1, const ScoreTcArgs& g,
                              int grid, cudaStream_t st) {
-  const size_t smem = tc_smem_need<MODE, TOPK, BN>(g.BNq, g.K);
-  cudaError_t e = cudaFuncSetAttribute(k_score_tc<MODE, TOPK, BN>,
+  const size_t smem = tc_smem_need<MODE, TOPK, BN, AT>(g.BNq, g.K);
+  cudaError_t e = cudaFuncSetAttribute(k_score_tc<MODE, TOPK, BN, AT>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  k_score_tc<MODE, TOPK, BN><<<grid, kThreadsTc, smem, st>>>(t0, t1, g);
+  k_score_tc<MODE, TOPK, BN, AT><<<grid, kThreadsTc, smem, st>>>(t0, t1, g);
   return cudaGetLastError();
 }
 
 template <bool TOPK>
 cudaError_t dispatch_tc(int mode, int BN, const CUtensorMap& t0, const CUtensorMap& t1, const ScoreTcArgs& g,
                         int grid, cudaStream_t st) {
-  if (mode == EOGP_SCORE_PAPER) return launch_tc_kernel<EOGP_SCORE_PAPER, TOPK, 128>(t0, t1, g, grid, st);
-  if (BN == 256) return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 256>(t0, t1, g, grid, st);
-  return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 128>(t0, t1, g, grid, st);
+  if (BN == 256 && g.U != 1) return cudaErrorInvalidValue;  // 256-query tiles keep no running score
+  if (mode == EOGP_SCORE_PAPER) return launch_tc_kernel<EOGP_SCORE_PAPER, TOPK, 128, false>(t0, t1, g, grid, st);
+  if (tc_a_in_tmem(mode)) {
+    if (BN == 256) return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 256, true>(t0, t1, g, grid, st);
+    return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 128, true>(t0, t1, g, grid, st);
+  }
+  if (BN == 256) return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 256, false>(t0, t1, g, grid, st);
+  return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 128, false>(t0, t1, g, grid, st);
 }
 
 }  // namespace
@@ -717,7 +793,7 @@ bool score_tc_topk_fits(int mode, int U, int Q, int K) {
   const int BN = tc_bn(mode, U, Q, K);
   const int bq = bnq_for(Q, BN);
   const size_t need = mode == EOGP_SCORE_PAPER ? tc_smem_need<EOGP_SCORE_PAPER, true, 128>(bq, K)
-                      : BN == 256              ? tc_smem_need<EOGP_SCORE_CODES, true, 256>(bq, K)
+                      : BN > 128               ? tc_smem_need<EOGP_SCORE_CODES, true, 256>(bq, K)
                                                : tc_smem_need<EOGP_SCORE_CODES, true, 128>(bq, K);
   return need <= 232448;
 }
