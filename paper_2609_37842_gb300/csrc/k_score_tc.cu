@@ -114,8 +114,17 @@ constexpr uint32_t tc_b_offset() {
 // 128 (A slots in columns 384-511).
 template <int MODE, bool TOPK, int BN, bool AT>
 constexpr int tc_stages() {
-  return AT ? (BN == 256 ? 6 : 4) : ((MODE == EOGP_SCORE_CODES && BN == 128) ? 6 : 4);
+  return AT ? (BN == 256 ? 6 : 8) : ((MODE == EOGP_SCORE_CODES && BN == 128) ? 6 : 4);
 }
+
+// 128-query tiles with operand A in TMEM keep the running score in shared
+// memory (row stride kAccLd floats: conflict-free float4 rows), leaving 256
+// TMEM columns for eight A slots next to the two d_u accumulators.
+template <int BN, bool AT>
+constexpr bool tc_acc_smem() {
+  return AT && BN == 128;
+}
+constexpr int kAccLd = 132;
 
 // Stages the expanders fill per synchronisation round (one wait, fence and
 // arrive round): two with six stages, so that the MMAs always have at least
@@ -134,21 +143,23 @@ constexpr int tc_dbufs() {
 }
 constexpr int kMaxDbufs = 3;
 
-// First TMEM column of A slot s (TMEM A), after the accumulators.
+// First TMEM column of A slot s (TMEM A), after the accumulators (one of 256
+// columns, or two of 128).
 template <int BN>
 __device__ __forceinline__ uint32_t tc_acol(int s) {
-  return static_cast<uint32_t>((BN == 256 ? 256 : 384) + 32 * s);
+  return static_cast<uint32_t>(256 + 32 * s);
 }
 
 // Shared-memory carve-up (byte offsets after 1024-byte alignment).
 struct TcSmem {
-  uint32_t sq, bars, lists, total;
+  uint32_t acc, sq, bars, lists, total;
 };
 template <int MODE, bool TOPK, int BN, bool AT>
 __host__ __device__ inline TcSmem tc_smem_layout(int BNq, int K) {
   constexpr int S = tc_stages<MODE, TOPK, BN, AT>();
   TcSmem l;
-  l.sq = S * tc_stage_bytes<MODE, BN, AT>();
+  l.acc = S * tc_stage_bytes<MODE, BN, AT>();
+  l.sq = l.acc + (tc_acc_smem<BN, AT>() ? 128u * kAccLd * 4u : 0u);
   l.bars = l.sq + 2 * BN * 4;  // query scales, double-buffered by module
   l.lists = l.bars + (2 * S + 2 * kMaxDbufs) * 8 + 16;
   // per-column held count, own threshold and shared threshold (the list buffers
@@ -244,6 +255,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   using HalfBits = typename TcMode<MODE>::HalfBits;
   constexpr int kG = 8;  // stages of code bits prefetched at a time
   constexpr int kP = tc_group<MODE, TOPK, BN, AT>();
+  constexpr bool kAccS = tc_acc_smem<BN, AT>();
   static_assert(kG % kP == 0, "prefetch groups hold whole expansion rounds");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
@@ -543,6 +555,16 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
         const bool last = u + 1 == g.U;
         const uint32_t dcol = tmem + lane_base + buf * static_cast<uint32_t>(BN);
         const uint32_t acol = tmem + lane_base + kAcc;
+        float* accrow = reinterpret_cast<float*>(smem + L.acc) + ep * kAccLd;  // kAccS: this row's running score
+        auto acc_load = [&](int c0, uint32_t* ar, int n) {  // n floats from the shared running score
+          for (int j = 0; j < n; j += 4) {
+            const float4 v = *reinterpret_cast<const float4*>(accrow + c0 + j);
+            ar[j] = __float_as_uint(v.x);
+            ar[j + 1] = __float_as_uint(v.y);
+            ar[j + 2] = __float_as_uint(v.z);
+            ar[j + 3] = __float_as_uint(v.w);
+          }
+        };
         // the module's term: fl(fl(s_q s_i) d) (CODES) or fl(s_i d) (PAPER)
         auto term = [&](int c, uint32_t dv) {
           return MODE == EOGP_SCORE_CODES ? __fmul_rn(__fmul_rn(sqb[c], si), __uint_as_float(dv))
@@ -553,7 +575,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
           // are in flight while this one is combined and stored back.
           uint32_t dr[16], ar[16];
           tmem_ld16_issue(dcol, dr);
-          if (u > 0) {
+          if (!kAccS && u > 0) {
             tmem_ld16_issue(acol, ar);
           } else {
 #pragma unroll
@@ -564,31 +586,45 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
             const int c0 = 16 * ci;
             if (c0 < g.BNq) {
               tmem_wait_ld(dr);
-              tmem_wait_ld(ar);
+              if constexpr (kAccS) {
+                if (u > 0) acc_load(c0, ar, 16);
+              } else {
+                tmem_wait_ld(ar);
+              }
               uint32_t o[16];
 #pragma unroll
               for (int j = 0; j < 16; ++j)
                 o[j] = __float_as_uint(__fadd_rn(__uint_as_float(ar[j]), term(c0 + j, dr[j])));
               if (c0 + 16 < g.BNq) {
                 tmem_ld16_issue(dcol + c0 + 16, dr);
-                if (u > 0) tmem_ld16_issue(acol + c0 + 16, ar);
+                if (!kAccS && u > 0) tmem_ld16_issue(acol + c0 + 16, ar);
               }
-              tmem_st16_issue(acol + c0, o);
+              if constexpr (kAccS) {
+#pragma unroll
+                for (int j = 0; j < 16; j += 4)
+                  *reinterpret_cast<float4*>(accrow + c0 + j) =
+                      make_float4(__uint_as_float(o[j]), __uint_as_float(o[j + 1]), __uint_as_float(o[j + 2]),
+                                  __uint_as_float(o[j + 3]));
+              } else {
+                tmem_st16_issue(acol + c0, o);
+              }
             }
           }
-          tmem_wait_st();  // stored before the next module reads them
+          if constexpr (!kAccS) tmem_wait_st();  // stored before the next module reads them
         } else {
           for (int c0 = 0; c0 < g.BNq; c0 += 32) {
             uint32_t dr[32], ar[32];
             tmem_ld32_issue(dcol + c0, dr);
-            if (u > 0) {
+            if (u > 0 && kAccS) {
+              acc_load(c0, ar, 32);
+            } else if (u > 0) {
               tmem_ld32_issue(acol + c0, ar);
             } else {
 #pragma unroll
               for (int j = 0; j < 32; ++j) ar[j] = 0u;
             }
             tmem_wait_ld(dr);
-            tmem_wait_ld(ar);
+            if constexpr (!kAccS) tmem_wait_ld(ar);
             float a[32];
 #pragma unroll
             for (int j = 0; j < 32; ++j) a[j] = __fadd_rn(__uint_as_float(ar[j]), term(c0 + j, dr[j]));
@@ -792,9 +828,12 @@ bool score_tc_topk_fits(int mode, int U, int Q, int K) {
   if (K < 1 || K > kTopKMax) return false;
   const int BN = tc_bn(mode, U, Q, K);
   const int bq = bnq_for(Q, BN);
-  const size_t need = mode == EOGP_SCORE_PAPER ? tc_smem_need<EOGP_SCORE_PAPER, true, 128>(bq, K)
-                      : BN > 128               ? tc_smem_need<EOGP_SCORE_CODES, true, 256>(bq, K)
-                                               : tc_smem_need<EOGP_SCORE_CODES, true, 128>(bq, K);
+  const size_t need =
+      mode == EOGP_SCORE_PAPER ? tc_smem_need<EOGP_SCORE_PAPER, true, 128>(bq, K)
+      : BN == 256 ? std::max(tc_smem_need<EOGP_SCORE_CODES, true, 256, false>(bq, K),
+                             tc_smem_need<EOGP_SCORE_CODES, true, 256, true>(bq, K))
+                  : std::max(tc_smem_need<EOGP_SCORE_CODES, true, 128, false>(bq, K),
+                             tc_smem_need<EOGP_SCORE_CODES, true, 128, true>(bq, K));
   return need <= 232448;
 }
 
