@@ -90,9 +90,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
+      int rs = 0;
+      uint32_t rph = 0;
       for (int i = 0; i < nkb; ++i) {
-        const int s = i % g.stages;
-        const uint32_t ph = static_cast<uint32_t>(i / g.stages) & 1u;
+        const int s = rs;
+        const uint32_t ph = rph;
+        if (++rs == g.stages) {
+          rs = 0;
+          rph ^= 1u;
+        }
         if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) break;
         uint8_t* st = smem + static_cast<size_t>(s) * stage_bytes;
         mbar_arrive_expect_tx(&full[s], stage_bytes);
@@ -106,9 +112,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16_f32(128, g.BN, 0, 0);
+      int rs = 0;
+      uint32_t rph = 0;
       for (int i = 0; i < nkb; ++i) {
-        const int s = i % g.stages;
-        const uint32_t ph = static_cast<uint32_t>(i / g.stages) & 1u;
+        const int s = rs;
+        const uint32_t ph = rph;
+        if (++rs == g.stages) {
+          rs = 0;
+          rph ^= 1u;
+        }
         if (!mbar_wait(&full[s], ph, g.status)) break;
         tc_fence_after();
         const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
@@ -250,14 +262,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       uint32_t it = 0;
+      int rs = 0;         // ring slot of pipeline iteration it (it % stages)
+      uint32_t rph = 0;  // and its phase parity ((it / stages) & 1)
       bool ok = true;
       for (int item = blockIdx.x; item < g.n_items && ok; item += gridDim.x) {
         const int b = item / g.n_tiles, tile = item % g.n_tiles;
         const int rc = g.tile_rc[tile];
         const int zs = b * g.nblkS + (rc >> 16), za = b * g.nblkA + (rc & 0xFFFF);
         for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const int s = static_cast<int>(it % g.stages);
-          const uint32_t ph = (it / g.stages) & 1u;
+          const int s = rs;
+          const uint32_t ph = rph;
+          if (++rs == g.stages) {
+            rs = 0;
+            rph ^= 1u;
+          }
           if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) {
             ok = false;
             break;
@@ -281,6 +299,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16_f32(128, 128, 1, 1);
       uint32_t it = 0;
+      int rs = 0;         // ring slot of pipeline iteration it (it % stages)
+      uint32_t rph = 0;  // and its phase parity ((it / stages) & 1)
       int i = 0;
       bool ok = true;
       for (int item = blockIdx.x; item < g.n_items && ok; item += gridDim.x, ++i) {
@@ -290,8 +310,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         const uint32_t d = tmem + buf * 128u;
         for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const int s = static_cast<int>(it % g.stages);
-          const uint32_t ph = (it / g.stages) & 1u;
+          const int s = rs;
+          const uint32_t ph = rph;
+          if (++rs == g.stages) {
+            rs = 0;
+            rph ^= 1u;
+          }
           if (!mbar_wait(&full[s], ph, g.status)) {
             ok = false;
             break;
@@ -425,6 +449,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       uint32_t it = 0;
+      int rs = 0;         // ring slot of pipeline iteration it (it % stages)
+      uint32_t rph = 0;  // and its phase parity ((it / stages) & 1)
       bool ok = true;
       for (int item = blockIdx.x; item < g.n_items && ok; item += gridDim.x) {
         const int chunk = item / g.n_tiles, tile = item % g.n_tiles;
@@ -433,8 +459,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int b = chunk * g.bpc; b < b1 && ok; ++b) {
           const int zs = b * g.nblkS + rt, za = b * g.nblkA + ct;
           for (int kb = 0; kb < nkb; ++kb, ++it) {
-            const int s = static_cast<int>(it % g.stages);
-            const uint32_t ph = (it / g.stages) & 1u;
+            const int s = rs;
+            const uint32_t ph = rph;
+            if (++rs == g.stages) {
+              rs = 0;
+              rph ^= 1u;
+            }
             if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) {
               ok = false;
               break;
@@ -459,6 +489,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16_f32(128, 128, 1, 1);
       uint32_t it = 0;
+      int rs = 0;         // ring slot of pipeline iteration it (it % stages)
+      uint32_t rph = 0;  // and its phase parity ((it / stages) & 1)
       int i = 0;  // examples issued by this CTA (selects the TMEM buffer)
       bool ok = true;
       for (int item = blockIdx.x; item < g.n_items && ok; item += gridDim.x) {
@@ -474,8 +506,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_after();
           const uint32_t d = tmem + buf * 128u;
           for (int kb = 0; kb < nkb; ++kb, ++it) {
-            const int s = static_cast<int>(it % g.stages);
-            const uint32_t ph = (it / g.stages) & 1u;
+            const int s = rs;
+            const uint32_t ph = rph;
+            if (++rs == g.stages) {
+              rs = 0;
+              rph ^= 1u;
+            }
             if (!mbar_wait(&full[s], ph, g.status)) {
               ok = false;
               break;
@@ -699,12 +735,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       uint32_t it = 0;
+      int rs = 0;         // ring slot of pipeline iteration it (it % stages)
+      uint32_t rph = 0;  // and its phase parity ((it / stages) & 1)
       bool ok = true;
       for (int t = blockIdx.x; t < g.n_tiles && ok; t += gridDim.x) {
         const int m0 = (t / g.nN) * 128, n0 = (t % g.nN) * g.BN;
         for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const int s = static_cast<int>(it % g.stages);
-          const uint32_t ph = (it / g.stages) & 1u;
+          const int s = rs;
+          const uint32_t ph = rph;
+          if (++rs == g.stages) {
+            rs = 0;
+            rph ^= 1u;
+          }
           if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) {
             ok = false;
             break;
@@ -719,8 +761,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp == 1) {
     if (lane == 0) {
+      // The issuing thread's own work per K block is kept minimal (one lane issues
+      // every MMA, so its instruction latency paces the tensor pipe): ring slot,
+      // phase and operand descriptors advance incrementally. A descriptor's
+      // address field is (byte address >> 4), so +2 steps 32 bytes (K = 16 bf16).
       const uint32_t idesc = idesc_bf16_f32(128, g.BN, 0, 0);
-      uint32_t it = 0;
+      const uint64_t dbase = sdesc_sw128(smem_u32(smem), 16, 1024);
+      const uint64_t dstage = stage_bytes >> 4, dab = kABytes >> 4;
+      uint64_t da = dbase;  // descriptor of operand A in ring slot rs
+      int rs = 0;           // ring slot of the next K block
+      uint32_t rph = 0;     // and its phase parity
       int i = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < g.n_tiles && ok; t += gridDim.x, ++i) {
@@ -729,21 +779,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(&tempty[buf], aph ^ 1u, g.status)) break;
         tc_fence_after();
         const uint32_t d = tmem + buf * bstride;
-        for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const int s = static_cast<int>(it % g.stages);
-          const uint32_t ph = (it / g.stages) & 1u;
+        for (int kb = 0; kb < nkb; ++kb) {
+          const int s = rs;
+          const uint32_t ph = rph;
+          const uint64_t a0 = da, b0 = da + dab;
+          if (++rs == g.stages) {
+            rs = 0;
+            rph ^= 1u;
+            da = dbase;
+          } else {
+            da += dstage;
+          }
           if (!mbar_wait(&full[s], ph, g.status)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
-          const uint32_t sb = sa + kABytes;
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk) {
-            tc_mma_f16(d, sdesc_sw128(sa + kk * 32, 16, 1024), sdesc_sw128(sb + kk * 32, 16, 1024),
-                       idesc, (kb | kk) != 0 ? 1u : 0u);
-          }
+          tc_mma_f16(d, a0, b0, idesc, kb != 0 ? 1u : 0u);
+          tc_mma_f16(d, a0 + 2, b0 + 2, idesc, 1u);
+          tc_mma_f16(d, a0 + 4, b0 + 4, idesc, 1u);
+          tc_mma_f16(d, a0 + 6, b0 + 6, idesc, 1u);
           tc_commit(&empty[s]);
         }
         tc_commit(&tfull[buf]);
@@ -832,13 +887,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       uint32_t it = 0;
+      int rs = 0;         // ring slot of pipeline iteration it (it % stages)
+      uint32_t rph = 0;  // and its phase parity ((it / stages) & 1)
       bool ok = true;
       for (int t = cl; t < g.n_tiles && ok; t += ncl) {
         const int m0 = (t / g.nN) * 256 + static_cast<int>(rank) * 128;
         const int n0 = (t % g.nN) * g.BN + static_cast<int>(rank) * half;
         for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const int s = static_cast<int>(it % g.stages);
-          const uint32_t ph = (it / g.stages) & 1u;
+          const int s = rs;
+          const uint32_t ph = rph;
+          if (++rs == g.stages) {
+            rs = 0;
+            rph ^= 1u;
+          }
           if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) {
             ok = false;
             break;
@@ -854,8 +915,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp == 1) {
     if (lane == 0 && rank == 0) {
+      // as in k_tc_rotate: slot, phase and descriptors advance incrementally
       const uint32_t idesc = idesc_bf16_f32(256, g.BN, 0, 0);
-      uint32_t it = 0;
+      const uint64_t dbase = sdesc_sw128(smem_u32(smem), 16, 1024);
+      const uint64_t dstage = stage_bytes >> 4, dab = kABytes >> 4;
+      uint64_t da = dbase;
+      int rs = 0;
+      uint32_t rph = 0;
       int i = 0;
       bool ok = true;
       for (int t = cl; t < g.n_tiles && ok; t += ncl, ++i) {
@@ -864,20 +930,26 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (!mbar_wait(&tempty[buf], aph ^ 1u, g.status)) break;
         tc_fence_after();
         const uint32_t d = tmem + buf * bstride;
-        for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const int s = static_cast<int>(it % g.stages);
-          const uint32_t ph = (it / g.stages) & 1u;
+        for (int kb = 0; kb < nkb; ++kb) {
+          const int s = rs;
+          const uint32_t ph = rph;
+          const uint64_t a0 = da, b0 = da + dab;
+          if (++rs == g.stages) {
+            rs = 0;
+            rph ^= 1u;
+            da = dbase;
+          } else {
+            da += dstage;
+          }
           if (!mbar_wait(&full[s], ph, g.status)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
-          const uint32_t sb = sa + kABytes;
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            tc_mma_f16_pair(d, sdesc_sw128(sa + kk * 32, 16, 1024), sdesc_sw128(sb + kk * 32, 16, 1024),
-                            idesc, (kb | kk) != 0 ? 1u : 0u);
+          tc_mma_f16_pair(d, a0, b0, idesc, kb != 0 ? 1u : 0u);
+          tc_mma_f16_pair(d, a0 + 2, b0 + 2, idesc, 1u);
+          tc_mma_f16_pair(d, a0 + 4, b0 + 4, idesc, 1u);
+          tc_mma_f16_pair(d, a0 + 6, b0 + 6, idesc, 1u);
           tc_commit_pair_mc(&empty[s], 0x3);
         }
         tc_commit_pair_mc(&tfull[buf], 0x3);
