@@ -303,6 +303,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t rph = 0;  // and its phase parity ((it / stages) & 1)
       int i = 0;
       bool ok = true;
+      // descriptor of S hi in ring slot rs (MN-major operands: LBO 8192, SBO 1024)
+      const uint64_t dbase = sdesc_sw128(smem_u32(smem), 8192, 1024);
+      uint64_t dsh = dbase;
       for (int item = blockIdx.x; item < g.n_items && ok; item += gridDim.x, ++i) {
         const int buf = i & 1;
         const uint32_t aph = static_cast<uint32_t>(i >> 1) & 1u;
@@ -312,23 +315,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kb = 0; kb < nkb; ++kb, ++it) {
           const int s = rs;
           const uint32_t ph = rph;
+          const uint64_t sh0 = dsh;  // S hi of this slot; S lo, A hi, A lo follow kOpBytes apart
           if (++rs == g.stages) {
             rs = 0;
             rph ^= 1u;
+            dsh = dbase;
+          } else {
+            dsh += kCStage >> 4;
           }
           if (!mbar_wait(&full[s], ph, g.status)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * kCStage);
+          constexpr uint64_t kOp = kOpBytes >> 4, kRow16 = 2048u >> 4;  // 16 token rows of 128 bytes
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk) {
-            const uint32_t o = kk * 2048u;  // 16 token rows of 128 bytes
-            const uint64_t sh = sdesc_sw128(sa + 0 * kOpBytes + o, 8192, 1024);
-            const uint64_t sl = sdesc_sw128(sa + 1 * kOpBytes + o, 8192, 1024);
-            const uint64_t ah = sdesc_sw128(sa + 2 * kOpBytes + o, 8192, 1024);
-            const uint64_t al = sdesc_sw128(sa + 3 * kOpBytes + o, 8192, 1024);
+            const uint64_t sh = sh0 + kk * kRow16, sl = sh + kOp, ah = sh + 2 * kOp, al = sh + 3 * kOp;
             tc_mma_f16(d, sh, ah, idesc, (kb | kk) != 0 ? 1u : 0u);
             tc_mma_f16(d, sh, al, idesc, 1u);
             tc_mma_f16(d, sl, ah, idesc, 1u);
