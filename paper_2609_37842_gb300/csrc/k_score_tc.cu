@@ -651,7 +651,14 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
     if (lane == 0) {
       const uint32_t idesc =
           MODE == EOGP_SCORE_CODES ? idesc_e4m3_f32(128, g.BNq) : idesc_bf16_f32(128, g.BNq, 0, 0);
-      uint32_t it = 0, gm = 0;
+      // One lane issues every MMA, so its own work per stage is kept minimal:
+      // ring slot, phase, A slot and descriptors advance incrementally (a
+      // descriptor's address field is byte address >> 4: +2 steps 32 bytes).
+      const uint64_t dbase = sdesc_sw128(smem_u32(smem), 16, 1024);
+      uint64_t dst = dbase;  // descriptor of ring slot rs (its first operand tile)
+      uint32_t acl = tmem + tc_acol<BN>(0);  // TMEM A slot of ring slot rs (AT)
+      int rs = 0;
+      uint32_t rph = 0, gm = 0;
       bool ok = true;
       for (int tile = tile_begin<TOPK>(g), tstep = tile_step<TOPK>(), tend = tile_end<TOPK>(g);
            tile < tend && ok; tile += tstep) {
@@ -665,26 +672,36 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
           tc_fence_after();
           const uint32_t d = tmem + buf * static_cast<uint32_t>(BN);
           const int nkb = g.k[u] / kBits;
-          for (int kb = 0; kb < nkb; ++kb, ++it) {
-            const int s = static_cast<int>(it % S);
-            const uint32_t ph = (it / S) & 1u;
+          for (int kb = 0; kb < nkb; ++kb) {
+            const int s = rs;
+            const uint32_t ph = rph;
+            const uint64_t a0 = dst;  // A (shared-memory A) or the query operand (TMEM A)
+            const uint64_t b0 = dst + (kAB >> 4), b1 = b0 + ((static_cast<uint32_t>(BN) * 128u) >> 4);
+            const uint32_t at0 = acl;
+            if (++rs == S) {
+              rs = 0;
+              rph ^= 1u;
+              dst = dbase;
+              acl = tmem + tc_acol<BN>(0);
+            } else {
+              dst += kStage >> 4;
+              acl += 32u;
+            }
             if (!mbar_wait(&full[s], ph, g.status)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t sa = smem_u32(smem + static_cast<size_t>(s) * kStage);
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
-              const uint64_t ad = sdesc_sw128(sa + kk * 32, 16, 1024);
               const uint32_t acc = (kb | kk) != 0 ? 1u : 0u;
               if constexpr (AT) {
-                tc_mma_f8_ta(d, tmem + tc_acol<BN>(s) + 8u * kk, sdesc_sw128(sa + kk * 32, 16, 1024), idesc, acc);
+                tc_mma_f8_ta(d, at0 + 8u * kk, a0 + 2 * kk, idesc, acc);
               } else if (MODE == EOGP_SCORE_CODES) {
-                tc_mma_f8(d, ad, sdesc_sw128(sa + kAB + kk * 32, 16, 1024), idesc, acc);
+                tc_mma_f8(d, a0 + 2 * kk, b0 + 2 * kk, idesc, acc);
               } else {
-                tc_mma_f16(d, ad, sdesc_sw128(sa + kAB + kk * 32, 16, 1024), idesc, acc);
-                tc_mma_f16(d, ad, sdesc_sw128(sa + kAB + BN * 128u + kk * 32, 16, 1024), idesc, 1u);
+                tc_mma_f16(d, a0 + 2 * kk, b0 + 2 * kk, idesc, acc);
+                tc_mma_f16(d, a0 + 2 * kk, b1 + 2 * kk, idesc, 1u);
               }
             }
             tc_commit(&empty[s]);
