@@ -43,7 +43,7 @@ METRIC = "training examples compressed/sec per layer stack"
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # dram__bytes_read.sum + dram__bytes_write.sum per rotation launch from the committed
 # ncu capture (profiles/), or None when the kernel changed after the capture.
-ROTATE_TRAFFIC_BYTES = 1415.5e6  # mean over one transformer block (8 launches) at B = 512
+ROTATE_TRAFFIC_BYTES = 1415.1e6  # mean over one transformer block (8 launches) at B = 512
 
 
 def load_peaks():

@@ -13,6 +13,7 @@
 #include <unistd.h>
 
 #include <cstdio>
+#include <cstring>
 #include <cstdint>
 #include <mutex>
 #include <unordered_map>
@@ -67,6 +68,10 @@ extern "C" int eogp_host_alloc(size_t bytes, void** ptr) {
   if (tail) munmap(reinterpret_cast<void*>(a + len), tail);
   void* p = reinterpret_cast<void*>(a);
   madvise(p, len, MADV_HUGEPAGE);  // advice only: without it the region still works
+  // Fault the region in from the CPU before registering it, so that the pages
+  // are placed by ordinary first-touch faults on the advised, aligned range:
+  // the configuration the ~211 GB/s copy rate above was measured with.
+  std::memset(p, 0, len);
   const cudaError_t e = cudaHostRegister(p, len, cudaHostRegisterDefault);
   if (e != cudaSuccess) {
     munmap(p, len);
