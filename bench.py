@@ -46,6 +46,25 @@ PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 ROTATE_TRAFFIC_BYTES = 1415.1e6  # mean over one transformer block (8 launches) at B = 512
 
 
+def score_peak(ks, probes, bf16_burst, peaks_src):
+    """Denominator of a one-bit tensor-core scoring rate: the measured rate of the
+    MMA the library issues for these module sizes (e2m1 kind::mxf4 when every
+    module is a multiple of 256 bits, else e4m3 kind::f8f6f4), as (TFLOP/s,
+    source, mode label). Without the probes: the bf16 burst peak times the
+    nominal dense ratio (fp8 2x, fp4 6x)."""
+    f4 = (os.environ.get("EOGP_SCORE_F4", "1") != "0" and os.environ.get("EOGP_SCORE_AT", "1") != "0"
+          and all(k % 256 == 0 for k in ks))
+    if f4:
+        mode = "tcgen05 kind::mxf4, +-1 e2m1 operands, unit ue8m0 scales"
+        if probes:
+            return probes["e2m1_tflops"], "eogp_measure_peaks e2m1", mode
+        return 6.0 * bf16_burst, f"6 x {peaks_src} bf16_tflops (nominal fp4 ratio)", mode
+    mode = "tcgen05 kind::f8f6f4, +-1 e4m3 operands"
+    if probes:
+        return probes["e4m3_tflops"], "eogp_measure_peaks e4m3", mode
+    return 2.0 * bf16_burst, f"2 x {peaks_src} bf16_tflops (nominal fp8 ratio)", mode
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -611,10 +630,10 @@ def main():
     # ---- measured e4m3 tensor-core and popcount rates (scoring rooflines) ----
     probes = None
     if rank == 0 and not args.no_score:
-        f8, pc = E.measure_peaks()
-        probes = {"e4m3_tflops": f8, "popc_words_per_s": pc,
-                  "what": "eogp_measure_peaks: back-to-back kind::f8f6f4 MMAs from shared memory; "
-                          "XOR + popcount chains on every core"}
+        f8, f4, pc = E.measure_peaks()
+        probes = {"e4m3_tflops": f8, "e2m1_tflops": f4, "popc_words_per_s": pc,
+                  "what": "eogp_measure_peaks: back-to-back kind::f8f6f4 (e4m3) and kind::mxf4 (e2m1, unit "
+                          "scales) MMAs; XOR + popcount chains on every core"}
 
     # ---- context: cuBLAS bf16 on the largest rotation shape (not on the path) ----
     ref_gemm = None
@@ -661,15 +680,15 @@ def main():
         E.sync_status()
         sms = e0.elapsed_time(e1) / reps
         D = U * w.k
-        f8_peak = probes["e4m3_tflops"] if probes else 2.0 * bf16_burst
+        pk, pk_src, pk_mode = score_peak(ks, probes, bf16_burst, peaks_src)
         alg = 2.0 * N * Q * D               # +-1 multiply-adds of the inner products
         scoring = {"metric": "query x train scores/sec", "value": N * Q / (sms / 1000.0),
                    "unit": "scores/s", "ms_per_call": sms, "N": N, "Q": Q, "bits": D,
-                   "mode": "CODES (tcgen05 kind::f8f6f4, +-1 e4m3 operands)",
+                   "mode": f"CODES ({pk_mode})",
                    "tensor_TFLOPs": alg / (sms / 1000.0) / 1e12,
-                   "tensor_frac": alg / (sms / 1000.0) / 1e12 / f8_peak,
-                   "tensor_peak": f8_peak,
-                   "tensor_peak_source": "eogp_measure_peaks e4m3" if probes else f"2 x {peaks_src} bf16_tflops"}
+                   "tensor_frac": alg / (sms / 1000.0) / 1e12 / pk,
+                   "tensor_peak": pk,
+                   "tensor_peak_source": pk_src}
         # paper mode (unquantised queries), dense and with the ranking fused (K = 20)
         y = torch.randn((Q, D), generator=g, device=dev)
         wsp = E.workspace(E.score_workspace_size(N, ks, E.SCORE_PAPER, Q), dev)
@@ -839,12 +858,11 @@ def main():
             ent = {"ms": qms, "scores_per_s": N * Q / (qms / 1000.0),
                    "GBps": byts / (qms / 1000.0) / 1e9,
                    "frac_of_hbm": byts / (qms / 1000.0) / 1e9 / hbm}
-            if Q >= 64:   # tensor-core kernel: +-1 multiply-adds against the e4m3 peak
+            if Q >= 64:   # tensor-core kernel: +-1 multiply-adds against the rate of the MMA it issues
                 tfl = 2.0 * N * ksc * Q / (qms / 1000.0) / 1e12
-                ent.update({"kernel": "k_score_tc", "tensor_TFLOPs": tfl,
-                            "tensor_frac": tfl / (probes["e4m3_tflops"] if probes else 2.0 * bf16_burst),
-                            "tensor_peak_source": "eogp_measure_peaks e4m3" if probes
-                            else "2 x measured bf16 burst"})
+                pk, pk_src, pk_mode = score_peak([ksc], probes, bf16_burst, peaks_src)
+                ent.update({"kernel": f"k_score_tc ({pk_mode})", "tensor_TFLOPs": tfl,
+                            "tensor_frac": tfl / pk, "tensor_peak_source": pk_src})
             else:
                 wops = N * Q * Wsc / (qms / 1000.0)
                 ent.update({"kernel": "k_score_codes_smallq (popcount)", "word_ops_per_s": wops})

@@ -98,11 +98,13 @@ int eogp_profile_read(int kind, int* launches, double* total_ms, int reset);
 
 /* Throughput probes for the scoring rooflines (no counterpart in the paper: a
  * library convenience). Measures on the current device, synchronously: the dense
- * tcgen05 kind::f8f6f4 e4m3 rate (TFLOP/s, back-to-back M = 128, N = 256, K = 32
- * MMAs from shared memory, one CTA per SM) and the CUDA-core XOR + popcount rate
- * (32-bit words per second). Either output may be NULL.
+ * tcgen05 rates of the two +-1 scoring MMAs in TFLOP/s (one CTA per SM issuing
+ * back-to-back M = 128, N = 256 MMAs: kind::f8f6f4 e4m3 with K = 32 from shared
+ * memory, kind::mxf4 e2m1 with unit ue8m0 scales, K = 64, A from tensor memory)
+ * and the CUDA-core XOR + popcount rate (32-bit words per second). Any output
+ * may be NULL.
  * Errors: EOGP_ECUDA, EOGP_ETIMEOUT. */
-int eogp_measure_peaks(double* e4m3_tflops, double* popc_words_per_s);
+int eogp_measure_peaks(double* e4m3_tflops, double* e2m1_tflops, double* popc_words_per_s);
 
 /* ========================================================================
  * Retained-set plan (host; once per module)

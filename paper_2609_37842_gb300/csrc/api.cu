@@ -1006,18 +1006,19 @@ extern "C" int eogp_payload_unpack(const uint8_t* payload, size_t ld_payload, in
 
 // ================================================================ probes
 
-extern "C" int eogp_measure_peaks(double* e4m3_tflops, double* popc_words_per_s) {
+extern "C" int eogp_measure_peaks(double* e4m3_tflops, double* e2m1_tflops, double* popc_words_per_s) {
   clear_error();
   unsigned* status = status_word();
   if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
   unsigned* sink = nullptr;
   CUDA_TRY(cudaMalloc(reinterpret_cast<void**>(&sink), sizeof(unsigned)));
-  double f8 = 0.0, pc = 0.0;
-  const cudaError_t e = run_peak_probes(sm_count(), status, sink, &f8, &pc, nullptr);
+  double f8 = 0.0, f4 = 0.0, pc = 0.0;
+  const cudaError_t e = run_peak_probes(sm_count(), status, sink, &f8, &f4, &pc, nullptr);
   cudaFree(sink);
   if (e != cudaSuccess) return set_error(EOGP_ECUDA, "%s", cudaGetErrorString(e));
   if (int rc = eogp_sync_status(nullptr)) return rc;
   if (e4m3_tflops) *e4m3_tflops = f8;
+  if (e2m1_tflops) *e2m1_tflops = f4;
   if (popc_words_per_s) *popc_words_per_s = pc;
   return EOGP_OK;
 }

@@ -248,6 +248,22 @@ __device__ __forceinline__ void tc_mma_f8(uint32_t d_tmem, uint64_t adesc, uint6
       : "memory");
 }
 
+// Block-scaled e2m1 MMA (kind::mxf4, K = 64 per instruction, one ue8m0 scale
+// per 32 elements) with operand A in tensor memory: a_tmem addresses the first
+// of 8 columns (8 e2m1 values per 32-bit column, element 8n + i in bits 4i..4i+3
+// of column n); B from shared memory as in tc_mma_f8 (two e2m1 per byte, the
+// lower K index in the low nibble); sfa / sfb address the scale factors in TMEM.
+__device__ __forceinline__ void tc_mma_f4_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                             uint32_t sfa, uint32_t sfb, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %6, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%0], [%1], %2, %3, [%4], [%5], p;\n\t}\n" ::"r"(
+          d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
+      : "memory");
+}
+
 // Same MMA with operand A in tensor memory: a_tmem addresses the first of the
 // K / 4 32-bit columns holding A (TMEM lane = row of A, four e4m3 elements per
 // column, element 4c + e in byte e of column c).
@@ -427,6 +443,16 @@ __host__ __device__ constexpr uint32_t idesc_e4m3_f32(int M, int N) {
          | (0u << 10)                             // B format: e4m3
          | (static_cast<uint32_t>(N >> 3) << 17)  // N / 8
          | (static_cast<uint32_t>(M >> 4) << 24); // M / 16
+}
+
+// Instruction descriptor for kind::mxf4 (block-scaled e2m1 A and B, fp32 D):
+// A, B format e2m1, K-major, scale format ue8m0, scale-factor ids 0, dense K = 64.
+__host__ __device__ constexpr uint32_t idesc_mxf4_f32(int M, int N) {
+  return (1u << 7)                                 // A format: e2m1
+         | (1u << 10)                              // B format: e2m1
+         | (static_cast<uint32_t>(N >> 3) << 17)   // N / 8
+         | (1u << 23)                              // scale format: ue8m0
+         | (static_cast<uint32_t>(M >> 4) << 24);  // M / 16
 }
 
 // Instruction descriptor for kind::f16 with bf16 A/B and fp32 D.

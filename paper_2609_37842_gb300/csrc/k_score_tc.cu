@@ -2,10 +2,12 @@
 // in two modes and with two outputs.
 //
 // CODES: both sides one-bit. For module u the +-1 inner product d_u = <b_q, b_i>
-//   is an integer with |d_u| <= k_u. Both sides are expanded to e4m3 bytes
-//   (+1 = 0x38, -1 = 0xB8, exact) and multiplied with tcgen05.mma kind::f8f6f4
-//   into fp32 TMEM: every partial sum is an integer far below 2^24, so d_u is
-//   exact. The epilogue dequantises in the same fixed fp32 order as the
+//   is an integer with |d_u| <= k_u. Both sides are expanded to +-1 and
+//   multiplied on the tensor cores into fp32 TMEM: as e2m1 values (+1 = 0x2,
+//   -1 = 0xA) with tcgen05.mma kind::mxf4 and every block scale 1 when each
+//   module is a multiple of 256 bits (twice the e4m3 rate), else as e4m3 bytes
+//   (+1 = 0x38, -1 = 0xB8) with kind::f8f6f4. Both encodings are exact and
+//   every partial sum is an integer far below 2^24, so d_u is exact. The epilogue dequantises in the same fixed fp32 order as the
 //   popcount kernels, acc = fl(acc + fl(fl(s_qu * s_iu) * d_u)) in module order,
 //   keeping acc in TMEM between modules, so scores are bitwise identical to the
 //   popcount path and to the oracle's float32 evaluation.
@@ -26,11 +28,11 @@
 // matrix never reaches HBM.
 //
 // Tiles: 128 stored rows (MMA M, operand A) x BNq queries (MMA N, operand B),
-// BNq <= 256 for CODES with one module, else <= 128. Queries are prepared once
-// per call in the workspace (e4m3 bytes, or bf16 hi and lo rows) and fetched
-// by TMA; stored rows are expanded from their bits into shared memory
-// (128-byte swizzled rows) by eight warps, so the store is read from HBM as
-// bits. Dense output runs tiles query-tile-major: one query tile stays in L2
+// BNq <= 256 for CODES with one module, else <= 128. Queries are prepared
+// once per call in the workspace (e2m1 pairs or e4m3 bytes, or bf16 hi and lo
+// rows) and fetched by TMA; stored rows are expanded from their bits by eight
+// warps into tensor memory (CODES) or into 128-byte swizzled shared-memory rows
+// (PAPER), so the store is read from HBM as bits. Dense output runs tiles query-tile-major: one query tile stays in L2
 // while the stored codes stream past it.
 //
 // Warps: 0-7 expand stored rows, two threads per row (warp 0 lane 0 also
@@ -42,6 +44,7 @@
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <type_traits>
 #include <cmath>
 #include <cstdlib>
 
@@ -112,9 +115,9 @@ constexpr uint32_t tc_b_offset() {
 // queries, 128 per tile), else four (48 KB stages). TMEM A: six 32 KB query
 // stages with 256 queries per tile (A slots in TMEM columns 256-447), four with
 // 128 (A slots in columns 384-511).
-template <int MODE, bool TOPK, int BN, bool AT>
+template <int MODE, bool TOPK, int BN, bool AT, bool F4 = false>
 constexpr int tc_stages() {
-  return AT ? (BN == 256 ? 6 : 8) : ((MODE == EOGP_SCORE_CODES && BN == 128) ? 6 : 4);
+  return AT ? (BN == 256 ? 6 : (F4 ? 7 : 8)) : ((MODE == EOGP_SCORE_CODES && BN == 128) ? 6 : 4);
 }
 
 // 128-query tiles with operand A in TMEM keep the running score in shared
@@ -129,9 +132,9 @@ constexpr int kAccLd = 132;
 // Stages the expanders fill per synchronisation round (one wait, fence and
 // arrive round): two with six stages, so that the MMAs always have at least
 // four stages to work on, else one.
-template <int MODE, bool TOPK, int BN, bool AT>
+template <int MODE, bool TOPK, int BN, bool AT, bool F4 = false>
 constexpr int tc_group() {
-  return tc_stages<MODE, TOPK, BN, AT>() >= 6 ? 2 : 1;
+  return tc_stages<MODE, TOPK, BN, AT, F4>() >= 6 ? 2 : 1;
 }
 
 // Accumulator buffers d_u in TMEM (BN columns each). Shared-memory A: three of
@@ -150,13 +153,21 @@ __device__ __forceinline__ uint32_t tc_acol(int s) {
   return static_cast<uint32_t>(256 + 32 * s);
 }
 
+// e2m1 path: the unit scale factors (ue8m0 0x7F = 1.0) of operands A and B,
+// 16 TMEM columns each, after the S A slots (columns 448-479 with 256 queries
+// per tile and six slots, 480-511 with 128 and seven).
+template <int S>
+constexpr uint32_t tc_sf_col() {
+  return static_cast<uint32_t>(256 + 32 * S);
+}
+
 // Shared-memory carve-up (byte offsets after 1024-byte alignment).
 struct TcSmem {
   uint32_t acc, sq, bars, lists, total;
 };
-template <int MODE, bool TOPK, int BN, bool AT>
+template <int MODE, bool TOPK, int BN, bool AT, bool F4 = false>
 __host__ __device__ inline TcSmem tc_smem_layout(int BNq, int K) {
-  constexpr int S = tc_stages<MODE, TOPK, BN, AT>();
+  constexpr int S = tc_stages<MODE, TOPK, BN, AT, F4>();
   TcSmem l;
   l.acc = S * tc_stage_bytes<MODE, BN, AT>();
   l.sq = l.acc + (tc_acc_smem<BN, AT>() ? 128u * kAccLd * 4u : 0u);
@@ -222,7 +233,28 @@ __device__ __forceinline__ void expand_half_tmem(uint32_t taddr, uint2 bits) {
   }
   tmem_st16_issue(taddr, v);
 }
-__device__ __forceinline__ void expand_half_tmem(uint32_t, uint32_t) {}  // bf16: shared memory only
+
+// e2m1 (fp4) one-bit operands. Word c of 32 code bits -> four 32-bit columns
+// of eight e2m1 values (+1 = 0x2 if the bit is set, -1 = 0xA if clear):
+// column j holds bits j, j + 4, ..., j + 28 in its nibbles 0..7, so each column
+// is one shift and one masked XOR. This permutes the K index within the word;
+// the query operand is expanded with the same permutation (k_expand_queries_f4),
+// and an inner product is unchanged by a permutation applied to both sides.
+__device__ __forceinline__ uint32_t e2m1x8(uint32_t c, int j) {
+  return ((c << (3 - j)) & 0x88888888u) ^ 0xAAAAAAAAu;
+}
+
+// Half a stage of one stored row (128 code bits) -> 16 TMEM columns of e2m1:
+// word q of the half gives columns 4q .. 4q + 3, stored without waiting.
+__device__ __forceinline__ void expand_half_tmem(uint32_t taddr, uint4 bits) {
+  const uint32_t w[4] = {bits.x, bits.y, bits.z, bits.w};
+  uint32_t v[16];
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) v[4 * q + j] = e2m1x8(w[q], j);
+  tmem_st16_issue(taddr, v);
+}
 
 // Tiles of a CTA. Dense output: strided over the grid, so all CTAs work on the
 // same query tile at a time. Ranking: a contiguous run of tiles, so a CTA
@@ -240,26 +272,31 @@ __device__ __forceinline__ int tile_step() {
   return TOPK ? 1 : gridDim.x;
 }
 
-template <int MODE, bool TOPK, int BN, bool AT>
+template <int MODE, bool TOPK, int BN, bool AT, bool F4 = false>
 __global__ void __launch_bounds__(kThreadsTc, 1)
     k_score_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQlo,
                const __grid_constant__ ScoreTcArgs g) {
-  static_assert(!AT || MODE == EOGP_SCORE_CODES, "operand A in TMEM is the e4m3 (one-bit) path");
-  constexpr int S = tc_stages<MODE, TOPK, BN, AT>();
+  static_assert(!AT || MODE == EOGP_SCORE_CODES, "operand A in TMEM is the one-bit path");
+  static_assert(!F4 || AT, "e2m1 operands are read from TMEM");
+  constexpr int S = tc_stages<MODE, TOPK, BN, AT, F4>();
   constexpr uint32_t kStage = tc_stage_bytes<MODE, BN, AT>();
   constexpr uint32_t kBOff = tc_b_offset<AT>();
-  constexpr int kBits = TcMode<MODE>::kBits;
+  // code bits per pipeline stage, and the query operand's TMA x coordinate per
+  // stage (elements of its tensor map: e4m3 / e2m1-pair bytes or bf16 values)
+  constexpr int kBits = F4 ? 256 : TcMode<MODE>::kBits;
+  constexpr int kQx = F4 ? 128 : kBits;
+  constexpr uint32_t kSfa = tc_sf_col<S>(), kSfb = kSfa + 16u;
   constexpr int ND = tc_dbufs<BN, AT>();
   // running-score columns: only 128-query tiles keep one (several modules)
   constexpr uint32_t kAcc = static_cast<uint32_t>(ND * BN);
-  using HalfBits = typename TcMode<MODE>::HalfBits;
+  using HalfBits = std::conditional_t<F4, uint4, typename TcMode<MODE>::HalfBits>;
   constexpr int kG = 8;  // stages of code bits prefetched at a time
-  constexpr int kP = tc_group<MODE, TOPK, BN, AT>();
+  constexpr int kP = tc_group<MODE, TOPK, BN, AT, F4>();
   constexpr bool kAccS = tc_acc_smem<BN, AT>();
   static_assert(kG % kP == 0, "prefetch groups hold whole expansion rounds");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  const TcSmem L = tc_smem_layout<MODE, TOPK, BN, AT>(g.BNq, g.K);
+  const TcSmem L = tc_smem_layout<MODE, TOPK, BN, AT, F4>(g.BNq, g.K);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   float* sq = reinterpret_cast<float*>(smem + L.sq);  // [2][BN] query scales of module u (CODES)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bars);
@@ -300,6 +337,18 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
     // TMEM A: this thread's row is TMEM lane r (warp w holds lanes 32 (w % 4) ..),
     // its half stage 16 columns of the stage's A slot.
     const uint32_t a_lane = tmem + (static_cast<uint32_t>(r & ~31) << 16) + 16u * static_cast<uint32_t>(half);
+    if constexpr (F4) {
+      // unit scale factors, once: warps 0-3 cover the four TMEM lane quarters
+      if (half == 0) {
+        uint32_t v[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) v[e] = 0x7F7F7F7Fu;
+        const uint32_t q_lane = tmem + (static_cast<uint32_t>(r & ~31) << 16);
+        tmem_st16_issue(q_lane + kSfa, v);
+        tmem_st16_issue(q_lane + kSfb, v);
+        tmem_wait_st();  // ordered before this warp's first arrive on a full barrier
+      }
+    }
     auto put = [&](int s, uint8_t* st, HalfBits bits) {
       if constexpr (AT) {
         tc_fence_after();  // the MMAs that read the slot before (released through empty[s]) are done
@@ -352,9 +401,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
                 uint8_t* st = smem + static_cast<size_t>(s) * kStage;
                 if (warp == 0 && lane == 0) {
                   mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(g.BNq) * 128u * TcMode<MODE>::kQBoxes);
-                  tma_load_2d(st + kBOff, &tmQ, j * kBits, q0, &full[s]);
+                  tma_load_2d(st + kBOff, &tmQ, j * kQx, q0, &full[s]);
                   if (MODE == EOGP_SCORE_PAPER)
-                    tma_load_2d(st + kBOff + static_cast<uint32_t>(BN) * 128u, &tmQlo, j * kBits, q0, &full[s]);
+                    tma_load_2d(st + kBOff + static_cast<uint32_t>(BN) * 128u, &tmQlo, j * kQx, q0, &full[s]);
                 }
                 put(s, st, cur[jj]);
                 publish();
@@ -387,10 +436,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
                 if (warp == 0 && lane == 0) {
                   const uint32_t qbytes = static_cast<uint32_t>(g.BNq) * 128u * TcMode<MODE>::kQBoxes;
                   mbar_arrive_expect_tx(&full[s0], qbytes);
-                  tma_load_2d(st0 + kBOff, &tmQ, j * kBits, q0, &full[s0]);
+                  tma_load_2d(st0 + kBOff, &tmQ, j * kQx, q0, &full[s0]);
                   if (two) {
                     mbar_arrive_expect_tx(&full[s1], qbytes);
-                    tma_load_2d(st1 + kBOff, &tmQ, (j + 1) * kBits, q0, &full[s1]);
+                    tma_load_2d(st1 + kBOff, &tmQ, (j + 1) * kQx, q0, &full[s1]);
                   }
                 }
                 put(s0, st0, cur[jj]);
@@ -649,8 +698,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   } else {
     // ---------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      const uint32_t idesc =
-          MODE == EOGP_SCORE_CODES ? idesc_e4m3_f32(128, g.BNq) : idesc_bf16_f32(128, g.BNq, 0, 0);
+      const uint32_t idesc = F4 ? idesc_mxf4_f32(128, g.BNq)
+                             : MODE == EOGP_SCORE_CODES ? idesc_e4m3_f32(128, g.BNq)
+                                                        : idesc_bf16_f32(128, g.BNq, 0, 0);
+      const uint32_t sfa = tmem + kSfa, sfb = tmem + kSfb;  // e2m1: unit scale factors
       // One lane issues every MMA, so its own work per stage is kept minimal:
       // ring slot, phase, A slot and descriptors advance incrementally (a
       // descriptor's address field is byte address >> 4: +2 steps 32 bytes).
@@ -695,7 +746,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
               const uint32_t acc = (kb | kk) != 0 ? 1u : 0u;
-              if constexpr (AT) {
+              if constexpr (F4) {
+                tc_mma_f4_ta(d, at0 + 8u * kk, a0 + 2 * kk, idesc, sfa, sfb, acc);
+              } else if constexpr (AT) {
                 tc_mma_f8_ta(d, at0 + 8u * kk, a0 + 2 * kk, idesc, acc);
               } else if (MODE == EOGP_SCORE_CODES) {
                 tc_mma_f8(d, a0 + 2 * kk, b0 + 2 * kk, idesc, acc);
@@ -736,6 +789,20 @@ __global__ void k_expand_queries(const uint32_t* __restrict__ query, int ldq, in
   }
 }
 
+// Query codes -> e2m1 +-1 in the stored rows' TMEM order (e2m1x8): word w of a
+// row gives output bytes 16 w .. 16 w + 15, column j of the word in bytes
+// 16 w + 4 j .. + 3 (two values per byte, the lower K index in the low nibble).
+__global__ void k_expand_queries_f4(const uint32_t* __restrict__ query, int ldq, int row_bytes,
+                                    uint8_t* __restrict__ out) {
+  const int q = blockIdx.y;
+  const int wtot = row_bytes >> 4;  // words per row (32 bits -> 16 bytes)
+  for (int w = blockIdx.x * blockDim.x + threadIdx.x; w < wtot; w += gridDim.x * blockDim.x) {
+    const uint32_t v = query[static_cast<size_t>(q) * ldq + w];
+    reinterpret_cast<uint4*>(out + static_cast<size_t>(q) * row_bytes)[w] =
+        make_uint4(e2m1x8(v, 0), e2m1x8(v, 1), e2m1x8(v, 2), e2m1x8(v, 3));
+  }
+}
+
 // Query coordinates y (fp32) -> bf16 hi = rn(y) and lo = rn(y - hi), dense rows of D.
 __global__ void k_split_queries(const float* __restrict__ y, int ldq, int D,
                                 __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __restrict__ lo) {
@@ -748,9 +815,9 @@ __global__ void k_split_queries(const float* __restrict__ y, int ldq, int D,
   }
 }
 
-template <int MODE, bool TOPK, int BN, bool AT = false>
+template <int MODE, bool TOPK, int BN, bool AT = false, bool F4 = false>
 size_t tc_smem_need(int BNq, int K) {
-  return 1024 + tc_smem_layout<MODE, TOPK, BN, AT>(BNq, K).total;
+  return 1024 + tc_smem_layout<MODE, TOPK, BN, AT, F4>(BNq, K).total;
 }
 
 // Operand A of the one-bit (CODES) kernel in TMEM unless EOGP_SCORE_AT = 0
@@ -759,6 +826,20 @@ bool tc_a_in_tmem(int mode) {
   if (mode != EOGP_SCORE_CODES) return false;
   const char* e = getenv("EOGP_SCORE_AT");
   return !(e && atoi(e) == 0);
+}
+
+// e2m1 (fp4) operands for the one-bit kernel with operand A in TMEM: the MMA
+// (kind::mxf4 with unit scales, exact for +-1) runs at twice the e4m3 rate and
+// a stage carries 256 code bits. Needs every module a multiple of 256 bits and
+// 16-byte aligned stored rows; EOGP_SCORE_F4 = 0 keeps e4m3 (read at every call).
+bool tc_f4(int mode, const int* ks, int U, const uint32_t* train, int ldt) {
+  if (!tc_a_in_tmem(mode)) return false;
+  const char* e = getenv("EOGP_SCORE_F4");
+  if (e && atoi(e) == 0) return false;
+  if (ldt % 4 || (reinterpret_cast<uintptr_t>(train) & 15)) return false;
+  for (int u = 0; u < U; ++u)
+    if (ks[u] % 256) return false;
+  return true;
 }
 
 // Queries per tile: 256 for CODES with one module and enough queries (when the
@@ -777,22 +858,26 @@ int tc_bn(int mode, int U, int Q, int K) {
 
 int bnq_for(int Q, int BN) { return std::min(BN, (Q + 31) / 32 * 32); }
 
-template <int MODE, bool TOPK, int BN, bool AT>
+template <int MODE, bool TOPK, int BN, bool AT, bool F4 = false>
 cudaError_t launch_tc_kernel(const CUtensorMap& t0, const CUtensorMap& t1, const ScoreTcArgs& g,
                              int grid, cudaStream_t st) {
-  const size_t smem = tc_smem_need<MODE, TOPK, BN, AT>(g.BNq, g.K);
-  cudaError_t e = cudaFuncSetAttribute(k_score_tc<MODE, TOPK, BN, AT>,
+  const size_t smem = tc_smem_need<MODE, TOPK, BN, AT, F4>(g.BNq, g.K);
+  cudaError_t e = cudaFuncSetAttribute(k_score_tc<MODE, TOPK, BN, AT, F4>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  k_score_tc<MODE, TOPK, BN, AT><<<grid, kThreadsTc, smem, st>>>(t0, t1, g);
+  k_score_tc<MODE, TOPK, BN, AT, F4><<<grid, kThreadsTc, smem, st>>>(t0, t1, g);
   return cudaGetLastError();
 }
 
 template <bool TOPK>
-cudaError_t dispatch_tc(int mode, int BN, const CUtensorMap& t0, const CUtensorMap& t1, const ScoreTcArgs& g,
-                        int grid, cudaStream_t st) {
+cudaError_t dispatch_tc(int mode, int BN, bool f4, const CUtensorMap& t0, const CUtensorMap& t1,
+                        const ScoreTcArgs& g, int grid, cudaStream_t st) {
   if (BN == 256 && g.U != 1) return cudaErrorInvalidValue;  // 256-query tiles keep no running score
   if (mode == EOGP_SCORE_PAPER) return launch_tc_kernel<EOGP_SCORE_PAPER, TOPK, 128, false>(t0, t1, g, grid, st);
+  if (f4) {
+    if (BN == 256) return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 256, true, true>(t0, t1, g, grid, st);
+    return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 128, true, true>(t0, t1, g, grid, st);
+  }
   if (tc_a_in_tmem(mode)) {
     if (BN == 256) return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 256, true>(t0, t1, g, grid, st);
     return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 128, true>(t0, t1, g, grid, st);
@@ -847,10 +932,12 @@ bool score_tc_topk_fits(int mode, int U, int Q, int K) {
   const int bq = bnq_for(Q, BN);
   const size_t need =
       mode == EOGP_SCORE_PAPER ? tc_smem_need<EOGP_SCORE_PAPER, true, 128>(bq, K)
-      : BN == 256 ? std::max(tc_smem_need<EOGP_SCORE_CODES, true, 256, false>(bq, K),
-                             tc_smem_need<EOGP_SCORE_CODES, true, 256, true>(bq, K))
-                  : std::max(tc_smem_need<EOGP_SCORE_CODES, true, 128, false>(bq, K),
-                             tc_smem_need<EOGP_SCORE_CODES, true, 128, true>(bq, K));
+      : BN == 256 ? std::max({tc_smem_need<EOGP_SCORE_CODES, true, 256, false>(bq, K),
+                              tc_smem_need<EOGP_SCORE_CODES, true, 256, true>(bq, K),
+                              tc_smem_need<EOGP_SCORE_CODES, true, 256, true, true>(bq, K)})
+                  : std::max({tc_smem_need<EOGP_SCORE_CODES, true, 128, false>(bq, K),
+                              tc_smem_need<EOGP_SCORE_CODES, true, 128, true>(bq, K),
+                              tc_smem_need<EOGP_SCORE_CODES, true, 128, true, true>(bq, K)});
   return need <= 232448;
 }
 
@@ -891,14 +978,20 @@ cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const floa
   g.D = D;
   const int grid = score_tc_grid(mode, U, N, Q, topk ? topk->K : 0, num_sms);
   CUtensorMap t0, t1;
+  const bool f4 = mode == EOGP_SCORE_CODES && tc_f4(mode, ks, U, train, ldt);
   if (mode == EOGP_SCORE_CODES) {
+    // expanded query rows: D e4m3 bytes, or D / 2 bytes of e2m1 pairs
     uint8_t* qx = static_cast<uint8_t*>(ws);
+    const int row_bytes = f4 ? D / 2 : D;
     dim3 eg(std::max(1, std::min((D / 32 + 255) / 256, 64)), Q);
-    k_expand_queries<<<eg, 256, 0, st>>>(static_cast<const uint32_t*>(query), ldq, D, qx);
+    if (f4)
+      k_expand_queries_f4<<<eg, 256, 0, st>>>(static_cast<const uint32_t*>(query), ldq, row_bytes, qx);
+    else
+      k_expand_queries<<<eg, 256, 0, st>>>(static_cast<const uint32_t*>(query), ldq, D, qx);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    const uint64_t dims[2] = {static_cast<uint64_t>(D), static_cast<uint64_t>(Q)};
-    const uint64_t strides[1] = {static_cast<uint64_t>(D)};
+    const uint64_t dims[2] = {static_cast<uint64_t>(row_bytes), static_cast<uint64_t>(Q)};
+    const uint64_t strides[1] = {static_cast<uint64_t>(row_bytes)};
     const uint32_t box[2] = {128, static_cast<uint32_t>(g.BNq)};
     if (make_tmap(&t0, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, qx, dims, strides, box,
                   CU_TENSOR_MAP_SWIZZLE_128B))
@@ -927,10 +1020,10 @@ cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const floa
     if (e != cudaSuccess) return e;
     e = cudaMemsetAsync(topk->gtau, 0, static_cast<size_t>(Q) * sizeof(unsigned), st);  // key 0: none yet
     if (e != cudaSuccess) return e;
-    e = dispatch_tc<true>(mode, BN, t0, t1, g, grid, st);
+    e = dispatch_tc<true>(mode, BN, f4, t0, t1, g, grid, st);
     if (e != cudaSuccess) return e;
     return launch_topk_merge(topk->lst, topk->lsi, grid, Q, topk->K, topk->out_s, topk->ld_os,
                              topk->out_i, topk->ld_oi, st);
   }
-  return dispatch_tc<false>(mode, BN, t0, t1, g, grid, st);
+  return dispatch_tc<false>(mode, BN, f4, t0, t1, g, grid, st);
 }

@@ -58,7 +58,7 @@ EXPORTS = {
     "eogp_last_error": (ctypes.c_char_p, []),
     "eogp_version": (ctypes.c_char_p, []),
     "eogp_sync_status": (c_int, [c_void_p]),
-    "eogp_measure_peaks": (c_int, [POINTER(c_double), POINTER(c_double)]),
+    "eogp_measure_peaks": (c_int, [POINTER(c_double), POINTER(c_double), POINTER(c_double)]),
     "eogp_profile_enable": (c_int, [c_int]),
     "eogp_profile_read": (c_int, [c_int, POINTER(c_int), POINTER(c_double), c_int]),
     "eogp_plan_layer": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_double,
@@ -611,12 +611,14 @@ def read_store(path: str, ks: Sequence[int], device) -> "torch.Tensor":
     return torch.from_numpy(raw.reshape(-1, rb)).to(device)
 
 
-def measure_peaks() -> Tuple[float, float]:
-    """(e4m3 tensor-core TFLOP/s, XOR + popcount words/s) measured on the current device."""
+def measure_peaks() -> Tuple[float, float, float]:
+    """(e4m3 and e2m1 tensor-core TFLOP/s, XOR + popcount words/s) measured on the
+    current device."""
     f8 = c_double()
+    f4 = c_double()
     pc = c_double()
-    _check(lib().eogp_measure_peaks(ctypes.byref(f8), ctypes.byref(pc)))
-    return f8.value, pc.value
+    _check(lib().eogp_measure_peaks(ctypes.byref(f8), ctypes.byref(f4), ctypes.byref(pc)))
+    return f8.value, f4.value, pc.value
 
 
 def second_moment(Z, C=None, accumulate: bool = False, stream=None):

@@ -223,14 +223,16 @@ def test_gpt2_query_scoring_all_scores(monkeypatch):
     qs = rng.lognormal(0, 0.5, (Q, 48)).astype(np.float32)
     d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(DEV)
     tcd, qcd = d(tc.view(np.int32)), d(qc.view(np.int32))
-    got = E.score(tcd, d(ts), ks, E.SCORE_CODES, qcd, d(qs))
-    E.sync_status()
     want = O.score_codes_f32(tc, ts, ks, qc, qs)
-    np.testing.assert_array_equal(got.cpu().numpy(), want)
     want_v, want_i = O.top_k(want, 20)
-    for fused in ("1", "0"):     # ranking fused into the scoring kernel, and the dense path
-        monkeypatch.setenv("EOGP_TOPK_FUSED", fused)
-        vals, idx = E.score_topk(tcd, d(ts), ks, E.SCORE_CODES, qcd, 20, query_scales=d(qs))
+    for f4 in ("1", "0"):            # e2m1 operands (the default here) and e4m3
+        monkeypatch.setenv("EOGP_SCORE_F4", f4)
+        got = E.score(tcd, d(ts), ks, E.SCORE_CODES, qcd, d(qs))
         E.sync_status()
-        np.testing.assert_array_equal(idx.cpu().numpy(), want_i)
-        np.testing.assert_array_equal(vals.cpu().numpy().astype(np.float64), want_v)
+        np.testing.assert_array_equal(got.cpu().numpy(), want)
+        for fused in ("1", "0"):     # ranking fused into the scoring kernel, and the dense path
+            monkeypatch.setenv("EOGP_TOPK_FUSED", fused)
+            vals, idx = E.score_topk(tcd, d(ts), ks, E.SCORE_CODES, qcd, 20, query_scales=d(qs))
+            E.sync_status()
+            np.testing.assert_array_equal(idx.cpu().numpy(), want_i)
+            np.testing.assert_array_equal(vals.cpu().numpy().astype(np.float64), want_v)

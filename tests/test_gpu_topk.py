@@ -116,10 +116,13 @@ def codes_case(N, Q, ks, seed, dup=True):
                                       (3000, 300, [512, 1024, 128], 20),   # several modules, two query tiles
                                       (5000, 130, [1024, 1024], 64)])
 @pytest.mark.parametrize("fused", ["1", "0"])
-def test_topk_codes_fused_exact(N, Q, ks, K, fused, monkeypatch):
+@pytest.mark.parametrize("f4", ["1", "0"])
+def test_topk_codes_fused_exact(N, Q, ks, K, fused, f4, monkeypatch):
     """K <= 32 ranks inside the tensor-core epilogue when fused; K = 64 always
-    takes the dense path. Both paths give the oracle's lists exactly."""
+    takes the dense path. Both paths give the oracle's lists exactly, with e2m1
+    operands (modules of multiples of 256 bits) and with e4m3 (EOGP_SCORE_F4=0)."""
     monkeypatch.setenv("EOGP_TOPK_FUSED", fused)
+    monkeypatch.setenv("EOGP_SCORE_F4", f4)
     tc, ts, qc, qs = codes_case(N, Q, ks, N + K)
     vals, idx = E.score_topk(dev(tc), dev(ts), ks, E.SCORE_CODES, dev(qc), K, query_scales=dev(qs))
     E.sync_status()
