@@ -407,7 +407,10 @@ int eogp_score_workspace_size(int N, const int* k_per_module, int U, int mode, i
  * bytes (0 bytes for the CUDA-core kernels); CODES and PAPER use the tensor
  * cores when it is given, the shape allows (CODES: Q >= 64, k_u % 128 == 0;
  * PAPER: k_u % 64 == 0) and the code rows are aligned (CODES: ld_train % 4 == 0
- * and a 16-byte aligned base; PAPER: ld_train % 2 == 0, 8-byte base).
+ * and a 16-byte aligned base; PAPER: ld_train % 2 == 0, 8-byte base). CODES on
+ * the tensor cores multiplies exact +-1 operands: e2m1 through the block-scaled
+ * fp4 MMA with unit scales when every k_u is a multiple of 256, else e4m3; the
+ * scores are the same bit for bit either way.
  * Errors: EOGP_EINVAL, EOGP_EWORKSPACE, EOGP_ECUDA. */
 int eogp_score(const void* train, int ld_train, const float* train_scales, int ld_tscale, int N,
                const int* k_per_module, int U, int mode, const void* query, int ld_query,
