@@ -52,8 +52,7 @@ def score_peak(ks, probes, bf16_burst, peaks_src):
     module is a multiple of 256 bits, else e4m3 kind::f8f6f4), as (TFLOP/s,
     source, mode label). Without the probes: the bf16 burst peak times the
     nominal dense ratio (fp8 2x, fp4 6x)."""
-    f4 = (os.environ.get("EOGP_SCORE_F4", "1") != "0" and os.environ.get("EOGP_SCORE_AT", "1") != "0"
-          and all(k % 256 == 0 for k in ks))
+    f4 = all(k % 256 == 0 for k in ks)
     if f4:
         mode = "tcgen05 kind::mxf4, +-1 e2m1 operands, unit ue8m0 scales"
         if probes:

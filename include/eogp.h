@@ -96,6 +96,25 @@ int eogp_sync_status(eogp_stream_t stream);
 int eogp_profile_enable(int on);
 int eogp_profile_read(int kind, int* launches, double* total_ms, int reset);
 
+/* ---- process-wide dispatch options (no counterpart in the paper) ---------
+ * Two choices between implementations that give identical results. They are
+ * read, under one setting, by both the workspace-size query and the call, so
+ * change them only while no eogp_score / eogp_score_topk call is being
+ * prepared or issued on another thread; a workspace sized under one setting
+ * may be too small under the other (the call then returns EOGP_EWORKSPACE).
+ *   EOGP_OPT_SCORE_OPERAND: one-bit operands of the tensor-core CODES scoring
+ *     kernel. 0 (default): e2m1 (kind::mxf4, unit scales) when every module is
+ *     a multiple of 256 bits and the stored rows are 16-byte aligned, else
+ *     e4m3; 1: always e4m3 (kind::f8f6f4). Scores are bit-identical.
+ *   EOGP_OPT_TOPK_PATH: ranking path of eogp_score_topk. 0 (default): chosen
+ *     by size; 1: ranking fused into the tensor-core scoring kernel where it
+ *     applies; 2: dense scores then a ranking kernel.
+ * eogp_set_option returns EOGP_EINVAL for an unknown option or value. */
+#define EOGP_OPT_SCORE_OPERAND 0
+#define EOGP_OPT_TOPK_PATH     1
+int eogp_set_option(int option, int value);
+int eogp_get_option(int option, int* value);
+
 /* Throughput probes for the scoring rooflines (no counterpart in the paper: a
  * library convenience). Measures on the current device, synchronously: the dense
  * tcgen05 rates of the two +-1 scoring MMAs in TFLOP/s (one CTA per SM issuing
@@ -235,7 +254,8 @@ int eogp_compress_layer(const eogp_layer_desc* L, const void* a, const void* s, 
  * transparent huge pages, registered with cudaHostRegister. Measured on GB300
  * systems, host-to-device copies from it ran at the link rate (~211 GB/s) in
  * every trial, where cudaHostAlloc'd buffers varied from ~80 to ~210 GB/s
- * between allocations. The size is rounded up to whole huge pages; the memory
+ * between allocations. Requests of at least one huge page are rounded up to
+ * whole huge pages, smaller ones to whole base pages (no huge-page advice); the memory
  * is zero-filled. eogp_host_free takes only the pointer (NULL is a no-op).
  * A library convenience with no counterpart in the paper.
  * Errors: EOGP_EINVAL (bytes == 0, ptr NULL, mapping failed, pointer not from
@@ -279,8 +299,11 @@ int eogp_compress_layer_host(const eogp_layer_desc* L, const void* a, const void
  *  - All calls on a device share the one array and it keeps the last call's
  *    contents. Calls whose kernels overlap on the GPU (e.g. on two streams
  *    without ordering between them) race on it and corrupt each other's results.
- *  - The first call on each device looks up the array's device address
- *    (cudaGetSymbolAddress); make that first call before any stream capture. */
+ *  - Every call looks up the array's device address on the current device
+ *    (cudaGetSymbolAddress, which allocates nothing), so the address stays
+ *    right if the device's context is destroyed and created again. The first
+ *    call on a device may also load the library's device code there; make
+ *    that first call before any stream capture. */
 #define EOGP_STATIC_WORKSPACE_BYTES (32u << 20)
 int eogp_compress_layer_static(const eogp_layer_desc* L, const void* a, const void* s, int B,
                                int out_mode, float* out, int ld_out, uint32_t* codes, int ld_codes,

@@ -8,6 +8,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 #include <numeric>
 #include <vector>
@@ -32,19 +33,18 @@ int set_error(int code, const char* fmt, ...) {
 
 void clear_error() { g_err[0] = '\0'; }
 
+// Looked up on every call (cudaGetSymbolAddress allocates nothing and is
+// cheap): a cached address would go stale if the device's context were
+// destroyed and recreated.
 unsigned* status_word() {
-  static unsigned* addr[128] = {nullptr};
-  static std::mutex mu;
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 128) return nullptr;
-  std::lock_guard<std::mutex> lk(mu);
-  if (!addr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_eogp_status) != cudaSuccess) return nullptr;
-    addr[dev] = static_cast<unsigned*>(p);
-  }
-  return addr[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_eogp_status) != cudaSuccess) return nullptr;
+  return static_cast<unsigned*>(p);
 }
+
+static std::atomic<int> g_opt[2] = {{0}, {0}};
+
+int option(int which) { return (which >= 0 && which < 2) ? g_opt[which].load(std::memory_order_relaxed) : 0; }
 
 static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
@@ -92,17 +92,19 @@ using namespace eogp;
 static inline size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
 static inline int round_up(int x, int a) { return (x + a - 1) / a * a; }
 
+// SM count of the current device, cached per device index.
 static int sm_count() {
-  static int n = 0;
-  if (n == 0) {
-    int dev = 0, v = 0;
-    if (cudaGetDevice(&dev) == cudaSuccess &&
-        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && v > 0)
-      n = v;
-    else
-      return 148;
+  static std::atomic<int> cache[128];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 148;
+  if (dev < 128) {
+    const int c = cache[dev].load(std::memory_order_relaxed);
+    if (c > 0) return c;
   }
-  return n;
+  int v = 0;
+  if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) return 148;
+  if (dev < 128) cache[dev].store(v, std::memory_order_relaxed);
+  return v;
 }
 
 static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
@@ -1006,6 +1008,26 @@ extern "C" int eogp_payload_unpack(const uint8_t* payload, size_t ld_payload, in
 
 // ================================================================ probes
 
+extern "C" int eogp_set_option(int opt, int value) {
+  clear_error();
+  if (opt == EOGP_OPT_SCORE_OPERAND && (value == 0 || value == 1)) {
+    g_opt[opt].store(value);
+    return EOGP_OK;
+  }
+  if (opt == EOGP_OPT_TOPK_PATH && value >= 0 && value <= 2) {
+    g_opt[opt].store(value);
+    return EOGP_OK;
+  }
+  return set_error(EOGP_EINVAL, "eogp_set_option: unknown option %d or value %d", opt, value);
+}
+
+extern "C" int eogp_get_option(int opt, int* value) {
+  clear_error();
+  if (!value || opt < 0 || opt > 1) return set_error(EOGP_EINVAL, "eogp_get_option: bad option %d", opt);
+  *value = g_opt[opt].load();
+  return EOGP_OK;
+}
+
 extern "C" int eogp_measure_peaks(double* e4m3_tflops, double* e2m1_tflops, double* popc_words_per_s) {
   clear_error();
   unsigned* status = status_word();
@@ -1254,12 +1276,11 @@ struct TopkPlan {
 // the ranking is fused into the tensor-core scoring kernel when it supports the
 // request (the Q x N matrix then never reaches HBM), else dense scores, per-slot
 // lists and a merge. Measured on the GPT-2 query workload (N = 16384, Q = 1024,
-// top 20): fused 2.4 ms, dense + per-slot lists 2.9 ms. EOGP_TOPK_FUSED = 1 / 0
-// forces the fused / a dense path (tests); it is read at every call, so the
-// workspace query and the call must see the same setting.
+// top 20): fused 2.4 ms, dense + per-slot lists 2.9 ms. EOGP_OPT_TOPK_PATH = 1 / 2
+// forces the fused / a dense path.
 static int topk_fused_override() {
-  const char* e = getenv("EOGP_TOPK_FUSED");
-  return e ? atoi(e) : -1;
+  const int v = option(EOGP_OPT_TOPK_PATH);
+  return v == 1 ? 1 : v == 2 ? 0 : -1;
 }
 
 static TopkPlan topk_plan(int N, const int* ks, int U, int mode, int Q, int K) {

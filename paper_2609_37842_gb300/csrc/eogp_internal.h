@@ -20,6 +20,9 @@ void clear_error();
 // Address of the device status word on the current device (nullptr on failure).
 unsigned* status_word();
 
+// Current value of a process-wide dispatch option (EOGP_OPT_*).
+int option(int which);
+
 // Encodes a tiled TMA descriptor (driver entry point resolved once).
 // dims/strides: innermost first; strides in bytes for dims 1..rank-1.
 int make_tmap(CUtensorMap* tm, CUtensorMapDataType dt, int rank, const void* base,

@@ -55,10 +55,15 @@ extern "C" int eogp_host_alloc(size_t bytes, void** ptr) {
   if (!ptr) return set_error(EOGP_EINVAL, "ptr is NULL");
   *ptr = nullptr;
   if (bytes == 0) return set_error(EOGP_EINVAL, "bytes must be > 0");
-  const size_t hp = huge_page_bytes();
+  // Requests of at least one huge page are aligned to and advised for huge
+  // pages; smaller ones are rounded to the base page only (on 64 KB-page arm64
+  // hosts a huge page is 512 MB, far too much to pin for a small buffer).
+  const size_t huge = huge_page_bytes();
+  const long ps = sysconf(_SC_PAGESIZE);
+  const size_t hp = bytes >= huge ? huge : static_cast<size_t>(ps > 0 ? ps : 4096);
   const size_t len = (bytes + hp - 1) / hp * hp;
   if (len < bytes || len + hp < len) return set_error(EOGP_EINVAL, "size too large");
-  // Map one huge page more than needed and keep the aligned part.
+  // Map one alignment unit more than needed and keep the aligned part.
   void* raw = mmap(nullptr, len + hp, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
   if (raw == MAP_FAILED) return set_error(EOGP_EINVAL, "mmap of %zu bytes failed", len + hp);
   const uintptr_t r = reinterpret_cast<uintptr_t>(raw);
@@ -67,7 +72,7 @@ extern "C" int eogp_host_alloc(size_t bytes, void** ptr) {
   const size_t tail = (r + len + hp) - (a + len);
   if (tail) munmap(reinterpret_cast<void*>(a + len), tail);
   void* p = reinterpret_cast<void*>(a);
-  madvise(p, len, MADV_HUGEPAGE);  // advice only: without it the region still works
+  if (hp == huge) madvise(p, len, MADV_HUGEPAGE);  // advice only: without it the region still works
   // Fault the region in from the CPU before registering it, so that the pages
   // are placed by ordinary first-touch faults on the advised, aligned range:
   // the configuration the ~211 GB/s copy rate above was measured with.

@@ -820,22 +820,17 @@ size_t tc_smem_need(int BNq, int K) {
   return 1024 + tc_smem_layout<MODE, TOPK, BN, AT, F4>(BNq, K).total;
 }
 
-// Operand A of the one-bit (CODES) kernel in TMEM unless EOGP_SCORE_AT = 0
-// (shared memory, for comparisons; read at every call).
-bool tc_a_in_tmem(int mode) {
-  if (mode != EOGP_SCORE_CODES) return false;
-  const char* e = getenv("EOGP_SCORE_AT");
-  return !(e && atoi(e) == 0);
-}
+// Operand A of the one-bit (CODES) kernel is written to TMEM; the PAPER kernel
+// keeps its bf16 +-1 operand in shared memory.
+bool tc_a_in_tmem(int mode) { return mode == EOGP_SCORE_CODES; }
 
-// e2m1 (fp4) operands for the one-bit kernel with operand A in TMEM: the MMA
-// (kind::mxf4 with unit scales, exact for +-1) runs at twice the e4m3 rate and
-// a stage carries 256 code bits. Needs every module a multiple of 256 bits and
-// 16-byte aligned stored rows; EOGP_SCORE_F4 = 0 keeps e4m3 (read at every call).
+// e2m1 (fp4) operands for the one-bit kernel: the MMA (kind::mxf4 with unit
+// scales, exact for +-1) runs at twice the e4m3 rate and a stage carries 256
+// code bits. Needs every module a multiple of 256 bits and 16-byte aligned
+// stored rows; EOGP_OPT_SCORE_OPERAND = 1 keeps e4m3.
 bool tc_f4(int mode, const int* ks, int U, const uint32_t* train, int ldt) {
   if (!tc_a_in_tmem(mode)) return false;
-  const char* e = getenv("EOGP_SCORE_F4");
-  if (e && atoi(e) == 0) return false;
+  if (eogp::option(EOGP_OPT_SCORE_OPERAND) == 1) return false;
   if (ldt % 4 || (reinterpret_cast<uintptr_t>(train) & 15)) return false;
   for (int u = 0; u < U; ++u)
     if (ks[u] % 256) return false;
@@ -846,11 +841,9 @@ bool tc_f4(int mode, const int* ks, int U, const uint32_t* train, int ldt) {
 // shared memory allows), else 128. (Measured with operand A in TMEM on the
 // 4.2M-code scan at Q = 1024: 48.0 ms with 256-query tiles and one accumulator,
 // 63.2 ms with 192-query tiles and two: the expansion is repeated per query
-// tile.) EOGP_SCORE_BN = 128 forces 128 (comparisons).
+// tile.)
 int tc_bn(int mode, int U, int Q, int K) {
-  const char* e = getenv("EOGP_SCORE_BN");
-  const bool force128 = e && atoi(e) == 128;
-  if (mode == EOGP_SCORE_CODES && U == 1 && Q >= 256 && !force128 &&
+  if (mode == EOGP_SCORE_CODES && U == 1 && Q >= 256 &&
       (K == 0 || tc_smem_need<EOGP_SCORE_CODES, true, 256>(256, K) <= 232448))
     return 256;
   return 128;
@@ -878,12 +871,8 @@ cudaError_t dispatch_tc(int mode, int BN, bool f4, const CUtensorMap& t0, const 
     if (BN == 256) return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 256, true, true>(t0, t1, g, grid, st);
     return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 128, true, true>(t0, t1, g, grid, st);
   }
-  if (tc_a_in_tmem(mode)) {
-    if (BN == 256) return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 256, true>(t0, t1, g, grid, st);
-    return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 128, true>(t0, t1, g, grid, st);
-  }
-  if (BN == 256) return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 256, false>(t0, t1, g, grid, st);
-  return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 128, false>(t0, t1, g, grid, st);
+  if (BN == 256) return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 256, true>(t0, t1, g, grid, st);
+  return launch_tc_kernel<EOGP_SCORE_CODES, TOPK, 128, true>(t0, t1, g, grid, st);
 }
 
 }  // namespace
@@ -932,11 +921,9 @@ bool score_tc_topk_fits(int mode, int U, int Q, int K) {
   const int bq = bnq_for(Q, BN);
   const size_t need =
       mode == EOGP_SCORE_PAPER ? tc_smem_need<EOGP_SCORE_PAPER, true, 128>(bq, K)
-      : BN == 256 ? std::max({tc_smem_need<EOGP_SCORE_CODES, true, 256, false>(bq, K),
-                              tc_smem_need<EOGP_SCORE_CODES, true, 256, true>(bq, K),
+      : BN == 256 ? std::max({tc_smem_need<EOGP_SCORE_CODES, true, 256, true>(bq, K),
                               tc_smem_need<EOGP_SCORE_CODES, true, 256, true, true>(bq, K)})
-                  : std::max({tc_smem_need<EOGP_SCORE_CODES, true, 128, false>(bq, K),
-                              tc_smem_need<EOGP_SCORE_CODES, true, 128, true>(bq, K),
+                  : std::max({tc_smem_need<EOGP_SCORE_CODES, true, 128, true>(bq, K),
                               tc_smem_need<EOGP_SCORE_CODES, true, 128, true, true>(bq, K)});
   return need <= 232448;
 }

@@ -1055,29 +1055,14 @@ cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, 
 
 // CTA pairs measured faster for short reductions (K <= 1536: the hi/lo
 // epilogue dominates and halving the per-SM operand stream helps) and slower
-// for long ones; EOGP_ROT_PAIRS = 0 / 1 forces one choice.
-static bool rotate_pairs(int K) {
-  static int v = -2;
-  if (v == -2) {
-    const char* e = getenv("EOGP_ROT_PAIRS");
-    v = e ? atoi(e) : -1;
-  }
-  if (v >= 0) return v != 0;
-  return K <= 1536;
-}
+// for long ones.
+static bool rotate_pairs(int K) { return K <= 1536; }
 
 // N tile width for `n` output columns: as few tiles of at most 256 columns as
 // is cheapest, each a multiple of `gran` (16: the tcgen05 N granularity, for one
 // CTA and for CTA pairs, whose halves of N / 2 rows are whole 8-row swizzle
-// atoms), counting a fixed per-tile overhead of 32 columns. EOGP_ROT_BN
-// overrides for sweeps.
+// atoms), counting a fixed per-tile overhead of 32 columns.
 int rotate_bn(int n, int gran) {
-  static int forced = -1;
-  if (forced < 0) {
-    const char* e = getenv("EOGP_ROT_BN");
-    forced = e ? atoi(e) : 0;
-  }
-  if (forced > 0 && forced % gran == 0 && forced <= 256) return forced;
   const int n0 = (n + 255) / 256;
   int best = 0, best_cost = 1 << 30;
   for (int nN = n0; nN <= n0 + 1; ++nN) {
@@ -1097,16 +1082,9 @@ cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W
   if (M <= 0) return cudaSuccess;
   const bool pairs = rotate_pairs(K);
   const int BN = rotate_bn(Wrows, 16);
-  // As many pipeline stages as fit in 227 KB of shared memory (at most 8);
-  // EOGP_ROT_STAGES overrides for tuning sweeps.
-  static int forced_stages = -1;
-  if (forced_stages < 0) {
-    const char* e = getenv("EOGP_ROT_STAGES");
-    forced_stages = e ? atoi(e) : 0;
-  }
+  // As many pipeline stages as fit in 227 KB of shared memory (at most 8).
   int stages = 2;
   while (stages < 8 && rotate_smem_bytes(BN, stages + 1) <= 232448) ++stages;
-  if (forced_stages >= 2 && rotate_smem_bytes(BN, forced_stages) <= 232448) stages = forced_stages;
   CUtensorMap tX, tW;
   if (tmap_bf16_2d(&tX, X, static_cast<uint64_t>(K), static_cast<uint64_t>(M), ldx, 64, 128) ||
       tmap_bf16_2d(&tW, W, K, Wrows, ldw, 64, BN))
@@ -1132,7 +1110,6 @@ cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W
     if (tmap_bf16_2d(&tWh, W, K, Wrows, ldw, 64, BN / 2)) return cudaErrorInvalidValue;
     int st2 = 2;
     while (st2 < 8 && rotate2_smem_bytes(BN, st2 + 1) <= 232448) ++st2;
-    if (forced_stages >= 2 && rotate2_smem_bytes(BN, forced_stages) <= 232448) st2 = forced_stages;
     g.stages = st2;
     g.n_tiles = ((M + 255) / 256) * g.nN;
     const size_t smem = rotate2_smem_bytes(BN, st2);

@@ -10,8 +10,6 @@
 // EOGP_STATIC_WORKSPACE_BYTES, which every GPU that loads the library holds
 // until the process exits. The entry point itself calls no cudaMalloc,
 // cudaFree or other allocating routine.
-#include <mutex>
-
 #include "eogp_dev.cuh"
 #include "eogp_internal.h"
 
@@ -19,27 +17,18 @@ static __device__ __align__(256) unsigned char g_eogp_static_ws[EOGP_STATIC_WORK
 
 namespace {
 
-std::mutex g_static_mu;
-void* g_static_addr[128] = {nullptr};
-
 // Device address of the scratch array on the current device. In host code the
-// array's name is only a host-side stand-in, so the address is looked up once
-// per device (with that device current) and cached.
+// array's name is only a host-side stand-in, so the address is looked up with
+// the device current, on every call: the lookup allocates nothing, and an
+// address kept from an earlier call would be stale if the device's context had
+// been destroyed and created again since.
 int static_scratch(void** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return eogp::set_error(EOGP_ECUDA, "cudaGetDevice failed: %s", cudaGetErrorString(e));
-  if (dev < 0 || dev >= 128) return eogp::set_error(EOGP_EUNSUPPORTED, "device index %d too large", dev);
-  std::lock_guard<std::mutex> lk(g_static_mu);
-  if (!g_static_addr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_eogp_static_ws);
-    if (e != cudaSuccess || !p)
-      return eogp::set_error(EOGP_ECUDA, "cudaGetSymbolAddress of the built-in scratch failed: %s",
-                             cudaGetErrorString(e));
-    g_static_addr[dev] = p;
-  }
-  *out = g_static_addr[dev];
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_eogp_static_ws);
+  if (e != cudaSuccess || !p)
+    return eogp::set_error(EOGP_ECUDA, "cudaGetSymbolAddress of the built-in scratch failed: %s",
+                           cudaGetErrorString(e));
+  *out = p;
   return EOGP_OK;
 }
 

@@ -60,6 +60,8 @@ EXPORTS = {
     "eogp_sync_status": (c_int, [c_void_p]),
     "eogp_measure_peaks": (c_int, [POINTER(c_double), POINTER(c_double), POINTER(c_double)]),
     "eogp_profile_enable": (c_int, [c_int]),
+    "eogp_set_option": (c_int, [c_int, c_int]),
+    "eogp_get_option": (c_int, [c_int, POINTER(c_int)]),
     "eogp_profile_read": (c_int, [c_int, POINTER(c_int), POINTER(c_double), c_int]),
     "eogp_plan_layer": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_double,
                                 POINTER(c_void_p)]),
@@ -609,6 +611,43 @@ def read_store(path: str, ks: Sequence[int], device) -> "torch.Tensor":
     if raw.size % rb:
         raise ValueError(f"{path}: {raw.size} bytes is not a whole number of {rb}-byte records")
     return torch.from_numpy(raw.reshape(-1, rb)).to(device)
+
+
+OPT_SCORE_OPERAND = 0   # 0: e2m1 where it applies (default), 1: e4m3
+OPT_TOPK_PATH = 1       # 0: by size (default), 1: fused ranking, 2: dense scores + ranking kernel
+
+
+def set_option(option: int, value: int) -> None:
+    """eogp_set_option: a process-wide dispatch choice between implementations
+    with identical results (read by the workspace queries and the calls)."""
+    _check(lib().eogp_set_option(option, value))
+
+
+def get_option(option: int) -> int:
+    v = c_int()
+    _check(lib().eogp_get_option(option, ctypes.byref(v)))
+    return v.value
+
+
+class options:
+    """Context manager setting dispatch options and restoring them on exit:
+    `with options(score_operand=1, topk_path=2): ...`."""
+
+    def __init__(self, score_operand: Optional[int] = None, topk_path: Optional[int] = None):
+        self.want = {OPT_SCORE_OPERAND: score_operand, OPT_TOPK_PATH: topk_path}
+        self.old = {}
+
+    def __enter__(self):
+        for o, v in self.want.items():
+            if v is not None:
+                self.old[o] = get_option(o)
+                set_option(o, v)
+        return self
+
+    def __exit__(self, *exc):
+        for o, v in self.old.items():
+            set_option(o, v)
+        return False
 
 
 def measure_peaks() -> Tuple[float, float, float]:

@@ -208,7 +208,7 @@ def test_fit_pca_gpt2_size():
 
 # ------------------------------------------------------ GPT-2 query scoring
 
-def test_gpt2_query_scoring_all_scores(monkeypatch):
+def test_gpt2_query_scoring_all_scores(eogp_options):
     """Q = 1024 queries x 48 modules x 1024 bits (the bench's query workload: the
     running score kept in TMEM across modules) against N = 300 stored codes (a
     ragged last row tile): every score equals the oracle's float32 evaluation
@@ -226,12 +226,12 @@ def test_gpt2_query_scoring_all_scores(monkeypatch):
     want = O.score_codes_f32(tc, ts, ks, qc, qs)
     want_v, want_i = O.top_k(want, 20)
     for f4 in ("1", "0"):            # e2m1 operands (the default here) and e4m3
-        monkeypatch.setenv("EOGP_SCORE_F4", f4)
+        eogp_options(score_operand=0 if f4 == "1" else 1)
         got = E.score(tcd, d(ts), ks, E.SCORE_CODES, qcd, d(qs))
         E.sync_status()
         np.testing.assert_array_equal(got.cpu().numpy(), want)
         for fused in ("1", "0"):     # ranking fused into the scoring kernel, and the dense path
-            monkeypatch.setenv("EOGP_TOPK_FUSED", fused)
+            eogp_options(topk_path=1 if fused == "1" else 2)
             vals, idx = E.score_topk(tcd, d(ts), ks, E.SCORE_CODES, qcd, 20, query_scales=d(qs))
             E.sync_status()
             np.testing.assert_array_equal(idx.cpu().numpy(), want_i)

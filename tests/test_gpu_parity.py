@@ -109,11 +109,11 @@ def rand_store(rng, n, ks):
                                     (129, 200, [1024, 128, 2048]), (777, 257, [512] * 5),
                                     (1000, 300, [256, 768, 1024]), (500, 300, [2048])])
 @pytest.mark.parametrize("f4", ["1", "0"])
-def test_score_codes_bit_exact(N, Q, ks, f4, monkeypatch):
+def test_score_codes_bit_exact(N, Q, ks, f4, eogp_options):
     """CODES scores equal the oracle's float32 evaluation bit for bit. Where every
     module is a multiple of 256 bits the tensor-core kernel takes e2m1 operands
-    (kind::mxf4, unit scales) unless EOGP_SCORE_F4=0 keeps e4m3: both run."""
-    monkeypatch.setenv("EOGP_SCORE_F4", f4)
+    (kind::mxf4, unit scales) unless EOGP_OPT_SCORE_OPERAND = 1 keeps e4m3: both run."""
+    eogp_options(score_operand=0 if f4 == "1" else 1)
     rng = np.random.default_rng(N * 7 + Q)
     tc, qc = rand_store(rng, N, ks), rand_store(rng, Q, ks)
     U = len(ks)

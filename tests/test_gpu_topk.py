@@ -10,7 +10,7 @@
 * The three paths: up to 49,152 stored rows, dense scores and a radix select
   per query row (the library's choice there); beyond, the ranking fused into
   the tensor-core epilogue (K <= 32), else dense scores, per-slot lists and a
-  merge. EOGP_TOPK_FUSED=1 / 0 forces the fused / a dense path, which the
+  merge. EOGP_OPT_TOPK_PATH = 1 / 2 forces the fused / a dense path, which the
   tests use to run both on the same cases; edge cases N < K and N = 0, ties.
 * Full scan scale (4,194,304 stored 16,384-bit codes, Q = 1024): the fused
   lists equal the oracle ranking of the dense scores of sampled queries.
@@ -117,12 +117,12 @@ def codes_case(N, Q, ks, seed, dup=True):
                                       (5000, 130, [1024, 1024], 64)])
 @pytest.mark.parametrize("fused", ["1", "0"])
 @pytest.mark.parametrize("f4", ["1", "0"])
-def test_topk_codes_fused_exact(N, Q, ks, K, fused, f4, monkeypatch):
+def test_topk_codes_fused_exact(N, Q, ks, K, fused, f4, eogp_options):
     """K <= 32 ranks inside the tensor-core epilogue when fused; K = 64 always
     takes the dense path. Both paths give the oracle's lists exactly, with e2m1
-    operands (modules of multiples of 256 bits) and with e4m3 (EOGP_SCORE_F4=0)."""
-    monkeypatch.setenv("EOGP_TOPK_FUSED", fused)
-    monkeypatch.setenv("EOGP_SCORE_F4", f4)
+    operands (modules of multiples of 256 bits) and with e4m3 (EOGP_OPT_SCORE_OPERAND = 1)."""
+    eogp_options(topk_path=1 if fused == "1" else 2)
+    eogp_options(score_operand=0 if f4 == "1" else 1)
     tc, ts, qc, qs = codes_case(N, Q, ks, N + K)
     vals, idx = E.score_topk(dev(tc), dev(ts), ks, E.SCORE_CODES, dev(qc), K, query_scales=dev(qs))
     E.sync_status()
@@ -147,8 +147,8 @@ def test_topk_codes_dense_exact(N, Q, ks, K):
 @pytest.mark.parametrize("N,Q,ks,K", [(1500, 70, [64, 128], 20), (4000, 3, [256], 10),
                                       (600, 130, [128], 100)])
 @pytest.mark.parametrize("fused", ["1", "0"])
-def test_topk_paper_valid(N, Q, ks, K, fused, monkeypatch):
-    monkeypatch.setenv("EOGP_TOPK_FUSED", fused)
+def test_topk_paper_valid(N, Q, ks, K, fused, eogp_options):
+    eogp_options(topk_path=1 if fused == "1" else 2)
     rng = np.random.default_rng(N + Q + K)
     tc = rand_store(rng, N, ks)
     ts = rng.lognormal(0, 0.5, (N, len(ks))).astype(np.float32)

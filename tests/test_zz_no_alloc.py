@@ -9,6 +9,8 @@ ABI twice in a row and checks both results against eogp_compress_layer with a
 caller workspace, then checks that an oversized batch is refused.
 """
 import ctypes
+import os
+import re
 
 import numpy as np
 import pytest
@@ -19,7 +21,28 @@ pytestmark = pytest.mark.gpu
 from paper_2609_37842_gb300 import eogp as E  # noqa: E402
 from paper_2609_37842_gb300 import synth  # noqa: E402
 
-STATIC_BYTES = 32 << 20  # EOGP_STATIC_WORKSPACE_BYTES in include/eogp.h
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _static_bytes():
+    """EOGP_STATIC_WORKSPACE_BYTES as the public header defines it."""
+    with open(os.path.join(ROOT, "include", "eogp.h")) as f:
+        m = re.search(r"#define\s+EOGP_STATIC_WORKSPACE_BYTES\s+\((\d+)u\s*<<\s*(\d+)\)", f.read())
+    assert m, "EOGP_STATIC_WORKSPACE_BYTES not found in include/eogp.h"
+    return int(m.group(1)) << int(m.group(2))
+
+
+STATIC_BYTES = _static_bytes()
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_37842_gb300 import build
+    build.build()
+    E.lib()
+    yield
 
 
 def _module(dev):
@@ -49,10 +72,6 @@ def _static_call(desc, a, s, mode, out=None, codes=None, scales=None):
 
 
 def test_static_scratch_matches_workspace_path():
-    if not torch.cuda.is_available():
-        pytest.skip("no CUDA device")
-    from paper_2609_37842_gb300 import build
-    build.build()
     dev = torch.device("cuda:0")
     desc, rng, T, d_in, d_out, k = _module(dev)
     B = 6
@@ -83,8 +102,6 @@ def test_static_scratch_matches_workspace_path():
 
 
 def test_static_scratch_rejects_oversized_batch():
-    if not torch.cuda.is_available():
-        pytest.skip("no CUDA device")
     dev = torch.device("cuda:0")
     desc, rng, T, d_in, d_out, k = _module(dev)
     B = 256
