@@ -44,6 +44,9 @@ PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # dram__bytes_read.sum + dram__bytes_write.sum per rotation launch from the committed
 # ncu capture (profiles/), or None when the kernel changed after the capture.
 ROTATE_TRAFFIC_BYTES = 1415.1e6  # mean over one transformer block (8 launches) at B = 512
+# Examples per compression call (one step) of each workload's throughput line.
+CONFIG_BATCH = {"gpt2_small_bf16": 512, "tiny_f32": 4096, "olmo2_1b_bf16": 128, "olmo2_7b_bf16": 32,
+                "olmo2_32b_gate_bf16": 64}
 
 
 def score_peak(ks, probes, bf16_burst, peaks_src):
@@ -319,10 +322,13 @@ def _config_stack(name, B, dev, gh, g):
     return w, per_layer, keys
 
 
-def bench_config(name, B, steps, warmup, dev, stream_bases=False):
-    """Examples/s per layer stack for one workload; with stream_bases the retained
-    eigenvector rows of every layer live in pinned host memory and are copied to
-    the device one layer ahead of its compute on a side stream."""
+def config_setup(name, B, dev):
+    """Everything one step of a workload's throughput line launches with: the
+    workload, per-module-type plans, retained eigenvector rows and inputs
+    (`per_layer`), the module-type key of every module of the stack (`keys`),
+    the PCA directions `Pt`, one layer descriptor per module type (`descs`) and
+    a workspace for B examples (`ws`). The tests call this too, so that they
+    check the launches the bench times."""
     import torch
     from paper_2609_37842_gb300 import eogp as E
     from paper_2609_37842_gb300 import synth
@@ -333,6 +339,19 @@ def bench_config(name, B, steps, warmup, dev, stream_bases=False):
     w, per_layer, keys = _config_stack(name, B, dev, gh, g)
     Pt = synth.torch_eigvec_rows(w.m, w.k, dev, gh,
                                  torch.bfloat16 if w.dtype == "bf16" else torch.float32)
+    descs = {key: E.layer_desc(L["plan"], w.T, w.k, L["VA"], L["VS"], Pt) for key, L in per_layer.items()}
+    ws = E.workspace(max(E.compress_workspace_size(d, B, E.OUT_CODES) for d in descs.values()), dev)
+    return dict(w=w, per_layer=per_layer, keys=keys, Pt=Pt, descs=descs, ws=ws)
+
+
+def bench_config(name, B, steps, warmup, dev, stream_bases=False):
+    """Examples/s per layer stack for one workload; with stream_bases the retained
+    eigenvector rows of every layer live in pinned host memory and are copied to
+    the device one layer ahead of its compute on a side stream."""
+    import torch
+    from paper_2609_37842_gb300 import eogp as E
+    cs = config_setup(name, B, dev)
+    w, per_layer, keys, Pt, descs, ws = (cs[x] for x in ("w", "per_layer", "keys", "Pt", "descs", "ws"))
     words = (w.k + 31) // 32
     U = len(w.modules)
     codes = torch.empty((B, U * words), dtype=torch.int32, device=dev)
@@ -340,10 +359,6 @@ def bench_config(name, B, steps, warmup, dev, stream_bases=False):
     stream = torch.cuda.current_stream()
     nmod_layer = len(set(keys))
     layers = U // nmod_layer if name.startswith("olmo") else 1
-    descs = {}
-    for key, L in per_layer.items():
-        descs[key] = E.layer_desc(L["plan"], w.T, w.k, L["VA"], L["VS"], Pt)
-    ws = E.workspace(max(E.compress_workspace_size(d, B, E.OUT_CODES) for d in descs.values()), dev)
     host_bases = dev_bases = None
     if stream_bases:
         # one pinned host copy per module type (every layer copies it again) and two
@@ -889,10 +904,12 @@ def main():
     if rank == 0 and not args.no_configs:
         torch.cuda.empty_cache()
         configs = {
-            "tiny_f32": bench_config("tiny_f32", 4096, 5, 3, dev),
-            "olmo2_1b_bf16": bench_config("olmo2_1b_bf16", 128, 3, 3, dev),
-            "olmo2_7b_bf16": bench_config("olmo2_7b_bf16", 32, 3, 3, dev, stream_bases=True),
-            "olmo2_32b_gate_bf16": bench_config("olmo2_32b_gate_bf16", 64, 5, 3, dev),
+            "tiny_f32": bench_config("tiny_f32", CONFIG_BATCH["tiny_f32"], 5, 3, dev),
+            "olmo2_1b_bf16": bench_config("olmo2_1b_bf16", CONFIG_BATCH["olmo2_1b_bf16"], 3, 3, dev),
+            "olmo2_7b_bf16": bench_config("olmo2_7b_bf16", CONFIG_BATCH["olmo2_7b_bf16"], 3, 3, dev,
+                                          stream_bases=True),
+            "olmo2_32b_gate_bf16": bench_config("olmo2_32b_gate_bf16", CONFIG_BATCH["olmo2_32b_gate_bf16"],
+                                                5, 3, dev),
         }
         fit = bench_fit(dev)
         configs["ekfac_correction"] = [bench_ekfac(dev, 768, 3072, 512, 32),

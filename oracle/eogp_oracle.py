@@ -35,6 +35,7 @@ Function map:
   onebit                Sec. 3.3, Eq. onebit; App. A.3 Eq. app_onebit_scale
   pack_bits/unpack_bits App. E.1 (per-module byte packing, Eq. app_payload)
   score_codes           Sec. 3.3 Eq. onebit_influence with both sides one-bit
+  onebit_dot_xor        the same +-1 inner product counted as k - 2 * (differing signs)
   score_paper           Sec. 3.3 Eq. onebit_influence; App. B.3 Eq. app_stored_influence
   score_fp              Sec. 3.1 (influence as an inner product of coordinates)
   srht                  Sec. 3.2 "A scalable alternative to PCA"; App. B.2 Eq. app_srht_definition
@@ -351,6 +352,25 @@ def score_codes_f32(train_codes: np.ndarray, train_scales: np.ndarray, ks: Seque
         sp = (qs[:, u, None] * ts[None, :, u]).astype(np.float32)
         acc = (acc + (sp * d).astype(np.float32)).astype(np.float32)
     return acc
+
+
+def onebit_dot_xor(train_words: np.ndarray, query_words: np.ndarray, k: int) -> np.ndarray:
+    """<b_i, b_q> of +-1 vectors of one module, for every stored row i of
+    train_words [N, ceil(k/32)] against one query row query_words [ceil(k/32)],
+    through the identity <b, b'> = k - 2 * #{c : b_c != b'_c}: the differing
+    signs are the set bits of the XOR of the packed codes (pad bits are 0 on
+    both sides), counted per word. A closed form of the +-1 sum that
+    score_codes forms explicitly, for checks over millions of stored rows.
+    Returns int64 [N]."""
+    t = np.asarray(train_words, np.uint32)
+    q = np.asarray(query_words, np.uint32)
+    x = np.bitwise_xor(t, q[None, :])
+    if hasattr(np, "bitwise_count"):
+        diff = np.bitwise_count(x).sum(axis=1, dtype=np.int64)
+    else:
+        table = np.array([bin(v).count("1") for v in range(256)], np.int64)
+        diff = table[x.view(np.uint8)].sum(axis=1)
+    return k - 2 * diff
 
 
 def score_paper(train_codes: np.ndarray, train_scales: np.ndarray, ks: Sequence[int],

@@ -3,14 +3,21 @@
 * GPT-2 stack: the compression in the exact launch configuration bench.py
   times (B = 512 examples per call, T = 512, m = 4096, k = 1024, device-side
   inputs), checked on sampled examples of one module of each shape.
-* OLMo 2 1B / 7B shapes and the 32B gate projection (T = 2048, m = 8192,
-  k = 2048): a few examples per distinct module shape.
+* OLMo 2 1B / 7B stacks and the 32B gate projection in the launch
+  configuration bench.py times (B = 128 / 32 / 64 examples per call, T = 2048,
+  m = 8192, k = 2048, device-side inputs): sampled examples of one module of
+  each distinct shape, with the oracle's own retained-set selection on the
+  full eigenvalue table checked against the plan's sets; and the same shapes
+  at B = 1-2 with host-drawn inputs and Haar bases.
+* OLMo 2 1B query scoring: Q = 4096 one-bit queries of 112 modules x 2048
+  bits against 65,536 stored codes, sampled stored rows bit for bit.
 * GPT-2 query scoring: Q = 1024 one-bit queries of 48 modules x 1024 bits
   (the bench's query workload) against 300 stored codes, every score bit for
   bit, dense and with the top-20 ranking fused.
 * Scoring sweep: 4,194,304 stored 16,384-bit codes, Q in {1, 64, 1024, 8192};
   sampled stored rows are checked bit for bit.
-* PCA fit at the GPT-2 size (10,000 fitting rows, m = 4096, k = 1024).
+* PCA fit at the GPT-2 size (10,000 fitting rows, m = 4096, k = 1024) and at
+  the OLMo size (10,000 rows, m = 8192, k = 2048).
 
 The oracle is given only the retained eigenvector columns: G~[j, i] for a
 retained (j, i) depends on Q_S[:, j] and Q_A[:, i] alone, so restricting Q_A,
@@ -99,6 +106,63 @@ def test_gpt2_stack_in_bench_launch_configuration():
         check_x_codes(x[examples].cpu().numpy().astype(np.float64),
                       codes[examples, u * words:(u + 1) * words].cpu().numpy().view(np.uint32),
                       scales[examples, u].cpu().numpy(), x_or, w.k)
+
+
+# ------------------------------------- OLMo / 32B in the bench's launch shape
+
+@pytest.mark.parametrize("name,n_ex", [("olmo2_1b_bf16", 3), ("olmo2_7b_bf16", 2),
+                                       ("olmo2_32b_gate_bf16", 3)])
+def test_bench_launch_configuration(name, n_ex):
+    """One module of each distinct shape compressed exactly as bench.py's
+    throughput line launches it (its batch, its inputs, codes written into the
+    stack's strided code matrix), checked on n_ex sampled examples against the
+    oracle."""
+    import bench
+    B = bench.CONFIG_BATCH[name]
+    dev = torch.device(DEV)
+    cs = bench.config_setup(name, B, dev)
+    w, per_layer, keys, Pt, descs, ws = (cs[x] for x in ("w", "per_layer", "keys", "Pt", "descs", "ws"))
+    words = w.k // 32
+    U = len(w.modules)
+    codes = torch.empty((B, U * words), dtype=torch.int32, device=dev)
+    scales = torch.empty((B, U), dtype=torch.float32, device=dev)
+    first = {}
+    for u, key in enumerate(keys):
+        first.setdefault((key[0], key[1]), u)
+    examples = np.linspace(0, B - 1, n_ex).astype(int)
+    P = Pt.float().cpu().numpy().T.astype(np.float64)
+    for (d_in, d_out), u in first.items():
+        key = keys[u]
+        L = per_layer[key]
+        E.compress_layer(descs[key], L["a"], L["s"], E.OUT_CODES,
+                         codes=codes[:, u * words:(u + 1) * words], scales=scales[:, u], ws=ws)
+        x = E.compress_layer(descs[key], L["a"], L["s"], E.OUT_COORDS, ws=ws)
+        E.sync_status()
+        if w.spectrum == "channel":
+            sp = synth.layer_spec(w, u, 1, 1)
+            lamA, lamS = sp.lam_A, sp.lam_S
+        else:
+            lamA, lamS = synth.power_spectrum(d_in, w.alpha), synth.power_spectrum(d_out, w.alpha)
+        Lam = O.kfac_eigenvalues(lamS, lamA)
+        lam = O.damping(Lam, w.damping_rel)
+        # the oracle's own top-m selection on the full table gives the plan's sets
+        j_or, i_or = O.select_retained(Lam, w.m)
+        R, C = L["plan"].sets()
+        np.testing.assert_array_equal(R, np.unique(j_or))
+        np.testing.assert_array_equal(C, np.unique(i_or))
+        a = L["a"][examples].float().cpu().numpy()
+        s_ = L["s"][examples].float().cpu().numpy()
+        QA_cols = L["VA"].float().cpu().numpy().T.astype(np.float64)
+        QS_cols = L["VS"].float().cpu().numpy().T.astype(np.float64)
+        z_or = oracle_retained(a, s_, QA_cols, QS_cols, R, C, Lam, lam, w.m)
+        x_or = O.project(z_or, P)
+        print(f"{name} module {u} ({d_in}->{d_out}) B={B} examples {list(examples)}")
+        check_x_codes(x[examples].cpu().numpy().astype(np.float64),
+                      codes[examples, u * words:(u + 1) * words].cpu().numpy().view(np.uint32),
+                      scales[examples, u].cpu().numpy(), x_or, w.k)
+        del x
+    del cs, per_layer, descs, ws, codes, scales
+    torch.cuda.empty_cache()
 
 
 # --------------------------------------------------------- OLMo-shaped layers
@@ -190,6 +254,35 @@ def test_scan_sweep_sampled_rows(Q):
     torch.cuda.empty_cache()
 
 
+# ------------------------------------------------- OLMo-1B query scoring
+
+def test_olmo2_1b_query_scoring_sampled_rows():
+    """Q = 4096 one-bit queries of 112 modules x 2048 bits (the OLMo-1B stack's
+    codes) against 65,536 stored codes: every score of 16 sampled stored rows
+    equals the oracle's float32 evaluation bit for bit."""
+    w = synth.WORKLOADS["olmo2_1b_bf16"]
+    U, k = len(w.modules), w.k
+    ks = [k] * U
+    N, Q = 65536, w.Q
+    W = U * k // 32
+    g = torch.Generator(device=DEV)
+    g.manual_seed(4096)
+    train = torch.randint(-2 ** 31, 2 ** 31 - 1, (N, W), generator=g, device=DEV, dtype=torch.int32)
+    query = torch.randint(-2 ** 31, 2 ** 31 - 1, (Q, W), generator=g, device=DEV, dtype=torch.int32)
+    tsc = torch.exp(0.5 * torch.randn((N, U), generator=g, device=DEV))
+    qsc = torch.exp(0.5 * torch.randn((Q, U), generator=g, device=DEV))
+    out = E.score(train, tsc, ks, E.SCORE_CODES, query, qsc)
+    E.sync_status()
+    rows = np.arange(0, N, 4099)
+    got = out[:, rows].cpu().numpy()
+    del out
+    want = O.score_codes_f32(train[rows].cpu().numpy().view(np.uint32), tsc[rows].cpu().numpy(), ks,
+                             query.cpu().numpy().view(np.uint32), qsc.cpu().numpy())
+    np.testing.assert_array_equal(got, want)
+    del train, query
+    torch.cuda.empty_cache()
+
+
 # -------------------------------------------------------------------- PCA fit
 
 def test_fit_pca_gpt2_size():
@@ -236,3 +329,13 @@ def test_gpt2_query_scoring_all_scores(eogp_options):
             E.sync_status()
             np.testing.assert_array_equal(idx.cpu().numpy(), want_i)
             np.testing.assert_array_equal(vals.cpu().numpy().astype(np.float64), want_v)
+
+
+def test_fit_pca_olmo_size():
+    """The fit at the OLMo workloads' size: 10,000 fitting rows, m = 8192, k = 2048."""
+    from test_gpu_parity import subspace_checks
+    n, m, k = 10000, 8192, 2048
+    Z = synth.first_stage_like(n, m, seed=6)
+    Pt, eig = E.fit_pca(torch.from_numpy(Z).to(DEV), k)
+    E.sync_status()
+    subspace_checks(Pt.cpu().numpy(), eig.cpu().numpy(), Z, k)

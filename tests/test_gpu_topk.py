@@ -201,11 +201,23 @@ def test_topk_scan_scale_sampled_queries():
     want_v, want_i = O.top_k(dn, K)
     np.testing.assert_array_equal(idx[qsel].cpu().numpy(), want_i)
     np.testing.assert_array_equal(vals[qsel].cpu().numpy().astype(np.float64), want_v)
-    # the dense scores behind the comparison are the oracle's, on sampled stored rows
+    # the dense scores behind the comparison are the oracle's: on sampled stored
+    # rows by explicit +-1 sums, and on every stored row by the XOR / population
+    # count form, in the same float32 order (one module: fl(fl(s_q s_i) d))
     rows = np.unique(np.concatenate([want_i.reshape(-1), np.arange(0, N, 524287)]))
     tr = train[rows].cpu().numpy().view(np.uint32)
     ref = O.score_codes_f32(tr, tsc[rows].cpu().numpy(), [k], query[qsel].cpu().numpy().view(np.uint32),
                             qsc[qsel].cpu().numpy())
     np.testing.assert_array_equal(dn[:, rows], ref)
+    qh = query[qsel].cpu().numpy().view(np.uint32)
+    qsh = qsc[qsel].cpu().numpy()[:, 0]
+    ts_all = tsc.cpu().numpy()[:, 0]
+    step = 1 << 18
+    for r0 in range(0, N, step):
+        tw = train[r0:r0 + step].cpu().numpy().view(np.uint32)
+        for j in range(len(qsel)):
+            d = O.onebit_dot_xor(tw, qh[j], k).astype(np.float32)
+            sp = (qsh[j] * ts_all[r0:r0 + step]).astype(np.float32)
+            np.testing.assert_array_equal(dn[j, r0:r0 + step], (sp * d).astype(np.float32))
     del train, query, dense
     torch.cuda.empty_cache()

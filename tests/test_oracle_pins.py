@@ -331,6 +331,22 @@ def test_scores():
     check_scores(O, 23)
 
 
+@pytest.mark.parametrize("counter", ["bitwise_count", "byte_table"])
+def test_onebit_dot_xor_equals_pm1_sums(counter, monkeypatch):
+    """The XOR / population-count form of the one-bit inner product equals the
+    explicit +-1 sum, for ragged and word-multiple k (both counting routes)."""
+    if counter == "byte_table":
+        monkeypatch.delattr(np, "bitwise_count", raising=False)
+    rng = np.random.default_rng(41)
+    for k in (1, 31, 32, 33, 100, 1024, 2049):
+        bt = rng.integers(0, 2, (50, k)).astype(bool)
+        bq = rng.integers(0, 2, (3, k)).astype(bool)
+        tw, qw = O.pack_bits(bt), O.pack_bits(bq)
+        for q in range(3):
+            want = np.where(bt, 1, -1) @ np.where(bq[q], 1, -1)
+            np.testing.assert_array_equal(O.onebit_dot_xor(tw, qw[q], k), want)
+
+
 def test_norm_preservation():
     """An orthogonal rotation preserves the Frobenius norm and inner products."""
     rng = np.random.default_rng(29)
