@@ -1075,29 +1075,11 @@ extern "C" int eogp_fit_pca_workspace_size(int n, int m, int k, size_t* bytes) {
   clear_error();
   if (!bytes) return set_error(EOGP_EINVAL, "bytes is NULL");
   if (n < 1 || m < 1 || k < 1 || k > std::min(n, m)) return set_error(EOGP_EINVAL, "need 1 <= k <= min(n, m)");
-  if (std::min(n, m) > 12288) return set_error(EOGP_EUNSUPPORTED, "min(n, m) > 12288");
+  if (!fit_pca_supported(n, m, k))
+    return set_error(EOGP_EUNSUPPORTED, "fit size out of range (dense solver: min(n, m) <= 12288; subspace "
+                     "solver: min(n, m) <= 32768 and k + max(64, k / 4) <= 12288)");
   *bytes = fit_pca_ws_bytes(n, m, k);
   return EOGP_OK;
-}
-
-static PcaWs carve_pca_ws(void* ws, int n, int m, int k) {
-  const int nn = std::min(n, m);
-  char* w = static_cast<char*>(ws);
-  size_t off = 0;
-  auto take = [&](size_t bytes) {
-    char* p = w + off;
-    off += al256(bytes);
-    return p;
-  };
-  PcaWs pw;
-  pw.A = reinterpret_cast<double*>(take(static_cast<size_t>(nn) * nn * 8));
-  pw.Vt = reinterpret_cast<double*>(take(static_cast<size_t>(nn) * nn * 8));
-  pw.cs = reinterpret_cast<double*>(take((static_cast<size_t>(nn) / 2 + 1) * 2 * 8));
-  pw.mu = reinterpret_cast<double*>(take(static_cast<size_t>(nn) * 8));
-  pw.sel = reinterpret_cast<int*>(take(static_cast<size_t>(k) * 4));
-  pw.red = reinterpret_cast<double*>(take(4 * 8));
-  pw.Pr = n < m ? reinterpret_cast<double*>(take(static_cast<size_t>(k) * m * 8)) : nullptr;
-  return pw;
 }
 
 extern "C" int eogp_fit_pca(const float* Z, int n, int m, int ldz, int k, void* Pt, int ld_pt,
@@ -1110,7 +1092,7 @@ extern "C" int eogp_fit_pca(const float* Z, int n, int m, int ldz, int k, void* 
   if (pt_dtype != EOGP_F32 && pt_dtype != EOGP_BF16) return set_error(EOGP_EINVAL, "bad pt_dtype");
   if (!ws || ws_bytes < need) return set_error(EOGP_EWORKSPACE, "workspace of %zu bytes needed", need);
   if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
-  return fit_pca_device(Z, n, m, ldz, k, Pt, ld_pt, pt_dtype, eig, carve_pca_ws(ws, n, m, k), status_word(),
+  return fit_pca_device(Z, n, m, ldz, k, Pt, ld_pt, pt_dtype, eig, ws, status_word(),
                         reinterpret_cast<cudaStream_t>(stream));
 }
 
@@ -1145,8 +1127,8 @@ extern "C" int eogp_fit_pca_from_moment(const double* C, int m, int ldc, int n_t
   if (pt_dtype != EOGP_F32 && pt_dtype != EOGP_BF16) return set_error(EOGP_EINVAL, "bad pt_dtype");
   if (!ws || ws_bytes < need) return set_error(EOGP_EWORKSPACE, "workspace of %zu bytes needed", need);
   if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
-  return fit_pca_device(nullptr, n_total, m, m, k, Pt, ld_pt, pt_dtype, eig, carve_pca_ws(ws, m, m, k),
-                        status_word(), reinterpret_cast<cudaStream_t>(stream), C, ldc);
+  return fit_pca_device(nullptr, n_total, m, m, k, Pt, ld_pt, pt_dtype, eig, ws, status_word(),
+                        reinterpret_cast<cudaStream_t>(stream), C, ldc);
 }
 
 // ============================================================== pack, score

@@ -181,6 +181,13 @@ cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, 
                            const void* W, int ldw, int Wrows, int splits, int epi, void* out0,
                            void* out1, int ldo, size_t slab, TcGemmCfg cfg, unsigned* status,
                            cudaStream_t st);
+// out[M x N] (row stride ldo, fp32) = alpha * (Ah Bh^T + Ah Bl^T + Al Bh^T): both
+// operands bf16 hi/lo pairs, K-major ([M x K] and [N x K], row strides lda, ldb
+// multiples of 8 elements, 16-byte aligned); an operand pair stands for an fp32
+// matrix to about 16 significant bits, and lo x lo is below that.
+cudaError_t launch_tc_gemm_hl(int M, int N, int K, const void* Ah, const void* Al, int lda, const void* Bh,
+                              const void* Bl, int ldb, float* out, int ldo, float alpha, unsigned* status,
+                              cudaStream_t st);
 // Persistent rotation GEMM: hi/lo = split(X[M x K] W[Wrows x K]^T), columns < ldo
 // (a multiple of 128), rows M = B * T, written in the blocked layout
 // [B][ldo / 128][T][128] that launch_tc_contract reads.
@@ -196,19 +203,14 @@ cudaError_t launch_tc_contract(const void* St_hi, const void* St_lo, int ldS, co
                                int num_sms, unsigned* status, cudaStream_t st);
 
 // k_pca.cu
-struct PcaWs {
-  double* A;     // [n' x n'] symmetric matrix, diagonalised in place
-  double* Vt;    // [n' x n'] eigenvectors as rows
-  double* cs;    // [n'/2+1][2] rotation (c, s)
-  double* mu;    // [n']
-  int* sel;      // [k]
-  double* red;   // [4] reduction scratch
-  double* Pr;    // [k x m] raw directions (Gram route)
-};
+// Whether the fit handles this size (the subspace solver for large problems,
+// the dense Jacobi solver otherwise), and the workspace it needs.
+bool fit_pca_supported(int n, int m, int k);
 // C_in (optional): a summed second moment sum_r z_r z_r^T [m x ldc] of n rows in
-// place of Z (covariance route; Z is then unused).
+// place of Z (covariance route; Z is then unused). ws: fit_pca_ws_bytes(n, m, k)
+// bytes, 256-byte aligned (fit_pca_ws_bytes(m, m, k) with C_in).
 int fit_pca_device(const float* Z, int n, int m, int ldz, int k, void* Pt, int ld_pt, int pt_dtype,
-                   float* eig, PcaWs ws, unsigned* status, cudaStream_t st, const double* C_in = nullptr,
+                   float* eig, void* ws, unsigned* status, cudaStream_t st, const double* C_in = nullptr,
                    int ldc = 0);
 cudaError_t second_moment_device(const float* Z, int n, int m, int ldz, double* C, int ldc, int accumulate,
                                  cudaStream_t st);

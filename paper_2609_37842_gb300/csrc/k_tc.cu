@@ -36,7 +36,8 @@ constexpr int kThreads = 192;
 constexpr uint32_t kABytes = 128u * 64u * 2u;  // 128 rows x 64 bf16 (one 128-byte swizzle row each)
 
 struct GemmArgs {
-  int M, N, K, BN, stages, nA, kbps, epi, ldo;
+  int M, N, K, BN, stages, nA, nW, kbps, epi, ldo;
+  float alpha;  // epilogue 1: output scale
   void* out0;
   void* out1;
   size_t slab;
@@ -54,12 +55,13 @@ __device__ __forceinline__ uint32_t tmem_cols_for(int n) {
 
 __global__ void __launch_bounds__(kThreads, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__ CUtensorMap tmX1,
-              const __grid_constant__ CUtensorMap tmW, const GemmArgs g) {
+              const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmW1,
+              const GemmArgs g) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t b_bytes = static_cast<uint32_t>(g.BN) * 128u;
-  const uint32_t stage_bytes = static_cast<uint32_t>(g.nA) * kABytes + b_bytes;
+  const uint32_t stage_bytes = static_cast<uint32_t>(g.nA) * kABytes + static_cast<uint32_t>(g.nW) * b_bytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(g.stages) * stage_bytes);
   uint64_t* empty = full + g.stages;
   uint64_t* done = empty + g.stages;
@@ -75,6 +77,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tmX0);
     if (g.nA > 1) tma_prefetch_desc(&tmX1);
     tma_prefetch_desc(&tmW);
+    if (g.nW > 1) tma_prefetch_desc(&tmW1);
     for (int s = 0; s < g.stages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
@@ -106,6 +109,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_2d(st, &tmX0, kx, m0, &full[s]);
         if (g.nA > 1) tma_load_2d(st + kABytes, &tmX1, kx, m0, &full[s]);
         tma_load_2d(st + g.nA * kABytes, &tmW, kx, n0, &full[s]);
+        if (g.nW > 1) tma_load_2d(st + g.nA * kABytes + b_bytes, &tmW1, kx, n0, &full[s]);
       }
     }
     __syncwarp();
@@ -127,10 +131,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t sb = sa + g.nA * kABytes;
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk) {
-          const uint64_t bd = sdesc_sw128(sb + kk * 32, 16, 1024);
-          for (int a = 0; a < g.nA; ++a) {
-            const uint64_t ad = sdesc_sw128(sa + a * kABytes + kk * 32, 16, 1024);
-            tc_mma_f16(tmem, ad, bd, idesc, (i | kk | a) != 0 ? 1u : 0u);
+          for (int w = 0; w < g.nW; ++w) {
+            const uint64_t bd = sdesc_sw128(sb + w * b_bytes + kk * 32, 16, 1024);
+            for (int a = 0; a < g.nA; ++a) {
+              if (a == 1 && w == 1) continue;  // lo x lo: below the hi/lo pair's precision
+              const uint64_t ad = sdesc_sw128(sa + a * kABytes + kk * 32, 16, 1024);
+              tc_mma_f16(tmem, ad, bd, idesc, (i | kk | a | w) != 0 ? 1u : 0u);
+            }
           }
         }
         tc_commit(&empty[s]);
@@ -183,6 +190,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int col = n0 + c;
           if (row < g.M && col < g.N) {
             float* o = out + static_cast<size_t>(row) * g.ldo + col;
+            if (g.alpha != 1.0f) {
+#pragma unroll
+              for (int e = 0; e < 16; ++e) v[e] *= g.alpha;
+            }
             if (col + 16 <= g.N) {
 #pragma unroll
               for (int e = 0; e < 4; ++e)
@@ -608,8 +619,8 @@ __global__ void k_ekfac_finalize(const float* __restrict__ part, int n_chunks, i
   }
 }
 
-size_t gemm_smem_bytes(int BN, int stages, int nA) {
-  return 1024 + static_cast<size_t>(stages) * (nA * kABytes + BN * 128u) + (2 * stages + 1) * 8 + 16;
+size_t gemm_smem_bytes(int BN, int stages, int nA, int nW = 1) {
+  return 1024 + static_cast<size_t>(stages) * (nA * kABytes + nW * BN * 128u) + (2 * stages + 1) * 8 + 16;
 }
 
 size_t contract_smem_bytes(int stages) {
@@ -1011,13 +1022,14 @@ static int tmap_bf16_blocked(CUtensorMap* tm, const void* base, uint64_t T, uint
                    CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
-cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, int ldx,
-                                const void* W, int ldw, int Wrows, int splits, int epi,
-                                void* out0, void* out1, int ldo, size_t slab, TcGemmCfg cfg,
-                                unsigned* status, cudaStream_t st) {
+static cudaError_t launch_tc_gemm_impl(int M, int N, int K, const void* X0, const void* X1, int ldx,
+                                      const void* W, const void* W1, int ldw, int Wrows, int splits, int epi,
+                                      void* out0, void* out1, int ldo, size_t slab, float alpha,
+                                      TcGemmCfg cfg, unsigned* status, cudaStream_t st) {
   if (M <= 0 || N <= 0) return cudaSuccess;
   const int nA = X1 ? 2 : 1;
-  CUtensorMap tX0, tX1, tW;
+  const int nW = W1 ? 2 : 1;
+  CUtensorMap tX0, tX1, tW, tW1;
   if (tmap_bf16_2d(&tX0, X0, static_cast<uint64_t>(K), static_cast<uint64_t>(M), ldx, 64, 128))
     return cudaErrorInvalidValue;
   if (nA > 1) {
@@ -1026,6 +1038,11 @@ cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, 
     tX1 = tX0;
   }
   if (tmap_bf16_2d(&tW, W, K, Wrows, ldw, 64, cfg.BN)) return cudaErrorInvalidValue;
+  if (nW > 1) {
+    if (tmap_bf16_2d(&tW1, W1, K, Wrows, ldw, 64, cfg.BN)) return cudaErrorInvalidValue;
+  } else {
+    tW1 = tW;
+  }
   const int nkb = (K + 63) / 64;
   splits = max(1, min(splits, nkb));
   const int kbps = (nkb + splits - 1) / splits;
@@ -1037,20 +1054,38 @@ cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, 
   g.BN = cfg.BN;
   g.stages = cfg.stages;
   g.nA = nA;
+  g.nW = nW;
   g.kbps = kbps;
   g.epi = epi;
   g.ldo = ldo;
+  g.alpha = alpha;
   g.out0 = out0;
   g.out1 = out1;
   g.slab = slab;
   g.status = status;
-  const size_t smem = gemm_smem_bytes(cfg.BN, cfg.stages, nA);
+  const size_t smem = gemm_smem_bytes(cfg.BN, cfg.stages, nA, nW);
   cudaError_t e = cudaFuncSetAttribute(k_tc_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   dim3 grid((N + cfg.BN - 1) / cfg.BN, (M + 127) / 128, splits);
-  k_tc_gemm<<<grid, kThreads, smem, st>>>(tX0, tX1, tW, g);
+  k_tc_gemm<<<grid, kThreads, smem, st>>>(tX0, tX1, tW, tW1, g);
   return cudaGetLastError();
+}
+
+cudaError_t launch_tc_gemm(int M, int N, int K, const void* X0, const void* X1, int ldx,
+                                const void* W, int ldw, int Wrows, int splits, int epi,
+                                void* out0, void* out1, int ldo, size_t slab, TcGemmCfg cfg,
+                                unsigned* status, cudaStream_t st) {
+  return launch_tc_gemm_impl(M, N, K, X0, X1, ldx, W, nullptr, ldw, Wrows, splits, epi, out0, out1, ldo,
+                             slab, 1.0f, cfg, status, st);
+}
+
+cudaError_t launch_tc_gemm_hl(int M, int N, int K, const void* Ah, const void* Al, int lda, const void* Bh,
+                              const void* Bl, int ldb, float* out, int ldo, float alpha, unsigned* status,
+                              cudaStream_t st) {
+  // 128-column tiles: a stage holds 2 x 16 KB of A and 2 x 16 KB of B, three stages.
+  return launch_tc_gemm_impl(M, N, K, Ah, Al, lda, Bh, Bl, ldb, N, 1, 1, out, nullptr, ldo, 0, alpha,
+                             TcGemmCfg{128, 3}, status, st);
 }
 
 // CTA pairs measured faster for short reductions (K <= 1536: the hi/lo

@@ -291,7 +291,9 @@ def subspace_checks(Pt, eig, Z, k):
         assert s.min() > 1 - 1e-3
 
 
-@pytest.mark.parametrize("n,m,k", [(256, 512, 128), (1000, 300, 64), (77, 40, 40)])
+@pytest.mark.parametrize("n,m,k", [(256, 512, 128), (1000, 300, 64), (77, 40, 40),
+                                   (1500, 3000, 256),    # subspace solver, Gram route (n < m)
+                                   (4000, 2000, 300)])   # subspace solver, covariance route
 def test_fit_pca(n, m, k):
     Z = synth.first_stage_like(n, m, seed=n + m)
     Pt, eig = E.fit_pca(torch.from_numpy(Z).to(DEV), k)
@@ -299,7 +301,8 @@ def test_fit_pca(n, m, k):
     subspace_checks(Pt.cpu().numpy(), eig.cpu().numpy(), Z, k)
 
 
-@pytest.mark.parametrize("n,m,k", [(1000, 300, 64), (900, 512, 128)])
+@pytest.mark.parametrize("n,m,k", [(1000, 300, 64), (900, 512, 128),
+                                   (3000, 1536, 200)])   # subspace solver on the summed moment
 def test_fit_pca_from_summed_moments(n, m, k):
     """The sharded fit: second moments of three row shards added on the device
     (accumulate) and the fit from the sum match the oracle like a direct fit."""
