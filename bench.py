@@ -1,23 +1,30 @@
 #!/usr/bin/env python
 """Throughput of the EOGP hot path on GB300.
 
-One step compresses one batch of B = 256 training examples through every module of
-the GPT-2-small-shaped stack (48 linears, T = 512 tokens, m = 4096 retained
-first-stage coordinates, k = 1024 PCA coordinates per module) into one-bit
-codes: Kronecker rotations, per-example contraction with the scale-and-gather
-epilogue, PCA projection, sign packing (Alg. 1 "Storing one training
-example"). Inputs are synthetic (Gaussian a and s, Haar eigenbases,
-power-law spectra with exponent 1.2), drawn on the device before timing; each
-step reads B x 151 MB of inputs, far more than L2, so no flush is needed.
+Headline: one step compresses one batch of B = 32 training examples through all
+224 modules of the OLMo-2-7B-shaped stack (32 layers x {q, k, v, o 4096 x
+4096; gate, up 4096 -> 11008; down 11008 -> 4096}, T = 2048 tokens, m = 8192
+retained first-stage coordinates, k = 2048 PCA coordinates per module) into
+one-bit codes: Kronecker rotations, per-example contraction with the
+scale-and-gather epilogue, PCA projection, sign packing (Alg. 1 "Storing one
+training example"). The retained eigenvector rows of every layer live in
+page-locked host memory and are copied one layer ahead of its compute on a side
+stream. Inputs are synthetic (Gaussian a and s, Haar eigenbases, power-law
+spectra with exponent 1.0), drawn on the device before timing; one input buffer
+per module type serves the 32 layers, and each module's inputs (0.5-2 GB) exceed
+L2, so no flush is needed.
 
-The JSON line's `value` is examples compressed per second per layer stack
-(whole job, all ranks). `scoring` reports the query x train scan (Q = 1024
-one-bit queries against N = 16384 stored codes). `e2e` repeats the
-compression through the C-ABI's host-input call (eogp_compress_layer_host)
-with the inputs in pinned host memory: the call's host-to-device copies and
-the device-to-host read of the codes are inside the timed region.
+`value` is examples compressed per second per layer stack (whole job, all
+ranks). `e2e` repeats the step through the C-ABI's host-input call
+(eogp_compress_layer_host) with a, s and the eigenbases in page-locked host
+memory: the call's host-to-device copies and the device-to-host read of the
+codes are inside the timed region; the plain host-to-device copy rate of the
+same run is reported beside it. `roofline` is that of the rotation kernels,
+and `roofline.others` carries the other timed kernels' rooflines, the
+query x train scoring rates included. The GPT-2, OLMo-1B, 32B-gate and fp32
+stacks, the scoring workloads and the PCA fit follow in the same line.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--batch B]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--batch B] [--workload NAME]
     python bench.py --impl reference ...   # the CPU oracle on the host cores
 """
 from __future__ import annotations
@@ -38,15 +45,18 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-WORKLOAD = "gpt2_small_bf16"
+HEADLINE = "olmo2_7b_bf16"
 METRIC = "training examples compressed/sec per layer stack"
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-# dram__bytes_read.sum + dram__bytes_write.sum per rotation launch from the committed
-# ncu capture (profiles/), or None when the kernel changed after the capture.
-ROTATE_TRAFFIC_BYTES = 1415.1e6  # mean over one transformer block (8 launches) at B = 512
 # Examples per compression call (one step) of each workload's throughput line.
 CONFIG_BATCH = {"gpt2_small_bf16": 512, "tiny_f32": 4096, "olmo2_1b_bf16": 128, "olmo2_7b_bf16": 32,
                 "olmo2_32b_gate_bf16": 64}
+# dram__bytes_read.sum + dram__bytes_write.sum per rotation launch from the committed
+# ncu captures (profiles/), as (bytes per launch, examples per launch at capture), or
+# None when the kernel changed after the capture. Traffic grows with the examples
+# per launch, so it is scaled to the bench's batch.
+ROTATE_TRAFFIC = {"gpt2_small_bf16": (1415.1e6, 512), "olmo2_7b_bf16": (267.2e6, 8)}
+E2E_BATCH = {"olmo2_7b_bf16": 8, "gpt2_small_bf16": 128}
 
 
 def score_peak(ks, probes, bf16_burst, peaks_src):
@@ -132,7 +142,8 @@ class ClockSampler:
 
 # ----------------------------------------------------------- workload
 def build_stack(w, B, dev, seed):
-    """Per-module plans, retained eigenvector rows, PCA directions and inputs."""
+    """Per-module plans, retained eigenvector rows, PCA directions and inputs
+    (one input buffer per module)."""
     import torch
     from paper_2609_37842_gb300 import eogp as E
     from paper_2609_37842_gb300 import synth
@@ -178,100 +189,6 @@ def rotate_flops(mods, B, T):
     return sum(2.0 * B * T * (md["d_in"] * md["nC"] + md["d_out"] * md["nR"]) for md in mods)
 
 
-# ------------------------------------------------------------ CPU oracle
-def cpu_sample(w, n_examples, seed=1):
-    """Time the oracle compressing `n_examples` examples through one module of each
-    distinct shape; returns (seconds per example per stack, cores, description)."""
-    import numpy as np
-    from oracle import eogp_oracle as O
-    from paper_2609_37842_gb300 import synth
-    shapes = {}
-    for u, mod in enumerate(w.modules):
-        shapes.setdefault((mod.d_in, mod.d_out), []).append(u)
-    rng = np.random.default_rng(seed)
-    total = 0.0
-    per_shape = {}
-    flops = 0.0
-    for (d_in, d_out), us in shapes.items():
-        u = us[0]
-        QA = synth.round_bf16(synth.haar_orthogonal(d_in, rng))
-        QS = synth.round_bf16(synth.haar_orthogonal(d_out, rng))
-        lamA, lamS = synth.power_spectrum(d_in, w.alpha), synth.power_spectrum(d_out, w.alpha)
-        P = synth.round_bf16(synth.haar_orthogonal(w.m, rng, w.k))
-        a, s = synth.layer_inputs(w, u, n_examples)
-        t0 = time.perf_counter()
-        Lam = O.kfac_eigenvalues(lamS, lamA)
-        lam = O.damping(Lam, w.damping_rel)
-        O.compress_layer(a, s, QA, QS, Lam, lam, w.m, P)
-        dt = (time.perf_counter() - t0) / n_examples
-        total += dt * len(us)
-        per_shape[f"{d_in}->{d_out}"] = 1.0 / dt
-        # the oracle's dense work per example: G (2 T d_out d_in), Q_S^T G Q_A
-        # (2 d_out d_in (d_in + d_out)), P^T z (2 m k)
-        flops += len(us) * (2.0 * w.T * d_out * d_in + 2.0 * d_out * d_in * (d_in + d_out) +
-                            2.0 * w.m * w.k)
-    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
-    desc = (f"{n_examples} example(s) x one module of each of the {len(shapes)} distinct shapes, "
-            f"scaled by the shape counts to the {len(w.modules)}-module stack")
-    cpu_sample.details = {"examples_per_s_per_shape": per_shape,
-                          "oracle_GFLOPs": flops / total / 1e9 if total else None}
-    return total, cores, desc
-
-
-def cpu_score_sample(seconds=3.0):
-    """Oracle one-bit scores/s (float32 evaluation order) on the GPT-2 query shape
-    (48 modules of 1024 bits): repeated batches of 64 stored rows x 4 queries for
-    about `seconds` of scoring (input generation not timed)."""
-    import numpy as np
-    from oracle import eogp_oracle as O
-    rng = np.random.default_rng(3)
-    ks = [1024] * 48
-    Q, n = 4, 64
-    qc = O.pack_concat([rng.integers(0, 2, (Q, k)).astype(bool) for k in ks])
-    qs = rng.lognormal(0, 0.5, (Q, len(ks))).astype(np.float32)
-    done, busy = 0, 0.0
-    while busy < seconds:
-        tc = O.pack_concat([rng.integers(0, 2, (n, k)).astype(bool) for k in ks])
-        ts = rng.lognormal(0, 0.5, (n, len(ks))).astype(np.float32)
-        t1 = time.perf_counter()
-        O.score_codes_f32(tc, ts, ks, qc, qs)
-        busy += time.perf_counter() - t1
-        done += n * Q
-    return done / busy
-
-
-def run_reference(args):
-    rank = int(os.environ.get("RANK", "0"))
-    if rank != 0:
-        return 0
-    from paper_2609_37842_gb300 import synth
-    w = synth.WORKLOADS[WORKLOAD]
-    for _ in range(args.warmup):
-        cpu_sample(w, 1)
-    ts = []
-    cores, desc = None, None
-    for _ in range(args.steps):
-        t, cores, desc = cpu_sample(w, 1)
-        ts.append(t)
-    sec = sum(ts)
-    value = args.steps / sec
-    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "examples/s",
-            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": 1000 * sec / args.steps, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "batch": 1, "seq_len": w.T, "m": w.m, "k": w.k,
-                       "modules": len(w.modules)},
-            "cpu_baseline": {"value": value, "unit": "examples/s", "cores": cores,
-                             "kind": "oracle", "sample": desc},
-            "e2e": {"value": value, "unit": "examples/s", "h2d_bytes_per_step": 0,
-                    "d2h_bytes_per_step": 0}}
-    print(json.dumps(line))
-    return 0
-
-
-
-
-# ------------------------------------------------ other workloads (throughput)
 def _config_stack(name, B, dev, gh, g):
     """Plans, retained eigenvector rows and inputs for one layer's module types of a
     workload; the per-layer inputs are reused by every layer (the work per layer is
@@ -344,113 +261,259 @@ def config_setup(name, B, dev):
     return dict(w=w, per_layer=per_layer, keys=keys, Pt=Pt, descs=descs, ws=ws)
 
 
-def bench_config(name, B, steps, warmup, dev, stream_bases=False):
-    """Examples/s per layer stack for one workload; with stream_bases the retained
-    eigenvector rows of every layer live in pinned host memory and are copied to
-    the device one layer ahead of its compute on a side stream."""
-    import torch
-    from paper_2609_37842_gb300 import eogp as E
-    cs = config_setup(name, B, dev)
-    w, per_layer, keys, Pt, descs, ws = (cs[x] for x in ("w", "per_layer", "keys", "Pt", "descs", "ws"))
-    words = (w.k + 31) // 32
-    U = len(w.modules)
-    codes = torch.empty((B, U * words), dtype=torch.int32, device=dev)
-    scales = torch.empty((B, U), dtype=torch.float32, device=dev)
-    stream = torch.cuda.current_stream()
-    nmod_layer = len(set(keys))
-    layers = U // nmod_layer if name.startswith("olmo") else 1
-    host_bases = dev_bases = None
-    if stream_bases:
-        # one pinned host copy per module type (every layer copies it again) and two
-        # device slots, so layer l+1's rows land while layer l computes
-        host_one = {k: (L["VA"].cpu().pin_memory(), L["VS"].cpu().pin_memory())
-                    for k, L in per_layer.items()}
-        host_bases = [host_one] * layers
-        dev_bases = [{k: (torch.empty_like(L["VA"]), torch.empty_like(L["VS"]))
-                      for k, L in per_layer.items()} for _ in range(2)]
-        slot_descs = [{k: E.layer_desc(per_layer[k]["plan"], w.T, w.k, dev_bases[sl][k][0],
-                                       dev_bases[sl][k][1], Pt) for k in per_layer} for sl in range(2)]
-        cstream = torch.cuda.Stream()
-        landed = [torch.cuda.Event() for _ in range(2)]
-        freed = [None, None]
+class Stack:
+    """One workload's compression step: B examples through every module of the
+    stack into one-bit codes. With stream_bases the retained eigenvector rows of
+    every layer live in page-locked host memory and are copied to the device one
+    layer ahead of its compute on a side stream (two device slots)."""
 
-    def step():
-        if not stream_bases:
-            for u, key in enumerate(keys):
-                L = per_layer[key]
-                E.compress_layer(descs[key], L["a"], L["s"], E.OUT_CODES,
-                                 codes=codes[:, u * words:(u + 1) * words], scales=scales[:, u], ws=ws)
+    def __init__(self, name, B, dev, stream_bases=False, modules=0):
+        import dataclasses
+        import torch
+        from paper_2609_37842_gb300 import eogp as E
+        self.E = E
+        self.name, self.B, self.dev = name, B, dev
+        cs = config_setup(name, B, dev)
+        self.w, self.per_layer, self.keys, self.Pt, self.descs, self.ws = (
+            cs[x] for x in ("w", "per_layer", "keys", "Pt", "descs", "ws"))
+        if modules:
+            self.keys = self.keys[:modules]
+            self.w = dataclasses.replace(self.w, modules=self.w.modules[:modules])
+        w = self.w
+        self.words = (w.k + 31) // 32
+        self.U = len(self.keys)
+        self.codes = torch.empty((B, self.U * self.words), dtype=torch.int32, device=dev)
+        self.scales = torch.empty((B, self.U), dtype=torch.float32, device=dev)
+        self.stream = torch.cuda.current_stream()
+        self.nmod_layer = len(set(self.keys))
+        self.layers = max(1, self.U // self.nmod_layer) if name.startswith("olmo") else 1
+        self.stream_bases = stream_bases and self.layers > 1
+        if self.stream_bases:
+            pl = self.per_layer
+            self.host_one = {k: (L["VA"].cpu().pin_memory(), L["VS"].cpu().pin_memory()) for k, L in pl.items()}
+            self.dev_bases = [{k: (torch.empty_like(L["VA"]), torch.empty_like(L["VS"])) for k, L in pl.items()}
+                              for _ in range(2)]
+            self.slot_descs = [{k: E.layer_desc(pl[k]["plan"], w.T, w.k, self.dev_bases[sl][k][0],
+                                                self.dev_bases[sl][k][1], self.Pt) for k in pl} for sl in range(2)]
+            self.cstream = torch.cuda.Stream()
+            self.landed = [torch.cuda.Event() for _ in range(2)]
+            self.freed = [None, None]
+
+    def _module(self, u, desc):
+        L = self.per_layer[self.keys[u]]
+        wd = self.words
+        self.E.compress_layer(desc, L["a"], L["s"], self.E.OUT_CODES, codes=self.codes[:, u * wd:(u + 1) * wd],
+                              scales=self.scales[:, u], ws=self.ws)
+
+    def step(self):
+        import torch
+        if not self.stream_bases:
+            for u, key in enumerate(self.keys):
+                self._module(u, self.descs[key])
             return
 
         def issue_copy(layer):
             sl = layer % 2
-            if freed[sl] is not None:
-                cstream.wait_event(freed[sl])
-            with torch.cuda.stream(cstream):
-                for k in per_layer:
-                    dev_bases[sl][k][0].copy_(host_bases[layer][k][0], non_blocking=True)
-                    dev_bases[sl][k][1].copy_(host_bases[layer][k][1], non_blocking=True)
-                landed[sl].record(cstream)
+            if self.freed[sl] is not None:
+                self.cstream.wait_event(self.freed[sl])
+            with torch.cuda.stream(self.cstream):
+                for k in self.per_layer:
+                    self.dev_bases[sl][k][0].copy_(self.host_one[k][0], non_blocking=True)
+                    self.dev_bases[sl][k][1].copy_(self.host_one[k][1], non_blocking=True)
+                self.landed[sl].record(self.cstream)
         issue_copy(0)
-        for layer in range(layers):
+        for layer in range(self.layers):
             sl = layer % 2
-            if layer + 1 < layers:
+            if layer + 1 < self.layers:
                 issue_copy(layer + 1)
-            stream.wait_event(landed[sl])
-            for j in range(nmod_layer):
-                u = layer * nmod_layer + j
-                key = keys[u]
-                L = per_layer[key]
-                E.compress_layer(slot_descs[sl][key], L["a"], L["s"], E.OUT_CODES,
-                                 codes=codes[:, u * words:(u + 1) * words], scales=scales[:, u], ws=ws)
+            self.stream.wait_event(self.landed[sl])
+            for j in range(self.nmod_layer):
+                u = layer * self.nmod_layer + j
+                self._module(u, self.slot_descs[sl][self.keys[u]])
             ev = torch.cuda.Event()
-            ev.record(stream)
-            freed[sl] = ev
+            ev.record(self.stream)
+            self.freed[sl] = ev
 
-    for _ in range(warmup):
-        step()
+    def timed(self, steps, warmup, clocks=None, barrier=None):
+        """Warm-up, then `steps` steps between CUDA events on the compute stream with
+        every library launch bracketed by events; returns (ms, per-kind kernel times)."""
+        import torch
+        E = self.E
+        for _ in range(warmup):
+            self.step()
+        torch.cuda.synchronize()
+        E.sync_status()
+        for kk in E.KERNEL_KINDS:
+            E.profile_read(kk, reset=True)
+        E.profile_enable(True)
+        if barrier:
+            barrier()
+        torch.cuda.synchronize()
+        if clocks:
+            clocks.start()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(self.stream)
+        for _ in range(steps):
+            self.step()
+        e1.record(self.stream)
+        torch.cuda.synchronize()
+        if barrier:
+            barrier()
+        clk = clocks.stop() if clocks else None
+        E.profile_enable(False)
+        E.sync_status()
+        kern = {}
+        for kk, nm in E.KERNEL_KINDS.items():
+            n, kms = E.profile_read(kk, reset=True)
+            if n:
+                kern[nm] = {"launches": n, "ms": kms}
+        ktot = sum(v["ms"] for v in kern.values())
+        for v in kern.values():
+            v["share"] = v["ms"] / ktot if ktot else None
+        return e0.elapsed_time(e1), kern, clk
+
+    def rot_flops(self):
+        pl = self.per_layer
+        return sum(2.0 * self.B * self.w.T * (pl[k]["d_in"] * pl[k]["nC"] + pl[k]["d_out"] * pl[k]["nR"])
+                   for k in self.keys)
+
+    def in_bytes(self):
+        pl = self.per_layer
+        return sum(2.0 * self.B * self.w.T * (pl[k]["d_in"] + pl[k]["d_out"]) * (2 if self.w.dtype == "f32" else 1)
+                   for k in self.keys)
+
+    def summary(self, ms, steps, kern, peaks):
+        """examples/s, stack and rotation TFLOP/s, input GB/s and the rotation roofline."""
+        w, B = self.w, self.B
+        sec = ms / 1000.0
+        rot = kern.get("rotate", {"launches": 0, "ms": 0.0})
+        rf = self.rot_flops()
+        out = {"examples_per_s": B * steps / sec, "ms_per_step": ms / steps, "batch": B,
+               "modules": self.U, "T": w.T, "m": w.m, "k": w.k,
+               "stack_TFLOPs": rf * steps / sec / 1e12,
+               "input_GBps": self.in_bytes() * steps / sec / 1e9,
+               "alg_GFLOP_per_example": rf / B / 1e9,
+               "input_MB_per_example": self.in_bytes() / B / 1e6,
+               "kernels": kern}
+        hbm = peaks.get("hbm_gbs") or PEAKS_FALLBACK["hbm_gbs"]
+        out["input_frac_of_hbm"] = out["input_GBps"] / hbm
+        if rot["launches"]:
+            per_launch = rf * steps / rot["launches"]
+            avg_ms = rot["ms"] / rot["launches"]
+            ach = per_launch / (avg_ms / 1000.0) / 1e12
+            peak = peaks.get("bf16_tflops_sustained") or PEAKS_FALLBACK["bf16_tflops_sustained"]
+            tr = ROTATE_TRAFFIC.get(self.name)
+            out["roofline"] = {"bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+                               "frac": ach / peak,
+                               "traffic": tr[0] * B / tr[1] if tr and self.U == len(self.w.modules) else None,
+                               "kernel": "k_tc_rotate / k_tc_rotate2 (Kronecker rotations)",
+                               "flops_per_launch": per_launch}
+        if self.stream_bases:
+            out["eigenbases"] = "host-pinned, one layer ahead on a side stream"
+            out["h2d_bytes_per_step"] = self.layers * sum(2 * (L["VA"].numel() + L["VS"].numel())
+                                                          for L in self.per_layer.values())
+        if self.layers > 1:
+            out["inputs"] = f"one buffer per module type, shared by the {self.layers} layers"
+        return out
+
+    def release(self):
+        import torch
+        for k in list(vars(self)):
+            if k not in ("name", "B", "w", "U", "keys", "layers"):
+                setattr(self, k, None)
+        torch.cuda.empty_cache()
+
+
+def h2d_link_rate(dev, nbytes=1 << 30, reps=3):
+    """Plain host-to-device copy rate of one page-locked buffer (eogp_host_alloc) with
+    one cudaMemcpyAsync per repetition, GB/s."""
+    import torch
+    from paper_2609_37842_gb300 import eogp as E
+    h = E.host_empty((nbytes,), torch.uint8)
+    d = torch.empty((nbytes,), dtype=torch.uint8, device=dev)
+    d.copy_(h, non_blocking=True)
     torch.cuda.synchronize()
-    E.sync_status()
-    for kk in E.KERNEL_KINDS:
-        E.profile_read(kk, reset=True)
-    E.profile_enable(True)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(steps):
-        step()
-    e1.record(stream)
+    e0.record()
+    for _ in range(reps):
+        d.copy_(h, non_blocking=True)
+    e1.record()
     torch.cuda.synchronize()
-    E.profile_enable(False)
-    E.sync_status()
     ms = e0.elapsed_time(e1)
-    kern = {}
-    for kk, nm in E.KERNEL_KINDS.items():
-        n, kms = E.profile_read(kk, reset=True)
-        if n:
-            kern[nm] = {"launches": n, "ms": kms}
-    rms = kern.get("rotate", {}).get("ms", 0.0)
-    peaks, _ = load_peaks()
-    hbm_peak = peaks.get("hbm_gbs") or PEAKS_FALLBACK["hbm_gbs"]
-    rot_flops = sum(2.0 * B * w.T * (per_layer[k]["d_in"] * per_layer[k]["nC"] +
-                                     per_layer[k]["d_out"] * per_layer[k]["nR"]) for k in keys)
-    in_bytes = sum(2.0 * B * w.T * (per_layer[k]["d_in"] + per_layer[k]["d_out"]) for k in keys)
-    sec = ms / 1000.0
-    out = {"examples_per_s": B * steps / sec, "ms_per_step": ms / steps, "batch": B,
-           "modules": U, "T": w.T, "m": w.m, "k": w.k,
-           "rotate_TFLOPs": rot_flops * steps / (rms / 1000.0) / 1e12 if rms else None,
-           "stack_TFLOPs": rot_flops * steps / sec / 1e12,
-           "input_GBps": in_bytes * steps / sec / 1e9,
-           "alg_GFLOP_per_example": rot_flops / B / 1e9,
-           "input_MB_per_example": in_bytes / B / 1e6,
-           "input_frac_of_hbm": in_bytes * steps / sec / 1e9 / hbm_peak,
-           "kernels": kern}
-    if stream_bases:
-        out["eigenbases"] = "host-pinned, one layer ahead on a side stream"
-        out["h2d_bytes_per_step"] = layers * sum(2 * (L["VA"].numel() + L["VS"].numel())
-                                                 for L in per_layer.values())
-    if layers > 1:
-        out["inputs"] = f"one buffer per module type, shared by the {layers} layers"
-    del per_layer, descs, ws
+    del h, d
+    return nbytes * reps / (ms / 1000.0) / 1e9
+
+
+def e2e_run(st, Be, steps, chunk, dev, world, barrier):
+    """The step through the public host-input call (eogp_compress_layer_host): per
+    module, a and s in page-locked host memory (one buffer per module type) and,
+    for streamed-eigenbasis stacks, the retained eigenvector rows too (descriptor
+    bases_on_host); every call copies its inputs chunk by chunk into its workspace
+    while the previous chunk is compressed; the step ends with the device-to-host
+    read of the stack's codes and scales."""
+    import torch
+    E = st.E
+    w = st.w
+    hdt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    host = {}
+    hdesc = {}
+    bases_bytes = 0
+    for key, L in st.per_layer.items():
+        ha = E.host_empty((Be, w.T, L["d_in"]), hdt)
+        hs = E.host_empty((Be, w.T, L["d_out"]), hdt)
+        ha.copy_(L["a"][:Be])
+        hs.copy_(L["s"][:Be])
+        host[key] = (ha, hs)
+        if st.stream_bases:
+            hva, hvs = st.host_one[key]
+            hdesc[key] = E.layer_desc(L["plan"], w.T, w.k, hva, hvs, st.Pt)
+        else:
+            hdesc[key] = st.descs[key]
+    if st.stream_bases:
+        bases_bytes = sum(2 * (st.per_layer[k]["VA"].numel() + st.per_layer[k]["VS"].numel()) for k in st.keys)
+    hws = E.workspace(max(E.compress_host_workspace_size(d, Be, E.OUT_CODES, chunk) for d in hdesc.values()), dev)
+    wd = st.words
+    ecodes, escales = st.codes[:Be], st.scales[:Be]
+    hcodes = torch.empty(ecodes.shape, dtype=ecodes.dtype, pin_memory=True)
+    hscales = torch.empty(escales.shape, dtype=escales.dtype, pin_memory=True)
+    h2d = sum(host[k][0].numel() * host[k][0].element_size() + host[k][1].numel() * host[k][1].element_size()
+              for k in st.keys) + bases_bytes
+    d2h = hcodes.numel() * 4 + hscales.numel() * 4
+
+    def e2e_step():
+        for u, key in enumerate(st.keys):
+            ha, hs = host[key]
+            E.compress_layer_host(hdesc[key], ha, hs, E.OUT_CODES, dev, chunk=chunk,
+                                  codes=ecodes[:, u * wd:(u + 1) * wd], scales=escales[:, u], ws=hws,
+                                  stream=st.stream)
+        hcodes.copy_(ecodes, non_blocking=True)
+        hscales.copy_(escales, non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        e2e_step()
+    torch.cuda.synchronize()
+    ems = (time.perf_counter() - t0) * 1000.0
+    E.sync_status()
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([ems], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ems = float(tt.item())
+    link = h2d_link_rate(dev)
+    rate = h2d * steps / (ems / 1000.0) / 1e9
+    out = {"value": world * Be * steps / (ems / 1000.0), "unit": "examples/s", "batch": Be,
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
+           "h2d_GBps": rate, "link_GBps": link, "frac_of_link": rate / link if link else None,
+           "link": "one cudaMemcpyAsync of a 1 GiB page-locked buffer, same run",
+           "api": "eogp_compress_layer_host (host inputs, chunked copies inside the call)",
+           "chunk": chunk or "library default (about 64 MB of inputs)"}
+    if st.stream_bases:
+        out["eigenbases"] = "page-locked host memory, copied by each call (bases_on_host)"
+    del host, hdesc, hws
     torch.cuda.empty_cache()
     return out
 
@@ -510,13 +573,345 @@ def bench_fit(dev, n=10000, m=4096, k=1024):
     return {"n": n, "m": m, "k": k, "seconds": sec,
             "route": "covariance; tensor-core Gram, subspace iteration with Rayleigh-Ritz"}
 
+
+# ------------------------------------------------------------ CPU oracle
+def _shapes(w):
+    shapes = {}
+    for u, mod in enumerate(w.modules):
+        shapes.setdefault((mod.d_in, mod.d_out), []).append(u)
+    return shapes
+
+
+def _dense_orthogonal(d, rng):
+    """A dense orthogonal d x d matrix (I - 2 u u^T)(I - 2 v v^T) for random unit
+    u, v: cheap to form at d = 11008, where a Haar draw (QR of a Gaussian) takes
+    minutes on the host cores. The oracle's cost does not depend on the values
+    of the eigenbases, only on their (dense) shape."""
+    u = rng.standard_normal(d)
+    v = rng.standard_normal(d)
+    u /= np.linalg.norm(u)
+    v /= np.linalg.norm(v)
+    H = np.eye(d) - 2.0 * np.outer(u, u)
+    return H - 2.0 * np.outer(H @ v, v)
+
+
+class OracleSample:
+    """The oracle compressing one example through one module of each distinct shape
+    of a workload (inputs prepared once, not timed): dense orthogonal eigenbases
+    and P rounded to the workload dtype, the workload's spectra and inputs."""
+
+    def __init__(self, w, seed=1):
+        from paper_2609_37842_gb300 import synth
+        from oracle import eogp_oracle as O
+        self.O, self.w = O, w
+        rng = np.random.default_rng(seed)
+        qcache = {}
+
+        def q(d):
+            if d not in qcache:
+                qcache[d] = synth.round_to(_dense_orthogonal(d, rng), w.dtype)
+            return qcache[d]
+        self.P = synth.round_to(_dense_orthogonal(w.m, rng)[:, :w.k], w.dtype)
+        self.cases = []
+        for (d_in, d_out), us in _shapes(w).items():
+            u = us[0]
+            if w.spectrum == "channel":
+                sp = synth.layer_spec(w, u, 1, 1)
+                lamA, lamS = sp.lam_A, sp.lam_S
+            else:
+                lamA, lamS = synth.power_spectrum(d_in, w.alpha), synth.power_spectrum(d_out, w.alpha)
+            a, s = synth.layer_inputs(w, u, 1)
+            self.cases.append(dict(shape=f"{d_in}->{d_out}", count=len(us), QA=q(d_in), QS=q(d_out),
+                                   lamA=lamA, lamS=lamS, a=a, s=s, d_in=d_in, d_out=d_out))
+
+    def run(self, i):
+        """Seconds for the oracle on case i (one example, one module)."""
+        c, O, w = self.cases[i], self.O, self.w
+        t0 = time.perf_counter()
+        Lam = O.kfac_eigenvalues(c["lamS"], c["lamA"])
+        lam = O.damping(Lam, w.damping_rel)
+        O.compress_layer(c["a"], c["s"], c["QA"], c["QS"], Lam, lam, w.m, self.P)
+        return time.perf_counter() - t0
+
+    def flops(self, i):
+        # the oracle's dense work per example: G (2 T d_out d_in), Q_S^T G Q_A
+        # (2 d_out d_in (d_in + d_out)), P^T z (2 m k)
+        c, w = self.cases[i], self.w
+        return (2.0 * w.T * c["d_out"] * c["d_in"] + 2.0 * c["d_out"] * c["d_in"] * (c["d_in"] + c["d_out"]) +
+                2.0 * w.m * w.k)
+
+
+def _cores():
+    return len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+
+
+def cpu_baseline(w):
+    """Examples/s per stack of the oracle, from one example through one module of
+    each distinct shape, scaled by the shape counts (1 / sum_s count_s t_s)."""
+    smp = OracleSample(w)
+    total, per_shape, flops = 0.0, {}, 0.0
+    for i, c in enumerate(smp.cases):
+        t = smp.run(i)
+        total += c["count"] * t
+        per_shape[c["shape"]] = 1.0 / t
+        flops += c["count"] * smp.flops(i)
+    desc = (f"1 example x one module of each of the {len(smp.cases)} distinct shapes, "
+            f"scaled by the shape counts to the {len(w.modules)}-module stack")
+    return {"value": 1.0 / total, "unit": "examples/s", "cores": _cores(), "kind": "oracle",
+            "sample": desc, "examples_per_s_per_shape": per_shape,
+            "oracle_GFLOPs": flops / total / 1e9}
+
+
+def cpu_score_sample(ks, seconds=3.0):
+    """Oracle one-bit scores/s (float32 evaluation order) for stored codes of the
+    given modules: repeated batches of 16 stored rows x 4 queries for about
+    `seconds` of scoring (input generation not timed)."""
+    from oracle import eogp_oracle as O
+    rng = np.random.default_rng(3)
+    Q, n = 4, 16
+    qc = O.pack_concat([rng.integers(0, 2, (Q, k)).astype(bool) for k in ks])
+    qs = rng.lognormal(0, 0.5, (Q, len(ks))).astype(np.float32)
+    done, busy = 0, 0.0
+    while busy < seconds:
+        tc = O.pack_concat([rng.integers(0, 2, (n, k)).astype(bool) for k in ks])
+        ts = rng.lognormal(0, 0.5, (n, len(ks))).astype(np.float32)
+        t1 = time.perf_counter()
+        O.score_codes_f32(tc, ts, ks, qc, qs)
+        busy += time.perf_counter() - t1
+        done += n * Q
+    return done / busy
+
+
+def headline_config(w, B, world, name):
+    cfg = {"workload": name, "batch_per_gpu": B, "seq_len": w.T, "m": w.m, "k": w.k,
+           "modules": len(w.modules), "parallelism": f"replicas x{world}",
+           "l2": "inputs > L2 (each module's inputs exceed 129 MB every step)"}
+    if name == "olmo2_7b_bf16":
+        cfg["eigenbases"] = "page-locked host memory, streamed one layer ahead"
+    return cfg
+
+
+def run_reference(args):
+    """The reference arm: the oracle on the host cores, on the headline workload.
+    A step is the oracle compressing one example through one module, the
+    distinct module shapes taken in turn; the timed steps give each shape's mean
+    time t_s, and value = 1 / sum_s count_s t_s examples/s per stack."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    from paper_2609_37842_gb300 import synth
+    name = args.workload
+    w = synth.WORKLOADS[name]
+    B = args.batch or CONFIG_BATCH[name]
+    smp = OracleSample(w)
+    nc = len(smp.cases)
+    for i in range(args.warmup):
+        smp.run(i % nc)
+    times = [[] for _ in range(nc)]
+    wall0 = time.perf_counter()
+    for i in range(args.steps):
+        times[i % nc].append(smp.run(i % nc))
+    wall = time.perf_counter() - wall0
+    mean = [statistics.mean(t) if t else smp.run(i) for i, t in enumerate(times)]
+    value = 1.0 / sum(c["count"] * t for c, t in zip(smp.cases, mean))
+    world = int(os.environ.get("WORLD_SIZE", str(args.gpus)))
+    sample = (f"each step: 1 example through one module, the {nc} distinct module shapes in turn; value = 1 / "
+              f"sum over shapes of (modules of that shape x mean step time of that shape)")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "examples/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000.0 * wall / max(1, args.steps), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": headline_config(w, B, world, name),
+            "value_basis": "per-shape step times scaled to the stack (a step is one module, not one stack)",
+            "cpu_baseline": {"value": value, "unit": "examples/s", "cores": _cores(), "kind": "oracle",
+                             "sample": sample,
+                             "seconds_per_shape": {c["shape"]: t for c, t in zip(smp.cases, mean)}},
+            "e2e": {"value": value, "unit": "examples/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+# ------------------------------------------------------------- scoring
+def timed_call(fn, stream, reps=3):
+    import torch
+    from paper_2609_37842_gb300 import eogp as E
+    fn()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(reps):
+        fn()
+    b.record(stream)
+    torch.cuda.synchronize()
+    E.sync_status()
+    return a.elapsed_time(b) / reps
+
+
+def bench_query_scoring(w, N, Q, dev, stream, probes, bf16_burst, peaks_src, seed, paper=True):
+    """CODES scores (dense and with the top 20 fused) of Q one-bit queries against N
+    stored codes of the workload's modules; PAPER mode (unquantised queries) too."""
+    import torch
+    from paper_2609_37842_gb300 import eogp as E
+    U, words = len(w.modules), (w.k + 31) // 32
+    ks = [w.k] * U
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    tc = torch.randint(-2 ** 31, 2 ** 31 - 1, (N, U * words), generator=g, device=dev, dtype=torch.int32)
+    qc = torch.randint(-2 ** 31, 2 ** 31 - 1, (Q, U * words), generator=g, device=dev, dtype=torch.int32)
+    tsc = torch.exp(0.5 * torch.randn((N, U), generator=g, device=dev))
+    qsc = torch.exp(0.5 * torch.randn((Q, U), generator=g, device=dev))
+    out = torch.empty((Q, N), dtype=torch.float32, device=dev)
+    sms = timed_call(lambda: E.score(tc, tsc, ks, E.SCORE_CODES, qc, qsc, out=out), stream)
+    D = U * w.k
+    pk, pk_src, pk_mode = score_peak(ks, probes, bf16_burst, peaks_src)
+    alg = 2.0 * N * Q * D               # +-1 multiply-adds of the inner products
+    res = {"metric": "query x train scores/sec", "value": N * Q / (sms / 1000.0), "unit": "scores/s",
+           "ms_per_call": sms, "N": N, "Q": Q, "modules": U, "bits": D, "mode": f"CODES ({pk_mode})",
+           "tensor_TFLOPs": alg / (sms / 1000.0) / 1e12,
+           "tensor_frac": alg / (sms / 1000.0) / 1e12 / pk,
+           "tensor_peak": pk, "tensor_peak_source": pk_src}
+    del out
+    K = 20
+    wtc = E.workspace(E.score_topk_workspace_size(N, ks, E.SCORE_CODES, Q, K), dev)
+    cms = timed_call(lambda: E.score_topk(tc, tsc, ks, E.SCORE_CODES, qc, K, query_scales=qsc, ws=wtc), stream)
+    res["codes_top20"] = {"ms_per_call": cms, "scores_per_s": N * Q / (cms / 1000.0)}
+    del wtc
+    if paper:
+        y = torch.randn((Q, D), generator=g, device=dev)
+        out = torch.empty((Q, N), dtype=torch.float32, device=dev)
+        wsp = E.workspace(E.score_workspace_size(N, ks, E.SCORE_PAPER, Q), dev)
+        pms = timed_call(lambda: E.score(tc, tsc, ks, E.SCORE_PAPER, y, out=out, ws=wsp), stream)
+        res["paper_dense"] = {"ms_per_call": pms, "scores_per_s": N * Q / (pms / 1000.0),
+                              "tensor_TFLOPs_issued": 2 * alg / (pms / 1000.0) / 1e12,
+                              "tensor_frac_issued": 2 * alg / (pms / 1000.0) / 1e12 / bf16_burst,
+                              "note": "bf16 hi + lo query split: 2 MMAs per algorithmic one"}
+        del out, wsp
+        wtp = E.workspace(E.score_topk_workspace_size(N, ks, E.SCORE_PAPER, Q, K), dev)
+        tms = timed_call(lambda: E.score_topk(tc, tsc, ks, E.SCORE_PAPER, y, K, ws=wtp), stream)
+        res["paper_top20"] = {"ms_per_call": tms, "scores_per_s": N * Q / (tms / 1000.0)}
+        del y, wtp
+    del tc, qc, tsc, qsc
+    torch.cuda.empty_cache()
+    return res
+
+
+def bench_scan(dev, stream, probes, bf16_burst, peaks_src, hbm, rows=0, qs_arg=""):
+    """The scoring-bound sweep: 4,194,304 stored 16,384-bit codes, Q in {1, 64, 1024,
+    8192} (chunks of 1024 queries), top 20 fused for Q >= 1024."""
+    import torch
+    from paper_2609_37842_gb300 import eogp as E
+    from paper_2609_37842_gb300 import synth
+    g = torch.Generator(device=dev)
+    g.manual_seed(99)
+    sc = synth.SCAN
+    N, ksc = (rows or sc["N"]), sc["k"]
+    scan_qs = [int(q) for q in qs_arg.split(",")] if qs_arg else list(sc["Qs"])
+    Wsc = ksc // 32
+    tr = torch.randint(-2 ** 31, 2 ** 31 - 1, (N, Wsc), generator=g, device=dev, dtype=torch.int32)
+    tsc = torch.exp(sc["scale_sigma"] * torch.randn((N, 1), generator=g, device=dev))
+    qmax = 1024
+    out = torch.empty((qmax, N), dtype=torch.float32, device=dev)
+    scan = {"N": N, "bits": ksc, "mode": "CODES", "per_Q": {}}
+    for Q in scan_qs:
+        qc = torch.randint(-2 ** 31, 2 ** 31 - 1, (Q, Wsc), generator=g, device=dev, dtype=torch.int32)
+        qs = torch.exp(sc["scale_sigma"] * torch.randn((Q, 1), generator=g, device=dev))
+        chunks = [(q0, min(Q, q0 + qmax)) for q0 in range(0, Q, qmax)]
+
+        def run():
+            for q0, q1 in chunks:
+                E.score(tr, tsc, [ksc], E.SCORE_CODES, qc[q0:q1], qs[q0:q1], out=out[:q1 - q0])
+        qms = timed_call(run, stream, reps=1)
+        byts = len(chunks) * (N * Wsc * 4 + N * 4) + Q * N * 4
+        ent = {"ms": qms, "scores_per_s": N * Q / (qms / 1000.0), "GBps": byts / (qms / 1000.0) / 1e9,
+               "frac_of_hbm": byts / (qms / 1000.0) / 1e9 / hbm}
+        if Q >= 64:   # tensor-core kernel: +-1 multiply-adds against the rate of the MMA it issues
+            tfl = 2.0 * N * ksc * Q / (qms / 1000.0) / 1e12
+            pk, pk_src, pk_mode = score_peak([ksc], probes, bf16_burst, peaks_src)
+            ent.update({"kernel": f"k_score_tc ({pk_mode})", "tensor_TFLOPs": tfl,
+                        "tensor_frac": tfl / pk, "tensor_peak_source": pk_src})
+        else:
+            wops = N * Q * Wsc / (qms / 1000.0)
+            ent.update({"kernel": "k_score_codes_smallq (popcount)", "word_ops_per_s": wops})
+            if probes:
+                ent["popc_frac"] = wops / probes["popc_words_per_s"]
+        if Q >= 1024:  # per-query top 20 in the scoring epilogue: no Q x N output
+            K = 20
+            wt = E.workspace(E.score_topk_workspace_size(N, [ksc], E.SCORE_CODES, Q, K), dev)
+            kms = timed_call(lambda: E.score_topk(tr, tsc, [ksc], E.SCORE_CODES, qc, K, query_scales=qs, ws=wt),
+                             stream, reps=1)
+            ent["top20"] = {"ms": kms, "scores_per_s": N * Q / (kms / 1000.0), "output_bytes_avoided": Q * N * 4}
+            del wt
+        scan["per_Q"][str(Q)] = ent
+        del qc, qs
+    del tr, out
+    torch.cuda.empty_cache()
+    return scan
+
+
+def bench_pack(dev, stream, hbm):
+    import torch
+    from paper_2609_37842_gb300 import eogp as E
+    g = torch.Generator(device=dev)
+    g.manual_seed(98)
+    xs = torch.randn((262144, 1024), generator=g, device=dev)
+    pc = torch.empty((262144, 32), dtype=torch.int32, device=dev)
+    psc = torch.empty((262144,), dtype=torch.float32, device=dev)
+    pms = timed_call(lambda: E.pack_sign(xs, pc, psc), stream, reps=5)
+    pbytes = xs.numel() * 4 + pc.numel() * 4 + psc.numel() * 4
+    del xs, pc, psc
+    torch.cuda.empty_cache()
+    return {"rows": 262144, "k": 1024, "ms": pms, "GBps": pbytes / (pms / 1000.0) / 1e9,
+            "frac_of_hbm": pbytes / (pms / 1000.0) / 1e9 / hbm}
+
+
+def compact_rooflines(scoring, scan, pack, others, fit):
+    """Other kernels' roofline fractions and rates, for the record's `roofline`."""
+    r = {}
+    for nm, sc in (scoring or {}).items():
+        r[f"score_codes_{nm}"] = {"bound": "tensor (+-1 MMA)", "scores_per_s": sc["value"],
+                                  "achieved": sc["tensor_TFLOPs"], "peak": sc["tensor_peak"], "unit": "TFLOP/s",
+                                  "frac": sc["tensor_frac"], "peak_source": sc["tensor_peak_source"],
+                                  "ms": sc["ms_per_call"], "N": sc["N"], "Q": sc["Q"], "bits": sc["bits"]}
+        if "codes_top20" in sc:
+            r[f"score_codes_{nm}"]["top20_scores_per_s"] = sc["codes_top20"]["scores_per_s"]
+        if "paper_dense" in sc:
+            r[f"score_paper_{nm}"] = {"bound": "tensor (bf16, hi/lo issued)",
+                                      "scores_per_s": sc["paper_dense"]["scores_per_s"],
+                                      "frac": sc["paper_dense"]["tensor_frac_issued"]}
+    for q, ent in ((scan or {}).get("per_Q") or {}).items():
+        e = {"scores_per_s": ent["scores_per_s"], "ms": ent["ms"], "hbm_frac": ent["frac_of_hbm"]}
+        if "tensor_frac" in ent:
+            e.update({"bound": "tensor (+-1 MMA)" if int(q) >= 1024 else "hbm or tensor", "tensor_frac": ent["tensor_frac"]})
+        else:
+            e.update({"bound": "hbm", "popc_frac": ent.get("popc_frac")})
+        if "top20" in ent:
+            e["top20_scores_per_s"] = ent["top20"]["scores_per_s"]
+        r[f"scan_4M_q{q}"] = e
+    if pack:
+        r["pack_sign"] = {"bound": "hbm", "achieved": pack["GBps"], "unit": "GB/s", "frac": pack["frac_of_hbm"]}
+    for nm, o in (others or {}).items():
+        if isinstance(o, dict) and "roofline" in o:
+            rf = o["roofline"]
+            r[f"rotate_{nm}"] = {"bound": "tensor", "achieved": rf["achieved"], "peak": rf["peak"],
+                                 "unit": "TFLOP/s", "frac": rf["frac"], "traffic": rf["traffic"],
+                                 "examples_per_s": o["examples_per_s"]}
+        if isinstance(o, dict) and nm == "olmo2_1b_bf16":
+            r["olmo2_1b_input_hbm"] = {"bound": "hbm", "frac": o["input_frac_of_hbm"],
+                                      "achieved": o["input_GBps"], "unit": "GB/s"}
+    if fit:
+        r["fit_pca_seconds"] = {f"m{f['m']}_k{f['k']}": f["seconds"] for f in fit}
+    return r
+
+
 # ------------------------------------------------------------------ main
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--batch", type=int, default=512)
+    ap.add_argument("--workload", default=HEADLINE,
+                    help="headline stack (default: the OLMo-2-7B-shaped stack)")
+    ap.add_argument("--batch", type=int, default=0, help="examples per step (default: the workload's)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -524,8 +919,7 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--e2e-chunk", type=int, default=0,
                     help="examples per host-to-device chunk inside the call (0: about 64 MB)")
-    ap.add_argument("--e2e-batch", type=int, default=128,
-                    help="examples per e2e step (pinned host staging is sized by it)")
+    ap.add_argument("--e2e-batch", type=int, default=0, help="examples per e2e step (default: the workload's)")
     ap.add_argument("--no-scan", action="store_true")
     ap.add_argument("--scan-rows", type=int, default=0,
                     help="stored codes in the scan (default: the 4,194,304 of the scan workload)")
@@ -535,14 +929,13 @@ def main():
                     help="time only the EK-FAC correction (GPT-2 c_fc and OLMo-1B gate modules); "
                          "the case profiles/ captures for k_tc_ekfac")
     ap.add_argument("--no-configs", action="store_true",
-                    help="skip the OLMo / 32B / tiny-fp32 throughput and the PCA-fit timing")
+                    help="skip the other stacks and the PCA-fit timing")
     ap.add_argument("--modules", type=int, default=0,
-                    help="use only the first N modules of the stack (small profiling cases)")
+                    help="use only the first N modules of the headline stack (small profiling cases)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
 
-    import numpy as np
     import torch
     import torch.distributed as dist
 
@@ -564,65 +957,21 @@ def main():
         if rank == 0:
             print(json.dumps({"ekfac_correction": ek}))
         return
-    w = synth.WORKLOADS[WORKLOAD]
-    if args.modules:
-        import dataclasses
-        w = dataclasses.replace(w, modules=w.modules[:args.modules])
-    B, T, U = args.batch, w.T, len(w.modules)
-    words = (w.k + 31) // 32
+    name = args.workload
+    B = args.batch or CONFIG_BATCH[name]
     peaks, peaks_src = load_peaks()
     bf16_burst = peaks.get("bf16_tflops") or PEAKS_FALLBACK["bf16_tflops"]
-
-    # Page-locked, huge-page backed staging of the end-to-end inputs
-    # (eogp_host_alloc): cudaHostAlloc'd buffers fed host-to-device copies at
-    # anywhere from ~80 to ~210 GB/s between allocations on the GB300 machines
-    # measured, these at ~211 GB/s every time.
-    Be = min(B, args.e2e_batch)
-    host_in = None
-    if not args.no_e2e:
-        hdt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
-        host_in = [(E.host_empty((Be, T, mdl.d_in), hdt), E.host_empty((Be, T, mdl.d_out), hdt))
-                   for mdl in w.modules]
-
-    mods = build_stack(w, B, dev, seed=1000 + rank)
-    ws_bytes = max(E.compress_workspace_size(md["desc"], B, E.OUT_CODES) for md in mods)
-    ws = E.workspace(ws_bytes, dev)
-    codes = torch.empty((B, U * words), dtype=torch.int32, device=dev)
-    scales = torch.empty((B, U), dtype=torch.float32, device=dev)
-    stream = torch.cuda.current_stream()
+    hbm = peaks.get("hbm_gbs") or PEAKS_FALLBACK["hbm_gbs"]
 
     def barrier():
         if world > 1:
             dist.barrier()
 
-    for _ in range(args.warmup):
-        compress_step(mods, E, codes, scales, ws, words)
-    E.sync_status()
-
-    # ---- timed region: K compression steps, kernel events on ----
-    for kk in E.KERNEL_KINDS:
-        E.profile_read(kk, reset=True)
-    E.profile_enable(True)
+    # ---- headline: K compression steps of the stack, kernel events on ----
+    st = Stack(name, B, dev, stream_bases=(name == "olmo2_7b_bf16"), modules=args.modules)
+    w = st.w
     clocks = ClockSampler(local)
-    barrier()
-    torch.cuda.synchronize()
-    clocks.start()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    ev0.record(stream)
-    for _ in range(args.steps):
-        compress_step(mods, E, codes, scales, ws, words)
-    ev1.record(stream)
-    torch.cuda.synchronize()
-    barrier()
-    clk = clocks.stop()
-    E.profile_enable(False)
-    E.sync_status()
-    ms = ev0.elapsed_time(ev1)
-    kern = {}
-    for kk, name in E.KERNEL_KINDS.items():
-        n, t = E.profile_read(kk, reset=True)
-        if n:
-            kern[name] = {"launches": n, "ms": t}
+    ms, kern, clk = st.timed(args.steps, args.warmup, clocks=clocks, barrier=barrier)
     t_max = ms
     if world > 1:
         tt = torch.tensor([ms], device=dev)
@@ -630,24 +979,21 @@ def main():
         t_max = float(tt.item())
     value = world * B * args.steps / (t_max / 1000.0)
     launches = sum(v["launches"] for v in kern.values())
-    ktot = sum(v["ms"] for v in kern.values())
-    for v in kern.values():
-        v["share"] = v["ms"] / ktot if ktot else None
+    head = st.summary(ms, args.steps, kern, peaks)
+    roofline = dict(head.get("roofline") or {"bound": "tensor", "achieved": None, "peak": None,
+                                             "unit": "TFLOP/s", "frac": None, "traffic": None})
+    roofline["peak_source"] = f"{peaks_src} bf16_tflops_sustained"
 
-    rot = kern.get("rotate", {"launches": 0, "ms": 0.0})
-    flops_per_launch = rotate_flops(mods, B, T) / (2 * U)
-    avg_ms = rot["ms"] / max(1, rot["launches"])
-    achieved = flops_per_launch / (avg_ms / 1000.0) / 1e12 if avg_ms > 0 else None
-    peak = peaks.get("bf16_tflops_sustained") or PEAKS_FALLBACK["bf16_tflops_sustained"]
-    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": (achieved / peak) if achieved else None,
-                # captured on the full stack's block structure at the default batch only
-                "traffic": ROTATE_TRAFFIC_BYTES if (B == 512 and U % 4 == 0) else None,
-                "kernel": "k_tc_rotate / k_tc_rotate2 (Kronecker rotations)",
-                "peak_source": f"{peaks_src} bf16_tflops_sustained",
-                "flops_per_launch": flops_per_launch}
+    # ---- end to end through the public host-input call ----
+    e2e = None
+    if not args.no_e2e:
+        Be = min(B, args.e2e_batch or E2E_BATCH.get(name, B))
+        e2e = e2e_run(st, Be, args.e2e_steps, args.e2e_chunk, dev, world, barrier)
+    st.release()
+    del st
+    torch.cuda.empty_cache()
 
-    # ---- measured e4m3 tensor-core and popcount rates (scoring rooflines) ----
+    # ---- measured +-1 MMA and popcount rates (scoring rooflines) ----
     probes = None
     if rank == 0 and not args.no_score:
         f8, f4, pc = E.measure_peaks()
@@ -655,294 +1001,63 @@ def main():
                   "what": "eogp_measure_peaks: back-to-back kind::f8f6f4 (e4m3) and kind::mxf4 (e2m1, unit "
                           "scales) MMAs; XOR + popcount chains on every core"}
 
-    # ---- context: cuBLAS bf16 on the largest rotation shape (not on the path) ----
-    ref_gemm = None
-    if rank == 0 and not args.no_score:
-        kmax = max(md["d_in"] for md in mods)
-        A = torch.randn((B * T, kmax), device=dev, dtype=torch.bfloat16)
-        Wt = torch.randn((640, kmax), device=dev, dtype=torch.bfloat16)
-        A @ Wt.t()
-        torch.cuda.synchronize()
-        a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a_ev.record(stream)
-        for _ in range(3):
-            A @ Wt.t()
-        b_ev.record(stream)
-        torch.cuda.synchronize()
-        gms = a_ev.elapsed_time(b_ev) / 3
-        ref_gemm = {"what": f"cuBLAS bf16 [{B * T} x {kmax}] x [{kmax} x 640] -> bf16 (context only)",
-                    "ms": gms, "TFLOPs": 2.0 * B * T * kmax * 640 / (gms / 1000.0) / 1e12}
-        del A, Wt
-
-    # ---- scoring: Q = 1024 one-bit queries x N = 16384 stored codes ----
+    # ---- query x train scoring: the headline's query workload and GPT-2's ----
+    stream = torch.cuda.current_stream()
     scoring = None
-    if not args.no_score:
-        N, Q = w.N, w.Q
-        g = torch.Generator(device=dev)
-        g.manual_seed(77 + rank)
-        tc = torch.randint(-2 ** 31, 2 ** 31 - 1, (N, U * words), generator=g, device=dev,
-                           dtype=torch.int32)
-        qc = torch.randint(-2 ** 31, 2 ** 31 - 1, (Q, U * words), generator=g, device=dev,
-                           dtype=torch.int32)
-        tsc = torch.exp(0.5 * torch.randn((N, U), generator=g, device=dev))
-        qsc = torch.exp(0.5 * torch.randn((Q, U), generator=g, device=dev))
-        out = torch.empty((Q, N), dtype=torch.float32, device=dev)
-        ks = [w.k] * U
-        E.score(tc, tsc, ks, E.SCORE_CODES, qc, qsc, out=out)
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        reps = 3
-        e0.record(stream)
-        for _ in range(reps):
-            E.score(tc, tsc, ks, E.SCORE_CODES, qc, qsc, out=out)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        E.sync_status()
-        sms = e0.elapsed_time(e1) / reps
-        D = U * w.k
-        pk, pk_src, pk_mode = score_peak(ks, probes, bf16_burst, peaks_src)
-        alg = 2.0 * N * Q * D               # +-1 multiply-adds of the inner products
-        scoring = {"metric": "query x train scores/sec", "value": N * Q / (sms / 1000.0),
-                   "unit": "scores/s", "ms_per_call": sms, "N": N, "Q": Q, "bits": D,
-                   "mode": f"CODES ({pk_mode})",
-                   "tensor_TFLOPs": alg / (sms / 1000.0) / 1e12,
-                   "tensor_frac": alg / (sms / 1000.0) / 1e12 / pk,
-                   "tensor_peak": pk,
-                   "tensor_peak_source": pk_src}
-        # paper mode (unquantised queries), dense and with the ranking fused (K = 20)
-        y = torch.randn((Q, D), generator=g, device=dev)
-        wsp = E.workspace(E.score_workspace_size(N, ks, E.SCORE_PAPER, Q), dev)
+    if rank == 0 and not args.no_score:
+        scoring = {}
+        if w.Q and len(w.modules) > 1:
+            scoring[name] = bench_query_scoring(w, w.N, w.Q, dev, stream, probes, bf16_burst, peaks_src, 77,
+                                                paper=False)
+        g2 = synth.WORKLOADS["gpt2_small_bf16"]
+        if name != "gpt2_small_bf16" or not scoring:
+            scoring["gpt2_small_bf16"] = bench_query_scoring(g2, g2.N, g2.Q, dev, stream, probes, bf16_burst,
+                                                             peaks_src, 78)
 
-        def timed(fn, reps=3):
-            fn()
-            torch.cuda.synchronize()
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a.record(stream)
-            for _ in range(reps):
-                fn()
-            b.record(stream)
-            torch.cuda.synchronize()
-            E.sync_status()
-            return a.elapsed_time(b) / reps
-
-        pms = timed(lambda: E.score(tc, tsc, ks, E.SCORE_PAPER, y, out=out, ws=wsp))
-        scoring["paper_dense"] = {"ms_per_call": pms, "scores_per_s": N * Q / (pms / 1000.0),
-                                  "tensor_TFLOPs_issued": 2 * alg / (pms / 1000.0) / 1e12,
-                                  "tensor_frac_issued": 2 * alg / (pms / 1000.0) / 1e12 / bf16_burst,
-                                  "note": "bf16 hi + lo query split: 2 MMAs per algorithmic one"}
-        del out
-        K = 20
-        wtc = E.workspace(E.score_topk_workspace_size(N, ks, E.SCORE_CODES, Q, K), dev)
-        wtp = E.workspace(E.score_topk_workspace_size(N, ks, E.SCORE_PAPER, Q, K), dev)
-        cms = timed(lambda: E.score_topk(tc, tsc, ks, E.SCORE_CODES, qc, K, query_scales=qsc, ws=wtc))
-        tms = timed(lambda: E.score_topk(tc, tsc, ks, E.SCORE_PAPER, y, K, ws=wtp))
-        scoring["codes_top20"] = {"ms_per_call": cms, "scores_per_s": N * Q / (cms / 1000.0)}
-        scoring["paper_top20"] = {"ms_per_call": tms, "scores_per_s": N * Q / (tms / 1000.0)}
-        del y, wsp, wtc, wtp
-
-    # ---- EOGP-R: the SRHT second stage in place of P (App. B.2), same stack ----
-    eogp_r = None
-    if not args.no_score:
-        eogp_r = {}
-        for kr in (w.k, 4 * w.k):
-            rdesc = []
-            for u, md in enumerate(mods):
-                plan, VA, VS, _ = md["desc"]._refs[:4]
-                sg, rw = synth.srht_draw(w.m, kr, seed=w.seed, module_index=u)
-                rdesc.append(E.layer_desc(plan, T, kr, VA, VS, None,
-                                          srht_signs=torch.from_numpy(sg).to(dev),
-                                          srht_rows=torch.from_numpy(rw).to(dev)))
-            rwords = (kr + 31) // 32
-            rcodes = torch.empty((B, U * rwords), dtype=torch.int32, device=dev)
-            rws = E.workspace(max(E.compress_workspace_size(d, B, E.OUT_CODES) for d in rdesc), dev)
-
-            def rstep():
-                for u, md in enumerate(mods):
-                    E.compress_layer(rdesc[u], md["a"], md["s"], E.OUT_CODES,
-                                     codes=rcodes[:, u * rwords:(u + 1) * rwords],
-                                     scales=scales[:, u], ws=rws)
-            rstep()
-            torch.cuda.synchronize()
-            a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a_ev.record(stream)
-            for _ in range(3):
-                rstep()
-            b_ev.record(stream)
-            torch.cuda.synchronize()
-            E.sync_status()
-            rms = a_ev.elapsed_time(b_ev) / 3
-            eogp_r[f"k{kr}"] = {"examples_per_s": B / (rms / 1000.0), "ms_per_step": rms,
-                                "bits_per_module": kr}
-            del rdesc, rcodes, rws
-
-    # ---- end to end through the public API with host buffers ----
-    # Per module, eogp_compress_layer_host on a and s in page-locked host memory:
-    # the call copies the batch into its workspace chunk by chunk (about 64 MB per
-    # chunk, double-buffered on a copy stream of its own) while the previous chunk
-    # is compressed; then the step's codes and scales are read back to the host.
-    e2e = None
-    if not args.no_e2e:
-        for md, (ha, hs) in zip(mods, host_in):
-            ha.copy_(md["a"][:Be])
-            hs.copy_(md["s"][:Be])
-        hws = E.workspace(max(E.compress_host_workspace_size(md["desc"], Be, E.OUT_CODES, args.e2e_chunk)
-                              for md in mods), dev)
-        ecodes, escales = codes[:Be], scales[:Be]
-        hcodes = torch.empty(ecodes.shape, dtype=codes.dtype, pin_memory=True)
-        hscales = torch.empty(escales.shape, dtype=scales.dtype, pin_memory=True)
-        h2d = sum(ha.numel() * ha.element_size() + hs.numel() * hs.element_size() for ha, hs in host_in)
-        d2h = hcodes.numel() * 4 + hscales.numel() * 4
-
-        def e2e_step():
-            for u, (md, (ha, hs)) in enumerate(zip(mods, host_in)):
-                E.compress_layer_host(md["desc"], ha, hs, E.OUT_CODES, dev, chunk=args.e2e_chunk,
-                                      codes=ecodes[:, u * words:(u + 1) * words], scales=escales[:, u],
-                                      ws=hws, stream=stream)
-            hcodes.copy_(ecodes, non_blocking=True)
-            hscales.copy_(escales, non_blocking=True)
-
-        e2e_step()
-        torch.cuda.synchronize()
-        barrier()
-        t0 = time.perf_counter()
-        for _ in range(args.e2e_steps):
-            e2e_step()
-        torch.cuda.synchronize()
-        ems = (time.perf_counter() - t0) * 1000.0
-        E.sync_status()
-        if world > 1:
-            tt = torch.tensor([ems], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            ems = float(tt.item())
-        e2e = {"value": world * Be * args.e2e_steps / (ems / 1000.0), "unit": "examples/s",
-               "batch": Be,
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
-               "h2d_GBps": h2d * args.e2e_steps / (ems / 1000.0) / 1e9,
-               "api": "eogp_compress_layer_host (host inputs, chunked copies inside the call)",
-               "chunk": args.e2e_chunk or "library default (about 64 MB of inputs)"}
-        del hws
-    host_in = None
-
-    # ---- standalone sign-pack and the scoring sweep (HBM-bound kernels) ----
-    hbm = peaks.get("hbm_gbs") or PEAKS_FALLBACK["hbm_gbs"]
-    pack = None
-    scan = None
+    # ---- standalone sign-pack and the scoring sweep ----
+    pack = scan = None
     if rank == 0 and not args.no_scan:
-        del mods
-        torch.cuda.empty_cache()
-        g = torch.Generator(device=dev)
-        g.manual_seed(99)
-        xs = torch.randn((262144, 1024), generator=g, device=dev)
-        pc = torch.empty((262144, 32), dtype=torch.int32, device=dev)
-        psc = torch.empty((262144,), dtype=torch.float32, device=dev)
-        E.pack_sign(xs, pc, psc)
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(5):
-            E.pack_sign(xs, pc, psc)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        E.sync_status()
-        pms = e0.elapsed_time(e1) / 5
-        pbytes = xs.numel() * 4 + pc.numel() * 4 + psc.numel() * 4
-        pack = {"rows": 262144, "k": 1024, "ms": pms, "GBps": pbytes / (pms / 1000.0) / 1e9,
-                "frac_of_hbm": pbytes / (pms / 1000.0) / 1e9 / hbm}
-        del xs, pc, psc
-        sc = synth.SCAN
-        N, ksc = (args.scan_rows or sc["N"]), sc["k"]
-        scan_qs = [int(q) for q in args.scan_qs.split(",")] if args.scan_qs else list(sc["Qs"])
-        Wsc = ksc // 32
-        tr = torch.randint(-2 ** 31, 2 ** 31 - 1, (N, Wsc), generator=g, device=dev, dtype=torch.int32)
-        tsc = torch.exp(sc["scale_sigma"] * torch.randn((N, 1), generator=g, device=dev))
-        qmax = 1024
-        out = torch.empty((qmax, N), dtype=torch.float32, device=dev)
-        scan = {"N": N, "bits": ksc, "mode": "CODES", "per_Q": {}}
-        for Q in scan_qs:
-            qc = torch.randint(-2 ** 31, 2 ** 31 - 1, (Q, Wsc), generator=g, device=dev,
-                               dtype=torch.int32)
-            qs = torch.exp(sc["scale_sigma"] * torch.randn((Q, 1), generator=g, device=dev))
-            chunks = [(q0, min(Q, q0 + qmax)) for q0 in range(0, Q, qmax)]
-            for q0, q1 in chunks[:1]:
-                E.score(tr, tsc, [ksc], E.SCORE_CODES, qc[q0:q1], qs[q0:q1], out=out[:q1 - q0])
-            torch.cuda.synchronize()
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            for q0, q1 in chunks:
-                E.score(tr, tsc, [ksc], E.SCORE_CODES, qc[q0:q1], qs[q0:q1], out=out[:q1 - q0])
-            e1.record(stream)
-            torch.cuda.synchronize()
-            E.sync_status()
-            qms = e0.elapsed_time(e1)
-            byts = len(chunks) * (N * Wsc * 4 + N * 4) + Q * N * 4
-            ent = {"ms": qms, "scores_per_s": N * Q / (qms / 1000.0),
-                   "GBps": byts / (qms / 1000.0) / 1e9,
-                   "frac_of_hbm": byts / (qms / 1000.0) / 1e9 / hbm}
-            if Q >= 64:   # tensor-core kernel: +-1 multiply-adds against the rate of the MMA it issues
-                tfl = 2.0 * N * ksc * Q / (qms / 1000.0) / 1e12
-                pk, pk_src, pk_mode = score_peak([ksc], probes, bf16_burst, peaks_src)
-                ent.update({"kernel": f"k_score_tc ({pk_mode})", "tensor_TFLOPs": tfl,
-                            "tensor_frac": tfl / pk, "tensor_peak_source": pk_src})
-            else:
-                wops = N * Q * Wsc / (qms / 1000.0)
-                ent.update({"kernel": "k_score_codes_smallq (popcount)", "word_ops_per_s": wops})
-                if probes:
-                    ent["popc_frac"] = wops / probes["popc_words_per_s"]
-            if Q >= 1024:  # per-query top 20 in the scoring epilogue: no Q x N output
-                K = 20
-                wt = E.workspace(E.score_topk_workspace_size(N, [ksc], E.SCORE_CODES, Q, K), dev)
-                E.score_topk(tr, tsc, [ksc], E.SCORE_CODES, qc, K, query_scales=qs, ws=wt)
-                torch.cuda.synchronize()
-                e0.record(stream)
-                E.score_topk(tr, tsc, [ksc], E.SCORE_CODES, qc, K, query_scales=qs, ws=wt)
-                e1.record(stream)
-                torch.cuda.synchronize()
-                E.sync_status()
-                kms = e0.elapsed_time(e1)
-                ent["top20"] = {"ms": kms, "scores_per_s": N * Q / (kms / 1000.0),
-                                "output_bytes_avoided": Q * N * 4}
-                del wt
-            scan["per_Q"][str(Q)] = ent
-        del tr, out
+        pack = bench_pack(dev, stream, hbm)
+        scan = bench_scan(dev, stream, probes, bf16_burst, peaks_src, hbm, args.scan_rows, args.scan_qs)
 
-    configs = None
-    fit = None
+    # ---- the other stacks, the EK-FAC correction and the PCA fit ----
+    configs = fit = None
     if rank == 0 and not args.no_configs:
-        torch.cuda.empty_cache()
-        configs = {
-            "tiny_f32": bench_config("tiny_f32", CONFIG_BATCH["tiny_f32"], 5, 3, dev),
-            "olmo2_1b_bf16": bench_config("olmo2_1b_bf16", CONFIG_BATCH["olmo2_1b_bf16"], 3, 3, dev),
-            "olmo2_7b_bf16": bench_config("olmo2_7b_bf16", CONFIG_BATCH["olmo2_7b_bf16"], 3, 3, dev,
-                                          stream_bases=True),
-            "olmo2_32b_gate_bf16": bench_config("olmo2_32b_gate_bf16", CONFIG_BATCH["olmo2_32b_gate_bf16"],
-                                                5, 3, dev),
-        }
-        fit = [bench_fit(dev, 10000, 4096, 1024), bench_fit(dev, 10000, 8192, 2048)]
+        configs = {}
+        for nm in ("gpt2_small_bf16", "olmo2_1b_bf16", "olmo2_7b_bf16", "olmo2_32b_gate_bf16", "tiny_f32"):
+            if nm == name:
+                continue
+            o = Stack(nm, CONFIG_BATCH[nm], dev, stream_bases=(nm == "olmo2_7b_bf16"))
+            steps = 3 if nm.startswith("olmo2_") and nm != "olmo2_32b_gate_bf16" else 5
+            oms, okern, _ = o.timed(steps, 3)
+            configs[nm] = o.summary(oms, steps, okern, peaks)
+            o.release()
+            del o
+            torch.cuda.empty_cache()
         configs["ekfac_correction"] = [bench_ekfac(dev, 768, 3072, 512, 32),
                                        bench_ekfac(dev, 2048, 8192, 2048, 4)]
+        fit = [bench_fit(dev, 10000, 4096, 1024), bench_fit(dev, 10000, 8192, 2048)]
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        sec, cores, desc = cpu_sample(w, 1)
-        cpu = {"value": 1.0 / sec, "unit": "examples/s", "cores": cores, "kind": "oracle",
-               "sample": desc, **cpu_sample.details,
-               "oracle_scores_per_s": cpu_score_sample(),
-               "scores_sample": "64 stored rows x 4 one-bit queries of 48 x 1024 bits, repeated for ~3 s"}
+        cpu = cpu_baseline(w)
+        ks = [w.k] * len(w.modules)
+        cpu["oracle_scores_per_s"] = cpu_score_sample(ks)
+        cpu["scores_sample"] = (f"16 stored rows x 4 one-bit queries of {len(ks)} x {w.k} bits, "
+                                f"repeated for ~3 s")
 
     if rank == 0:
+        roofline["others"] = compact_rooflines(scoring, scan, pack, configs, fit)
         line = {"metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": world,
                 "steps": args.steps, "warmup": args.warmup,
                 "ms_per_step": t_max / args.steps, "higher_is_better": True, "scaling": "weak",
-                "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-                "config": {"workload": WORKLOAD if not args.modules else
-                           f"{WORKLOAD} (first {U} modules)", "batch_per_gpu": B, "seq_len": T, "m": w.m,
-                           "k": w.k, "modules": U, "parallelism": f"replicas x{world}",
-                           "l2": "inputs > L2 (B x 151 MB per step)"},
-                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "scoring": scoring,
-                "pack_sign": pack, "scan": scan, "eogp_r_srht": eogp_r, "reference_gemm": ref_gemm,
-                "measured_rates": probes,
-                "other_workloads": configs,
-                "fit_pca": fit,
+                "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
+                "config": headline_config(w, B, world, name if not args.modules else
+                                          f"{name} (first {len(w.modules)} modules)"),
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+                "headline": {k: v for k, v in head.items() if k != "roofline"},
+                "scoring": scoring, "pack_sign": pack, "scan": scan,
+                "measured_rates": probes, "other_workloads": configs, "fit_pca": fit,
                 "gpu_launches": launches, "kernels": kern, "clocks": clk}
         print(json.dumps(line))
     if world > 1:
