@@ -250,14 +250,21 @@ int eogp_compress_layer(const eogp_layer_desc* L, const void* a, const void* s, 
                         eogp_stream_t stream);
 
 /* Page-locked host memory for inputs that eogp_compress_layer_host (or the
- * caller) copies to the device: an anonymous mapping aligned to and advised for
- * transparent huge pages, registered with cudaHostRegister. Measured on GB300
- * systems, host-to-device copies from it ran at the link rate (~211 GB/s) in
- * every trial, where cudaHostAlloc'd buffers varied from ~80 to ~210 GB/s
- * between allocations. Requests of at least one huge page are rounded up to
- * whole huge pages, smaller ones to whole base pages (no huge-page advice); the memory
- * is zero-filled. eogp_host_free takes only the pointer (NULL is a no-op).
- * A library convenience with no counterpart in the paper.
+ * caller) copies to the device, registered with cudaHostRegister and backed by
+ * transparent huge pages where that matters. Measured on GB300 systems,
+ * host-to-device copies from anonymous memory advised for huge pages ran at the
+ * link rate (~211 GB/s) in every trial; cudaHostAlloc'd buffers varied from ~80
+ * to ~210 GB/s between allocations, and the same memory on 64 KB base pages
+ * ran at ~51 GB/s. Size classes (H = the kernel's huge-page size, 2 MB on
+ * 4 KB-page hosts, 512 MB on 64 KB-page arm64 hosts):
+ *   bytes >= H/2           a region of its own, whole huge pages;
+ *   1 MB <= bytes < H/2    a 4 KB-aligned block of a shared arena of one huge
+ *                          page (first fit; the arena is released with its last
+ *                          block), so such buffers get huge pages without each
+ *                          pinning a whole one;
+ *   bytes < 1 MB           whole base pages, no huge-page advice.
+ * The memory is zero-filled. eogp_host_free takes only the pointer (NULL is a
+ * no-op). Thread-safe. A library convenience with no counterpart in the paper.
  * Errors: EOGP_EINVAL (bytes == 0, ptr NULL, mapping failed, pointer not from
  * eogp_host_alloc), EOGP_ECUDA (registration failed, e.g. no device). */
 int eogp_host_alloc(size_t bytes, void** ptr);

@@ -216,6 +216,48 @@ def test_host_empty_memory_round_trip():
     gc.collect()
 
 
+def test_host_alloc_size_classes():
+    """eogp_host_alloc in each size class (base pages below 1 MB, blocks of a
+    shared huge-page arena up to half a huge page, whole huge pages above):
+    blocks are 4 KB aligned, never overlap while live, come back zero-filled
+    after a freed block is reused, and copy to the device and back."""
+    import ctypes
+    L = E.lib()
+    sizes = [64 << 10, 1 << 20, (3 << 20) + 123, 5 << 20, 17 << 20]
+    ptrs = []
+    for n in sizes:
+        p = ctypes.c_void_p()
+        assert L.eogp_host_alloc(n, ctypes.byref(p)) == E.OK
+        assert p.value % 4096 == 0
+        ctypes.memset(p.value, 0x5A, n)
+        ptrs.append((p.value, n))
+    spans = sorted(ptrs)
+    for (a, na), (b, _) in zip(spans, spans[1:]):
+        assert a + na <= b, "live blocks overlap"
+    # free the middle blocks and take them again: the new blocks are zero-filled
+    for p, n in ptrs[1:3]:
+        assert L.eogp_host_free(ctypes.c_void_p(p)) == E.OK
+    again = []
+    for n in sizes[1:3]:
+        p = ctypes.c_void_p()
+        assert L.eogp_host_alloc(n, ctypes.byref(p)) == E.OK
+        buf = (ctypes.c_uint8 * n).from_address(p.value)
+        assert not any(bytes(buf)), "reused block not zero-filled"
+        again.append((p.value, n))
+    # device round trip through the largest arena-class block
+    p, n = again[1]
+    host = torch.frombuffer((ctypes.c_uint8 * n).from_address(p), dtype=torch.uint8)
+    host.copy_(torch.randint(0, 256, (n,), dtype=torch.uint8))
+    d = host.to(DEV, non_blocking=True)
+    back = torch.empty_like(host).pin_memory()
+    back.copy_(d, non_blocking=True)
+    torch.cuda.synchronize()
+    assert torch.equal(back, host)
+    del host
+    for p, _ in [ptrs[0], ptrs[3], ptrs[4]] + again:
+        assert L.eogp_host_free(ctypes.c_void_p(p)) == E.OK
+
+
 def test_measure_peaks_rates():
     """eogp_measure_peaks: the e4m3 and e2m1 one-bit MMA rates and the popcount
     rate are finite and positive, the e2m1 MMA (K = 64 per instruction) outruns
