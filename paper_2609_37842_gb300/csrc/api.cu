@@ -1270,20 +1270,20 @@ static TopkPlan topk_plan(int N, const int* ks, int U, int mode, int Q, int K) {
   const bool tc_ok = (mode == EOGP_SCORE_CODES || mode == EOGP_SCORE_PAPER) &&
                      score_tc_supported(mode, ks, U, Q);
   const int force = topk_fused_override();
-  p.fused = tc_ok && score_tc_topk_fits(mode, U, Q, K) && force != 0 &&
+  p.fused = tc_ok && score_tc_topk_fits(mode, ks, U, Q, K) && force != 0 &&
             (force == 1 || N > topk_select_max_n());
   p.select = !p.fused && N <= topk_select_max_n();
   p.q_bytes = tc_ok ? score_tc_ws_bytes(mode, ks, U, Q) : 0;
   if (p.fused) {
-    p.slots = score_tc_grid(mode, U, N, Q, K, sm_count());
+    p.slots = score_tc_grid(mode, ks, U, N, Q, K, sm_count());
     p.dense_bytes = 0;
   } else {
     p.slots = p.select ? 0 : topk_dense_slots(N);
     p.dense_bytes = al256(static_cast<size_t>(Q) * ((static_cast<size_t>(N) + 3) & ~size_t(3)) * 4);
   }
   p.list_bytes = al256(static_cast<size_t>(p.slots) * Q * K * 4);
-  p.buf_bytes = p.fused ? al256(score_tc_list_buf_bytes(mode, U, Q, K, p.slots)) : 0;
-  p.scr_bytes = p.fused ? al256(score_tc_scratch_bytes(mode, U, Q, K, p.slots)) : 0;
+  p.buf_bytes = p.fused ? al256(score_tc_list_buf_bytes(mode, ks, U, Q, K, p.slots)) : 0;
+  p.scr_bytes = p.fused ? al256(score_tc_scratch_bytes(mode, ks, U, Q, K, p.slots)) : 0;
   p.total = al256(p.q_bytes) + p.dense_bytes + 2 * p.list_bytes + 2 * p.buf_bytes +
             (p.fused ? al256(static_cast<size_t>(Q) * 4) : 0) + p.scr_bytes;
   return p;

@@ -264,6 +264,21 @@ __device__ __forceinline__ void tc_mma_f4_ta(uint32_t d_tmem, uint32_t a_tmem, u
       : "memory");
 }
 
+// The same block-scaled e2m1 MMA over a CTA pair (M = 256, issued by the
+// leader CTA): each CTA's TMEM holds its 128 rows of A at a_tmem and of D at
+// d_tmem, each CTA's shared memory its N / 2 rows of B at the descriptor's
+// address; the scale factors are read from each CTA's TMEM.
+__device__ __forceinline__ void tc_mma_f4_ta_pair(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                                  uint32_t sfa, uint32_t sfb, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %6, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::mxf4.block_scale.scale_vec::2X [%0], [%1], %2, %3, [%4], [%5], p;\n\t}\n" ::"r"(
+          d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
+      : "memory");
+}
+
 // Same MMA with operand A in tensor memory: a_tmem addresses the first of the
 // K / 4 32-bit columns holding A (TMEM lane = row of A, four e4m3 elements per
 // column, element 4c + e in byte e of column c).

@@ -103,10 +103,10 @@ struct TcTopK {
 };
 bool score_tc_supported(int mode, const int* ks, int U, int Q);
 size_t score_tc_ws_bytes(int mode, const int* ks, int U, int Q);
-int score_tc_grid(int mode, int U, int N, int Q, int K, int num_sms);
-bool score_tc_topk_fits(int mode, int U, int Q, int K);
-size_t score_tc_list_buf_bytes(int mode, int U, int Q, int K, int grid);  // each of bufs, bufi
-size_t score_tc_scratch_bytes(int mode, int U, int Q, int K, int grid);
+int score_tc_grid(int mode, const int* ks, int U, int N, int Q, int K, int num_sms);
+bool score_tc_topk_fits(int mode, const int* ks, int U, int Q, int K);
+size_t score_tc_list_buf_bytes(int mode, const int* ks, int U, int Q, int K, int grid);  // each of bufs, bufi
+size_t score_tc_scratch_bytes(int mode, const int* ks, int U, int Q, int K, int grid);
 cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const float* ts, int ldts, int N,
                             const int* ks, int U, const void* query, int ldq, const float* qs,
                             int ldqs, int Q, float* out, int ldo, const TcTopK* topk, void* ws,

@@ -107,7 +107,9 @@ def rand_store(rng, n, ks):
                                     (513, 70, [40, 1024, 7, 33]), (64, 64, [16384]),
                                     (1000, 64, [128, 1024]), (300, 100, [256]),
                                     (129, 200, [1024, 128, 2048]), (777, 257, [512] * 5),
-                                    (1000, 300, [256, 768, 1024]), (500, 300, [2048])])
+                                    (1000, 300, [256, 768, 1024]), (500, 300, [2048]),
+                                    (2000, 64, [256, 1280]), (5000, 200, [768]), (40000, 64, [1024]),
+                                    (3000, 1000, [256, 256, 512])])
 @pytest.mark.parametrize("f4", ["1", "0"])
 def test_score_codes_bit_exact(N, Q, ks, f4, eogp_options):
     """CODES scores equal the oracle's float32 evaluation bit for bit. Where every
