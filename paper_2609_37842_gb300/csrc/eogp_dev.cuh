@@ -504,6 +504,20 @@ __device__ __forceinline__ uint32_t __syncthreads_and_named(uint32_t pred) {
   return out;
 }
 
+// AND of `pred` over the `nthreads` threads of named barrier `id` (all of them wait).
+__device__ __forceinline__ uint32_t named_bar_and(int id, int nthreads, uint32_t pred) {
+  uint32_t out;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}\n"
+      : "=r"(out)
+      : "r"(pred), "r"(id), "r"(nthreads)
+      : "memory");
+  return out;
+}
+
 // OR of `pred` over the `nthreads` threads of named barrier `id` (all of them wait).
 __device__ __forceinline__ uint32_t named_bar_or(int id, int nthreads, uint32_t pred) {
   uint32_t out;

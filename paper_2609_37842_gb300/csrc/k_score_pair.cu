@@ -27,10 +27,9 @@
 //    round: at 256 bits per round the rounds, not the tensor pipe, set the pace
 //    (measured: 589 cycles per four N = 256 MMAs, 8.4 of 9.7 PFLOP/s), at
 //    512 bits the tensor pipe does (1024 cycles per eight, 9.7 PFLOP/s).
-// Each expander warp takes whole stages of its 32 rows (warps 0-3 the even
-// stages of a tile, 4-7 the odd ones): two 16-byte shared-memory loads, the
-// e2m1 expansion, the TMEM stores, and one relaxed arrive on the leader's
-// barrier of the group. That arrive orders enough: it is issued after
+// Each expander warp takes the 32 rows of one TMEM lane quarter, a whole group
+// per round: two 16-byte shared-memory loads and the e2m1 expansion per stage,
+// the TMEM stores, and one relaxed arrive on the leader's barrier of the group. That arrive orders enough: it is issued after
 // tcgen05.wait::st, which returns only once the thread's TMEM stores have
 // completed, and after the tcgen05 fence; the leader issues the MMAs only after
 // observing it; and in the pair MMA each SM's tensor core reads operand A from
@@ -40,8 +39,11 @@
 // 30.9 ms with cluster-scope release, 44.8 ms with one thread of the peer
 // forwarding every stage with one cluster-scope release.
 //
-// Warps: 0-7 expand, 8-11 dequantise, 12 owns TMEM and, in the leader, issues
-// the MMAs, 13 loads the code boxes, 14 the query tiles.
+// Warps: 0-3 expand, 4-11 dequantise (two per TMEM lane quarter, half of the
+// query columns each, which halves the drain of the accumulator the MMAs of a
+// 256-query tile wait for), 12 owns TMEM and, in the leader, issues the MMAs,
+// 13 loads the code boxes, 14 the query tiles. Fifteen warps leave 128
+// registers a thread (an SM sub-partition holds at most four of them).
 #include <algorithm>
 #include <atomic>
 
@@ -51,9 +53,13 @@ namespace eogp {
 namespace sc {
 namespace {
 
-constexpr int kPairThreads = (kExpWarps + 4 + 1 + 2) * 32;
-constexpr int kCodeWarp = kMmaWarp + 1;
-constexpr int kQueryWarp = kMmaWarp + 2;
+constexpr int kPrExpWarps = 4;                   // expander warps: one per TMEM lane quarter
+constexpr int kPrDq0 = kPrExpWarps;              // first dequantise warp
+constexpr int kPrDqWarps = 8;                    // dequantise warps: two per TMEM lane quarter
+constexpr int kPrMmaWarp = kPrDq0 + kPrDqWarps;
+constexpr int kCodeWarp = kPrMmaWarp + 1;
+constexpr int kQueryWarp = kPrMmaWarp + 2;
+constexpr int kPairThreads = (kQueryWarp + 1) * 32;
 constexpr int kCodeBoxWords = 32;            // 1024 code bits of a row per box (4 stages)
 constexpr uint32_t kCodeBox = 128u * 128u;   // 128 rows x 128 bytes
 
@@ -139,33 +145,35 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     tma_prefetch_desc(&tmC);
     for (int s = 0; s < NG; ++s) {
       // leader's copy: per CTA the query producer's expect_tx arrive (+ its TMA
-      // bytes) and, per stage of the group, its four expander warps
-      mbar_init(&full[s], 2 * (1 + G * kExpWarps / 2));
+      // bytes) and the four expander warps
+      mbar_init(&full[s], 2 * (1 + kPrExpWarps));
       mbar_init(&empty[s], 1);  // MMA completion, multicast to both CTAs
     }
     for (int b = 0; b < ND; ++b) {
       mbar_init(&dfull[b], 1);   // multicast to both CTAs
-      mbar_init(&dempty[b], 8);  // 4 dequantise warps x 2 CTAs (leader's copy)
+      mbar_init(&dempty[b], 2 * kPrDqWarps);  // every dequantise warp of both CTAs (leader's copy)
     }
     for (int b = 0; b < kCodeRing; ++b) {
       mbar_init(&cfull[b], 1);           // the producer's expect_tx arrive (+ TMA bytes)
-      mbar_init(&cempty[b], kExpWarps);  // every expander warp, once per box
+      mbar_init(&cempty[b], kPrExpWarps);  // every expander warp, once per box
     }
     fence_barrier_init();
   }
-  if (warp == kMmaWarp) tmem_alloc_pair(tslot, 512);
+  if (warp == kPrMmaWarp) tmem_alloc_pair(tslot, 512);
   tc_fence_before();
   __syncthreads();
   cluster_sync_all();  // both CTAs' barriers initialised before any remote arrive
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
-  if (warp < kExpWarps) {
+  if (warp < kPrExpWarps) {
     // ---------------------------------------------------------- expanders
-    const int q4 = warp & 3, par = warp >> 2;  // lane quarter, stage parity
-    const int r = q4 * 32 + lane;              // stored row in the CTA's tile = TMEM lane
-    const uint32_t a_lane = tmem + (static_cast<uint32_t>(q4 * 32) << 16);
-    if (par == 0) {  // unit scale factors (ue8m0 0x7F = 1.0) of A and B, once
+    // Warp w expands the rows of TMEM lane quarter w, a whole group (G stages,
+    // 32 G columns) per round: wait for the group's slots, two 16-byte loads and
+    // 32 e2m1 columns per stage, one tcgen05.wait::st, one arrive.
+    const int r = warp * 32 + lane;  // stored row in the CTA's tile = TMEM lane
+    const uint32_t a_lane = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    {  // unit scale factors (ue8m0 0x7F = 1.0) of A and B, once
       uint32_t v[16];
 #pragma unroll
       for (int e = 0; e < 16; ++e) v[e] = 0x7F7F7F7Fu;
@@ -186,21 +194,24 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           break;
         }
         const uint8_t* crow = smem + code_off + cs * kCodeBox + r * 128;
-        for (int sub = par; sub < 4; sub += 2) {
-          const int jt = 4 * bt + sub;  // stage within the tile
-          if (jt >= nst) break;
-          const uint32_t j = it + jt, gj = j / G;
+        // groups never cross a box: a box holds four stages, a group G of 1 or 2
+        for (int sub = 0; sub < 4 && 4 * bt + sub < nst; sub += G) {
+          const uint32_t gj = (it + 4 * bt + sub) / G;
           const int rp = static_cast<int>(gj % NG);
           if (!warp_wait(&empty[rp], ((gj / NG) & 1u) ^ 1u, g.status)) {
             ok = false;
             break;
           }
-          const uint4 w0 = *reinterpret_cast<const uint4*>(crow + (((2 * sub) ^ row_sw) << 4));
-          const uint4 w1 = *reinterpret_cast<const uint4*>(crow + (((2 * sub + 1) ^ row_sw) << 4));
-          tc_fence_after();  // the MMAs that read the slot before (released through empty) are done
-          const uint32_t acol = a_lane + pr_acol0<BN>() + 32u * static_cast<uint32_t>(rp * G + j % G);
-          expand_half_tmem(acol, w0);
-          expand_half_tmem(acol + 16u, w1);
+          tc_fence_after();  // the MMAs that read the slots before (released through empty) are done
+#pragma unroll
+          for (int st = 0; st < G; ++st) {
+            const int c = 2 * (sub + st);  // the stage's two 16-byte chunks of the row
+            const uint4 w0 = *reinterpret_cast<const uint4*>(crow + ((c ^ row_sw) << 4));
+            const uint4 w1 = *reinterpret_cast<const uint4*>(crow + (((c + 1) ^ row_sw) << 4));
+            const uint32_t acol = a_lane + pr_acol0<BN>() + 32u * static_cast<uint32_t>(rp * G + st);
+            expand_half_tmem(acol, w0);
+            expand_half_tmem(acol + 16u, w1);
+          }
           tmem_wait_st();
           tc_fence_before();
           __syncwarp();
@@ -212,9 +223,10 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       it += nst;
       bx += nbx;
     }
-  } else if (warp < kMmaWarp) {
-    dequant_role<EOGP_SCORE_CODES, TOPK, BN, ND, pr_acc_smem<BN>(), true>(g, smem, L, tmem, sq, dfull, dempty);
-  } else if (warp == kMmaWarp) {
+  } else if (warp < kPrMmaWarp) {
+    dequant_role<EOGP_SCORE_CODES, TOPK, BN, ND, pr_acc_smem<BN>(), true, kPrDqWarps, kPrDq0>(g, smem, L, tmem, sq,
+                                                                                              dfull, dempty);
+  } else if (warp == kPrMmaWarp) {
     if (lane == 0 && rank == 0) {
       // ---------------------------------------------------------- MMA issuer (leader)
       // Kept to waits, MMAs and commits: one thread issues every MMA of the pair.
@@ -330,7 +342,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   __syncthreads();
   cluster_sync_all();  // neither CTA leaves while its peer may still signal it
   tc_fence_after();
-  if (warp == kMmaWarp) tmem_dealloc_pair(tmem, 512);
+  if (warp == kPrMmaWarp) tmem_dealloc_pair(tmem, 512);
 }
 
 template <bool TOPK, int BN, int G>

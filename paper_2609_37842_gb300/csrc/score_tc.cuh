@@ -103,21 +103,30 @@ __device__ __forceinline__ int tile_row0(int ib) {
   return PAIR ? ib * 256 + static_cast<int>(cluster_ctarank()) * 128 : ib * 128;
 }
 
-// The dequantise role (warps kDqWarp0 .. kDqWarp0 + 3, one TMEM lane quarter
-// each; TMEM lane = stored row of the CTA's tile). Per module u of a tile: wait
+// The dequantise role (warps DQ0 .. DQ0 + NDW - 1; warp w reads TMEM
+// lane quarter w % 4, TMEM lane = stored row of the CTA's tile; with eight
+// warps the two of a lane quarter take half of the query columns each). Per module u of a tile: wait
 // for the MMAs of d_u, fold acc = fl(acc + term(d_u)) into the running score
 // (TMEM columns after the ND accumulators, or shared memory when ACCS), release
 // the accumulator; after the last module write the scores (dense) or screen and
 // rank them (TOPK). In a CTA pair (PAIR) each CTA drains its own 128 rows and
 // releases the accumulator on the leader CTA's barrier.
-template <int MODE, bool TOPK, int BN, int ND, bool ACCS, bool PAIR>
+template <int MODE, bool TOPK, int BN, int ND, bool ACCS, bool PAIR, int NDW = 4, int DQ0 = kDqWarp0>
 __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem, const TcSmem& L, uint32_t tmem,
                                              float* sq, uint64_t* dfull, uint64_t* dempty) {
+  static_assert(NDW == 4 || NDW == 8, "four or eight dequantise warps");
+  static_assert(DQ0 % 4 == 0, "warp w reads TMEM lane quarter w % 4");
   constexpr uint32_t kAcc = static_cast<uint32_t>(ND * BN);
   constexpr bool kAccS = ACCS;
+  constexpr int kThr = NDW * 32;     // dequantise threads
+  constexpr int CW = BN * 4 / NDW;   // query columns of a warp (all of them, or half)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int q4 = warp & 3;
-  const int ep = threadIdx.x - 32 * kDqWarp0;  // TMEM lane (stored row in the tile)
+  const int wid = warp - DQ0;        // dequantise warp 0 .. NDW - 1
+  const int ep = wid * 32 + lane;    // dequantise thread
+  const int rr = q4 * 32 + lane;     // TMEM lane = stored row of the CTA's tile
+  const int cbeg = (wid >> 2) * CW;  // this warp's first query column
+  const int cend = min(g.BNq, cbeg + CW);
   const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
   float* lsb = g.bufs + static_cast<size_t>(blockIdx.x) * g.BNq * kFusedCap;
   int* lib = g.bufi + static_cast<size_t>(blockIdx.x) * g.BNq * kFusedCap;
@@ -130,11 +139,10 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
     return WarpTopk{lsb + static_cast<size_t>(col) * kFusedCap, lib + static_cast<size_t>(col) * kFusedCap,
                     cntb + col, taub + col, g.K, g.gtau + q0_cur + col};
   };
-  const int dw = ep >> 5;  // dequantise warp 0..3
   int seg_qt = -1;
-  // Lists of the finished query tile to global memory; warp dw writes columns dw, dw + 4, ...
+  // Lists of the finished query tile to global memory; warp wid writes columns wid, wid + NDW, ...
   auto flush = [&]() {
-    for (int col = dw; col < g.BNq; col += 4) {
+    for (int col = wid; col < g.BNq; col += NDW) {
       const int q = seg_qt * g.BNq + col;
       if (q < g.Q) {
         const size_t off = (static_cast<size_t>(blockIdx.x) * g.Q + q) * g.K;
@@ -142,40 +150,37 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
       }
     }
   };
-  // Ranks one chunk of 32 query columns (values a[] of this thread's stored row):
-  // if no value beats its column's threshold (the usual case once the lists
-  // have filled), nothing is staged; otherwise the chunk is staged column-major
-  // and warp dw offers 8 of the columns to their lists.
   // Last module of a tile, per chunk of 32 query columns: keep the scores in this
   // CTA's scratch (column-major) and note which columns hold a row that can
-  // enter the column's list (one bit per column, per warp).
+  // enter the column's list (one bit per column, per lane quarter); a column no
+  // row of which beats its threshold (the usual case once the lists have
+  // filled) is not offered.
   float* scr = g.scr + static_cast<size_t>(blockIdx.x) * BN * 128;
-  auto screen_chunk = [&](int c0, int q0, int row, const float (&a)[32]) {
-    uint32_t bits = 0;
+  // One 16-column half of a 32-column chunk: candidates' bits into `bits` (bit
+  // c0 % 32 + j), the scores into the scratch.
+  auto screen16 = [&](int c0, int q0, int row, const float (&a)[16], uint32_t& bits) {
     if (row < g.N) {
       const float4* t4 = reinterpret_cast<const float4*>(taub + c0);
       const float4* g4 = reinterpret_cast<const float4*>(gtb + c0);
 #pragma unroll
-      for (int j4 = 0; j4 < 8; ++j4) {
+      for (int j4 = 0; j4 < 4; ++j4) {
         const float4 t = t4[j4], u = g4[j4];
         const float tj[4] = {t.x, t.y, t.z, t.w}, uj[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const float x = a[4 * j4 + e];
           const bool live = q0 + c0 + 4 * j4 + e < g.Q;
-          bits |= (live && x >= uj[e] && (tj[e] != tj[e] ? x == x : x > tj[e])) ? (1u << (4 * j4 + e)) : 0u;
+          if (live && x >= uj[e] && (tj[e] != tj[e] ? x == x : x > tj[e])) bits |= 1u << ((c0 & 31) + 4 * j4 + e);
         }
       }
     }
-    const uint32_t wbits = __reduce_or_sync(0xffffffffu, bits);
-    if (lane == 0) cmask[(c0 >> 5) * 4 + dw] = wbits;
 #pragma unroll
-    for (int j = 0; j < 32; ++j) scr[static_cast<size_t>(c0 + j) * 128 + ep] = a[j];
+    for (int j = 0; j < 16; ++j) scr[static_cast<size_t>(c0 + j) * 128 + rr] = a[j];
   };
   // After the D buffer is released: the flagged columns, dealt round-robin to
-  // the four warps, offered to their lists from the scratch.
+  // the warps, offered to their lists from the scratch.
   auto rank_tile = [&](int q0, int i0) {
-    named_bar_sync(3, 128);  // scratch and masks of every warp visible
+    named_bar_sync(3, kThr);  // scratch and masks of every warp visible
     const int nr = min(128, g.N - i0);
     int n = 0;
     for (int c0 = 0; c0 < g.BNq; c0 += 32) {
@@ -184,12 +189,12 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
       for (; colmask; ++n) {
         const int cc = __ffs(colmask) - 1;
         colmask &= colmask - 1;
-        if ((n & 3) == dw)
+        if (n % NDW == wid)
           topk_warp_offer<2>(scr + static_cast<size_t>(c0 + cc) * 128, nr, i0, list_of(c0 + cc), lane,
                              gtb[c0 + cc]);
       }
     }
-    named_bar_sync(3, 128);  // lists settled before the next tile screens or flushes
+    named_bar_sync(3, kThr);  // lists settled before the next tile screens or flushes
   };
   uint32_t gm = 0;
   bool ok = true;
@@ -197,36 +202,36 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
        tile < tend && ok; tile += tstep) {
     const int qt = tile / g.n_it, ib = tile % g.n_it;
     const int i0 = tile_row0<PAIR>(ib), q0 = qt * g.BNq;
-    const int row = i0 + ep;
+    const int row = i0 + rr;
     if (TOPK && qt != seg_qt) {
       if (seg_qt >= 0) {
         flush();
-        named_bar_sync(3, 128);  // every list written before any is reset
+        named_bar_sync(3, kThr);  // every list written before any is reset
       }
       seg_qt = qt;
       q0_cur = q0;
-      for (int col = ep; col < BN; col += 128) {
+      for (int col = ep; col < BN; col += kThr) {
         cntb[col] = 0;
         taub[col] = NAN;
       }
-      named_bar_sync(3, 128);
+      named_bar_sync(3, kThr);
     }
     if (TOPK) {
       // Thresholds other CTAs' lists of these queries have reached (read before the
       // last module's ranking, after the barriers of the module loop).
-      for (int col = ep; col < BN; col += 128)
+      for (int col = ep; col < BN; col += kThr)
         gtb[col] = q0 + col < g.Q ? topk_unkey32(__ldcg(g.gtau + q0 + col)) : INFINITY;
     }
     // Scales of module u + 1 are loaded while module u is dequantised. The
     // query scales go through shared memory (buffer gm & 1): buffer gm & 1 was
     // last read in module gm - 2, which every thread finished before the
     // barrier of module gm - 1.
-    constexpr int kSqPer = (BN + 127) / 128;  // query columns of a tile per dequantise thread
+    constexpr int kSqPer = (BN + kThr - 1) / kThr;  // query columns of a tile per dequantise thread
     float si_next = row < g.N ? g.ts[static_cast<size_t>(row) * g.ldts] : 0.f;
     float sq_next[kSqPer];
 #pragma unroll
     for (int e = 0; e < kSqPer; ++e) {
-      const int c = ep + 128 * e;
+      const int c = ep + kThr * e;
       sq_next[e] = (MODE == EOGP_SCORE_CODES && c < g.BNq && q0 + c < g.Q)
                        ? g.qs[static_cast<size_t>(q0 + c) * g.ldqs] : 0.f;
     }
@@ -238,13 +243,13 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
       if (MODE == EOGP_SCORE_CODES) {
 #pragma unroll
         for (int e = 0; e < kSqPer; ++e)
-          if (ep + 128 * e < BN) sqb[ep + 128 * e] = sq_next[e];
+          if (ep + kThr * e < BN) sqb[ep + kThr * e] = sq_next[e];
       }
       if (u + 1 < g.U) {
         si_next = row < g.N ? g.ts[static_cast<size_t>(row) * g.ldts + u + 1] : 0.f;
 #pragma unroll
         for (int e = 0; e < kSqPer; ++e) {
-          const int c = ep + 128 * e;
+          const int c = ep + kThr * e;
           sq_next[e] = (MODE == EOGP_SCORE_CODES && c < g.BNq && q0 + c < g.Q)
                            ? g.qs[static_cast<size_t>(q0 + c) * g.ldqs + u + 1] : 0.f;
         }
@@ -254,14 +259,14 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
       w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
       __syncwarp();
       tc_fence_after();
-      if (!__syncthreads_and_named(w_ok)) {  // also publishes sqb
+      if (!named_bar_and(2, kThr, w_ok)) {  // also publishes sqb
         ok = false;
         break;
       }
       const bool last = u + 1 == g.U;
       const uint32_t dcol = tmem + lane_base + buf * static_cast<uint32_t>(BN);
       const uint32_t acol = tmem + lane_base + kAcc;
-      float* accrow = reinterpret_cast<float*>(smem + L.acc) + ep * kAccLd;  // kAccS: this row's running score
+      float* accrow = reinterpret_cast<float*>(smem + L.acc) + rr * kAccLd;  // kAccS: this row's running score
       auto acc_load = [&](int c0, uint32_t* ar, int n) {  // n floats from the shared running score
         for (int j = 0; j < n; j += 4) {
           const float4 v = *reinterpret_cast<const float4*>(accrow + c0 + j);
@@ -280,17 +285,17 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
         // Running score, 16 columns at a time: the TMEM loads of the next chunk
         // are in flight while this one is combined and stored back.
         uint32_t dr[16], ar[16];
-        tmem_ld16_issue(dcol, dr);
-        if (!kAccS && u > 0) {
-          tmem_ld16_issue(acol, ar);
+        if (cbeg < cend) tmem_ld16_issue(dcol + cbeg, dr);
+        if (!kAccS && u > 0 && cbeg < cend) {
+          tmem_ld16_issue(acol + cbeg, ar);
         } else {
 #pragma unroll
           for (int j = 0; j < 16; ++j) ar[j] = 0u;
         }
 #pragma unroll
-        for (int ci = 0; ci < BN / 16; ++ci) {
-          const int c0 = 16 * ci;
-          if (c0 < g.BNq) {
+        for (int ci = 0; ci < CW / 16; ++ci) {
+          const int c0 = cbeg + 16 * ci;
+          if (c0 < cend) {
             tmem_wait_ld(dr);
             if constexpr (kAccS) {
               if (u > 0) acc_load(c0, ar, 16);
@@ -301,7 +306,7 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
 #pragma unroll
             for (int j = 0; j < 16; ++j)
               o[j] = __float_as_uint(__fadd_rn(__uint_as_float(ar[j]), term(c0 + j, dr[j])));
-            if (c0 + 16 < g.BNq) {
+            if (c0 + 16 < cend) {
               tmem_ld16_issue(dcol + c0 + 16, dr);
               if (!kAccS && u > 0) tmem_ld16_issue(acol + c0 + 16, ar);
             }
@@ -318,41 +323,59 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
         }
         if constexpr (!kAccS) tmem_wait_st();  // stored before the next module reads them
       } else {
-        for (int c0 = 0; c0 < g.BNq; c0 += 32) {
-          uint32_t dr[32], ar[32];
-          tmem_ld32_issue(dcol + c0, dr);
-          if (u > 0 && kAccS) {
-            acc_load(c0, ar, 32);
-          } else if (u > 0) {
-            tmem_ld32_issue(acol + c0, ar);
-          } else {
+        // Last module: 16 columns at a time, the next chunk's TMEM loads in
+        // flight while this one is finished and written out (or screened).
+        uint32_t dr[16], ar[16];
+        if (cbeg < cend) {
+          tmem_ld16_issue(dcol + cbeg, dr);
+          if (!kAccS && u > 0) tmem_ld16_issue(acol + cbeg, ar);
+        }
+        uint32_t bits = 0;  // TOPK: candidates of the current 32-column chunk
 #pragma unroll
-            for (int j = 0; j < 32; ++j) ar[j] = 0u;
-          }
-          tmem_wait_ld(dr);
-          if constexpr (!kAccS) tmem_wait_ld(ar);
-          float a[32];
+        for (int ci = 0; ci < CW / 16; ++ci) {
+          const int c0 = cbeg + 16 * ci;
+          if (c0 < cend) {
+            tmem_wait_ld(dr);
+            if (u > 0 && kAccS) {
+              acc_load(c0, ar, 16);
+            } else if (u > 0) {
+              tmem_wait_ld(ar);
+            } else {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) a[j] = __fadd_rn(__uint_as_float(ar[j]), term(c0 + j, dr[j]));
-          if (!TOPK) {
-            if (row < g.N) {
-#pragma unroll
-              for (int j = 0; j < 32; ++j)
-                if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
+              for (int j = 0; j < 16; ++j) ar[j] = 0u;
             }
-          } else {
-            screen_chunk(c0, q0, row, a);
+            float a[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) a[j] = __fadd_rn(__uint_as_float(ar[j]), term(c0 + j, dr[j]));
+            if (c0 + 16 < cend) {
+              tmem_ld16_issue(dcol + c0 + 16, dr);
+              if (!kAccS && u > 0) tmem_ld16_issue(acol + c0 + 16, ar);
+            }
+            if (!TOPK) {
+              if (row < g.N) {
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                  if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
+              }
+            } else {
+              screen16(c0, q0, row, a, bits);
+              if ((c0 & 31) == 16) {  // the 32-column chunk is complete (BNq is a multiple of 32)
+                const uint32_t wbits = __reduce_or_sync(0xffffffffu, bits);
+                if (lane == 0) cmask[(c0 >> 5) * 4 + q4] = wbits;  // a chunk's rows: the four lane quarters
+                bits = 0;
+              }
+            }
           }
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {  // D buffer free: the MMAs run on
-      if constexpr (PAIR)  // the pair's MMA issuer waits on the leader CTA's barrier
-        mbar_arrive_relaxed_cluster(mapa_shared(smem_u32(&dempty[buf]), 0));
-      else
-        mbar_arrive(&dempty[buf]);
-    }
+        if constexpr (PAIR)  // the pair's MMA issuer waits on the leader CTA's barrier
+          mbar_arrive_relaxed_cluster(mapa_shared(smem_u32(&dempty[buf]), 0));
+        else
+          mbar_arrive(&dempty[buf]);
+      }
       if (TOPK && last) rank_tile(q0, i0);
     }
   }
