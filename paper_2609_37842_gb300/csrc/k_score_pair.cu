@@ -19,10 +19,14 @@
 //    128-byte swizzle, loaded by TMA by a producer warp as far ahead as the
 //    ring allows, so HBM latency is hidden by the ring rather than by registers;
 //  * pipeline groups of G 256-bit stages: per stage a query operand tile in
-//    shared memory (BNq / 2 rows x 128 bytes, loaded by a second producer warp
-//    as soon as the MMAs release the group) and an A slot of 32 TMEM columns
-//    (the expanded stored rows). One barrier pair per group: the MMA issuer
-//    waits once, issues 4 G MMAs and commits once. A single thread issues all
+//    shared memory (BNq / 2 rows x 128 bytes, loaded by a second producer warp)
+//    and an A slot of 32 TMEM columns (the expanded stored rows). One barrier
+//    pair per group: the MMA issuer waits once, issues 4 G MMAs and commits
+//    once. The query tiles sit in a deeper ring (NQ groups) than the A slots
+//    (NG groups, all TMEM leaves): the query stages of group gj are loaded once
+//    group gj - NQ is done, its A slots refilled once group gj - NG is done,
+//    both read from the one commit per group, so the queries' L2 latency is off
+//    the A slots' round trip. A single thread issues all
 //    MMAs at about one per 64 cycles, plus ~330 cycles per wait-fence-commit
 //    round: at 256 bits per round the rounds, not the tensor pipe, set the pace
 //    (measured: 589 cycles per four N = 256 MMAs, 8.4 of 9.7 PFLOP/s), at
@@ -81,11 +85,15 @@ template <int BN>
 constexpr bool pr_acc_smem() {
   return BN == 128;
 }
-// Code boxes in flight: as many as the shared memory holds next to the query
-// tiles (and the running score of several modules).
+// Code boxes in flight and query stages: as many as the shared memory holds
+// next to the running score of several modules.
 template <int BN>
 constexpr int pr_code_ring() {
-  return BN == 64 ? 8 : BN == 256 ? 6 : 4;
+  return BN == 64 ? 8 : BN == 256 ? 3 : 4;
+}
+template <int BN>
+constexpr int pr_qstages() {
+  return BN == 64 ? 20 : 10;
 }
 template <int BN>
 constexpr uint32_t pr_acol0() {
@@ -96,18 +104,18 @@ constexpr uint32_t pr_sf_col() {
   return pr_acol0<BN>() + 32u * static_cast<uint32_t>(pr_slots<BN>());
 }
 
-// Shared memory: query tiles (one per A slot), the code ring, then the layout
-// the dequantise role shares with the one-CTA kernel.
+// Shared memory: the query ring, the code ring, then the layout the dequantise
+// role shares with the one-CTA kernel.
 template <bool TOPK, int BN, int G>
 __host__ __device__ inline TcSmem pr_smem_layout(uint32_t* code_off) {
-  constexpr int NG = pr_slots<BN>() / G, kCodeRing = pr_code_ring<BN>();
+  constexpr int NQ = pr_qstages<BN>() / G, kCodeRing = pr_code_ring<BN>();
   constexpr uint32_t kStage = static_cast<uint32_t>(BN / 2) * 128u;
   TcSmem l;
-  *code_off = NG * G * kStage;
+  *code_off = NQ * G * kStage;
   l.acc = *code_off + kCodeRing * kCodeBox;
   l.sq = l.acc + (pr_acc_smem<BN>() ? 128u * kAccLd * 4u : 0u);
   l.bars = l.sq + 2 * BN * 4;
-  l.lists = l.bars + (2 * NG + 2 * pr_dbufs<BN>() + 2 * kCodeRing) * 8 + 16;
+  l.lists = l.bars + (2 * NQ + 2 * pr_dbufs<BN>() + 2 * kCodeRing) * 8 + 16;
   l.total = l.lists + (TOPK ? BN * 12 + 8 * 4 * 4 : 0);
   return l;
 }
@@ -116,13 +124,14 @@ template <bool TOPK, int BN, int G>
 __global__ void __launch_bounds__(kPairThreads, 1)
     k_score_pair(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmC,
                  const __grid_constant__ ScoreTcArgs g) {
-  constexpr int NG = pr_slots<BN>() / G;  // groups in the ring
+  constexpr int NG = pr_slots<BN>() / G;      // groups of A slots in TMEM
+  constexpr int NQ = pr_qstages<BN>() / G;    // groups of query stages in shared memory
   constexpr int ND = pr_dbufs<BN>();
   constexpr int kCodeRing = pr_code_ring<BN>();
   constexpr uint32_t kStage = static_cast<uint32_t>(BN / 2) * 128u;
   constexpr uint32_t kSfa = pr_sf_col<BN>(), kSfb = kSfa + 16u;
   static_assert(kSfb + 16u <= 512u, "TMEM budget");
-  static_assert(NG >= 2, "the ring needs two groups");
+  static_assert(NG >= 2 && NQ >= NG, "rings: at least two A groups, at least as many query groups");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint32_t code_off;
@@ -130,9 +139,11 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
   float* sq = reinterpret_cast<float*>(smem + L.sq);
+  // group gj: full / empty barrier gj % NQ, query stages of slot gj % NQ, A
+  // slots of slot gj % NG
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bars);
-  uint64_t* empty = full + NG;
-  uint64_t* dfull = empty + NG;
+  uint64_t* empty = full + NQ;
+  uint64_t* dfull = empty + NQ;
   uint64_t* dempty = dfull + ND;
   uint64_t* cfull = dempty + ND;
   uint64_t* cempty = cfull + kCodeRing;
@@ -143,11 +154,11 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tmQ);
     tma_prefetch_desc(&tmC);
-    for (int s = 0; s < NG; ++s) {
+    for (int s = 0; s < NQ; ++s) {
       // leader's copy: per CTA the query producer's expect_tx arrive (+ its TMA
       // bytes) and the four expander warps
       mbar_init(&full[s], 2 * (1 + kPrExpWarps));
-      mbar_init(&empty[s], 1);  // MMA completion, multicast to both CTAs
+      mbar_init(&empty[s], 1);  // MMA completion of the group, multicast to both CTAs
     }
     for (int b = 0; b < ND; ++b) {
       mbar_init(&dfull[b], 1);   // multicast to both CTAs
@@ -198,11 +209,15 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         for (int sub = 0; sub < 4 && 4 * bt + sub < nst; sub += G) {
           const uint32_t gj = (it + 4 * bt + sub) / G;
           const int rp = static_cast<int>(gj % NG);
-          if (!warp_wait(&empty[rp], ((gj / NG) & 1u) ^ 1u, g.status)) {
-            ok = false;
-            break;
+          // the A slots are free once the MMAs of group gj - NG are done
+          if (gj >= NG) {
+            const uint32_t gp = gj - NG;
+            if (!warp_wait(&empty[gp % NQ], (gp / NQ) & 1u, g.status)) {
+              ok = false;
+              break;
+            }
           }
-          tc_fence_after();  // the MMAs that read the slots before (released through empty) are done
+          tc_fence_after();  // the MMAs that read the slots before are done
 #pragma unroll
           for (int st = 0; st < G; ++st) {
             const int c = 2 * (sub + st);  // the stage's two 16-byte chunks of the row
@@ -215,7 +230,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           tmem_wait_st();
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive_relaxed_cluster(mapa_shared(smem_u32(&full[rp]), 0));
+          if (lane == 0) mbar_arrive_relaxed_cluster(mapa_shared(smem_u32(&full[gj % NQ]), 0));
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&cempty[cs]);  // this warp is done reading box b
@@ -234,9 +249,9 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       const uint32_t sfa = tmem + kSfa, sfb = tmem + kSfb;
       const uint64_t dbase = sdesc_sw128(smem_u32(smem), 16, 1024);
       constexpr uint64_t kGroupDesc = (static_cast<uint64_t>(G) * kStage) >> 4;  // descriptor step per group
-      uint64_t dq = dbase;                   // query tile of the group's first stage
-      uint32_t acl = tmem + pr_acol0<BN>();  // its A slot
-      int rg = 0;
+      uint64_t dq = dbase;                   // query stages of query slot rq
+      uint32_t acl = tmem + pr_acol0<BN>();  // A slots of A slot ra
+      int rq = 0, ra = 0;
       uint32_t rph = 0, gm = 0;
       bool ok = true;
       for (int tile = tile_begin<TOPK, true>(g), tstep = tile_step<TOPK, true>(), tend = tile_end<TOPK, true>(g);
@@ -251,17 +266,21 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           const uint32_t d = tmem + buf * static_cast<uint32_t>(BN);
           const int ngr = g.k[u] / (256 * G);
           for (int gi = 0; gi < ngr; ++gi) {
-            const int s = rg;
+            const int s = rq;
             const uint32_t ph = rph;
             const uint64_t b0 = dq;
             const uint32_t at0 = acl;
-            if (++rg == NG) {
-              rg = 0;
+            if (++rq == NQ) {
+              rq = 0;
               rph ^= 1u;
               dq = dbase;
-              acl = tmem + pr_acol0<BN>();
             } else {
               dq += kGroupDesc;
+            }
+            if (++ra == NG) {
+              ra = 0;
+              acl = tmem + pr_acol0<BN>();
+            } else {
               acl += 32u * G;
             }
             // both CTAs' query bytes and expander warps (the MMAs read the
@@ -322,8 +341,8 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         const int qrow = (tile / g.n_it) * g.BNq + static_cast<int>(rank) * (g.BNq / 2);
         for (int jt = 0; jt < nst; jt += G) {
           const uint32_t gj = (it + jt) / G;
-          const int s = static_cast<int>(gj % NG);
-          if (!mbar_wait(&empty[s], ((gj / NG) & 1u) ^ 1u, g.status)) {
+          const int s = static_cast<int>(gj % NQ);  // free once the MMAs of group gj - NQ are done
+          if (!mbar_wait(&empty[s], ((gj / NQ) & 1u) ^ 1u, g.status)) {
             ok = false;
             break;
           }
