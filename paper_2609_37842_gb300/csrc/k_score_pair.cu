@@ -30,7 +30,9 @@
 //    MMAs at about one per 64 cycles, plus ~330 cycles per wait-fence-commit
 //    round: at 256 bits per round the rounds, not the tensor pipe, set the pace
 //    (measured: 589 cycles per four N = 256 MMAs, 8.4 of 9.7 PFLOP/s), at
-//    512 bits the tensor pipe does (1024 cycles per eight, 9.7 PFLOP/s).
+//    512 bits the tensor pipe does (1024 cycles per eight, 9.7 PFLOP/s). An
+//    N = 64 MMA takes as long to issue as an N = 128 one, so 64-query tiles
+//    (one module of a multiple of 1024 bits) take four stages per group.
 // Each expander warp takes the 32 rows of one TMEM lane quarter, a whole group
 // per round: two 16-byte shared-memory loads and the e2m1 expansion per stage,
 // the TMEM stores, and one relaxed arrive on the leader's barrier of the group. That arrive orders enough: it is issued after
@@ -205,7 +207,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           break;
         }
         const uint8_t* crow = smem + code_off + cs * kCodeBox + r * 128;
-        // groups never cross a box: a box holds four stages, a group G of 1 or 2
+        // groups never cross a box: a box holds four stages, a group G of 1, 2 or 4
         for (int sub = 0; sub < 4 && 4 * bt + sub < nst; sub += G) {
           const uint32_t gj = (it + 4 * bt + sub) / G;
           const int rp = static_cast<int>(gj % NG);
@@ -396,6 +398,7 @@ cudaError_t launch_bn(int BN, int G, const CUtensorMap& tq, const CUtensorMap& t
                       cudaStream_t st) {
   if (BN == 256) return G == 2 ? launch<TOPK, 256, 2>(tq, tc, g, grid, st) : launch<TOPK, 256, 1>(tq, tc, g, grid, st);
   if (BN == 128) return G == 2 ? launch<TOPK, 128, 2>(tq, tc, g, grid, st) : launch<TOPK, 128, 1>(tq, tc, g, grid, st);
+  if (G == 4) return launch<TOPK, 64, 4>(tq, tc, g, grid, st);
   return G == 2 ? launch<TOPK, 64, 2>(tq, tc, g, grid, st) : launch<TOPK, 64, 1>(tq, tc, g, grid, st);
 }
 
@@ -405,11 +408,11 @@ size_t pair_smem_need(int BN, int G, bool topk) {
   if (topk) {
     if (BN == 256) return G == 2 ? smem_need<true, 256, 2>() : smem_need<true, 256, 1>();
     if (BN == 128) return G == 2 ? smem_need<true, 128, 2>() : smem_need<true, 128, 1>();
-    return G == 2 ? smem_need<true, 64, 2>() : smem_need<true, 64, 1>();
+    return G == 4 ? smem_need<true, 64, 4>() : G == 2 ? smem_need<true, 64, 2>() : smem_need<true, 64, 1>();
   }
   if (BN == 256) return G == 2 ? smem_need<false, 256, 2>() : smem_need<false, 256, 1>();
   if (BN == 128) return G == 2 ? smem_need<false, 128, 2>() : smem_need<false, 128, 1>();
-  return G == 2 ? smem_need<false, 64, 2>() : smem_need<false, 64, 1>();
+  return G == 4 ? smem_need<false, 64, 4>() : G == 2 ? smem_need<false, 64, 2>() : smem_need<false, 64, 1>();
 }
 
 int pair_cluster_cap(int num_sms) {
@@ -447,7 +450,7 @@ int pair_cluster_cap(int num_sms) {
 cudaError_t launch_pair(int BN, int G, bool topk, const CUtensorMap& tq, const ScoreTcArgs& g, int grid,
                         cudaStream_t st) {
   if (BN != 64 && BN != 128 && BN != 256) return cudaErrorInvalidValue;
-  if (G != 1 && G != 2) return cudaErrorInvalidValue;
+  if (G != 1 && G != 2 && !(G == 4 && BN == 64)) return cudaErrorInvalidValue;
   if (BN == 256 && g.U != 1) return cudaErrorInvalidValue;  // 256-query tiles keep no running score
   if (BN == 64 && g.U != 1) return cudaErrorInvalidValue;   // 64-query tiles keep no running score
   for (int u = 0; u < g.U; ++u)

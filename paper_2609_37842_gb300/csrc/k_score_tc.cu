@@ -536,11 +536,12 @@ TcCfg tc_cfg(int mode, const int* ks, int U, int Q, int K) {
   c.BN = c.pair ? pr_bn(U, Q) : tc_bn(mode, U, Q, K);
   c.BNq = bnq_for(Q, c.BN);
   c.rows = c.pair ? 256 : 128;
-  // two stages per group when every module is a multiple of 512 bits (groups
-  // never straddle modules), else one
-  c.G = 2;
-  for (int u = 0; u < U; ++u)
-    if (ks[u] % 512) c.G = 1;
+  // stages per group of the pair kernel (groups never straddle modules): four
+  // with 64-query tiles when every module is a multiple of 1024 bits, two when
+  // a multiple of 512, else one
+  c.G = c.BN == 64 ? 4 : 2;
+  for (int u = 0; u < U && c.pair; ++u)
+    while (c.G > 1 && ks[u] % (256 * c.G)) c.G /= 2;
   return c;
 }
 

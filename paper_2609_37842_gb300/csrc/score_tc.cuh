@@ -388,7 +388,8 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsign
 }
 
 // Host side of the CTA-pair kernel (k_score_pair.cu): BN queries per tile (64,
-// 128 or 256), G 256-bit stages per pipeline group (1 or 2), fused ranking or not.
+// 128 or 256), G 256-bit stages per pipeline group (1 or 2; 4 with BN = 64),
+// fused ranking or not.
 size_t pair_smem_need(int BN, int G, bool topk);
 // Clusters of two that can be resident at once on the current device.
 int pair_cluster_cap(int num_sms);
