@@ -26,7 +26,10 @@
 //    (NG groups, all TMEM leaves): the query stages of group gj are loaded once
 //    group gj - NQ is done, its A slots refilled once group gj - NG is done,
 //    both read from the one commit per group, so the queries' L2 latency is off
-//    the A slots' round trip. A single thread issues all
+//    the A slots' round trip. This lagged reuse relies on groups completing in
+//    order, hence one issuing thread: with a second one (each owning one of two
+//    accumulators) completions came out of order, a parity wait could pass a
+//    phase early, and the full 4.2M-code scan faulted the GPU (Xid 13). A single thread issues all
 //    MMAs at about one per 64 cycles, plus ~330 cycles per wait-fence-commit
 //    round: at 256 bits per round the rounds, not the tensor pipe, set the pace
 //    (measured: 589 cycles per four N = 256 MMAs, 8.4 of 9.7 PFLOP/s), at
