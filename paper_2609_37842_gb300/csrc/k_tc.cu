@@ -1089,9 +1089,12 @@ cudaError_t launch_tc_gemm_hl(int M, int N, int K, const void* Ah, const void* A
 }
 
 // CTA pairs measured faster for short reductions (K <= 1536: the hi/lo
-// epilogue dominates and halving the per-SM operand stream helps) and slower
-// for long ones.
-static bool rotate_pairs(int K) { return K <= 1536; }
+// epilogue dominates and halving the per-SM operand stream helps) and for few
+// output columns (n <= 256: the activations stream from HBM and every 128-row
+// tile re-reads the whole eigenvector operand from L2, which the pair halves;
+// OLMo-2-1B stack 1,487 -> 1,557 examples/s), and slower for long reductions
+// with many columns.
+static bool rotate_pairs(int K, int n) { return K <= 1536 || n <= 256; }
 
 // N tile width for `n` output columns: as few tiles of at most 256 columns as
 // is cheapest, each a multiple of `gran` (16: the tcgen05 N granularity, for one
@@ -1115,7 +1118,7 @@ cudaError_t launch_tc_rotate(int M, int K, const void* X, int ldx, const void* W
                              void* hi, void* lo, int ldo, int T, const float* bias,
                              const int32_t* lengths, int num_sms, unsigned* status, cudaStream_t st) {
   if (M <= 0) return cudaSuccess;
-  const bool pairs = rotate_pairs(K);
+  const bool pairs = rotate_pairs(K, Wrows);
   const int BN = rotate_bn(Wrows, 16);
   // As many pipeline stages as fit in 227 KB of shared memory (at most 8).
   int stages = 2;
