@@ -14,13 +14,18 @@ spectra with exponent 1.0), drawn on the device before timing; one input buffer
 per module type serves the 32 layers, and each module's inputs (0.5-2 GB) exceed
 L2, so no flush is needed.
 
-`value` is examples compressed per second per layer stack (whole job, all
-ranks). `e2e` repeats the step through the C-ABI's host-input call
+Consecutive modules alternate between two streams with a workspace each (the
+modules are independent), so one module's contraction, projection and pack run
+beside the next module's rotations. `value` is examples compressed per second
+per layer stack (whole job, all ranks). `e2e` repeats the step through the C-ABI's host-input call
 (eogp_compress_layer_host) with a, s and the eigenbases in page-locked host
 memory: the call's host-to-device copies and the device-to-host read of the
 codes are inside the timed region; the plain host-to-device copy rate of the
 same run is reported beside it. `roofline` is that of the rotation kernels,
-and `roofline.others` carries the other timed kernels' rooflines, the
+timed launch by launch with CUDA events in a few profiled steps of the same
+configuration after the timed ones (every module on one stream, so that no
+launch overlaps another), and `roofline.others` carries the other timed
+kernels' rooflines, the
 query x train scoring rates included. The GPT-2, OLMo-1B, 32B-gate and fp32
 stacks, the scoring workloads and the PCA fit follow in the same line.
 
@@ -263,9 +268,12 @@ def config_setup(name, B, dev):
 
 class Stack:
     """One workload's compression step: B examples through every module of the
-    stack into one-bit codes. With stream_bases the retained eigenvector rows of
-    every layer live in page-locked host memory and are copied to the device one
-    layer ahead of its compute on a side stream (two device slots)."""
+    stack into one-bit codes. Consecutive modules alternate between two streams,
+    each with its own workspace (the modules are independent), so that one
+    module's contraction, projection and pack overlap the next module's
+    rotations. With stream_bases the retained eigenvector rows of every layer
+    live in page-locked host memory and are copied to the device one layer ahead
+    of its compute on a side stream (two device slots)."""
 
     def __init__(self, name, B, dev, stream_bases=False, modules=0):
         import dataclasses
@@ -285,6 +293,8 @@ class Stack:
         self.codes = torch.empty((B, self.U * self.words), dtype=torch.int32, device=dev)
         self.scales = torch.empty((B, self.U), dtype=torch.float32, device=dev)
         self.stream = torch.cuda.current_stream()
+        self.streams = [self.stream, torch.cuda.Stream()]
+        self.wss = [self.ws, E.workspace(self.ws.numel(), dev)]
         self.nmod_layer = len(set(self.keys))
         self.layers = max(1, self.U // self.nmod_layer) if name.startswith("olmo") else 1
         self.stream_bases = stream_bases and self.layers > 1
@@ -299,23 +309,30 @@ class Stack:
             self.landed = [torch.cuda.Event() for _ in range(2)]
             self.freed = [None, None]
 
-    def _module(self, u, desc):
+    def _module(self, u, desc, single=False):
         L = self.per_layer[self.keys[u]]
         wd = self.words
+        i = 0 if single else u % 2
         self.E.compress_layer(desc, L["a"], L["s"], self.E.OUT_CODES, codes=self.codes[:, u * wd:(u + 1) * wd],
-                              scales=self.scales[:, u], ws=self.ws)
+                              scales=self.scales[:, u], ws=self.wss[i], stream=self.streams[i])
 
-    def step(self):
+    def step(self, single=False):
+        """One step; `single` keeps every module on the main stream (the profiled
+        steps that time each kernel on its own)."""
         import torch
+        s0, s1 = self.streams
+        s1.wait_stream(s0)  # the step starts after everything before it on the main stream
         if not self.stream_bases:
             for u, key in enumerate(self.keys):
-                self._module(u, self.descs[key])
+                self._module(u, self.descs[key], single)
+            s0.wait_stream(s1)  # and ends after both streams' work
             return
 
         def issue_copy(layer):
             sl = layer % 2
             if self.freed[sl] is not None:
-                self.cstream.wait_event(self.freed[sl])
+                for ev in self.freed[sl]:
+                    self.cstream.wait_event(ev)
             with torch.cuda.stream(self.cstream):
                 for k in self.per_layer:
                     self.dev_bases[sl][k][0].copy_(self.host_one[k][0], non_blocking=True)
@@ -326,26 +343,30 @@ class Stack:
             sl = layer % 2
             if layer + 1 < self.layers:
                 issue_copy(layer + 1)
-            self.stream.wait_event(self.landed[sl])
+            s0.wait_event(self.landed[sl])
+            s1.wait_event(self.landed[sl])
             for j in range(self.nmod_layer):
                 u = layer * self.nmod_layer + j
-                self._module(u, self.slot_descs[sl][self.keys[u]])
-            ev = torch.cuda.Event()
-            ev.record(self.stream)
-            self.freed[sl] = ev
+                self._module(u, self.slot_descs[sl][self.keys[u]], single)
+            evs = (torch.cuda.Event(), torch.cuda.Event())  # the slot is free once both streams are done with it
+            evs[0].record(s0)
+            evs[1].record(s1)
+            self.freed[sl] = evs
+        s0.wait_stream(s1)
 
-    def timed(self, steps, warmup, clocks=None, barrier=None):
-        """Warm-up, then `steps` steps between CUDA events on the compute stream with
-        every library launch bracketed by events; returns (ms, per-kind kernel times)."""
+    def timed(self, steps, warmup, clocks=None, barrier=None, prof_steps=0):
+        """Warm-up, then `steps` steps between CUDA events on the main stream
+        (modules alternating between the two streams); then `prof_steps` (default:
+        min(steps, 3)) steps with every module on the main stream and every library
+        launch bracketed by CUDA events, which time each kernel on its own. Returns
+        (ms of the timed steps, per-kind kernel times of the profiled steps, clocks,
+        profiled steps)."""
         import torch
         E = self.E
         for _ in range(warmup):
             self.step()
         torch.cuda.synchronize()
         E.sync_status()
-        for kk in E.KERNEL_KINDS:
-            E.profile_read(kk, reset=True)
-        E.profile_enable(True)
         if barrier:
             barrier()
         torch.cuda.synchronize()
@@ -360,6 +381,14 @@ class Stack:
         if barrier:
             barrier()
         clk = clocks.stop() if clocks else None
+        E.sync_status()
+        prof_steps = prof_steps or min(steps, 3)
+        for kk in E.KERNEL_KINDS:
+            E.profile_read(kk, reset=True)
+        E.profile_enable(True)
+        for _ in range(prof_steps):
+            self.step(single=True)
+        torch.cuda.synchronize()
         E.profile_enable(False)
         E.sync_status()
         kern = {}
@@ -370,7 +399,7 @@ class Stack:
         ktot = sum(v["ms"] for v in kern.values())
         for v in kern.values():
             v["share"] = v["ms"] / ktot if ktot else None
-        return e0.elapsed_time(e1), kern, clk
+        return e0.elapsed_time(e1), kern, clk, prof_steps
 
     def rot_flops(self):
         pl = self.per_layer
@@ -382,8 +411,9 @@ class Stack:
         return sum(2.0 * self.B * self.w.T * (pl[k]["d_in"] + pl[k]["d_out"]) * (2 if self.w.dtype == "f32" else 1)
                    for k in self.keys)
 
-    def summary(self, ms, steps, kern, peaks):
-        """examples/s, stack and rotation TFLOP/s, input GB/s and the rotation roofline."""
+    def summary(self, ms, steps, kern, peaks, prof_steps):
+        """examples/s, stack and rotation TFLOP/s, input GB/s (timed steps) and the
+        rotation roofline (profiled steps)."""
         w, B = self.w, self.B
         sec = ms / 1000.0
         rot = kern.get("rotate", {"launches": 0, "ms": 0.0})
@@ -398,7 +428,7 @@ class Stack:
         hbm = peaks.get("hbm_gbs") or PEAKS_FALLBACK["hbm_gbs"]
         out["input_frac_of_hbm"] = out["input_GBps"] / hbm
         if rot["launches"]:
-            per_launch = rf * steps / rot["launches"]
+            per_launch = rf * prof_steps / rot["launches"]
             avg_ms = rot["ms"] / rot["launches"]
             ach = per_launch / (avg_ms / 1000.0) / 1e12
             peak = peaks.get("bf16_tflops_sustained") or PEAKS_FALLBACK["bf16_tflops_sustained"]
@@ -407,7 +437,10 @@ class Stack:
                                "frac": ach / peak,
                                "traffic": tr[0] * B / tr[1] if tr and self.U == len(self.w.modules) else None,
                                "kernel": "k_tc_rotate / k_tc_rotate2 (Kronecker rotations)",
-                               "flops_per_launch": per_launch}
+                               "flops_per_launch": per_launch,
+                               "timing": f"CUDA events around each launch in {prof_steps} profiled steps of the same "
+                                         "configuration after the timed ones, every module on one stream (the "
+                                         "timed steps alternate two streams, so launches overlap there)"}
         if self.stream_bases:
             out["eigenbases"] = "host-pinned, one layer ahead on a side stream"
             out["h2d_bytes_per_step"] = self.layers * sum(2 * (L["VA"].numel() + L["VS"].numel())
@@ -685,7 +718,8 @@ def cpu_score_sample(ks, seconds=3.0):
 def headline_config(w, B, world, name):
     cfg = {"workload": name, "batch_per_gpu": B, "seq_len": w.T, "m": w.m, "k": w.k,
            "modules": len(w.modules), "parallelism": f"replicas x{world}",
-           "l2": "inputs > L2 (each module's inputs exceed 129 MB every step)"}
+           "l2": "inputs > L2 (each module's inputs exceed 129 MB every step)",
+           "streams": "consecutive modules alternate between two streams, one workspace each"}
     if name == "olmo2_7b_bf16":
         cfg["eigenbases"] = "page-locked host memory, streamed one layer ahead"
     return cfg
@@ -971,15 +1005,16 @@ def main():
     st = Stack(name, B, dev, stream_bases=(name == "olmo2_7b_bf16"), modules=args.modules)
     w = st.w
     clocks = ClockSampler(local)
-    ms, kern, clk = st.timed(args.steps, args.warmup, clocks=clocks, barrier=barrier)
+    ms, kern, clk, psteps = st.timed(args.steps, args.warmup, clocks=clocks, barrier=barrier)
     t_max = ms
     if world > 1:
         tt = torch.tensor([ms], device=dev)
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         t_max = float(tt.item())
     value = world * B * args.steps / (t_max / 1000.0)
-    launches = sum(v["launches"] for v in kern.values())
-    head = st.summary(ms, args.steps, kern, peaks)
+    # library launches inside the timed region: per step as counted in the profiled steps
+    launches = round(sum(v["launches"] for v in kern.values()) / psteps * args.steps)
+    head = st.summary(ms, args.steps, kern, peaks, psteps)
     roofline = dict(head.get("roofline") or {"bound": "tensor", "achieved": None, "peak": None,
                                              "unit": "TFLOP/s", "frac": None, "traffic": None})
     roofline["peak_source"] = f"{peaks_src} bf16_tflops_sustained"
@@ -1029,8 +1064,8 @@ def main():
                 continue
             o = Stack(nm, CONFIG_BATCH[nm], dev, stream_bases=(nm == "olmo2_7b_bf16"))
             steps = 3 if nm.startswith("olmo2_") and nm != "olmo2_32b_gate_bf16" else 5
-            oms, okern, _ = o.timed(steps, 3)
-            configs[nm] = o.summary(oms, steps, okern, peaks)
+            oms, okern, _, opsteps = o.timed(steps, 3)
+            configs[nm] = o.summary(oms, steps, okern, peaks, opsteps)
             o.release()
             del o
             torch.cuda.empty_cache()
