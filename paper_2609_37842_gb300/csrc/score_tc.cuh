@@ -118,6 +118,10 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
   static_assert(DQ0 % 4 == 0, "warp w reads TMEM lane quarter w % 4");
   constexpr uint32_t kAcc = static_cast<uint32_t>(ND * BN);
   constexpr bool kAccS = ACCS;
+  // The running score of several modules: in shared memory (ACCS), else in the
+  // TMEM columns after the accumulators, which only the one-CTA kernel's
+  // 128-query tiles have (the pair kernel's other tile widths serve one module).
+  constexpr bool kAccT = !ACCS && BN == 128 && !PAIR;
   constexpr int kThr = NDW * 32;     // dequantise threads
   constexpr int CW = BN * 4 / NDW;   // query columns of a warp (all of them, or half)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -281,14 +285,62 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
         return MODE == EOGP_SCORE_CODES ? __fmul_rn(__fmul_rn(sqb[c], si), __uint_as_float(dv))
                                         : __fmul_rn(si, __uint_as_float(dv));
       };
-      if (!last) {
-        // Running score, 16 columns at a time: the TMEM loads of the next chunk
-        // are in flight while this one is combined and stored back.
+      if constexpr (!kAccT) {
+        // d_u in batches of 32 columns: the batch's TMEM loads are issued
+        // before its one wait (tcgen05.wait::ld waits for all of the thread's
+        // loads, so a load issued one 16-column chunk ahead is still waited for
+        // before that chunk is done); the running score, when there is one, is
+        // in shared memory.
+        uint32_t bits = 0;  // TOPK: candidates of the current 32-column chunk
+        for (int cb = cbeg; cb < cend; cb += 32) {
+          uint32_t d0[32];
+          tmem_ld32_issue(dcol + cb, d0);
+          tmem_wait_ld(d0);
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {  // 16-column halves of the batch
+            const int c0 = cb + 16 * h;
+            float a[16];
+            if (u > 0) {
+              uint32_t ar[16];
+              acc_load(c0, ar, 16);
+#pragma unroll
+              for (int j = 0; j < 16; ++j) a[j] = __uint_as_float(ar[j]);
+            } else {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) a[j] = 0.f;
+            }
+#pragma unroll
+            for (int j = 0; j < 16; ++j) a[j] = __fadd_rn(a[j], term(c0 + j, d0[16 * h + j]));
+            if (!last) {
+#pragma unroll
+              for (int j = 0; j < 16; j += 4)
+                *reinterpret_cast<float4*>(accrow + c0 + j) = make_float4(a[j], a[j + 1], a[j + 2], a[j + 3]);
+            } else if (!TOPK) {
+              if (row < g.N) {
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                  if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
+              }
+            } else {
+              screen16(c0, q0, row, a, bits);
+              if (h == 1) {  // the 32-column chunk is complete (BNq is a multiple of 32)
+                const uint32_t wbits = __reduce_or_sync(0xffffffffu, bits);
+                if (lane == 0) cmask[(c0 >> 5) * 4 + q4] = wbits;  // a chunk's rows: the four lane quarters
+                bits = 0;
+              }
+            }
+          }
+        }
+      } else if (!last) {
+        // Running score in TMEM (several modules, 128-query tiles of the bf16
+        // kernel), 16 columns at a time: the TMEM loads of the next chunk are in
+        // flight while this one is combined and stored back.
         uint32_t dr[16], ar[16];
-        if (cbeg < cend) tmem_ld16_issue(dcol + cbeg, dr);
-        if (!kAccS && u > 0 && cbeg < cend) {
-          tmem_ld16_issue(acol + cbeg, ar);
-        } else {
+        if (cbeg < cend) {
+          tmem_ld16_issue(dcol + cbeg, dr);
+          if (u > 0) tmem_ld16_issue(acol + cbeg, ar);
+        }
+        if (u == 0) {
 #pragma unroll
           for (int j = 0; j < 16; ++j) ar[j] = 0u;
         }
@@ -297,38 +349,29 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
           const int c0 = cbeg + 16 * ci;
           if (c0 < cend) {
             tmem_wait_ld(dr);
-            if constexpr (kAccS) {
-              if (u > 0) acc_load(c0, ar, 16);
-            } else {
-              tmem_wait_ld(ar);
-            }
+            if (u > 0) tmem_wait_ld(ar);
             uint32_t o[16];
 #pragma unroll
             for (int j = 0; j < 16; ++j)
               o[j] = __float_as_uint(__fadd_rn(__uint_as_float(ar[j]), term(c0 + j, dr[j])));
             if (c0 + 16 < cend) {
               tmem_ld16_issue(dcol + c0 + 16, dr);
-              if (!kAccS && u > 0) tmem_ld16_issue(acol + c0 + 16, ar);
+              if (u > 0) tmem_ld16_issue(acol + c0 + 16, ar);
             }
-            if constexpr (kAccS) {
-#pragma unroll
-              for (int j = 0; j < 16; j += 4)
-                *reinterpret_cast<float4*>(accrow + c0 + j) =
-                    make_float4(__uint_as_float(o[j]), __uint_as_float(o[j + 1]), __uint_as_float(o[j + 2]),
-                                __uint_as_float(o[j + 3]));
-            } else {
-              tmem_st16_issue(acol + c0, o);
-            }
+            tmem_st16_issue(acol + c0, o);
           }
         }
-        if constexpr (!kAccS) tmem_wait_st();  // stored before the next module reads them
+        tmem_wait_st();  // stored before the next module reads them
       } else {
-        // Last module: 16 columns at a time, the next chunk's TMEM loads in
-        // flight while this one is finished and written out (or screened).
+        // Last module, running score in TMEM: 16 columns at a time.
         uint32_t dr[16], ar[16];
         if (cbeg < cend) {
           tmem_ld16_issue(dcol + cbeg, dr);
-          if (!kAccS && u > 0) tmem_ld16_issue(acol + cbeg, ar);
+          if (u > 0) tmem_ld16_issue(acol + cbeg, ar);
+        }
+        if (u == 0) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) ar[j] = 0u;
         }
         uint32_t bits = 0;  // TOPK: candidates of the current 32-column chunk
 #pragma unroll
@@ -336,20 +379,13 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
           const int c0 = cbeg + 16 * ci;
           if (c0 < cend) {
             tmem_wait_ld(dr);
-            if (u > 0 && kAccS) {
-              acc_load(c0, ar, 16);
-            } else if (u > 0) {
-              tmem_wait_ld(ar);
-            } else {
-#pragma unroll
-              for (int j = 0; j < 16; ++j) ar[j] = 0u;
-            }
+            if (u > 0) tmem_wait_ld(ar);
             float a[16];
 #pragma unroll
             for (int j = 0; j < 16; ++j) a[j] = __fadd_rn(__uint_as_float(ar[j]), term(c0 + j, dr[j]));
             if (c0 + 16 < cend) {
               tmem_ld16_issue(dcol + c0 + 16, dr);
-              if (!kAccS && u > 0) tmem_ld16_issue(acol + c0 + 16, ar);
+              if (u > 0) tmem_ld16_issue(acol + c0 + 16, ar);
             }
             if (!TOPK) {
               if (row < g.N) {
@@ -359,9 +395,9 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
               }
             } else {
               screen16(c0, q0, row, a, bits);
-              if ((c0 & 31) == 16) {  // the 32-column chunk is complete (BNq is a multiple of 32)
+              if ((c0 & 31) == 16) {
                 const uint32_t wbits = __reduce_or_sync(0xffffffffu, bits);
-                if (lane == 0) cmask[(c0 >> 5) * 4 + q4] = wbits;  // a chunk's rows: the four lane quarters
+                if (lane == 0) cmask[(c0 >> 5) * 4 + q4] = wbits;
                 bits = 0;
               }
             }
