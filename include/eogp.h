@@ -125,6 +125,19 @@ int eogp_get_option(int option, int* value);
  * Errors: EOGP_ECUDA, EOGP_ETIMEOUT. */
 int eogp_measure_peaks(double* e4m3_tflops, double* e2m1_tflops, double* popc_words_per_s);
 
+/* Self-test of the bounded waits (no counterpart in the paper: a library
+ * convenience). Every wait in the library's kernels gives up after a limit
+ * (~2 s), sets the timeout bit of the device status word and lets its kernel
+ * finish instead of hanging. This call launches one thread on the current
+ * device that waits, through the same routine, on an mbarrier nothing will
+ * arrive on, with a limit of `limit_cycles` SM clock cycles (1 .. 1e9), then
+ * returns what eogp_sync_status(NULL) reports: EOGP_ETIMEOUT when the path
+ * works (that read clears the status word; the context stays usable). No fault,
+ * trap or hang is involved.
+ * Errors: EOGP_EINVAL (limit out of range, checked before any device call),
+ * EOGP_ECUDA. */
+int eogp_selftest_wait_timeout(long long limit_cycles);
+
 /* ========================================================================
  * Retained-set plan (host; once per module)
  *

@@ -1045,6 +1045,16 @@ extern "C" int eogp_measure_peaks(double* e4m3_tflops, double* e2m1_tflops, doub
   return EOGP_OK;
 }
 
+extern "C" int eogp_selftest_wait_timeout(long long limit_cycles) {
+  clear_error();
+  if (limit_cycles < 1 || limit_cycles > 1000000000LL)
+    return set_error(EOGP_EINVAL, "limit_cycles must be in [1, 1e9]");
+  unsigned* status = status_word();
+  if (!status) return set_error(EOGP_ECUDA, "device status word unavailable");
+  CUDA_TRY(run_wait_selftest(status, limit_cycles, nullptr));
+  return eogp_sync_status(nullptr);
+}
+
 // ================================================================ SRHT
 
 extern "C" int eogp_srht(const float* z, int B, int m, int ldz, const int8_t* signs, const int32_t* rows,

@@ -54,12 +54,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Bounded wait for the phase with the given parity to complete.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned* status) {
+// Bounded wait for the phase with the given parity to complete: after `limit`
+// SM cycles (default ~2 s) it sets the timeout bit of the status word and
+// returns false.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned* status,
+                                          long long limit = EOGP_WAIT_CYCLES) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > EOGP_WAIT_CYCLES) {
+    if (clock64() - t0 > limit) {
       flag_status(status, EOGP_ST_TIMEOUT);
       return false;
     }

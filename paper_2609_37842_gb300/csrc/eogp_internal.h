@@ -146,6 +146,7 @@ cudaError_t launch_payload_unpack(const uint8_t* in, size_t ld_in, int N, const 
                                   int ld_codes, float* scales, int ld_scales, cudaStream_t st);
 
 // k_peaks.cu: e4m3 tensor-core and XOR + popcount throughput probes.
+cudaError_t run_wait_selftest(unsigned* status, long long limit, cudaStream_t st);
 cudaError_t run_peak_probes(int num_sms, unsigned* status, unsigned* sink, double* f8_tflops, double* f4_tflops,
                             double* popc_words_per_s, cudaStream_t st);
 

@@ -155,7 +155,26 @@ __global__ void __launch_bounds__(256) k_peak_popc(int iters, unsigned* sink) {
   if (t == 0xFFFFFFFFu) atomicAdd(sink, t);
 }
 
+// Self-test of the bounded waits: one thread waits, through the same
+// mbar_wait every kernel uses, on an mbarrier that nothing arrives on, so the
+// wait runs out after `limit` cycles and sets the timeout bit.
+__global__ void k_wait_selftest(unsigned* status, long long limit) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) mbar_wait(&bar, 0, status, limit);
+  __syncthreads();
+}
+
 }  // namespace
+
+cudaError_t run_wait_selftest(unsigned* status, long long limit, cudaStream_t st) {
+  k_wait_selftest<<<1, 32, 0, st>>>(status, limit);
+  return cudaGetLastError();
+}
 
 cudaError_t run_peak_probes(int num_sms, unsigned* status, unsigned* sink, double* f8_tflops,
                             double* f4_tflops, double* popc_words_per_s, cudaStream_t st) {

@@ -59,6 +59,7 @@ EXPORTS = {
     "eogp_version": (ctypes.c_char_p, []),
     "eogp_sync_status": (c_int, [c_void_p]),
     "eogp_measure_peaks": (c_int, [POINTER(c_double), POINTER(c_double), POINTER(c_double)]),
+    "eogp_selftest_wait_timeout": (c_int, [ctypes.c_longlong]),
     "eogp_profile_enable": (c_int, [c_int]),
     "eogp_set_option": (c_int, [c_int, c_int]),
     "eogp_get_option": (c_int, [c_int, POINTER(c_int)]),
@@ -658,6 +659,12 @@ def measure_peaks() -> Tuple[float, float, float]:
     pc = c_double()
     _check(lib().eogp_measure_peaks(ctypes.byref(f8), ctypes.byref(f4), ctypes.byref(pc)))
     return f8.value, f4.value, pc.value
+
+
+def selftest_wait_timeout(limit_cycles: int = 2_000_000) -> int:
+    """eogp_selftest_wait_timeout: status code of a wait made to run out (ETIMEOUT
+    when the bounded-wait path works)."""
+    return lib().eogp_selftest_wait_timeout(int(limit_cycles))
 
 
 def second_moment(Z, C=None, accumulate: bool = False, stream=None):

@@ -185,6 +185,14 @@ def test_host_input_call_argument_checks():
     assert L.eogp_compress_layer_host(*args) == E.EWORKSPACE
 
 
+def test_selftest_wait_argument_checks():
+    """eogp_selftest_wait_timeout refuses limits outside [1, 1e9] before any device call."""
+    L = E.lib()
+    assert L.eogp_selftest_wait_timeout(0) == E.EINVAL
+    assert L.eogp_selftest_wait_timeout(-5) == E.EINVAL
+    assert L.eogp_selftest_wait_timeout(10 ** 10) == E.EINVAL
+
+
 def test_host_alloc_argument_checks():
     """eogp_host_alloc / eogp_host_free: argument checks, and clean failure (or
     success, with a GPU present) of the registration."""

@@ -258,6 +258,20 @@ def test_host_alloc_size_classes():
         assert L.eogp_host_free(ctypes.c_void_p(p)) == E.OK
 
 
+def test_bounded_wait_times_out_and_context_survives():
+    """A kernel wait made to run out (an mbarrier nothing arrives on, a limit of
+    2e6 cycles) reports EOGP_ETIMEOUT through eogp_sync_status, the report clears
+    the status word, and the next library call on the same context succeeds."""
+    assert E.selftest_wait_timeout(2_000_000) == E.ETIMEOUT
+    assert E.lib().eogp_sync_status(None) == E.OK
+    x = torch.randn(64, 256, device=DEV)
+    codes, scales = torch.empty(64, 8, dtype=torch.int32, device=DEV), torch.empty(64, device=DEV)
+    E.pack_sign(x, codes, scales)
+    E.sync_status()
+    bits, sc = O.onebit(x.cpu().double().numpy())
+    assert np.array_equal(O.unpack_bits(codes.cpu().numpy().view(np.uint32), 256), bits)
+
+
 def test_measure_peaks_rates():
     """eogp_measure_peaks: the e4m3 and e2m1 one-bit MMA rates and the popcount
     rate are finite and positive, the e2m1 MMA (K = 64 per instruction) outruns
