@@ -457,13 +457,12 @@ class Stack:
         torch.cuda.empty_cache()
 
 
-def h2d_link_rate(dev, nbytes=1 << 30, reps=3):
-    """Plain host-to-device copy rate of one page-locked buffer (eogp_host_alloc) with
-    one cudaMemcpyAsync per repetition, GB/s."""
+def h2d_link_rate(h, dev, reps=3):
+    """Plain host-to-device copy rate of the page-locked host tensor `h` (one of the
+    e2e run's own input buffers) with one cudaMemcpyAsync per repetition, GB/s."""
     import torch
-    from paper_2609_37842_gb300 import eogp as E
-    h = E.host_empty((nbytes,), torch.uint8)
-    d = torch.empty((nbytes,), dtype=torch.uint8, device=dev)
+    nbytes = h.numel() * h.element_size()
+    d = torch.empty(h.shape, dtype=h.dtype, device=dev)
     d.copy_(h, non_blocking=True)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -473,7 +472,7 @@ def h2d_link_rate(dev, nbytes=1 << 30, reps=3):
     e1.record()
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1)
-    del h, d
+    del d
     return nbytes * reps / (ms / 1000.0) / 1e9
 
 
@@ -536,12 +535,14 @@ def e2e_run(st, Be, steps, chunk, dev, world, barrier):
         tt = torch.tensor([ems], device=dev)
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         ems = float(tt.item())
-    link = h2d_link_rate(dev)
+    big = max((t for pair in host.values() for t in pair), key=lambda t: t.numel() * t.element_size())
+    link = h2d_link_rate(big, dev)
     rate = h2d * steps / (ems / 1000.0) / 1e9
     out = {"value": world * Be * steps / (ems / 1000.0), "unit": "examples/s", "batch": Be,
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
            "h2d_GBps": rate, "link_GBps": link, "frac_of_link": rate / link if link else None,
-           "link": "one cudaMemcpyAsync of a 1 GiB page-locked buffer, same run",
+           "link": "one cudaMemcpyAsync of the run's largest input buffer (the same page-locked memory), "
+                   "3 copies",
            "api": "eogp_compress_layer_host (host inputs, chunked copies inside the call)",
            "chunk": chunk or "library default (about 64 MB of inputs)"}
     if st.stream_bases:
