@@ -26,16 +26,24 @@
 //    (NG groups, all TMEM leaves): the query stages of group gj are loaded once
 //    group gj - NQ is done, its A slots refilled once group gj - NG is done,
 //    both read from the one commit per group, so the queries' L2 latency is off
-//    the A slots' round trip. This lagged reuse relies on groups completing in
-//    order, hence one issuing thread: with a second one (each owning one of two
-//    accumulators) completions came out of order, a parity wait could pass a
-//    phase early, and the full 4.2M-code scan faulted the GPU (Xid 13). A single thread issues all
-//    MMAs at about one per 64 cycles, plus ~330 cycles per wait-fence-commit
-//    round: at 256 bits per round the rounds, not the tensor pipe, set the pace
-//    (measured: 589 cycles per four N = 256 MMAs, 8.4 of 9.7 PFLOP/s), at
-//    512 bits the tensor pipe does (1024 cycles per eight, 9.7 PFLOP/s). An
-//    N = 64 MMA takes as long to issue as an N = 128 one, so 64-query tiles
-//    (one module of a multiple of 1024 bits) take four stages per group.
+//    the A slots' round trip.
+//  * issuing threads: a thread issues an MMA about every 64 cycles whatever N
+//    is, plus ~330 cycles per wait-fence-commit round: at 256 bits per round
+//    the rounds, not the tensor pipe, set the pace (measured: 589 cycles per
+//    four N = 256 MMAs, 8.4 of 9.7 PFLOP/s), at 512 bits the tensor pipe does
+//    (1024 cycles per eight, 9.7 PFLOP/s). An N = 64 MMA takes as long to issue
+//    as an N = 128 one, so 64-query tiles take four stages per group (and one
+//    module of 64 queries has its own two-issuer kernel, k_score_pair_ks.cu).
+//    128-query tiles of several modules have two accumulators and two issuers,
+//    issuer b running the modules of accumulator b, so one thread's rounds
+//    overlap the other's MMAs. Groups then complete out of order, which the
+//    lagged reuse allows as long as no thread waits on a barrier phase before
+//    it has seen the previous phase of that barrier complete (a parity wait
+//    cannot tell a phase from the one two ahead): the expanders and the query
+//    producer wait on every group's empty barrier in order, and both issuers
+//    wait on every group's full barrier in order, issuing only their own. (An
+//    earlier version whose issuers waited only on their own groups' barriers
+//    passed a phase early and faulted the GPU, Xid 13, on the 4.2M-code scan.)
 // Each expander warp takes the 32 rows of one TMEM lane quarter, a whole group
 // per round: two 16-byte shared-memory loads and the e2m1 expansion per stage,
 // the TMEM stores, and one relaxed arrive on the leader's barrier of the group. That arrive orders enough: it is issued after
@@ -50,9 +58,9 @@
 //
 // Warps: 0-3 expand, 4-11 dequantise (two per TMEM lane quarter, half of the
 // query columns each, which halves the drain of the accumulator the MMAs of a
-// 256-query tile wait for), 12 owns TMEM and, in the leader, issues the MMAs,
-// 13 loads the code boxes, 14 the query tiles. Fifteen warps leave 128
-// registers a thread (an SM sub-partition holds at most four of them).
+// 256-query tile wait for), 12 owns TMEM and, in the leader, issues the MMAs
+// (of accumulator 0 with two issuers), 13 loads the code boxes, 14 the query
+// tiles, 15 is the second issuer. Sixteen warps leave 128 registers a thread.
 #include <algorithm>
 #include <atomic>
 
@@ -68,7 +76,8 @@ constexpr int kPrDqWarps = 8;                    // dequantise warps: two per TM
 constexpr int kPrMmaWarp = kPrDq0 + kPrDqWarps;
 constexpr int kCodeWarp = kPrMmaWarp + 1;
 constexpr int kQueryWarp = kPrMmaWarp + 2;
-constexpr int kPairThreads = (kQueryWarp + 1) * 32;
+constexpr int kIss1Warp = kPrMmaWarp + 3;         // second MMA issuer (two accumulators of several modules)
+constexpr int kPairThreads = (kIss1Warp + 1) * 32;
 constexpr int kCodeBoxWords = 32;            // 1024 code bits of a row per box (4 stages)
 constexpr uint32_t kCodeBox = 128u * 128u;   // 128 rows x 128 bytes
 
@@ -83,22 +92,28 @@ template <int BN>
 constexpr int pr_slots() {
   return (512 - pr_dbufs<BN>() * BN - 32) / 32;
 }
-// The running score of several modules lives in shared memory; only 128-query
-// tiles serve several modules (64-query tiles have no room for it in TMEM
-// either, so they serve one module, and 256-query tiles keep one accumulator).
+// Only 128-query tiles serve several modules (a running score, kept in the
+// dequantise warps' registers); 64-query tiles serve one (their TMEM has no
+// room for a second accumulator pair), and 256-query tiles keep one
+// accumulator.
 template <int BN>
-constexpr bool pr_acc_smem() {
+constexpr bool pr_running() {
   return BN == 128;
 }
-// Code boxes in flight and query stages: as many as the shared memory holds
-// next to the running score of several modules.
+// Code boxes in flight and query stages: as many as the shared memory holds.
 template <int BN>
 constexpr int pr_code_ring() {
-  return BN == 64 ? 8 : BN == 256 ? 3 : 4;
+  return BN == 64 ? 8 : BN == 256 ? 3 : 6;
 }
 template <int BN>
 constexpr int pr_qstages() {
-  return BN == 64 ? 20 : 10;
+  return BN == 64 ? 20 : BN == 256 ? 10 : 12;
+}
+// MMA-issuing threads: two with two accumulators of several modules (each
+// issues the modules of one accumulator), else one.
+template <int BN>
+constexpr int pr_issuers() {
+  return pr_dbufs<BN>() == 2 && pr_running<BN>() ? 2 : 1;
 }
 template <int BN>
 constexpr uint32_t pr_acol0() {
@@ -118,7 +133,7 @@ __host__ __device__ inline TcSmem pr_smem_layout(uint32_t* code_off) {
   TcSmem l;
   *code_off = NQ * G * kStage;
   l.acc = *code_off + kCodeRing * kCodeBox;
-  l.sq = l.acc + (pr_acc_smem<BN>() ? 128u * kAccLd * 4u : 0u);
+  l.sq = l.acc;  // no running score in shared memory
   l.bars = l.sq + 2 * BN * 4;
   l.lists = l.bars + (2 * NQ + 2 * pr_dbufs<BN>() + 2 * kCodeRing) * 8 + 16;
   l.total = l.lists + (TOPK ? BN * 12 + 8 * 4 * 4 : 0);
@@ -244,12 +259,17 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       bx += nbx;
     }
   } else if (warp < kPrMmaWarp) {
-    dequant_role<EOGP_SCORE_CODES, TOPK, BN, ND, pr_acc_smem<BN>(), true, kPrDqWarps, kPrDq0>(g, smem, L, tmem, sq,
+    dequant_role<EOGP_SCORE_CODES, TOPK, BN, ND, pr_running<BN>(), true, kPrDqWarps, kPrDq0>(g, smem, L, tmem, sq,
                                                                                               dfull, dempty);
-  } else if (warp == kPrMmaWarp) {
-    if (lane == 0 && rank == 0) {
-      // ---------------------------------------------------------- MMA issuer (leader)
-      // Kept to waits, MMAs and commits: one thread issues every MMA of the pair.
+  } else if (warp == kPrMmaWarp || warp == kIss1Warp) {
+    constexpr int NI = pr_issuers<BN>();
+    const int me = warp == kPrMmaWarp ? 0 : 1;
+    if (lane == 0 && rank == 0 && me < NI) {
+      // ---------------------------------------------------------- MMA issuers (leader)
+      // Kept to waits, MMAs and commits. With two issuers, issuer b runs the
+      // modules of accumulator b; both wait on every group's full barrier in
+      // order (each phase of every barrier a thread waits on is seen by it), and
+      // only the owner of a group issues and commits it.
       const uint32_t idesc = idesc_mxf4_f32(256, g.BNq);
       const uint32_t sfa = tmem + kSfa, sfb = tmem + kSfb;
       const uint64_t dbase = sdesc_sw128(smem_u32(smem), 16, 1024);
@@ -263,11 +283,14 @@ __global__ void __launch_bounds__(kPairThreads, 1)
            tile < tend && ok; tile += tstep) {
         for (int u = 0; u < g.U && ok; ++u, ++gm) {
           const int buf = static_cast<int>(gm % ND);
-          if (!mbar_wait_cluster(&dempty[buf], ((gm / ND) & 1u) ^ 1u, g.status)) {
-            ok = false;
-            break;
+          const bool mine = NI == 1 || buf == me;
+          if (mine) {
+            if (!mbar_wait_cluster(&dempty[buf], ((gm / ND) & 1u) ^ 1u, g.status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
           }
-          tc_fence_after();
           const uint32_t d = tmem + buf * static_cast<uint32_t>(BN);
           const int ngr = g.k[u] / (256 * G);
           for (int gi = 0; gi < ngr; ++gi) {
@@ -295,6 +318,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
               ok = false;
               break;
             }
+            if (!mine) continue;
             tc_fence_after();
 #pragma unroll
             for (int st = 0; st < G; ++st)
@@ -304,7 +328,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
                                   sfb, (gi | st | kk) != 0 ? 1u : 0u);
             tc_commit_pair_mc(&empty[s], 0x3);
           }
-          tc_commit_pair_mc(&dfull[buf], 0x3);
+          if (mine && ok) tc_commit_pair_mc(&dfull[buf], 0x3);
         }
       }
     }
@@ -465,6 +489,8 @@ cudaError_t launch_pair(int BN, int G, bool topk, const CUtensorMap& tq, const S
   const uint32_t cbox[2] = {static_cast<uint32_t>(kCodeBoxWords), 128};
   if (make_tmap(&tc, CU_TENSOR_MAP_DATA_TYPE_UINT32, 2, g.train, cdims, cstr, cbox, CU_TENSOR_MAP_SWIZZLE_128B))
     return cudaErrorInvalidValue;
+  // 64 queries of one module in whole 1024-bit groups: two MMA-issuing threads
+  if (!topk && BN == 64 && G == 4 && g.Q <= g.BNq) return launch_pair_ks(tq, tc, g, grid, st);
   return topk ? launch_bn<true>(BN, G, tq, tc, g, grid, st) : launch_bn<false>(BN, G, tq, tc, g, grid, st);
 }
 

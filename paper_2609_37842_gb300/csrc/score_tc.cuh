@@ -107,7 +107,8 @@ __device__ __forceinline__ int tile_row0(int ib) {
 // lane quarter w % 4, TMEM lane = stored row of the CTA's tile; with eight
 // warps the two of a lane quarter take half of the query columns each). Per module u of a tile: wait
 // for the MMAs of d_u, fold acc = fl(acc + term(d_u)) into the running score
-// (TMEM columns after the ND accumulators, or shared memory when ACCS), release
+// (TMEM columns after the ND accumulators; with ACCS registers in a pair, else
+// shared memory), release
 // the accumulator; after the last module write the scores (dense) or screen and
 // rank them (TOPK). In a CTA pair (PAIR) each CTA drains its own 128 rows and
 // releases the accumulator on the leader CTA's barrier.
@@ -118,10 +119,16 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
   static_assert(DQ0 % 4 == 0, "warp w reads TMEM lane quarter w % 4");
   constexpr uint32_t kAcc = static_cast<uint32_t>(ND * BN);
   constexpr bool kAccS = ACCS;
-  // The running score of several modules: in shared memory (ACCS), else in the
-  // TMEM columns after the accumulators, which only the one-CTA kernel's
-  // 128-query tiles have (the pair kernel's other tile widths serve one module).
+  // The running score of several modules (ACCS): in registers in the pair
+  // kernel, whose eight warps hold 64 columns of one row a thread (measured on
+  // GPT-2 query scoring, the shared-memory running score cost more than the
+  // MMAs it waits for), else in shared memory (the one-CTA kernel's four warps
+  // would need 128 registers for it). Without ACCS, in the TMEM columns after
+  // the accumulators, which only the one-CTA kernel's 128-query tiles have (the
+  // pair kernel's other tile widths serve one module).
+  constexpr bool kAccR = ACCS && PAIR && NDW == 8;
   constexpr bool kAccT = !ACCS && BN == 128 && !PAIR;
+  static_assert(!kAccR || MODE == EOGP_SCORE_CODES, "the pair kernel scores one-bit queries");
   constexpr int kThr = NDW * 32;     // dequantise threads
   constexpr int CW = BN * 4 / NDW;   // query columns of a warp (all of them, or half)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -239,6 +246,9 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
       sq_next[e] = (MODE == EOGP_SCORE_CODES && c < g.BNq && q0 + c < g.Q)
                        ? g.qs[static_cast<size_t>(q0 + c) * g.ldqs] : 0.f;
     }
+    float accr[kAccR ? CW : 1];  // kAccR: this thread's running score, from +0
+#pragma unroll
+    for (int i = 0; i < (kAccR ? CW : 1); ++i) accr[i] = 0.f;
     for (int u = 0; u < g.U; ++u, ++gm) {
       const int buf = static_cast<int>(gm % ND);
       const uint32_t dph = (gm / ND) & 1u;
@@ -285,7 +295,54 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
         return MODE == EOGP_SCORE_CODES ? __fmul_rn(__fmul_rn(sqb[c], si), __uint_as_float(dv))
                                         : __fmul_rn(si, __uint_as_float(dv));
       };
-      if constexpr (!kAccT) {
+      if constexpr (kAccR) {
+        // Running score in registers (from +0: fl(0 + t) for the first
+        // module); d_u 16 columns at a time (one TMEM wait a batch), the query
+        // scales four at a time from shared memory.
+        constexpr int RB = 16;
+        uint32_t bits = 0;  // TOPK: candidates of the current 32-column chunk
+#pragma unroll
+        for (int b = 0; b < CW / RB; ++b) {
+          const int cb = cbeg + RB * b;
+          if (cb < cend) {
+            uint32_t d0[RB];
+            tmem_ld_issue(dcol + cb, d0);
+            tmem_wait_ld(d0);
+#pragma unroll
+            for (int h = 0; h < RB / 16; ++h) {  // 16-column parts of the batch
+              const int c0 = cb + 16 * h;
+              float a[16];
+#pragma unroll
+              for (int j4 = 0; j4 < 4; ++j4) {
+                const float4 s4 = *reinterpret_cast<const float4*>(sqb + c0 + 4 * j4);
+                const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  const int j = 4 * j4 + e, ai = RB * b + 16 * h + j;
+                  a[j] = accr[ai] =
+                      __fadd_rn(accr[ai], __fmul_rn(__fmul_rn(sv[e], si), __uint_as_float(d0[16 * h + j])));
+                }
+              }
+              if (last) {
+                if (!TOPK) {
+                  if (row < g.N) {
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                      if (q0 + c0 + j < g.Q) g.out[static_cast<size_t>(q0 + c0 + j) * g.ldo + row] = a[j];
+                  }
+                } else {
+                  screen16(c0, q0, row, a, bits);
+                  if ((c0 & 31) == 16) {  // the 32-column chunk is complete (BNq is a multiple of 32)
+                    const uint32_t wbits = __reduce_or_sync(0xffffffffu, bits);
+                    if (lane == 0) cmask[(c0 >> 5) * 4 + q4] = wbits;
+                    bits = 0;
+                  }
+                }
+              }
+            }
+          }
+        }
+      } else if constexpr (!kAccT) {
         // d_u in batches of 32 columns: the batch's TMEM loads are issued
         // before its one wait (tcgen05.wait::ld waits for all of the thread's
         // loads, so a load issued one 16-column chunk ahead is still waited for
@@ -429,6 +486,12 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsign
 size_t pair_smem_need(int BN, int G, bool topk);
 // Clusters of two that can be resident at once on the current device.
 int pair_cluster_cap(int num_sms);
+// The two-issuer pair kernel (k_score_pair_ks.cu): one module, at most 64
+// queries (one query tile), modules of a multiple of 1024 bits; tq and tc as
+// for launch_pair (tc: the stored codes' map, boxes of 32 words x 128 rows).
+size_t pair_ks_smem_need();
+cudaError_t launch_pair_ks(const CUtensorMap& tq, const CUtensorMap& tc, const ScoreTcArgs& g, int grid,
+                           cudaStream_t st);
 // tq: the expanded queries' tensor map (boxes of 128 bytes x BNq / 2 rows); the
 // stored codes' map is made here from g.train, g.ldt, g.D and g.N.
 cudaError_t launch_pair(int BN, int G, bool topk, const CUtensorMap& tq, const ScoreTcArgs& g, int grid,

@@ -109,6 +109,7 @@ def rand_store(rng, n, ks):
                                     (129, 200, [1024, 128, 2048]), (777, 257, [512] * 5),
                                     (1000, 300, [256, 768, 1024]), (500, 300, [2048]),
                                     (2000, 64, [256, 1280]), (5000, 200, [768]), (40000, 64, [1024]),
+                                    (70000, 64, [4096]), (3000, 64, [768]),
                                     (3000, 1000, [256, 256, 512])])
 @pytest.mark.parametrize("f4", ["1", "0"])
 def test_score_codes_bit_exact(N, Q, ks, f4, eogp_options):
