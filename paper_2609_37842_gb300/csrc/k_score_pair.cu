@@ -103,11 +103,13 @@ constexpr bool pr_running() {
 // Code boxes in flight and query stages: as many as the shared memory holds.
 template <int BN>
 constexpr int pr_code_ring() {
-  return BN == 64 ? 8 : BN == 256 ? 3 : 6;
+  return BN == 64 ? 8 : BN == 256 ? 3 : 4;
 }
+// (16 with 128-query tiles: a multiple of 2 G x the groups of a module, so
+// each query-stage slot serves one issuer only, for modules of up to 2048 bits.)
 template <int BN>
 constexpr int pr_qstages() {
-  return BN == 64 ? 20 : BN == 256 ? 10 : 12;
+  return BN == 64 ? 20 : BN == 256 ? 10 : 16;
 }
 // MMA-issuing threads: two with two accumulators of several modules (each
 // issues the modules of one accumulator), else one.
@@ -267,9 +269,12 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     if (lane == 0 && rank == 0 && me < NI) {
       // ---------------------------------------------------------- MMA issuers (leader)
       // Kept to waits, MMAs and commits. With two issuers, issuer b runs the
-      // modules of accumulator b; both wait on every group's full barrier in
-      // order (each phase of every barrier a thread waits on is seen by it), and
-      // only the owner of a group issues and commits it.
+      // modules of accumulator b and only the owner of a group issues and
+      // commits it. Every thread must see each phase of a barrier it waits on:
+      // when all modules have the same number of groups ng and NQ is a multiple
+      // of 2 ng, the groups of a full barrier all belong to one issuer, which
+      // waits only on its own; otherwise both wait on every group's full
+      // barrier in order.
       const uint32_t idesc = idesc_mxf4_f32(256, g.BNq);
       const uint32_t sfa = tmem + kSfa, sfb = tmem + kSfb;
       const uint64_t dbase = sdesc_sw128(smem_u32(smem), 16, 1024);
@@ -279,11 +284,33 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       int rq = 0, ra = 0;
       uint32_t rph = 0, gm = 0;
       bool ok = true;
+      const int ngu = g.kuni / (256 * G);  // groups of every module (0: modules differ)
+      const bool excl = NI == 2 && ngu > 0 && NQ % (2 * ngu) == 0;
+      // one group on: query slot rq (phase rph, descriptor dq), A slot ra (columns acl)
+      auto advance = [&]() {
+        if (++rq == NQ) {
+          rq = 0;
+          rph ^= 1u;
+          dq = dbase;
+        } else {
+          dq += kGroupDesc;
+        }
+        if (++ra == NG) {
+          ra = 0;
+          acl = tmem + pr_acol0<BN>();
+        } else {
+          acl += 32u * G;
+        }
+      };
       for (int tile = tile_begin<TOPK, true>(g), tstep = tile_step<TOPK, true>(), tend = tile_end<TOPK, true>(g);
            tile < tend && ok; tile += tstep) {
         for (int u = 0; u < g.U && ok; ++u, ++gm) {
           const int buf = static_cast<int>(gm % ND);
           const bool mine = NI == 1 || buf == me;
+          if (!mine && excl) {  // the other issuer's module: its slots, not its barriers
+            for (int gi = 0; gi < ngu; ++gi) advance();
+            continue;
+          }
           if (mine) {
             if (!mbar_wait_cluster(&dempty[buf], ((gm / ND) & 1u) ^ 1u, g.status)) {
               ok = false;
@@ -298,19 +325,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
             const uint32_t ph = rph;
             const uint64_t b0 = dq;
             const uint32_t at0 = acl;
-            if (++rq == NQ) {
-              rq = 0;
-              rph ^= 1u;
-              dq = dbase;
-            } else {
-              dq += kGroupDesc;
-            }
-            if (++ra == NG) {
-              ra = 0;
-              acl = tmem + pr_acol0<BN>();
-            } else {
-              acl += 32u * G;
-            }
+            advance();
             // both CTAs' query bytes and expander warps (the MMAs read the
             // queries through the async proxy, tracked by the barrier's
             // transaction count)

@@ -660,6 +660,9 @@ cudaError_t launch_score_tc(int mode, const uint32_t* train, int ldt, const floa
     D += ks[u];
   }
   g.D = D;
+  g.kuni = ks[0];
+  for (int u = 1; u < U; ++u)
+    if (ks[u] != ks[0]) g.kuni = 0;
   const int grid = tc_grid(c, N, Q, num_sms);
   CUtensorMap t0, t1;
   if (mode == EOGP_SCORE_CODES) {

@@ -29,6 +29,7 @@ constexpr int kAccLd = 132;           // row stride (floats) of a running score 
 
 struct ScoreTcArgs {
   int N, Q, U, D, BNq, n_it, n_tiles, ldt, ldts, ldqs, ldo, K;
+  int kuni;  // bits of every module when all modules are equal, else 0
   const uint32_t* train;
   const float* ts;
   const float* qs;
@@ -233,51 +234,52 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
       for (int col = ep; col < BN; col += kThr)
         gtb[col] = q0 + col < g.Q ? topk_unkey32(__ldcg(g.gtau + q0 + col)) : INFINITY;
     }
-    // Scales of module u + 1 are loaded while module u is dequantised. The
-    // query scales go through shared memory (buffer gm & 1): buffer gm & 1 was
-    // last read in module gm - 2, which every thread finished before the
-    // barrier of module gm - 1.
+    // Scales: the query scales of module u go through shared memory (buffer
+    // gm & 1), written after the drain of module u - 1 (at the tile's start for
+    // the first module) and published by the barrier that ends it, so that
+    // barrier is off the path from the MMAs' commit to the accumulator's
+    // release. Buffer gm & 1 was last read in module gm - 2, which every thread
+    // finished before the barrier that ended it. The scales of module u + 1
+    // are loaded from global memory while module u is drained.
     constexpr int kSqPer = (BN + kThr - 1) / kThr;  // query columns of a tile per dequantise thread
-    float si_next = row < g.N ? g.ts[static_cast<size_t>(row) * g.ldts] : 0.f;
-    float sq_next[kSqPer];
+    auto load_scales = [&](int u, float& si_u, float (&sq_u)[kSqPer]) {
+      si_u = row < g.N ? g.ts[static_cast<size_t>(row) * g.ldts + u] : 0.f;
 #pragma unroll
-    for (int e = 0; e < kSqPer; ++e) {
-      const int c = ep + kThr * e;
-      sq_next[e] = (MODE == EOGP_SCORE_CODES && c < g.BNq && q0 + c < g.Q)
-                       ? g.qs[static_cast<size_t>(q0 + c) * g.ldqs] : 0.f;
-    }
+      for (int e = 0; e < kSqPer; ++e) {
+        const int c = ep + kThr * e;
+        sq_u[e] = (MODE == EOGP_SCORE_CODES && c < g.BNq && q0 + c < g.Q)
+                      ? g.qs[static_cast<size_t>(q0 + c) * g.ldqs + u] : 0.f;
+      }
+    };
+    auto store_sq = [&](uint32_t gmod, const float (&sq_u)[kSqPer]) {
+      if (MODE == EOGP_SCORE_CODES) {
+        float* b = sq + (gmod & 1u) * BN;
+#pragma unroll
+        for (int e = 0; e < kSqPer; ++e)
+          if (ep + kThr * e < BN) b[ep + kThr * e] = sq_u[e];
+      }
+    };
+    float si_next, sq_next[kSqPer];
+    load_scales(0, si_next, sq_next);
+    store_sq(gm, sq_next);
+    float si_cur = si_next;
+    if (g.U > 1) load_scales(1, si_next, sq_next);
+    named_bar_sync(2, kThr);  // module 0's query scales (and TOPK thresholds) visible
     float accr[kAccR ? CW : 1];  // kAccR: this thread's running score, from +0
 #pragma unroll
     for (int i = 0; i < (kAccR ? CW : 1); ++i) accr[i] = 0.f;
     for (int u = 0; u < g.U; ++u, ++gm) {
       const int buf = static_cast<int>(gm % ND);
       const uint32_t dph = (gm / ND) & 1u;
-      const float si = si_next;
-      float* sqb = sq + (gm & 1u) * BN;
-      if (MODE == EOGP_SCORE_CODES) {
-#pragma unroll
-        for (int e = 0; e < kSqPer; ++e)
-          if (ep + kThr * e < BN) sqb[ep + kThr * e] = sq_next[e];
-      }
-      if (u + 1 < g.U) {
-        si_next = row < g.N ? g.ts[static_cast<size_t>(row) * g.ldts + u + 1] : 0.f;
-#pragma unroll
-        for (int e = 0; e < kSqPer; ++e) {
-          const int c = ep + kThr * e;
-          sq_next[e] = (MODE == EOGP_SCORE_CODES && c < g.BNq && q0 + c < g.Q)
-                           ? g.qs[static_cast<size_t>(q0 + c) * g.ldqs + u + 1] : 0.f;
-        }
-      }
+      const float si = si_cur;
+      const float* sqb = sq + (gm & 1u) * BN;
       uint32_t w_ok = 1;
       if (lane == 0) w_ok = mbar_wait(&dfull[buf], dph, g.status) ? 1u : 0u;
       w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
       __syncwarp();
       tc_fence_after();
-      if (!named_bar_and(2, kThr, w_ok)) {  // also publishes sqb
-        ok = false;
-        break;
-      }
       const bool last = u + 1 == g.U;
+      if (w_ok) {
       const uint32_t dcol = tmem + lane_base + buf * static_cast<uint32_t>(BN);
       const uint32_t acol = tmem + lane_base + kAcc;
       float* accrow = reinterpret_cast<float*>(smem + L.acc) + rr * kAccLd;  // kAccS: this row's running score
@@ -468,6 +470,16 @@ __device__ __forceinline__ void dequant_role(const ScoreTcArgs& g, uint8_t* smem
           mbar_arrive_relaxed_cluster(mapa_shared(smem_u32(&dempty[buf]), 0));
         else
           mbar_arrive(&dempty[buf]);
+      }
+      }  // w_ok
+      if (!last) {  // the next module's query scales into the other buffer
+        store_sq(gm + 1, sq_next);
+        si_cur = si_next;
+        if (u + 2 < g.U) load_scales(u + 2, si_next, sq_next);
+      }
+      if (!named_bar_and(2, kThr, w_ok)) {  // every warp's ok; publishes the next scales
+        ok = false;
+        break;
       }
       if (TOPK && last) rank_tile(q0, i0);
     }
