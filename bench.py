@@ -862,7 +862,8 @@ def bench_scan(dev, stream, probes, bf16_burst, peaks_src, hbm, rows=0, qs_arg="
         if Q >= 64:   # tensor-core kernel: +-1 multiply-adds against the rate of the MMA it issues
             tfl = 2.0 * N * ksc * Q / (qms / 1000.0) / 1e12
             pk, pk_src, pk_mode = score_peak([ksc], probes, bf16_burst, peaks_src)
-            ent.update({"kernel": f"k_score_tc ({pk_mode})", "tensor_TFLOPs": tfl,
+            kern = ("k_score_pair_ks" if Q <= 64 else "k_score_pair") if "mxf4" in pk_mode else "k_score_tc"
+            ent.update({"kernel": f"{kern} ({pk_mode})", "tensor_TFLOPs": tfl,
                         "tensor_frac": tfl / pk, "tensor_peak_source": pk_src})
         else:
             wops = N * Q * Wsc / (qms / 1000.0)
