@@ -300,7 +300,13 @@ class Stack:
         self.stream_bases = stream_bases and self.layers > 1
         if self.stream_bases:
             pl = self.per_layer
-            self.host_one = {k: (L["VA"].cpu().pin_memory(), L["VS"].cpu().pin_memory()) for k, L in pl.items()}
+            # page-locked through the library's allocator (huge-page backed): the
+            # same memory class the e2e inputs use, which copies at the link rate
+            def pinned(t):
+                h = E.host_empty(tuple(t.shape), t.dtype)
+                h.copy_(t)
+                return h
+            self.host_one = {k: (pinned(L["VA"]), pinned(L["VS"])) for k, L in pl.items()}
             self.dev_bases = [{k: (torch.empty_like(L["VA"]), torch.empty_like(L["VS"])) for k, L in pl.items()}
                               for _ in range(2)]
             self.slot_descs = [{k: E.layer_desc(pl[k]["plan"], w.T, w.k, self.dev_bases[sl][k][0],
