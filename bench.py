@@ -483,12 +483,14 @@ def h2d_link_rate(h, dev, reps=3):
 
 
 def e2e_run(st, Be, steps, chunk, dev, world, barrier):
-    """The step through the public host-input call (eogp_compress_layer_host): per
-    module, a and s in page-locked host memory (one buffer per module type) and,
-    for streamed-eigenbasis stacks, the retained eigenvector rows too (descriptor
-    bases_on_host); every call copies its inputs chunk by chunk into its workspace
-    while the previous chunk is compressed; the step ends with the device-to-host
-    read of the stack's codes and scales."""
+    """The step through the public host-input call for several modules
+    (eogp_compress_layers_host), all modules of the stack in one call: per module,
+    a and s in page-locked host memory (one buffer per module type) and, for
+    streamed-eigenbasis stacks, the retained eigenvector rows too (descriptor
+    bases_on_host); the call copies each module's inputs chunk by chunk into
+    staging sets that alternate between modules, so one module's copies overlap
+    the previous module's compute; the step ends with the device-to-host read of
+    the stack's codes and scales."""
     import torch
     E = st.E
     w = st.w
@@ -509,9 +511,14 @@ def e2e_run(st, Be, steps, chunk, dev, world, barrier):
             hdesc[key] = st.descs[key]
     if st.stream_bases:
         bases_bytes = sum(2 * (st.per_layer[k]["VA"].numel() + st.per_layer[k]["VS"].numel()) for k in st.keys)
-    hws = E.workspace(max(E.compress_host_workspace_size(d, Be, E.OUT_CODES, chunk) for d in hdesc.values()), dev)
     wd = st.words
     ecodes, escales = st.codes[:Be], st.scales[:Be]
+    sdescs = [hdesc[key] for key in st.keys]
+    sa = [host[key][0] for key in st.keys]
+    ss = [host[key][1] for key in st.keys]
+    scodes = [ecodes[:, u * wd:(u + 1) * wd] for u in range(len(st.keys))]
+    sscales = [escales[:, u] for u in range(len(st.keys))]
+    hws = E.workspace(E.compress_layers_host_workspace_size(sdescs, Be, E.OUT_CODES, chunk), dev)
     hcodes = torch.empty(ecodes.shape, dtype=ecodes.dtype, pin_memory=True)
     hscales = torch.empty(escales.shape, dtype=escales.dtype, pin_memory=True)
     h2d = sum(host[k][0].numel() * host[k][0].element_size() + host[k][1].numel() * host[k][1].element_size()
@@ -519,11 +526,8 @@ def e2e_run(st, Be, steps, chunk, dev, world, barrier):
     d2h = hcodes.numel() * 4 + hscales.numel() * 4
 
     def e2e_step():
-        for u, key in enumerate(st.keys):
-            ha, hs = host[key]
-            E.compress_layer_host(hdesc[key], ha, hs, E.OUT_CODES, dev, chunk=chunk,
-                                  codes=ecodes[:, u * wd:(u + 1) * wd], scales=escales[:, u], ws=hws,
-                                  stream=st.stream)
+        E.compress_layers_host(sdescs, sa, ss, E.OUT_CODES, dev, chunk=chunk, codes=scodes, scales=sscales,
+                               ws=hws, stream=st.stream)
         hcodes.copy_(ecodes, non_blocking=True)
         hscales.copy_(escales, non_blocking=True)
 
@@ -549,7 +553,8 @@ def e2e_run(st, Be, steps, chunk, dev, world, barrier):
            "h2d_GBps": rate, "link_GBps": link, "frac_of_link": rate / link if link else None,
            "link": "one cudaMemcpyAsync of the run's largest input buffer (the same page-locked memory), "
                    "3 copies",
-           "api": "eogp_compress_layer_host (host inputs, chunked copies inside the call)",
+           "api": "eogp_compress_layers_host (the stack's modules in one call: host inputs, chunked copies "
+                  "inside the call, one module's copies overlapping the previous module's compute)",
            "chunk": chunk or "library default (about 64 MB of inputs)"}
     if st.stream_bases:
         out["eigenbases"] = "page-locked host memory, copied by each call (bases_on_host)"

@@ -307,6 +307,37 @@ int eogp_compress_layer_host(const eogp_layer_desc* L, const void* a, const void
                              float* scales, int ld_scales, void* ws, size_t ws_bytes,
                              eogp_stream_t stream);
 
+/* Several modules (a layer, or a stack of layers) of one batch of B examples
+ * with host-memory inputs, in one call: module u (descriptor L[u], inputs a[u]
+ * and s[u] in page-locked host memory, outputs codes[u] and scales[u], or
+ * out[u]) gets exactly the computation and outputs of
+ * eogp_compress_layer_host(L[u], a[u], s[u], B, chunk, out_mode, ...). One
+ * out_mode and one set of leading dimensions (ld_out, ld_codes, ld_scales)
+ * serve all modules. What the single call adds is overlap across modules. The
+ * workspace holds two sets of staging buffers, and of eigenbasis copies with
+ * bases_on_host, used by alternate modules. The copies of module u therefore
+ * wait only for the compute of module u - 2, and run while module u - 1 is
+ * computed. One call per module would wait for each previous module's
+ * compute.
+ *  - The first two modules' copies wait for the work already queued on
+ *    `stream`, as in eogp_compress_layer_host.
+ *  - The compute of every module is queued on `stream` in module order.
+ *  - The call releases its copy stream and events itself.
+ *  - The workspace size is the largest module's staging set twice, plus the
+ *    largest eogp_compress_layer workspace. With n = 1 it equals
+ *    eogp_compress_host_workspace_size.
+ * A library convenience for inputs that live in host memory: the paper times
+ * store construction including its host-to-device transfers (App. E.3) but
+ * gives no interface for it.
+ * Errors: as eogp_compress_layer_host; EOGP_EINVAL for n < 1 or a NULL array
+ * or entry. */
+int eogp_compress_layers_host_workspace_size(const eogp_layer_desc* const* L, int n, int B, int chunk,
+                                             int out_mode, size_t* bytes);
+int eogp_compress_layers_host(const eogp_layer_desc* const* L, int n, const void* const* a,
+                              const void* const* s, int B, int chunk, int out_mode, float* const* out,
+                              int ld_out, uint32_t* const* codes, int ld_codes, float* const* scales,
+                              int ld_scales, void* ws, size_t ws_bytes, eogp_stream_t stream);
+
 /* Same computation and outputs as eogp_compress_layer, for callers that cannot
  * allocate device memory (a plugin whose host framework owns every device
  * allocation, a service confined to a memory budget fixed at start-up, a C

@@ -737,17 +737,145 @@ HostLayout host_layout(const eogp_layer_desc* L, int B, int chunk, int mode) {
   return h;
 }
 
+// Several modules of one host-input call share one workspace: nsets sets of
+// staging buffers (and eigenbasis copies), used by alternate modules, each as
+// large as the largest module's, then the eogp_compress_layer workspace of the
+// largest. With one module this is exactly that module's HostLayout.
+struct HostMultiLayout {
+  int nsets = 1;
+  size_t set_bytes = 0, comp = 0, comp_bytes = 0, total = 0;
+};
+
+HostMultiLayout host_multi_layout(const eogp_layer_desc* const* L, int n, int B, int chunk, int mode) {
+  HostMultiLayout m;
+  m.nsets = n > 1 ? 2 : 1;
+  for (int u = 0; u < n; ++u) {
+    const HostLayout h = host_layout(L[u], B, chunk, mode);
+    m.set_bytes = std::max(m.set_bytes, al256(h.comp));
+    m.comp_bytes = std::max(m.comp_bytes, h.comp_bytes);
+  }
+  m.comp = static_cast<size_t>(m.nsets) * m.set_bytes;
+  m.total = m.comp + m.comp_bytes;
+  return m;
+}
+
 // Stream and events of one host-input call, released when it returns (the
-// runtime frees them once the work queued on them has completed).
+// runtime frees them once the work queued on them has completed). Per set of
+// staging buffers: chunk buffer b landed / computed, and the set's last module
+// computed.
 struct HostCallRes {
   cudaStream_t cs = nullptr;
-  cudaEvent_t entry = nullptr, landed[2] = {nullptr, nullptr}, done[2] = {nullptr, nullptr};
+  cudaEvent_t entry = nullptr, landed[2][2] = {}, done[2][2] = {}, set_done[2] = {};
   ~HostCallRes() {
-    for (cudaEvent_t e : {entry, landed[0], landed[1], done[0], done[1]})
-      if (e) cudaEventDestroy(e);
+    if (entry) cudaEventDestroy(entry);
+    for (int i = 0; i < 2; ++i) {
+      for (int j = 0; j < 2; ++j) {
+        if (landed[i][j]) cudaEventDestroy(landed[i][j]);
+        if (done[i][j]) cudaEventDestroy(done[i][j]);
+      }
+      if (set_done[i]) cudaEventDestroy(set_done[i]);
+    }
     if (cs) cudaStreamDestroy(cs);
   }
 };
+
+int check_host_modules(const eogp_layer_desc* const* L, int n, const void* const* a, const void* const* s,
+                       int B, int chunk, int out_mode, float* const* out, uint32_t* const* codes,
+                       float* const* scales) {
+  if (n < 1) return set_error(EOGP_EINVAL, "n must be >= 1");
+  if (!L || !a || !s) return set_error(EOGP_EINVAL, "descriptor / a / s array is NULL");
+  if (chunk < 0) return set_error(EOGP_EINVAL, "chunk must be >= 0");
+  for (int u = 0; u < n; ++u) {
+    if (int rc = check_desc(L[u], B, out_mode)) return rc;
+    if (B == 0) continue;
+    if (!a[u] || !s[u]) return set_error(EOGP_EINVAL, "a / s of module %d is NULL", u);
+    if (out_mode == EOGP_OUT_CODES) {
+      if (!codes || !scales || !codes[u] || !scales[u])
+        return set_error(EOGP_EINVAL, "codes / scales of module %d is NULL", u);
+    } else if (!out || !out[u]) {
+      return set_error(EOGP_EINVAL, "out of module %d is NULL", u);
+    }
+  }
+  return EOGP_OK;
+}
+
+// The modules' chunks, in order: copies on a copy stream, compute on `st`.
+// Module u uses set u % nsets; its copies first wait for the compute of the
+// module that last used the set (u - nsets), or, for the first modules, for
+// the work already queued on `st`.
+int run_host_modules(const eogp_layer_desc* const* L, int n, const void* const* a, const void* const* s, int B,
+                     int chunk, int out_mode, float* const* out, int ld_out, uint32_t* const* codes,
+                     int ld_codes, float* const* scales, int ld_scales, void* ws, size_t ws_bytes,
+                     cudaStream_t st) {
+  const HostMultiLayout m = host_multi_layout(L, n, B, chunk, out_mode);
+  if (!ws || ws_bytes < m.total)
+    return set_error(EOGP_EWORKSPACE, "workspace of %zu bytes needed, %zu given", m.total, ws_bytes);
+  if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
+  for (int u = 0; u < n; ++u)
+    if (int rc = check_device(L[u]->plan)) return rc;
+  char* w = static_cast<char*>(ws);
+  HostCallRes r;
+  CUDA_TRY(cudaStreamCreateWithFlags(&r.cs, cudaStreamNonBlocking));
+  CUDA_TRY(cudaEventCreateWithFlags(&r.entry, cudaEventDisableTiming));
+  for (int i = 0; i < m.nsets; ++i) {
+    for (int j = 0; j < 2; ++j) {
+      CUDA_TRY(cudaEventCreateWithFlags(&r.landed[i][j], cudaEventDisableTiming));
+      CUDA_TRY(cudaEventCreateWithFlags(&r.done[i][j], cudaEventDisableTiming));
+    }
+    CUDA_TRY(cudaEventCreateWithFlags(&r.set_done[i], cudaEventDisableTiming));
+  }
+  // Work already queued on `st` (an earlier call) may still read the staging
+  // buffers: the first copies wait for it.
+  CUDA_TRY(cudaEventRecord(r.entry, st));
+  CUDA_TRY(cudaStreamWaitEvent(r.cs, r.entry, 0));
+  const bool cd = out_mode == EOGP_OUT_CODES;
+  for (int u = 0; u < n; ++u) {
+    const eogp_layer_desc* Lu = L[u];
+    const int set = u % m.nsets;
+    char* base = w + static_cast<size_t>(set) * m.set_bytes;
+    // the set is free once the module that used it before has been computed
+    if (u >= m.nsets) CUDA_TRY(cudaStreamWaitEvent(r.cs, r.set_done[set], 0));
+    const HostLayout h = host_layout(Lu, B, chunk, out_mode);
+    const size_t esz = Lu->dtype == EOGP_F32 ? 4 : 2;
+    const size_t a_row = static_cast<size_t>(Lu->T) * Lu->d_in * esz;  // bytes of one example's a
+    const size_t s_row = static_cast<size_t>(Lu->T) * Lu->d_out * esz;
+    eogp_layer_desc d = *Lu;
+    if (Lu->bases_on_host) {
+      CUDA_TRY(cudaMemcpyAsync(base + h.va, Lu->VA, static_cast<size_t>(Lu->plan->nC()) * Lu->d_in * esz,
+                               cudaMemcpyDefault, r.cs));
+      CUDA_TRY(cudaMemcpyAsync(base + h.vs, Lu->VS, static_cast<size_t>(Lu->plan->nR()) * Lu->d_out * esz,
+                               cudaMemcpyDefault, r.cs));
+      d.VA = base + h.va;
+      d.VS = base + h.vs;
+      d.bases_on_host = 0;
+    }
+    const int n_chunks = (B + h.chunk - 1) / h.chunk;
+    for (int c = 0; c < n_chunks; ++c) {
+      const int b0 = c * h.chunk, nb = std::min(h.chunk, B - b0), buf = c & 1;
+      char* sa = base + h.stage[buf];
+      char* ss = sa + al256(h.a_bytes);
+      // Copy stream: the staging buffer is free once chunk c - 2 has been computed.
+      if (c >= 2) CUDA_TRY(cudaStreamWaitEvent(r.cs, r.done[set][buf], 0));
+      CUDA_TRY(cudaMemcpyAsync(sa, static_cast<const char*>(a[u]) + b0 * a_row, nb * a_row, cudaMemcpyDefault,
+                               r.cs));
+      CUDA_TRY(cudaMemcpyAsync(ss, static_cast<const char*>(s[u]) + b0 * s_row, nb * s_row, cudaMemcpyDefault,
+                               r.cs));
+      CUDA_TRY(cudaEventRecord(r.landed[set][buf], r.cs));
+      // Compute stream: chunk c once its inputs have landed.
+      CUDA_TRY(cudaStreamWaitEvent(st, r.landed[set][buf], 0));
+      d.lengths = Lu->lengths ? Lu->lengths + b0 : nullptr;
+      if (int rc = eogp_compress_layer(&d, sa, ss, nb, out_mode,
+                                       cd ? nullptr : out[u] + static_cast<size_t>(b0) * ld_out, ld_out,
+                                       cd ? codes[u] + static_cast<size_t>(b0) * ld_codes : nullptr, ld_codes,
+                                       cd ? scales[u] + static_cast<size_t>(b0) * ld_scales : nullptr, ld_scales,
+                                       w + m.comp, m.comp_bytes, reinterpret_cast<eogp_stream_t>(st)))
+        return rc;
+      CUDA_TRY(cudaEventRecord(r.done[set][buf], st));
+    }
+    CUDA_TRY(cudaEventRecord(r.set_done[set], st));
+  }
+  return EOGP_OK;
+}
 
 }  // namespace
 
@@ -757,7 +885,7 @@ extern "C" int eogp_compress_host_workspace_size(const eogp_layer_desc* L, int B
   if (!bytes) return set_error(EOGP_EINVAL, "bytes is NULL");
   if (chunk < 0) return set_error(EOGP_EINVAL, "chunk must be >= 0");
   if (int rc = check_desc(L, B, out_mode)) return rc;
-  *bytes = host_layout(L, B, chunk, out_mode).total;
+  *bytes = host_multi_layout(&L, 1, B, chunk, out_mode).total;
   return EOGP_OK;
 }
 
@@ -766,70 +894,34 @@ extern "C" int eogp_compress_layer_host(const eogp_layer_desc* L, const void* a,
                                         int ld_codes, float* scales, int ld_scales, void* ws,
                                         size_t ws_bytes, eogp_stream_t stream) {
   clear_error();
-  if (chunk < 0) return set_error(EOGP_EINVAL, "chunk must be >= 0");
-  if (int rc = check_desc(L, B, out_mode)) return rc;
+  if (int rc = check_host_modules(&L, 1, &a, &s, B, chunk, out_mode, &out, &codes, &scales)) return rc;
   if (B == 0) return EOGP_OK;
-  if (!a || !s) return set_error(EOGP_EINVAL, "a / s is NULL");
-  if (out_mode == EOGP_OUT_CODES) {
-    if (!codes || !scales) return set_error(EOGP_EINVAL, "codes / scales is NULL");
-  } else if (!out) {
-    return set_error(EOGP_EINVAL, "out is NULL");
-  }
-  const HostLayout h = host_layout(L, B, chunk, out_mode);
-  if (!ws || ws_bytes < h.total)
-    return set_error(EOGP_EWORKSPACE, "workspace of %zu bytes needed, %zu given", h.total, ws_bytes);
-  if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(EOGP_EINVAL, "workspace must be 256-byte aligned");
-  if (int rc = check_device(L->plan)) return rc;
-  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  char* w = static_cast<char*>(ws);
-  const size_t esz = L->dtype == EOGP_F32 ? 4 : 2;
-  const size_t a_row = static_cast<size_t>(L->T) * L->d_in * esz;   // bytes of one example's a
-  const size_t s_row = static_cast<size_t>(L->T) * L->d_out * esz;
-  HostCallRes r;
-  CUDA_TRY(cudaStreamCreateWithFlags(&r.cs, cudaStreamNonBlocking));
-  CUDA_TRY(cudaEventCreateWithFlags(&r.entry, cudaEventDisableTiming));
-  for (int i = 0; i < 2; ++i) {
-    CUDA_TRY(cudaEventCreateWithFlags(&r.landed[i], cudaEventDisableTiming));
-    CUDA_TRY(cudaEventCreateWithFlags(&r.done[i], cudaEventDisableTiming));
-  }
-  // Work already queued on `stream` (an earlier call) may still read the staging
-  // buffers: the first copies wait for it.
-  CUDA_TRY(cudaEventRecord(r.entry, st));
-  CUDA_TRY(cudaStreamWaitEvent(r.cs, r.entry, 0));
-  eogp_layer_desc d = *L;
-  if (L->bases_on_host) {
-    CUDA_TRY(cudaMemcpyAsync(w + h.va, L->VA, static_cast<size_t>(L->plan->nC()) * L->d_in * esz,
-                             cudaMemcpyDefault, r.cs));
-    CUDA_TRY(cudaMemcpyAsync(w + h.vs, L->VS, static_cast<size_t>(L->plan->nR()) * L->d_out * esz,
-                             cudaMemcpyDefault, r.cs));
-    d.VA = w + h.va;
-    d.VS = w + h.vs;
-    d.bases_on_host = 0;
-  }
-  const int n_chunks = (B + h.chunk - 1) / h.chunk;
-  for (int c = 0; c < n_chunks; ++c) {
-    const int b0 = c * h.chunk, nb = std::min(h.chunk, B - b0), buf = c & 1;
-    char* sa = w + h.stage[buf];
-    char* ss = sa + al256(h.a_bytes);
-    // Copy stream: the staging buffer is free once chunk c - 2 has been computed.
-    if (c >= 2) CUDA_TRY(cudaStreamWaitEvent(r.cs, r.done[buf], 0));
-    CUDA_TRY(cudaMemcpyAsync(sa, static_cast<const char*>(a) + b0 * a_row, nb * a_row,
-                             cudaMemcpyDefault, r.cs));
-    CUDA_TRY(cudaMemcpyAsync(ss, static_cast<const char*>(s) + b0 * s_row, nb * s_row,
-                             cudaMemcpyDefault, r.cs));
-    CUDA_TRY(cudaEventRecord(r.landed[buf], r.cs));
-    // Compute stream: chunk c once its inputs have landed.
-    CUDA_TRY(cudaStreamWaitEvent(st, r.landed[buf], 0));
-    d.lengths = L->lengths ? L->lengths + b0 : nullptr;
-    const bool cd = out_mode == EOGP_OUT_CODES;
-    if (int rc = eogp_compress_layer(&d, sa, ss, nb, out_mode, cd ? nullptr : out + static_cast<size_t>(b0) * ld_out,
-                                     ld_out, cd ? codes + static_cast<size_t>(b0) * ld_codes : nullptr, ld_codes,
-                                     cd ? scales + static_cast<size_t>(b0) * ld_scales : nullptr, ld_scales,
-                                     w + h.comp, h.comp_bytes, stream))
-      return rc;
-    CUDA_TRY(cudaEventRecord(r.done[buf], st));
-  }
+  return run_host_modules(&L, 1, &a, &s, B, chunk, out_mode, &out, ld_out, &codes, ld_codes, &scales, ld_scales,
+                          ws, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+extern "C" int eogp_compress_layers_host_workspace_size(const eogp_layer_desc* const* L, int n, int B, int chunk,
+                                                        int out_mode, size_t* bytes) {
+  clear_error();
+  if (!bytes) return set_error(EOGP_EINVAL, "bytes is NULL");
+  if (n < 1) return set_error(EOGP_EINVAL, "n must be >= 1");
+  if (!L) return set_error(EOGP_EINVAL, "descriptor array is NULL");
+  if (chunk < 0) return set_error(EOGP_EINVAL, "chunk must be >= 0");
+  for (int u = 0; u < n; ++u)
+    if (int rc = check_desc(L[u], B, out_mode)) return rc;
+  *bytes = host_multi_layout(L, n, B, chunk, out_mode).total;
   return EOGP_OK;
+}
+
+extern "C" int eogp_compress_layers_host(const eogp_layer_desc* const* L, int n, const void* const* a,
+                                         const void* const* s, int B, int chunk, int out_mode, float* const* out,
+                                         int ld_out, uint32_t* const* codes, int ld_codes, float* const* scales,
+                                         int ld_scales, void* ws, size_t ws_bytes, eogp_stream_t stream) {
+  clear_error();
+  if (int rc = check_host_modules(L, n, a, s, B, chunk, out_mode, out, codes, scales)) return rc;
+  if (B == 0) return EOGP_OK;
+  return run_host_modules(L, n, a, s, B, chunk, out_mode, out, ld_out, codes, ld_codes, scales, ld_scales, ws,
+                          ws_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
 
 // ================================================================ EK-FAC correction

@@ -85,6 +85,11 @@ EXPORTS = {
     "eogp_compress_layer_host": (c_int, [POINTER(LayerDesc), c_void_p, c_void_p, c_int, c_int, c_int,
                                          c_void_p, c_int, c_void_p, c_int, c_void_p, c_int, c_void_p,
                                          c_size_t, c_void_p]),
+    "eogp_compress_layers_host_workspace_size": (c_int, [POINTER(POINTER(LayerDesc)), c_int, c_int, c_int, c_int,
+                                                         POINTER(c_size_t)]),
+    "eogp_compress_layers_host": (c_int, [POINTER(POINTER(LayerDesc)), c_int, POINTER(c_void_p), POINTER(c_void_p),
+                                          c_int, c_int, c_int, POINTER(c_void_p), c_int, POINTER(c_void_p), c_int,
+                                          POINTER(c_void_p), c_int, c_void_p, c_size_t, c_void_p]),
     "eogp_ekfac_workspace_size": (c_int, [POINTER(EkfacDesc), c_int, POINTER(c_size_t)]),
     "eogp_ekfac_accumulate": (c_int, [POINTER(EkfacDesc), c_void_p, c_void_p, c_int, c_void_p, c_int,
                                       c_int, c_void_p, c_size_t, c_void_p]),
@@ -390,6 +395,70 @@ def compress_layer_host(desc: LayerDesc, a, s, out_mode: int, device, chunk: int
     _check(lib().eogp_compress_layer_host(ctypes.byref(desc), _ptr(a), _ptr(s), B, int(chunk), out_mode,
                                           _ptr(out), out.stride(0), None, 0, None, 0, _ptr(ws),
                                           ws.numel(), _stream(stream)))
+    return out
+
+
+def _desc_array(descs):
+    return (POINTER(LayerDesc) * len(descs))(*[ctypes.pointer(d) for d in descs])
+
+
+def _ptr_array(ts):
+    return (c_void_p * len(ts))(*[t.data_ptr() for t in ts])
+
+
+def _common_ld(ts, name: str) -> int:
+    lds = {t.stride(0) for t in ts}
+    if len(lds) != 1:
+        raise ValueError(f"{name}: every module's view must have the same leading dimension")
+    return lds.pop()
+
+
+def compress_layers_host_workspace_size(descs: Sequence[LayerDesc], B: int, out_mode: int, chunk: int = 0) -> int:
+    n = c_size_t()
+    _check(lib().eogp_compress_layers_host_workspace_size(_desc_array(descs), len(descs), int(B), int(chunk),
+                                                          int(out_mode), ctypes.byref(n)))
+    return n.value
+
+
+def compress_layers_host(descs: Sequence[LayerDesc], a, s, out_mode: int, device, chunk: int = 0, out=None,
+                         codes=None, scales=None, ws=None, stream=None):
+    """eogp_compress_layers_host: module u compresses host tensors a[u] [B, T, d_in]
+    and s[u] [B, T, d_out] (page-locked) into codes[u] / scales[u] (OUT_CODES) or
+    out[u], all on `device`; the copies of one module overlap the compute of the
+    previous one. Output views of one kind share one leading dimension."""
+    import torch
+    n = len(descs)
+    if len(a) != n or len(s) != n:
+        raise ValueError("one a and one s per descriptor")
+    for t in list(a) + list(s):
+        _dense(t, "a / s")
+        if t.is_cuda:
+            raise ValueError("compress_layers_host takes host tensors (use compress_layer for device ones)")
+    B = a[0].shape[0]
+    if any(t.shape[0] != B for t in list(a) + list(s)):
+        raise ValueError("every module's a and s must hold the same B examples")
+    if ws is None:
+        ws = workspace(compress_layers_host_workspace_size(descs, B, out_mode, chunk), device)
+    if out_mode == OUT_CODES:
+        if codes is None:
+            codes = [torch.empty((B, (d.k + 31) // 32), dtype=torch.int32, device=device) for d in descs]
+        if scales is None:
+            scales = [torch.empty((B,), dtype=torch.float32, device=device) for _ in descs]
+        for t in codes:
+            _rows(t, "codes")
+        _check(lib().eogp_compress_layers_host(_desc_array(descs), n, _ptr_array(a), _ptr_array(s), B, int(chunk),
+                                               out_mode, None, 0, _ptr_array(codes), _common_ld(codes, "codes"),
+                                               _ptr_array(scales), _common_ld(scales, "scales"), _ptr(ws),
+                                               ws.numel(), _stream(stream)))
+        return codes, scales
+    if out is None:
+        out = [torch.empty((B, d.m if out_mode == OUT_FIRST_STAGE else d.k), dtype=torch.float32, device=device)
+               for d in descs]
+    for t in out:
+        _rows(t, "out")
+    _check(lib().eogp_compress_layers_host(_desc_array(descs), n, _ptr_array(a), _ptr_array(s), B, int(chunk),
+                                           out_mode, _ptr_array(out), _common_ld(out, "out"), None, 0, None, 0,
+                                           _ptr(ws), ws.numel(), _stream(stream)))
     return out
 
 

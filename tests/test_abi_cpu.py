@@ -185,6 +185,41 @@ def test_host_input_call_argument_checks():
     assert L.eogp_compress_layer_host(*args) == E.EWORKSPACE
 
 
+def test_several_modules_host_call_argument_checks():
+    """eogp_compress_layers_host / _workspace_size: argument checks that run before
+    any device work, and the workspace of one module equals the one-module call's."""
+    import ctypes
+    lam = np.arange(1, 9, dtype=np.float64) ** -1.0
+    plan = E.Plan.from_factors(lam, lam, 10, 0.1)
+    desc = E.LayerDesc(8, 8, 64, 10, 4, E.F32, 16, 16, 16, plan.handle)
+    desc2 = E.LayerDesc(8, 8, 32, 10, 4, E.F32, 16, 16, 16, plan.handle)   # T = 32: smaller staging
+    L = E.lib()
+    one, two, ref = ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_size_t()
+    arr1 = E._desc_array([desc])
+    arr2 = E._desc_array([desc, desc2])
+    assert L.eogp_compress_host_workspace_size(ctypes.byref(desc), 6, 2, E.OUT_CODES, ctypes.byref(ref)) == E.OK
+    assert L.eogp_compress_layers_host_workspace_size(arr1, 1, 6, 2, E.OUT_CODES, ctypes.byref(one)) == E.OK
+    assert one.value == ref.value
+    assert L.eogp_compress_layers_host_workspace_size(arr2, 2, 6, 2, E.OUT_CODES, ctypes.byref(two)) == E.OK
+    assert two.value > one.value    # two staging sets
+    assert L.eogp_compress_layers_host_workspace_size(arr2, 0, 6, 2, E.OUT_CODES, ctypes.byref(two)) == E.EINVAL
+    assert L.eogp_compress_layers_host_workspace_size(None, 1, 6, 2, E.OUT_CODES, ctypes.byref(two)) == E.EINVAL
+    assert L.eogp_compress_layers_host_workspace_size(arr1, 1, 6, -1, E.OUT_CODES, ctypes.byref(two)) == E.EINVAL
+    ptrs = (ctypes.c_void_p * 2)(16, 16)
+    args = [arr2, 2, ptrs, ptrs, 2, 0, E.OUT_CODES, None, 0, ptrs, 16, ptrs, 1, 256, two.value, None]
+    assert L.eogp_compress_layers_host(*args) == E.EINVAL          # host-only plan
+    args[1] = 0
+    assert L.eogp_compress_layers_host(*args) == E.EINVAL          # n < 1
+    args[1], args[2] = 2, None
+    assert L.eogp_compress_layers_host(*args) == E.EINVAL          # no a array
+    args[2], args[9] = ptrs, None
+    assert L.eogp_compress_layers_host(*args) == E.EINVAL          # no codes array
+    args[9], args[4] = ptrs, 0
+    assert L.eogp_compress_layers_host(*args) == E.OK              # empty batch: nothing to do
+    args[4], args[13] = 2, None
+    assert L.eogp_compress_layers_host(*args) == E.EWORKSPACE
+
+
 def test_selftest_wait_argument_checks():
     """eogp_selftest_wait_timeout refuses limits outside [1, 1e9] before any device call."""
     L = E.lib()

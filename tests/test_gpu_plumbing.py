@@ -197,6 +197,81 @@ def test_host_inputs_match_device_inputs(dtype, d_in, d_out, T, B, m, k, chunk, 
     assert torch.equal(c1, c2) and torch.equal(s1, s2)
 
 
+def _host_module(rng, d_in, d_out, T, m, k, host_bases, lengths=None):
+    """One bf16 module: plan, descriptor, its own inputs (host and device)."""
+    rnd = (lambda v: synth.round_to(v, "bf16"))
+    tdt = torch.bfloat16
+    QA, QS = rnd(synth.haar_orthogonal(d_in, rng)), rnd(synth.haar_orthogonal(d_out, rng))
+    plan = E.Plan.from_factors(synth.power_spectrum(d_out, 1.2), synth.power_spectrum(d_in, 1.2), m, 0.1)
+    R, C = plan.sets()
+    VA = torch.from_numpy(np.ascontiguousarray(QA.T[C], dtype=np.float32)).to(tdt)
+    VS = torch.from_numpy(np.ascontiguousarray(QS.T[R], dtype=np.float32)).to(tdt)
+    if host_bases:
+        hva, hvs = E.host_empty(VA.shape, tdt), E.host_empty(VS.shape, tdt)
+        hva.copy_(VA)
+        hvs.copy_(VS)
+        VA, VS = hva, hvs
+    else:
+        VA, VS = VA.to(DEV), VS.to(DEV)
+    Pt = dev(rnd(synth.haar_orthogonal(m, rng, k).T).astype(np.float32), tdt)
+    desc = E.layer_desc(plan, T, k, VA, VS, Pt, lengths=lengths)
+    return plan, desc, (VA, VS, Pt)
+
+
+@pytest.mark.parametrize("n,chunk,host_bases", [(5, 2, (True, False, True)), (1, 0, (True,)),
+                                                (4, 0, (False, True)), (3, 1, (True, True, True))])
+def test_several_modules_host_call_matches_device_inputs(n, chunk, host_bases):
+    """eogp_compress_layers_host (the modules of a stack in one call, staging sets
+    alternating between modules so that one module's copies overlap the previous
+    one's compute) gives each module the results of eogp_compress_layer on the
+    same inputs in device memory, bit for bit: modules of different shapes
+    (different staging sizes in one workspace), host and device eigenbases,
+    ragged chunks, per-example lengths, codes written into strided views of one
+    output like a stack's, and the coordinates mode."""
+    rng = np.random.default_rng(100 * n + chunk)
+    T, B, k, m = 64, 5, 256, 2048
+    shapes = [(768, 2304), (768, 768), (2304, 768)]
+    lv = rng.integers(1, T + 1, B).astype(np.int32)
+    lv[0] = T
+    lengths = dev(lv)
+    types = [_host_module(rng, di, do, T, m, k, host_bases[t % len(host_bases)], lengths)
+             for t, (di, do) in enumerate(shapes)]
+    descs, ah, sh, ad, sd = [], [], [], [], []
+    for u in range(n):
+        plan, desc, _ = types[u % len(types)]
+        di, do = shapes[u % len(types)]
+        a = torch.from_numpy(synth.round_to(rng.standard_normal((B, T, di)), "bf16").astype(np.float32))
+        s = torch.from_numpy(synth.round_to(rng.standard_normal((B, T, do)) * 0.1, "bf16").astype(np.float32))
+        a, s = a.to(torch.bfloat16), s.to(torch.bfloat16)
+        ha, hs = E.host_empty(a.shape, torch.bfloat16), E.host_empty(s.shape, torch.bfloat16)
+        ha.copy_(a)
+        hs.copy_(s)
+        descs.append(desc)
+        ah.append(ha)
+        sh.append(hs)
+        ad.append(a.to(DEV))
+        sd.append(s.to(DEV))
+    wd = (k + 31) // 32
+    codes = torch.zeros((B, n * wd), dtype=torch.int32, device=DEV)
+    scales = torch.zeros((B, n), dtype=torch.float32, device=DEV)
+    E.compress_layers_host(descs, ah, sh, E.OUT_CODES, DEV, chunk=chunk,
+                           codes=[codes[:, u * wd:(u + 1) * wd] for u in range(n)],
+                           scales=[scales[:, u] for u in range(n)])
+    outs = E.compress_layers_host(descs, ah, sh, E.OUT_COORDS, DEV, chunk=chunk)
+    if n == 1:
+        assert E.compress_layers_host_workspace_size(descs, B, E.OUT_CODES, chunk) == \
+            E.compress_host_workspace_size(descs[0], B, E.OUT_CODES, chunk)
+    torch.cuda.synchronize()
+    for u in range(n):
+        c1, s1 = E.compress_layer(descs[u], ad[u], sd[u], E.OUT_CODES)
+        x1 = E.compress_layer(descs[u], ad[u], sd[u], E.OUT_COORDS)
+        torch.cuda.synchronize()
+        assert torch.equal(codes[:, u * wd:(u + 1) * wd], c1), u
+        assert torch.equal(scales[:, u], s1), u
+        assert torch.equal(outs[u], x1), u
+    E.sync_status()
+
+
 def test_host_empty_memory_round_trip():
     """eogp_host_alloc memory (through host_empty): zero-filled, writable, copies
     to and from the device asynchronously, and is released with the tensor."""
